@@ -1,0 +1,246 @@
+/*
+ * lamb.h -- C ABI of the GB300 (sm_103a) layerwise-adaptive optimizer step.
+ *
+ * The library applies one step of LAMB (You et al., "Large Batch
+ * Optimization for Deep Learning: Training BERT in 76 minutes", ICLR 2020,
+ * Algorithm 2) or LARS (Algorithm 1 of the same paper) to every parameter
+ * tensor of a model in one call.  A "block" x^(i) of Section 2 is one
+ * parameter tensor here; norms, trust ratios and weight decay are per tensor.
+ *
+ * Per tensor k, with step count t >= 1, lambda_k = lambda * mask_k:
+ *   LAMB (Algorithm 2):
+ *     m <- beta1 m + (1-beta1) g,          v <- beta2 v + (1-beta2) g^2
+ *     r  = (m / (1-beta1^t)) / (sqrt(v / (1-beta2^t)) + eps) + lambda_k w
+ *     rho_k = phi(||w_k||) / ||r_k||       (1 if either norm is 0)
+ *     w <- w - eta * rho_k * r
+ *   LARS (Algorithm 1, with a trust coefficient kappa):
+ *     m <- beta1 m + (1-beta1) (g + lambda_k w)
+ *     rho_k = kappa * phi(||w_k||) / ||m_k|| (1 if either norm is 0)
+ *     w <- w - eta * rho_k * m
+ *   phi (Section 3) is the identity or min(max(z, gamma_l), gamma_u).
+ * m and v are stored without bias correction; the correction is applied only
+ * where r is formed.  eps is added outside the square root.
+ *
+ * Types and layout: w, m, v are contiguous float32 arrays (one per tensor);
+ * g is float32 or bfloat16; an optional bfloat16 copy of the new w is written
+ * with round-to-nearest-even.  All tensor pointers are DEVICE pointers on the
+ * plan's device.  Pointers aligned to 16 bytes (8 bytes for bfloat16 arrays)
+ * take the vectorised path; others are handled element by element.
+ *
+ * Ownership: the caller owns w, g, m, v, the bf16 copy, the step counter,
+ * the learning rate and the streams.  The plan owns its chunk table, pointer
+ * table, partial sums, norms, trust ratios and counters, and frees them in
+ * lamb_plan_destroy.  Bound pointers must stay valid until the last step
+ * that uses them has completed.
+ *
+ * Errors: every call returns a lamb_status_t; nothing throws across the ABI.
+ * Argument errors are detected on the host before any launch; a
+ * thread-local message is available from lamb_last_error().  CUDA launch
+ * errors are reported without synchronising.  Conditions only visible on
+ * the device (a step count < 1, non-finite norms) set bits in the plan's
+ * device status word, read with lamb_plan_query().
+ *
+ * Threading: a plan may be used from one host thread at a time.
+ */
+#ifndef LAMB_GB300_H
+#define LAMB_GB300_H
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define LAMB_ABI_VERSION 1
+
+/* Only the entry points below are exported from liblamb.so. */
+#if defined(__GNUC__)
+#define LAMB_API __attribute__((visibility("default")))
+#else
+#define LAMB_API
+#endif
+
+typedef enum {
+  LAMB_OK = 0,
+  LAMB_ERR_INVALID_ARG = 1,        /* bad size, count, pointer or value   */
+  LAMB_ERR_UNSUPPORTED_DTYPE = 2,  /* dtype code not supported here       */
+  LAMB_ERR_CUDA = 3,               /* a CUDA runtime call or launch failed */
+  LAMB_ERR_OOM = 4,                /* device allocation failed            */
+  LAMB_ERR_NOT_BOUND = 5           /* step before lamb_plan_bind, or the
+                                      array the step needs was not bound  */
+} lamb_status_t;
+
+typedef enum {
+  LAMB_DTYPE_NONE = -1,            /* "no bf16 copy"                      */
+  LAMB_F32 = 0,
+  LAMB_BF16 = 1
+} lamb_dtype_t;
+
+/* phi of Section 3 */
+typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
+
+/* lamb_hyper_t.flags */
+#define LAMB_FLAG_BIAS_CORRECTION 0x1u  /* divide by (1-beta^t), Alg. 2 and
+                                           the appendix on adam-correction */
+#define LAMB_FLAG_INCREMENT_STEP  0x2u  /* the step writes *d_step = t + 1
+                                           on the device when it completes */
+
+/* bits of the device status word (lamb_plan_query) */
+#define LAMB_STATUS_NONFINITE 0x1u      /* a tensor's sum of w^2 or of r^2
+                                           (LARS: m^2) was Inf/NaN         */
+#define LAMB_STATUS_BAD_STEP  0x2u      /* *d_step < 1 with bias correction:
+                                           the step was skipped, nothing was
+                                           written                          */
+
+/* Hyperparameters.  Doubles on purpose: (1 - beta) is formed in double and
+ * rounded once to float, so e.g. beta2 = 0.999 gives 1-beta2 = 0.001 to
+ * float precision.  eta and t are read from device memory instead (any
+ * schedule stays on the device; the step is CUDA-graph capturable). */
+typedef struct {
+  double beta1;          /* Alg. 1/2 beta1 (LARS momentum)                  */
+  double beta2;          /* Alg. 2 beta2 (ignored by lars_step)             */
+  double eps;            /* Alg. 2 epsilon (ignored by lars_step)           */
+  double weight_decay;   /* lambda; applied to tensors whose mask is 1      */
+  double gamma_l;        /* phi clip bounds, used when phi == LAMB_PHI_CLIP */
+  double gamma_u;
+  double trust_coef;     /* LARS kappa (ignored by lamb_step)               */
+  int32_t phi;           /* lamb_phi_t                                      */
+  uint32_t flags;        /* LAMB_FLAG_*                                     */
+} lamb_hyper_t;
+
+/* Optional plan-creation knobs (pass NULL for defaults). */
+typedef struct {
+  int32_t chunk_elems;   /* elements per chunk, multiple of 1024 in
+                            [1024, 1<<24]; 0 = default (16384)             */
+  int32_t blocks_per_sm; /* resident CTAs per SM for the persistent grid;
+                            0 = as many as the occupancy calculator allows */
+} lamb_plan_options_t;
+
+typedef struct {
+  int32_t n_tensors;
+  int32_t n_chunks;
+  int64_t n_params;
+  int32_t chunk_elems;
+  int32_t grid_blocks;       /* CTAs per launch (persistent grid)           */
+  int32_t threads_per_block;
+  int32_t num_sms;
+  int32_t device;
+  int32_t grad_dtype;
+  int32_t copy_dtype;
+  int32_t bound;             /* 1 after a successful lamb_plan_bind         */
+  int32_t n_vector_tensors;  /* tensors on the vectorised path (after bind) */
+  int64_t device_bytes;      /* device memory owned by the plan             */
+} lamb_plan_info_t;
+
+typedef struct lamb_plan* lamb_plan_t;
+
+/* Build a plan for n_tensors tensors of the given element counts.
+ *   sizes       host array [n_tensors], each >= 0 (0-element tensors are
+ *               allowed: they get trust ratio 1 and norms 0).
+ *   decay_mask  host array [n_tensors]; 1 = weight decay applies (lambda_k =
+ *               lambda), 0 = masked (lambda_k = 0).  NULL = all 1.
+ *   grad_dtype  LAMB_F32 or LAMB_BF16.
+ *   copy_dtype  LAMB_DTYPE_NONE or LAMB_BF16 (bf16 copy of the new w).
+ *   device      CUDA device ordinal; the plan's memory lives there.
+ *   opts        NULL or tuning knobs.
+ * Cuts every tensor into chunks of chunk_elems elements and uploads the chunk
+ * table (tensor id, offset, length) once.  Synchronous; not capturable.
+ * Errors: INVALID_ARG (n_tensors < 1, a negative size, total > 2^62 elements,
+ * more than 2^30 chunks, bad opts), UNSUPPORTED_DTYPE, CUDA, OOM. */
+LAMB_API lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
+                               const uint8_t* decay_mask, int32_t grad_dtype,
+                               int32_t copy_dtype, int32_t device,
+                               const lamb_plan_options_t* opts,
+                               lamb_plan_t* out);
+
+/* Bind the tensors' device pointers (host arrays of n_tensors pointers).
+ * w, g, m are required; v is required by lamb_step only (NULL for a
+ * LARS-only plan); w_copy is required iff the plan has a bf16 copy.  A
+ * pointer may be NULL only for a 0-element tensor.  Records per tensor
+ * whether every array is aligned for 128-bit access.  Uploads the pointer
+ * table on `stream` and synchronises it; not capturable.  Re-binding is
+ * allowed between steps. */
+LAMB_API lamb_status_t lamb_plan_bind(lamb_plan_t plan, void* const* w,
+                             const void* const* g, void* const* m,
+                             void* const* v, void* const* w_copy,
+                             cudaStream_t stream);
+
+/* One LAMB step (Algorithm 2) over every tensor, enqueued on `stream`.
+ *   d_step  DEVICE int64: t (>= 1 when bias correction is on).  Needed when
+ *           LAMB_FLAG_BIAS_CORRECTION or LAMB_FLAG_INCREMENT_STEP is set,
+ *           else may be NULL.
+ *   d_lr    DEVICE float: eta_t for this step.
+ * Updates w, m, v in place (and the bf16 copy); g is read only.  Writes the
+ * per-tensor norms and trust ratios (lamb_plan_trust_ratios).  No host
+ * synchronisation, allocation or pageable copy: capturable in a CUDA graph,
+ * and replays of the graph read the current *d_step and *d_lr. */
+LAMB_API lamb_status_t lamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                        int64_t* d_step, const float* d_lr,
+                        cudaStream_t stream);
+
+/* One LARS step (Algorithm 1 with trust coefficient kappa) over every
+ * tensor.  Uses w, g, m (v is not touched).  beta1 is the momentum; the
+ * momentum is damped by (1-beta1) as in Algorithm 1.  d_step is read only for
+ * LAMB_FLAG_INCREMENT_STEP (may be NULL otherwise).  Same capture and
+ * ownership rules as lamb_step. */
+LAMB_API lamb_status_t lars_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                        int64_t* d_step, const float* d_lr,
+                        cudaStream_t stream);
+
+/* DEVICE arrays [n_tensors] of the last step's trust ratio rho_k, ||w_k||
+ * and ||r_k|| (LARS: ||m_k||), in double.  Owned by the plan; valid until
+ * destroy; overwritten by the next step.  Any out pointer may be NULL. */
+LAMB_API lamb_status_t lamb_plan_trust_ratios(lamb_plan_t plan, const double** d_ratio,
+                                     const double** d_wnorm,
+                                     const double** d_unorm);
+
+/* Copy the last step's per-tensor results (as lamb_plan_trust_ratios) into
+ * caller-owned arrays of n_tensors doubles -- device or host memory, any of
+ * the three may be NULL -- with cudaMemcpyAsync on `stream` (kind inferred
+ * from the addresses).  Does not synchronise; with device destinations it is
+ * capturable. */
+LAMB_API lamb_status_t lamb_plan_copy_trust_ratios(lamb_plan_t plan, double* ratio,
+                                          double* wnorm, double* unorm,
+                                          cudaStream_t stream);
+
+/* Read (and optionally clear) the device status word (LAMB_STATUS_* bits).
+ * Synchronises `stream`; not capturable. */
+LAMB_API lamb_status_t lamb_plan_query(lamb_plan_t plan, uint32_t* status_bits,
+                              int32_t clear, cudaStream_t stream);
+
+LAMB_API lamb_status_t lamb_plan_get_info(lamb_plan_t plan, lamb_plan_info_t* info);
+
+/* Instrumentation: when enabled, each step records CUDA events on its
+ * stream around every kernel it launches (up to 4096 steps are kept).
+ * lamb_plan_read_timing waits for those events, returns the number of steps
+ * recorded and the summed device time of each kernel in milliseconds
+ * (ms_per_kernel[0..n_kernels-1]; a LAMB or LARS step launches 2 kernels),
+ * and clears the record. */
+LAMB_API lamb_status_t lamb_plan_set_timing(lamb_plan_t plan, int32_t enable);
+LAMB_API lamb_status_t lamb_plan_read_timing(lamb_plan_t plan, int32_t* n_steps,
+                                    double* ms_per_kernel, int32_t n_kernels);
+
+/* Frees everything the plan owns (synchronises the plan's device). */
+LAMB_API lamb_status_t lamb_plan_destroy(lamb_plan_t plan);
+
+/* Host-only planner, no device needed: the chunk table lamb_plan_create
+ * would build.  Writes up to `capacity` rows into the three host arrays
+ * (any may be NULL when capacity is 0) and the total row count into
+ * *n_chunks.  INVALID_ARG on bad sizes/chunk_elems or capacity too small
+ * (n_chunks is still written). */
+LAMB_API lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
+                                 int32_t chunk_elems, int32_t* chunk_tensor,
+                                 int64_t* chunk_offset, int32_t* chunk_len,
+                                 int32_t capacity, int32_t* n_chunks);
+
+/* Message of the last failed call on this host thread ("" if none). */
+LAMB_API const char* lamb_last_error(void);
+
+/* LAMB_ABI_VERSION of the built library. */
+LAMB_API int32_t lamb_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LAMB_GB300_H */

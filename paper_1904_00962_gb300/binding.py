@@ -1,0 +1,257 @@
+"""ctypes binding of liblamb.so -- argument marshalling only.
+
+Every function has the name of the C entry point it wraps (include/lamb.h)
+and raises LambError when the C call returns a non-zero status.  Pointers
+are Python ints (device addresses, e.g. ``tensor.data_ptr()``); streams are
+raw cudaStream_t handles as ints (``torch.cuda.current_stream().cuda_stream``)
+or 0 for the legacy default stream.  No arithmetic of the method happens
+here: every step runs in the CUDA kernels of the library.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+from ctypes import (POINTER, Structure, byref, c_char_p, c_double, c_int32,
+                    c_int64, c_uint8, c_uint32, c_void_p)
+
+import numpy as np
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_build",
+                        "liblamb.so")
+
+# status codes
+LAMB_OK = 0
+LAMB_ERR_INVALID_ARG = 1
+LAMB_ERR_UNSUPPORTED_DTYPE = 2
+LAMB_ERR_CUDA = 3
+LAMB_ERR_OOM = 4
+LAMB_ERR_NOT_BOUND = 5
+# dtypes
+LAMB_DTYPE_NONE = -1
+LAMB_F32 = 0
+LAMB_BF16 = 1
+# phi
+LAMB_PHI_IDENTITY = 0
+LAMB_PHI_CLIP = 1
+# flags / status bits
+LAMB_FLAG_BIAS_CORRECTION = 0x1
+LAMB_FLAG_INCREMENT_STEP = 0x2
+LAMB_STATUS_NONFINITE = 0x1
+LAMB_STATUS_BAD_STEP = 0x2
+
+EXPORTED = ["lamb_plan_create", "lamb_plan_bind", "lamb_step", "lars_step",
+            "lamb_plan_trust_ratios", "lamb_plan_copy_trust_ratios",
+            "lamb_plan_query", "lamb_plan_get_info",
+            "lamb_plan_set_timing", "lamb_plan_read_timing",
+            "lamb_plan_destroy", "lamb_layout_chunks", "lamb_last_error",
+            "lamb_abi_version"]
+
+
+class LambError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"liblamb status {status}: {message}")
+        self.status = status
+
+
+class LambLibraryMissing(ImportError):
+    pass
+
+
+class lamb_hyper_t(Structure):
+    _fields_ = [("beta1", c_double), ("beta2", c_double), ("eps", c_double),
+                ("weight_decay", c_double), ("gamma_l", c_double),
+                ("gamma_u", c_double), ("trust_coef", c_double),
+                ("phi", c_int32), ("flags", c_uint32)]
+
+
+class lamb_plan_options_t(Structure):
+    _fields_ = [("chunk_elems", c_int32), ("blocks_per_sm", c_int32)]
+
+
+class lamb_plan_info_t(Structure):
+    _fields_ = [("n_tensors", c_int32), ("n_chunks", c_int32),
+                ("n_params", c_int64), ("chunk_elems", c_int32),
+                ("grid_blocks", c_int32), ("threads_per_block", c_int32),
+                ("num_sms", c_int32), ("device", c_int32),
+                ("grad_dtype", c_int32), ("copy_dtype", c_int32),
+                ("bound", c_int32), ("n_vector_tensors", c_int32),
+                ("device_bytes", c_int64)]
+
+
+_lib = None
+
+
+def load(path: str | None = None) -> ctypes.CDLL:
+    """Load liblamb.so once; raises LambLibraryMissing if it is not built."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise LambLibraryMissing(
+            f"{p} not found: build it with `python -m "
+            f"paper_1904_00962_gb300.build` (needs nvcc)")
+    lib = ctypes.CDLL(p)
+    vp = c_void_p
+    lib.lamb_plan_create.argtypes = [POINTER(c_int64), c_int32,
+                                     POINTER(c_uint8), c_int32, c_int32,
+                                     c_int32, POINTER(lamb_plan_options_t),
+                                     POINTER(vp)]
+    lib.lamb_plan_bind.argtypes = [vp, POINTER(vp), POINTER(vp), POINTER(vp),
+                                   POINTER(vp), POINTER(vp), vp]
+    for name in ("lamb_step", "lars_step"):
+        getattr(lib, name).argtypes = [vp, POINTER(lamb_hyper_t), vp, vp, vp]
+    lib.lamb_plan_trust_ratios.argtypes = [vp, POINTER(vp), POINTER(vp),
+                                           POINTER(vp)]
+    lib.lamb_plan_copy_trust_ratios.argtypes = [vp, vp, vp, vp, vp]
+    lib.lamb_plan_query.argtypes = [vp, POINTER(c_uint32), c_int32, vp]
+    lib.lamb_plan_get_info.argtypes = [vp, POINTER(lamb_plan_info_t)]
+    lib.lamb_plan_set_timing.argtypes = [vp, c_int32]
+    lib.lamb_plan_read_timing.argtypes = [vp, POINTER(c_int32),
+                                          POINTER(c_double), c_int32]
+    lib.lamb_plan_destroy.argtypes = [vp]
+    lib.lamb_layout_chunks.argtypes = [POINTER(c_int64), c_int32, c_int32,
+                                       POINTER(c_int32), POINTER(c_int64),
+                                       POINTER(c_int32), c_int32,
+                                       POINTER(c_int32)]
+    for name in EXPORTED:
+        if name in ("lamb_last_error", "lamb_abi_version"):
+            continue
+        getattr(lib, name).restype = c_int32
+    lib.lamb_last_error.restype = c_char_p
+    lib.lamb_last_error.argtypes = []
+    lib.lamb_abi_version.restype = c_int32
+    lib.lamb_abi_version.argtypes = []
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def _check(status: int) -> None:
+    if status != LAMB_OK:
+        raise LambError(status, lamb_last_error())
+
+
+def _ptr_array(ptrs):
+    if ptrs is None:
+        return None
+    return (c_void_p * len(ptrs))(*[int(p) if p else None for p in ptrs])
+
+
+def lamb_last_error() -> str:
+    return load().lamb_last_error().decode()
+
+
+def lamb_abi_version() -> int:
+    return int(load().lamb_abi_version())
+
+
+def make_hyper(*, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01,
+               phi="identity", gamma_l=0.0, gamma_u=math.inf, trust_coef=1.0,
+               bias_correction=True, increment_step=False) -> lamb_hyper_t:
+    """Fill a lamb_hyper_t (plain field copy)."""
+    flags = (LAMB_FLAG_BIAS_CORRECTION if bias_correction else 0) | \
+            (LAMB_FLAG_INCREMENT_STEP if increment_step else 0)
+    return lamb_hyper_t(beta1, beta2, eps, weight_decay, gamma_l, gamma_u,
+                        trust_coef, LAMB_PHI_CLIP if phi == "clip"
+                        else LAMB_PHI_IDENTITY, flags)
+
+
+def lamb_plan_create(sizes, decay_mask=None, grad_dtype=LAMB_F32,
+                     copy_dtype=LAMB_DTYPE_NONE, device=0, chunk_elems=0,
+                     blocks_per_sm=0) -> int:
+    lib = load()
+    n = len(sizes)
+    sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
+    mask = None
+    if decay_mask is not None:
+        mask = (c_uint8 * max(n, 1))(*[1 if d else 0 for d in decay_mask])
+    opts = lamb_plan_options_t(int(chunk_elems), int(blocks_per_sm))
+    out = c_void_p()
+    _check(lib.lamb_plan_create(sz, n, mask, int(grad_dtype), int(copy_dtype),
+                                int(device), byref(opts), byref(out)))
+    return out.value
+
+
+def lamb_plan_bind(plan, w, g, m, v=None, w_copy=None, stream=0) -> None:
+    _check(load().lamb_plan_bind(c_void_p(plan), _ptr_array(w), _ptr_array(g),
+                                 _ptr_array(m), _ptr_array(v),
+                                 _ptr_array(w_copy), c_void_p(stream or None)))
+
+
+def lamb_step(plan, hyper: lamb_hyper_t, d_step, d_lr, stream=0) -> None:
+    _check(load().lamb_step(c_void_p(plan), byref(hyper),
+                            c_void_p(d_step or None), c_void_p(d_lr or None),
+                            c_void_p(stream or None)))
+
+
+def lars_step(plan, hyper: lamb_hyper_t, d_step, d_lr, stream=0) -> None:
+    _check(load().lars_step(c_void_p(plan), byref(hyper),
+                            c_void_p(d_step or None), c_void_p(d_lr or None),
+                            c_void_p(stream or None)))
+
+
+def lamb_plan_trust_ratios(plan):
+    r, w, u = c_void_p(), c_void_p(), c_void_p()
+    _check(load().lamb_plan_trust_ratios(c_void_p(plan), byref(r), byref(w),
+                                         byref(u)))
+    return r.value, w.value, u.value
+
+
+def lamb_plan_copy_trust_ratios(plan, ratio=0, wnorm=0, unorm=0,
+                                stream=0) -> None:
+    """Addresses (device or host) of caller-owned float64 arrays, or 0."""
+    _check(load().lamb_plan_copy_trust_ratios(
+        c_void_p(plan), c_void_p(ratio or None), c_void_p(wnorm or None),
+        c_void_p(unorm or None), c_void_p(stream or None)))
+
+
+def lamb_plan_query(plan, clear=False, stream=0) -> int:
+    bits = c_uint32()
+    _check(load().lamb_plan_query(c_void_p(plan), byref(bits), int(clear),
+                                  c_void_p(stream or None)))
+    return int(bits.value)
+
+
+def lamb_plan_get_info(plan) -> dict:
+    info = lamb_plan_info_t()
+    _check(load().lamb_plan_get_info(c_void_p(plan), byref(info)))
+    return {name: getattr(info, name) for name, _ in info._fields_}
+
+
+def lamb_plan_set_timing(plan, enable=True) -> None:
+    _check(load().lamb_plan_set_timing(c_void_p(plan), int(bool(enable))))
+
+
+def lamb_plan_read_timing(plan, n_kernels=2):
+    n = c_int32()
+    ms = (c_double * n_kernels)()
+    _check(load().lamb_plan_read_timing(c_void_p(plan), byref(n), ms,
+                                        n_kernels))
+    return int(n.value), [float(x) for x in ms]
+
+
+def lamb_plan_destroy(plan) -> None:
+    if plan:
+        _check(load().lamb_plan_destroy(c_void_p(plan)))
+
+
+def lamb_layout_chunks(sizes, chunk_elems=0):
+    """Host-only planner: returns (tensor, offset, length) int arrays."""
+    lib = load()
+    n = len(sizes)
+    sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
+    count = c_int32()
+    st = lib.lamb_layout_chunks(sz, n, int(chunk_elems), None, None, None, 0,
+                                byref(count))
+    _check(st)
+    cap = count.value
+    t = np.zeros(max(cap, 1), dtype=np.int32)
+    o = np.zeros(max(cap, 1), dtype=np.int64)
+    ln = np.zeros(max(cap, 1), dtype=np.int32)
+    _check(lib.lamb_layout_chunks(
+        sz, n, int(chunk_elems), t.ctypes.data_as(POINTER(c_int32)),
+        o.ctypes.data_as(POINTER(c_int64)), ln.ctypes.data_as(POINTER(c_int32)),
+        cap, byref(count)))
+    return t[:cap], o[:cap], ln[:cap]

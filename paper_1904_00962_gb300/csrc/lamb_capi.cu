@@ -1,0 +1,561 @@
+// C ABI of the library (declared in include/lamb.h): plan lifecycle, binding,
+// the LAMB / LARS step entry points, and queries.  Host code only; the
+// kernels live in lamb_kernels.cu.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "lamb.h"
+#include "lamb_internal.h"
+
+using namespace lamb;
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+lamb_status_t fail(lamb_status_t st, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return st;
+}
+
+lamb_status_t cuda_fail(cudaError_t e, const char* what) {
+  if (e == cudaErrorMemoryAllocation)
+    return fail(LAMB_ERR_OOM, "%s: %s", what, cudaGetErrorString(e));
+  return fail(LAMB_ERR_CUDA, "%s: %s (%d)", what, cudaGetErrorString(e),
+              (int)e);
+}
+
+constexpr int kMaxTimedSteps = 4096;
+constexpr int kKernelsPerStep = 2;
+
+// Restores the caller's current device on scope exit.
+struct DeviceGuard {
+  int prev = -1;
+  cudaError_t err = cudaSuccess;
+  explicit DeviceGuard(int dev) {
+    err = cudaGetDevice(&prev);
+    if (err == cudaSuccess && prev != dev) err = cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev)
+      cudaSetDevice(prev);
+  }
+};
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace
+
+struct lamb_plan {
+  int device = 0;
+  int n_tensors = 0;
+  int64_t n_chunks = 0;
+  int64_t n_params = 0;
+  int chunk_elems = kDefaultChunk;
+  int grad_bf16 = 0;
+  int copy_bf16 = 0;
+  int num_sms = 0;
+  int blocks_per_sm_opt = 0;
+  int grid[4] = {0, 0, 0, 0};  // lamb p1, lamb p2, lars p1, lars p2
+  bool bound = false;
+  bool has_v = false;
+  int n_vec = 0;
+  std::vector<TensorDesc> h_tensors;
+
+  void* arena = nullptr;
+  size_t arena_bytes = 0;
+  ChunkDesc* chunks = nullptr;
+  TensorDesc* tensors = nullptr;
+  TensorPtrs* ptrs = nullptr;
+  float2* slots = nullptr;
+  uint32_t* tickets = nullptr;
+  double* ratio = nullptr;
+  double* wnorm = nullptr;
+  double* unorm = nullptr;
+  StepScalars* scal = nullptr;
+  uint32_t* status = nullptr;
+  uint32_t* counters = nullptr;
+
+  bool timing = false;
+  int timed_steps = 0;
+  std::vector<cudaEvent_t> events;  // kMaxTimedSteps * (kKernelsPerStep + 1)
+};
+
+extern "C" {
+
+const char* lamb_last_error(void) { return g_err; }
+
+int32_t lamb_abi_version(void) { return LAMB_ABI_VERSION; }
+
+lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
+                                 int32_t chunk_elems, int32_t* chunk_tensor,
+                                 int64_t* chunk_offset, int32_t* chunk_len,
+                                 int32_t capacity, int32_t* n_chunks) {
+  if (n_chunks == nullptr) return fail(LAMB_ERR_INVALID_ARG, "n_chunks is NULL");
+  if (capacity < 0) return fail(LAMB_ERR_INVALID_ARG, "capacity < 0");
+  if (capacity > 0 && (!chunk_tensor || !chunk_offset || !chunk_len))
+    return fail(LAMB_ERR_INVALID_ARG, "output arrays are NULL");
+  if (chunk_elems == 0) chunk_elems = kDefaultChunk;
+  std::vector<ChunkDesc> rows;
+  try {
+    rows.resize((size_t)capacity);
+  } catch (const std::bad_alloc&) {
+    return fail(LAMB_ERR_OOM, "host allocation failed");
+  }
+  int64_t count = 0;
+  char err[256] = "";
+  const int rc = plan_chunks(sizes, n_tensors, chunk_elems,
+                             capacity ? rows.data() : nullptr, capacity,
+                             &count, nullptr, nullptr, err, sizeof(err));
+  *n_chunks = (int32_t)(count > INT32_MAX ? INT32_MAX : count);
+  if (rc) return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  if (count > capacity && capacity > 0)
+    return fail(LAMB_ERR_INVALID_ARG, "capacity %d < %lld chunks", capacity,
+                (long long)count);
+  for (int64_t i = 0; i < count && i < capacity; ++i) {
+    chunk_tensor[i] = rows[i].tensor;
+    chunk_offset[i] = rows[i].offset;
+    chunk_len[i] = rows[i].len;
+  }
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
+                               const uint8_t* decay_mask, int32_t grad_dtype,
+                               int32_t copy_dtype, int32_t device,
+                               const lamb_plan_options_t* opts,
+                               lamb_plan_t* out) {
+  if (out == nullptr) return fail(LAMB_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (grad_dtype != LAMB_F32 && grad_dtype != LAMB_BF16)
+    return fail(LAMB_ERR_UNSUPPORTED_DTYPE, "grad_dtype %d unsupported",
+                grad_dtype);
+  if (copy_dtype != LAMB_DTYPE_NONE && copy_dtype != LAMB_BF16)
+    return fail(LAMB_ERR_UNSUPPORTED_DTYPE,
+                "copy_dtype %d unsupported (NONE or BF16)", copy_dtype);
+  int chunk = kDefaultChunk, bps = 0;
+  if (opts) {
+    if (opts->chunk_elems) chunk = opts->chunk_elems;
+    if (opts->blocks_per_sm < 0)
+      return fail(LAMB_ERR_INVALID_ARG, "blocks_per_sm < 0");
+    bps = opts->blocks_per_sm;
+  }
+  if (device < 0) return fail(LAMB_ERR_INVALID_ARG, "device < 0");
+
+  lamb_plan* p = new (std::nothrow) lamb_plan();
+  if (!p) return fail(LAMB_ERR_OOM, "host allocation failed");
+  p->device = device;
+  p->n_tensors = n_tensors;
+  p->chunk_elems = chunk;
+  p->grad_bf16 = grad_dtype == LAMB_BF16;
+  p->copy_bf16 = copy_dtype == LAMB_BF16;
+  p->blocks_per_sm_opt = bps;
+
+  // ---- host planning ----------------------------------------------------
+  char err[256] = "";
+  int64_t nch = 0;
+  if (n_tensors < 1 || sizes == nullptr) {
+    delete p;
+    return fail(LAMB_ERR_INVALID_ARG, n_tensors < 1
+                                          ? "n_tensors must be >= 1"
+                                          : "sizes is NULL");
+  }
+  p->h_tensors.resize((size_t)n_tensors);
+  if (plan_chunks(sizes, n_tensors, chunk, nullptr, 0, &nch,
+                  p->h_tensors.data(), decay_mask, err, sizeof(err))) {
+    delete p;
+    return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  }
+  std::vector<ChunkDesc> h_chunks((size_t)nch);
+  if (plan_chunks(sizes, n_tensors, chunk, h_chunks.data(), nch, &nch,
+                  p->h_tensors.data(), decay_mask, err, sizeof(err))) {
+    delete p;
+    return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  }
+  p->n_chunks = nch;
+  for (int k = 0; k < n_tensors; ++k) p->n_params += sizes[k];
+
+  // ---- device ------------------------------------------------------------
+  DeviceGuard guard(device);
+  if (guard.err != cudaSuccess) {
+    delete p;
+    return cuda_fail(guard.err, "cudaSetDevice");
+  }
+  cudaError_t e = cudaDeviceGetAttribute(&p->num_sms,
+                                         cudaDevAttrMultiProcessorCount, device);
+  if (e != cudaSuccess) {
+    delete p;
+    return cuda_fail(e, "cudaDeviceGetAttribute");
+  }
+  int occ[4] = {0, 0, 0, 0};
+  int rc = occupancy_lamb_pass1(p->grad_bf16, &occ[0]);
+  if (!rc) rc = occupancy_lamb_pass2(p->copy_bf16, &occ[1]);
+  if (!rc) rc = occupancy_lars_pass1(p->grad_bf16, &occ[2]);
+  if (!rc) rc = occupancy_lars_pass2(p->copy_bf16, &occ[3]);
+  if (rc) {
+    delete p;
+    return cuda_fail((cudaError_t)rc, "occupancy query");
+  }
+  for (int i = 0; i < 4; ++i) {
+    int b = occ[i] < 1 ? 1 : occ[i];
+    if (bps > 0 && bps < b) b = bps;
+    int64_t g = (int64_t)p->num_sms * b;
+    if (g > nch) g = nch;      // never more CTAs than chunks
+    if (g < 1) g = 1;
+    p->grid[i] = (int)g;
+  }
+
+  const size_t n = (size_t)n_tensors, c = (size_t)nch;
+  size_t off = 0;
+  auto carve = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + (bytes ? bytes : 1), 256);
+    return at;
+  };
+  const size_t o_chunks = carve(c * sizeof(ChunkDesc));
+  const size_t o_tensors = carve(n * sizeof(TensorDesc));
+  const size_t o_ptrs = carve(n * sizeof(TensorPtrs));
+  const size_t o_slots = carve(c * sizeof(float2));
+  const size_t o_tickets = carve(n * sizeof(uint32_t));
+  const size_t o_ratio = carve(n * sizeof(double));
+  const size_t o_wnorm = carve(n * sizeof(double));
+  const size_t o_unorm = carve(n * sizeof(double));
+  const size_t o_scal = carve(sizeof(StepScalars));
+  const size_t o_status = carve(sizeof(uint32_t));
+  const size_t o_counters = carve(4 * sizeof(uint32_t));
+  p->arena_bytes = off;
+  e = cudaMalloc(&p->arena, p->arena_bytes);
+  if (e != cudaSuccess) {
+    delete p;
+    return cuda_fail(e, "cudaMalloc(plan)");
+  }
+  char* base = static_cast<char*>(p->arena);
+  p->chunks = reinterpret_cast<ChunkDesc*>(base + o_chunks);
+  p->tensors = reinterpret_cast<TensorDesc*>(base + o_tensors);
+  p->ptrs = reinterpret_cast<TensorPtrs*>(base + o_ptrs);
+  p->slots = reinterpret_cast<float2*>(base + o_slots);
+  p->tickets = reinterpret_cast<uint32_t*>(base + o_tickets);
+  p->ratio = reinterpret_cast<double*>(base + o_ratio);
+  p->wnorm = reinterpret_cast<double*>(base + o_wnorm);
+  p->unorm = reinterpret_cast<double*>(base + o_unorm);
+  p->scal = reinterpret_cast<StepScalars*>(base + o_scal);
+  p->status = reinterpret_cast<uint32_t*>(base + o_status);
+  p->counters = reinterpret_cast<uint32_t*>(base + o_counters);
+
+  // zero everything (tickets, counters, status, results, pointer table)
+  e = cudaMemset(p->arena, 0, p->arena_bytes);
+  if (e == cudaSuccess && c)
+    e = cudaMemcpy(p->chunks, h_chunks.data(), c * sizeof(ChunkDesc),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(p->tensors, p->h_tensors.data(), n * sizeof(TensorDesc),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) {
+    // trust ratio 1 for every tensor until a step computes it (0-element
+    // tensors keep it: Q6 zero-norm rule)
+    std::vector<double> ones(n, 1.0);
+    e = cudaMemcpy(p->ratio, ones.data(), n * sizeof(double),
+                   cudaMemcpyHostToDevice);
+  }
+  if (e != cudaSuccess) {
+    cudaFree(p->arena);
+    delete p;
+    return cuda_fail(e, "plan upload");
+  }
+  *out = p;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_bind(lamb_plan_t plan, void* const* w,
+                             const void* const* g, void* const* m,
+                             void* const* v, void* const* w_copy,
+                             cudaStream_t stream) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  if (!w || !g || !m)
+    return fail(LAMB_ERR_INVALID_ARG, "w, g and m pointer arrays are required");
+  if (plan->copy_bf16 && !w_copy)
+    return fail(LAMB_ERR_INVALID_ARG,
+                "plan writes a bf16 copy: w_copy pointer array is required");
+  const int n = plan->n_tensors;
+  std::vector<TensorPtrs> h((size_t)n);
+  int n_vec = 0;
+  const uintptr_t ga = plan->grad_bf16 ? 8 : 16;
+  for (int k = 0; k < n; ++k) {
+    TensorPtrs& t = h[(size_t)k];
+    std::memset(&t, 0, sizeof(t));
+    t.w = static_cast<float*>(w[k]);
+    t.g = g[k];
+    t.m = static_cast<float*>(m[k]);
+    t.v = v ? static_cast<float*>(v[k]) : nullptr;
+    t.copy = plan->copy_bf16 ? w_copy[k] : nullptr;
+    if (plan->h_tensors[(size_t)k].numel > 0) {
+      if (!t.w || !t.g || !t.m)
+        return fail(LAMB_ERR_INVALID_ARG, "tensor %d: NULL w/g/m pointer", k);
+      if (v && !t.v)
+        return fail(LAMB_ERR_INVALID_ARG, "tensor %d: NULL v pointer", k);
+      if (plan->copy_bf16 && !t.copy)
+        return fail(LAMB_ERR_INVALID_ARG, "tensor %d: NULL w_copy pointer", k);
+      if ((uintptr_t)t.w % 4 || (uintptr_t)t.m % 4 ||
+          (t.v && (uintptr_t)t.v % 4) ||
+          (uintptr_t)t.g % (plan->grad_bf16 ? 2 : 4) ||
+          (t.copy && (uintptr_t)t.copy % 2))
+        return fail(LAMB_ERR_INVALID_ARG,
+                    "tensor %d: pointer not aligned to its element size", k);
+    }
+    bool ok = (uintptr_t)t.w % 16 == 0 && (uintptr_t)t.m % 16 == 0 &&
+              (!t.v || (uintptr_t)t.v % 16 == 0) &&
+              (uintptr_t)t.g % ga == 0 && (!t.copy || (uintptr_t)t.copy % 8 == 0);
+    t.vec_ok = ok ? 1u : 0u;
+    n_vec += ok;
+  }
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  cudaError_t e = cudaMemcpyAsync(plan->ptrs, h.data(),
+                                  (size_t)n * sizeof(TensorPtrs),
+                                  cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "pointer table upload");
+  plan->bound = true;
+  plan->has_v = v != nullptr;
+  plan->n_vec = n_vec;
+  return LAMB_OK;
+}
+
+static lamb_status_t check_hyper(const lamb_hyper_t* h, bool lamb) {
+  if (!h) return fail(LAMB_ERR_INVALID_ARG, "hyper is NULL");
+  if (!(h->beta1 >= 0.0 && h->beta1 < 1.0))
+    return fail(LAMB_ERR_INVALID_ARG, "beta1 must be in [0, 1)");
+  if (lamb && !(h->beta2 >= 0.0 && h->beta2 < 1.0))
+    return fail(LAMB_ERR_INVALID_ARG, "beta2 must be in [0, 1)");
+  if (lamb && !(h->eps >= 0.0 && std::isfinite(h->eps)))
+    return fail(LAMB_ERR_INVALID_ARG, "eps must be finite and >= 0");
+  if (!std::isfinite(h->weight_decay))
+    return fail(LAMB_ERR_INVALID_ARG, "weight_decay must be finite");
+  if (h->phi != LAMB_PHI_IDENTITY && h->phi != LAMB_PHI_CLIP)
+    return fail(LAMB_ERR_INVALID_ARG, "phi must be IDENTITY or CLIP");
+  if (h->phi == LAMB_PHI_CLIP && !(h->gamma_l <= h->gamma_u))
+    return fail(LAMB_ERR_INVALID_ARG, "clip bounds need gamma_l <= gamma_u");
+  if (!lamb && !std::isfinite(h->trust_coef))
+    return fail(LAMB_ERR_INVALID_ARG, "trust_coef must be finite");
+  if (h->flags & ~(uint32_t)(LAMB_FLAG_BIAS_CORRECTION | LAMB_FLAG_INCREMENT_STEP))
+    return fail(LAMB_ERR_INVALID_ARG, "unknown flag bits 0x%x", h->flags);
+  return LAMB_OK;
+}
+
+static void fill_params(lamb_plan* p, const lamb_hyper_t* h, int64_t* d_step,
+                        const float* d_lr, StepParams* sp) {
+  std::memset(sp, 0, sizeof(*sp));
+  sp->chunks = p->chunks;
+  sp->tensors = p->tensors;
+  sp->ptrs = p->ptrs;
+  sp->slots = p->slots;
+  sp->tickets = p->tickets;
+  sp->counters = p->counters;
+  sp->ratio = p->ratio;
+  sp->wnorm = p->wnorm;
+  sp->unorm = p->unorm;
+  sp->scal = p->scal;
+  sp->status = p->status;
+  sp->d_step = d_step;
+  sp->d_lr = d_lr;
+  // (1 - beta) formed in double and rounded once
+  sp->b1 = (float)h->beta1;
+  sp->omb1 = (float)(1.0 - h->beta1);
+  sp->b2 = (float)h->beta2;
+  sp->omb2 = (float)(1.0 - h->beta2);
+  sp->eps = (float)h->eps;
+  sp->wd = (float)h->weight_decay;
+  sp->beta1 = h->beta1;
+  sp->beta2 = h->beta2;
+  sp->gamma_l = h->gamma_l;
+  sp->gamma_u = h->gamma_u;
+  sp->trust = h->trust_coef;
+  sp->phi = h->phi;
+  sp->flags = h->flags;
+  sp->n_chunks = (int32_t)p->n_chunks;
+}
+
+static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                              int64_t* d_step, const float* d_lr,
+                              cudaStream_t stream, bool lamb) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  lamb_status_t st = check_hyper(hyper, lamb);
+  if (st != LAMB_OK) return st;
+  if (!plan->bound) return fail(LAMB_ERR_NOT_BOUND, "plan is not bound");
+  if (lamb && !plan->has_v)
+    return fail(LAMB_ERR_NOT_BOUND, "lamb_step needs v: bind v pointers");
+  if (!d_lr) return fail(LAMB_ERR_INVALID_ARG, "d_lr is NULL");
+  const bool needs_step =
+      (hyper->flags & LAMB_FLAG_INCREMENT_STEP) ||
+      (lamb && (hyper->flags & LAMB_FLAG_BIAS_CORRECTION));
+  if (needs_step && !d_step)
+    return fail(LAMB_ERR_INVALID_ARG, "d_step is NULL but the flags need it");
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  StepParams sp;
+  fill_params(plan, hyper, d_step, d_lr, &sp);
+
+  const bool timed = plan->timing && plan->timed_steps < kMaxTimedSteps;
+  cudaEvent_t* ev = timed ? &plan->events[(size_t)plan->timed_steps *
+                                          (kKernelsPerStep + 1)]
+                          : nullptr;
+  cudaError_t e = cudaSuccess;
+  if (timed) e = cudaEventRecord(ev[0], stream);
+  int rc = (int)e;
+  if (!rc)
+    rc = lamb ? launch_lamb_pass1(sp, plan->grad_bf16, plan->grid[0], stream)
+              : launch_lars_pass1(sp, plan->grad_bf16, plan->grid[2], stream);
+  if (!rc && timed) rc = (int)cudaEventRecord(ev[1], stream);
+  if (!rc)
+    rc = lamb ? launch_lamb_pass2(sp, plan->copy_bf16, plan->grid[1], stream)
+              : launch_lars_pass2(sp, plan->copy_bf16, plan->grid[3], stream);
+  if (!rc && timed) rc = (int)cudaEventRecord(ev[2], stream);
+  if (rc) return cuda_fail((cudaError_t)rc, lamb ? "lamb_step" : "lars_step");
+  if (timed) ++plan->timed_steps;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                        int64_t* d_step, const float* d_lr,
+                        cudaStream_t stream) {
+  return run_step(plan, hyper, d_step, d_lr, stream, true);
+}
+
+lamb_status_t lars_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                        int64_t* d_step, const float* d_lr,
+                        cudaStream_t stream) {
+  return run_step(plan, hyper, d_step, d_lr, stream, false);
+}
+
+lamb_status_t lamb_plan_trust_ratios(lamb_plan_t plan, const double** d_ratio,
+                                     const double** d_wnorm,
+                                     const double** d_unorm) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  if (d_ratio) *d_ratio = plan->ratio;
+  if (d_wnorm) *d_wnorm = plan->wnorm;
+  if (d_unorm) *d_unorm = plan->unorm;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_copy_trust_ratios(lamb_plan_t plan, double* ratio,
+                                          double* wnorm, double* unorm,
+                                          cudaStream_t stream) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  const size_t bytes = (size_t)plan->n_tensors * sizeof(double);
+  const double* src[3] = {plan->ratio, plan->wnorm, plan->unorm};
+  double* dst[3] = {ratio, wnorm, unorm};
+  for (int i = 0; i < 3; ++i) {
+    if (!dst[i]) continue;
+    cudaError_t e = cudaMemcpyAsync(dst[i], src[i], bytes, cudaMemcpyDefault,
+                                    stream);
+    if (e != cudaSuccess) return cuda_fail(e, "trust ratio copy");
+  }
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_query(lamb_plan_t plan, uint32_t* status_bits,
+                              int32_t clear, cudaStream_t stream) {
+  if (!plan || !status_bits)
+    return fail(LAMB_ERR_INVALID_ARG, "plan or status_bits is NULL");
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  uint32_t h = 0;
+  cudaError_t e = cudaMemcpyAsync(&h, plan->status, sizeof(h),
+                                  cudaMemcpyDeviceToHost, stream);
+  if (e == cudaSuccess && clear)
+    e = cudaMemsetAsync(plan->status, 0, sizeof(uint32_t), stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "status query");
+  *status_bits = h;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_get_info(lamb_plan_t plan, lamb_plan_info_t* info) {
+  if (!plan || !info) return fail(LAMB_ERR_INVALID_ARG, "NULL argument");
+  std::memset(info, 0, sizeof(*info));
+  info->n_tensors = plan->n_tensors;
+  info->n_chunks = (int32_t)plan->n_chunks;
+  info->n_params = plan->n_params;
+  info->chunk_elems = plan->chunk_elems;
+  info->grid_blocks = plan->grid[0];
+  info->threads_per_block = kThreads;
+  info->num_sms = plan->num_sms;
+  info->device = plan->device;
+  info->grad_dtype = plan->grad_bf16 ? LAMB_BF16 : LAMB_F32;
+  info->copy_dtype = plan->copy_bf16 ? LAMB_BF16 : LAMB_DTYPE_NONE;
+  info->bound = plan->bound ? 1 : 0;
+  info->n_vector_tensors = plan->n_vec;
+  info->device_bytes = (int64_t)plan->arena_bytes;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_set_timing(lamb_plan_t plan, int32_t enable) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  if (enable && plan->events.empty()) {
+    DeviceGuard guard(plan->device);
+    if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+    plan->events.resize((size_t)kMaxTimedSteps * (kKernelsPerStep + 1));
+    for (auto& ev : plan->events) {
+      cudaError_t e = cudaEventCreate(&ev);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaEventCreate");
+    }
+  }
+  plan->timing = enable != 0;
+  plan->timed_steps = 0;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_read_timing(lamb_plan_t plan, int32_t* n_steps,
+                                    double* ms_per_kernel, int32_t n_kernels) {
+  if (!plan || !n_steps || (n_kernels > 0 && !ms_per_kernel))
+    return fail(LAMB_ERR_INVALID_ARG, "NULL argument");
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  for (int j = 0; j < n_kernels; ++j) ms_per_kernel[j] = 0.0;
+  for (int s = 0; s < plan->timed_steps; ++s) {
+    cudaEvent_t* ev = &plan->events[(size_t)s * (kKernelsPerStep + 1)];
+    cudaError_t e = cudaEventSynchronize(ev[kKernelsPerStep]);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
+    for (int j = 0; j < kKernelsPerStep && j < n_kernels; ++j) {
+      float ms = 0.f;
+      e = cudaEventElapsedTime(&ms, ev[j], ev[j + 1]);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+      ms_per_kernel[j] += ms;
+    }
+  }
+  *n_steps = plan->timed_steps;
+  plan->timed_steps = 0;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_destroy(lamb_plan_t plan) {
+  if (!plan) return LAMB_OK;
+  DeviceGuard guard(plan->device);
+  cudaError_t e = cudaSuccess;
+  if (guard.err == cudaSuccess) {
+    e = cudaDeviceSynchronize();
+    for (auto& ev : plan->events) cudaEventDestroy(ev);
+    if (plan->arena) {
+      cudaError_t e2 = cudaFree(plan->arena);
+      if (e == cudaSuccess) e = e2;
+    }
+  }
+  delete plan;
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  if (e != cudaSuccess) return cuda_fail(e, "lamb_plan_destroy");
+  return LAMB_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,106 @@
+// Internal layout of a plan and the kernel parameter block.
+//
+// HBM layout of a plan (one cudaMalloc, carved in this order, each piece
+// 256-byte aligned):
+//   ChunkDesc  chunks[n_chunks]   16 B  read-only after create
+//   TensorDesc tensors[n_tensors] 32 B  read-only after create
+//   TensorPtrs ptrs[n_tensors]    48 B  written by bind
+//   float2     slots[n_chunks]     8 B  per-chunk (sum w^2, sum u^2), pass 1
+//   uint32     tickets[n_tensors]  4 B  chunks of tensor k finished in pass 1;
+//                                       reset to 0 by the last one
+//   double     ratio/wnorm/unorm[n_tensors]  per-tensor results
+//   StepScalars, status word, work counters
+#pragma once
+#include <stdint.h>
+
+namespace lamb {
+
+constexpr int kDefaultChunk = 16384;
+constexpr int kThreads = 256;          // threads per CTA, all kernels
+constexpr int kWarps = kThreads / 32;
+constexpr int kMaxChunks = 1 << 30;
+
+struct __align__(16) ChunkDesc {
+  int64_t offset;   // first element of the chunk inside its tensor
+  int32_t tensor;   // tensor index k
+  int32_t len;      // elements in the chunk (1 .. chunk_elems)
+};
+
+struct __align__(16) TensorDesc {
+  int64_t numel;
+  int32_t first_chunk;
+  int32_t n_chunks;
+  float decay;      // 1.0f: weight decay applies, 0.0f: masked
+  uint32_t pad[3];
+};
+
+struct __align__(16) TensorPtrs {
+  float* w;
+  const void* g;    // float or bf16
+  float* m;
+  float* v;         // may be null (LARS-only binding)
+  void* copy;       // bf16 copy of w, or null
+  uint32_t vec_ok;  // every array aligned for 4-element vector access
+  uint32_t pad;
+};
+
+// Written by pass 1 (CTA 0) and read by pass 2, so both passes use the very
+// same float constants.
+struct __align__(16) StepScalars {
+  int64_t t;
+  float c1;         // 1/(1-beta1^t) (1 without bias correction)
+  float c2;         // 1/(1-beta2^t)
+  float lr;
+  int32_t skip;     // 1: bad step count, nothing is written
+  int32_t pad[2];
+};
+
+enum : uint32_t { kStatusNonfinite = 1u, kStatusBadStep = 2u };
+enum : uint32_t { kFlagBiasCorrection = 1u, kFlagIncrementStep = 2u };
+
+struct StepParams {
+  const ChunkDesc* chunks;
+  const TensorDesc* tensors;
+  const TensorPtrs* ptrs;
+  float2* slots;
+  uint32_t* tickets;
+  uint32_t* counters;     // [0] pass-1 work counter, [1] pass-2 work counter
+  double* ratio;
+  double* wnorm;
+  double* unorm;
+  StepScalars* scal;
+  uint32_t* status;
+  int64_t* d_step;
+  const float* d_lr;
+  // per-step constants, rounded once from double on the host
+  float b1, omb1, b2, omb2, eps, wd;
+  double beta1, beta2;    // for beta^t on the device
+  double gamma_l, gamma_u, trust;
+  int32_t phi;            // 0 identity, 1 clip
+  uint32_t flags;
+  int32_t n_chunks;
+};
+
+// Launchers (lamb_kernels.cu).  grid = number of CTAs of the persistent grid.
+// Return cudaError_t as int to keep this header free of CUDA includes.
+int launch_lamb_pass1(const StepParams& p, int grad_bf16, int grid,
+                      void* stream);
+int launch_lamb_pass2(const StepParams& p, int copy_bf16, int grid,
+                      void* stream);
+int launch_lars_pass1(const StepParams& p, int grad_bf16, int grid,
+                      void* stream);
+int launch_lars_pass2(const StepParams& p, int copy_bf16, int grid,
+                      void* stream);
+// Resident CTAs per SM of each kernel instantiation (occupancy calculator).
+int occupancy_lamb_pass1(int grad_bf16, int* blocks);
+int occupancy_lamb_pass2(int copy_bf16, int* blocks);
+int occupancy_lars_pass1(int grad_bf16, int* blocks);
+int occupancy_lars_pass2(int copy_bf16, int* blocks);
+
+// Host planner (planner.cpp).  Returns 0 on success, else writes a message.
+int plan_chunks(const int64_t* sizes, int32_t n, int32_t chunk_elems,
+                ChunkDesc* chunks, int64_t capacity, int64_t* n_chunks,
+                TensorDesc* tensors, const uint8_t* decay_mask, char* err,
+                int errlen);
+
+}  // namespace lamb

@@ -1,0 +1,631 @@
+// sm_103a kernels of the two-pass LAMB / LARS step.
+//
+// The step of Algorithm 2 needs, per tensor, ||x|| and ||r + lambda x|| over
+// the WHOLE tensor before any element of x may change, so it is split in two
+// streaming passes over HBM:
+//
+//   pass 1  reads g, m, v, w; writes the new m, v (Alg. 2 moment lines);
+//           forms u = r + lambda_k w in registers and accumulates sum w^2 and
+//           sum u^2 per chunk (fp32 per thread, fixed warp/CTA tree) into the
+//           chunk's slot.  The CTA that finishes the last chunk of a tensor
+//           (ticket counter) combines that tensor's slots in a fixed order in
+//           fp64 and writes ||w||, ||u|| and rho = phi(||w||)/||u|| (Alg. 2
+//           last line; rho = 1 on a zero norm).
+//   pass 2  reads m, v, w; recomputes u bit-identically (same __device__
+//           function, explicit round-to-nearest intrinsics, no contraction)
+//           and writes w - eta*rho*u (and its bf16 copy).
+//
+// LARS (Algorithm 1) has the same shape with u = m_t.
+//
+// Both passes are persistent grids (CTAs = SMs x resident CTAs per SM) that
+// draw chunks from a device work counter, so hundreds of tiny tensors and a
+// 31M-element embedding share one launch.  The grid never waits on itself:
+// tickets and counters only decide WHO does a piece of work, never block.
+// The last CTA to draw from a counter resets it (and the last chunk of a
+// tensor resets its ticket), so the kernels can be replayed from a CUDA
+// graph with no host involvement.
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+
+#include "lamb_internal.h"
+
+namespace lamb {
+namespace {
+
+constexpr int kUnroll1 = 4;   // 4-element packets in flight per thread, pass 1
+constexpr int kUnroll2 = 4;   // same for pass 2
+
+// ---------------------------------------------------------------------------
+// Element arithmetic.  Every operation is an explicit round-to-nearest
+// intrinsic, so the compiler cannot fuse differently in the two passes.
+// ---------------------------------------------------------------------------
+struct LambConsts {
+  float b1, omb1, b2, omb2;   // beta1, 1-beta1, beta2, 1-beta2
+  float c1, c2;               // 1/(1-beta1^t), 1/(1-beta2^t)
+  float eps;
+};
+
+// Alg. 2: m_t = beta1 m + (1-beta1) g ;  v_t = beta2 v + (1-beta2) g^2
+__device__ __forceinline__ void lamb_moments(float g, float& m, float& v,
+                                             const LambConsts& k) {
+  m = __fmaf_rn(k.b1, m, __fmul_rn(k.omb1, g));
+  v = __fmaf_rn(k.b2, v, __fmul_rn(k.omb2, __fmul_rn(g, g)));
+}
+
+// Alg. 2: u = (m_t c1) / (sqrt(v_t c2) + eps) + lambda_k w
+__device__ __forceinline__ float lamb_direction(float m, float v, float w,
+                                                float lam,
+                                                const LambConsts& k) {
+  const float mh = __fmul_rn(m, k.c1);
+  const float vh = __fmul_rn(v, k.c2);
+  const float den = __fadd_rn(__fsqrt_rn(vh), k.eps);
+  return __fmaf_rn(lam, w, __fdiv_rn(mh, den));
+}
+
+// Alg. 1: m_t = beta1 m + (1-beta1) (g + lambda_k w)
+__device__ __forceinline__ float lars_momentum(float g, float m, float w,
+                                               float lam, float b1,
+                                               float omb1) {
+  return __fmaf_rn(b1, m, __fmul_rn(omb1, __fmaf_rn(lam, w, g)));
+}
+
+// ---------------------------------------------------------------------------
+// Memory helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float4 ld4(const float* p) {
+  return *reinterpret_cast<const float4*>(p);
+}
+__device__ __forceinline__ float4 ld4_last(const float* p) {  // last use
+  return __ldcs(reinterpret_cast<const float4*>(p));
+}
+__device__ __forceinline__ void st4(float* p, float4 x) {
+  *reinterpret_cast<float4*>(p) = x;
+}
+__device__ __forceinline__ void st4_last(float* p, float4 x) {
+  __stcs(reinterpret_cast<float4*>(p), x);
+}
+
+// Gradients are read exactly once: streaming (evict-first) loads.
+__device__ __forceinline__ float4 ld_grad4(const float* p) {
+  return __ldcs(reinterpret_cast<const float4*>(p));
+}
+// bf16 -> f32 widening is exact: the bf16 pattern is the top half of the f32.
+__device__ __forceinline__ float4 ld_grad4(const __nv_bfloat16* p) {
+  const uint2 u = __ldcs(reinterpret_cast<const uint2*>(p));
+  return make_float4(__uint_as_float(u.x << 16),
+                     __uint_as_float(u.x & 0xffff0000u),
+                     __uint_as_float(u.y << 16),
+                     __uint_as_float(u.y & 0xffff0000u));
+}
+__device__ __forceinline__ float ld_grad1(const float* p) { return __ldcs(p); }
+__device__ __forceinline__ float ld_grad1(const __nv_bfloat16* p) {
+  const unsigned short h = __ldcs(reinterpret_cast<const unsigned short*>(p));
+  return __uint_as_float(uint32_t(h) << 16);
+}
+
+__device__ __forceinline__ void st_copy4(void* base, int64_t i, float4 x) {
+  const __nv_bfloat162 lo = __floats2bfloat162_rn(x.x, x.y);  // RNE
+  const __nv_bfloat162 hi = __floats2bfloat162_rn(x.z, x.w);
+  uint2 u;
+  u.x = *reinterpret_cast<const uint32_t*>(&lo);
+  u.y = *reinterpret_cast<const uint32_t*>(&hi);
+  __stcs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(base) + i), u);
+}
+__device__ __forceinline__ void st_copy1(void* base, int64_t i, float x) {
+  static_cast<__nv_bfloat16*>(base)[i] = __float2bfloat16_rn(x);
+}
+
+// ---------------------------------------------------------------------------
+// Reductions: fixed trees, so the result depends only on the data layout.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_down_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// Sum of (a, b) over the CTA, valid in thread 0.  Contains one barrier.
+__device__ __forceinline__ float2 cta_sum2(float a, float b,
+                                           float (*red)[kWarps]) {
+  a = warp_sum(a);
+  b = warp_sum(b);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) {
+    red[0][warp] = a;
+    red[1][warp] = b;
+  }
+  __syncthreads();
+  float2 r = make_float2(0.f, 0.f);
+  if (warp == 0) {
+    a = lane < kWarps ? red[0][lane] : 0.f;
+    b = lane < kWarps ? red[1][lane] : 0.f;
+    r = make_float2(warp_sum(a), warp_sum(b));
+  }
+  return r;
+}
+
+__device__ __forceinline__ double phi_of(double z, const StepParams& p) {
+  if (p.phi == 1) {  // clip; comparisons keep NaN as NaN
+    if (z < p.gamma_l) return p.gamma_l;
+    if (z > p.gamma_u) return p.gamma_u;
+  }
+  return z;
+}
+
+// Warp 0 of the CTA that finished tensor k's last chunk: fixed-order fp64
+// combine of the chunk slots -> norms and trust ratio.  Resets the ticket.
+__device__ __noinline__ void finalize_tensor(const StepParams& p, int k,
+                                             int first, int n, double coef) {
+  __threadfence();
+  const int lane = threadIdx.x & 31;
+  double aw = 0.0, au = 0.0;
+  for (int i = lane; i < n; i += 32) {
+    const float2 s = __ldcg(&p.slots[first + i]);
+    aw += (double)s.x;
+    au += (double)s.y;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    aw += __shfl_down_sync(0xffffffffu, aw, o);
+    au += __shfl_down_sync(0xffffffffu, au, o);
+  }
+  if (lane == 0) {
+    const double wn = sqrt(aw), un = sqrt(au);
+    double rho = 1.0;                                  // zero-norm rule
+    if (!(wn == 0.0 || un == 0.0)) rho = coef * phi_of(wn, p) / un;
+    p.ratio[k] = rho;
+    p.wnorm[k] = wn;
+    p.unorm[k] = un;
+    if (!isfinite(aw) || !isfinite(au)) atomicOr(p.status, kStatusNonfinite);
+    p.tickets[k] = 0u;
+  }
+}
+
+// Chunk epilogue of pass 1: publish the CTA's partial sums, take a ticket,
+// and let the last chunk of the tensor finalise it.
+__device__ __forceinline__ void publish_chunk(const StepParams& p, int c,
+                                              const ChunkDesc& ch,
+                                              const TensorDesc& td, float sw,
+                                              float su, float (*red)[kWarps],
+                                              int* s_last, double coef) {
+  const float2 tot = cta_sum2(sw, su, red);
+  if (threadIdx.x == 0) {
+    p.slots[c] = tot;
+    __threadfence();
+    const uint32_t prev = atomicAdd(&p.tickets[ch.tensor], 1u);
+    *s_last = (prev + 1u == (uint32_t)td.n_chunks);
+  }
+  __syncthreads();
+  if (*s_last && threadIdx.x < 32)
+    finalize_tensor(p, ch.tensor, td.first_chunk, td.n_chunks, coef);
+}
+
+// Work distribution.  Thread 0 draws chunk indices from counters[which];
+// indices >= n_chunks mean "done".  Every CTA draws exactly one such index,
+// so the CTA that draws n_chunks + gridDim.x - 1 is the last one to draw and
+// may reset the counter for the next launch.  Returns true for that CTA.
+__device__ __forceinline__ bool retire(const StepParams& p, int which,
+                                       uint32_t last_drawn) {
+  const bool last = last_drawn == (uint32_t)p.n_chunks + gridDim.x - 1u;
+  if (last && threadIdx.x == 0) atomicExch(&p.counters[which], 0u);
+  return last;
+}
+
+// ---------------------------------------------------------------------------
+// LAMB pass 1
+// ---------------------------------------------------------------------------
+template <typename GT>
+__device__ __forceinline__ void lamb1_elem(float g, float& m, float& v,
+                                           float w, float lam,
+                                           const LambConsts& k, float& sw,
+                                           float& su) {
+  lamb_moments(g, m, v, k);
+  const float u = lamb_direction(m, v, w, lam, k);
+  sw = __fmaf_rn(w, w, sw);
+  su = __fmaf_rn(u, u, su);
+}
+
+template <typename GT>
+__device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
+                                            const ChunkDesc& ch, float lam,
+                                            const LambConsts& k, float& sw,
+                                            float& su) {
+  float* __restrict__ w = tp.w + ch.offset;
+  float* __restrict__ m = tp.m + ch.offset;
+  float* __restrict__ v = tp.v + ch.offset;
+  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + ch.offset;
+  const int n = ch.len;
+  int scalar_from = 0;
+  if (tp.vec_ok) {
+    const int nv = n >> 2;
+    for (int base = threadIdx.x; base < nv; base += kThreads * kUnroll1) {
+      float4 wv[kUnroll1], mv[kUnroll1], vv[kUnroll1], gv[kUnroll1];
+#pragma unroll
+      for (int u = 0; u < kUnroll1; ++u) {
+        const int j = base + u * kThreads;
+        if (j < nv) {
+          gv[u] = ld_grad4(g + 4 * j);
+          mv[u] = ld4(m + 4 * j);
+          vv[u] = ld4(v + 4 * j);
+          wv[u] = ld4(w + 4 * j);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll1; ++u) {
+        const int j = base + u * kThreads;
+        if (j < nv) {
+          lamb1_elem<GT>(gv[u].x, mv[u].x, vv[u].x, wv[u].x, lam, k, sw, su);
+          lamb1_elem<GT>(gv[u].y, mv[u].y, vv[u].y, wv[u].y, lam, k, sw, su);
+          lamb1_elem<GT>(gv[u].z, mv[u].z, vv[u].z, wv[u].z, lam, k, sw, su);
+          lamb1_elem<GT>(gv[u].w, mv[u].w, vv[u].w, wv[u].w, lam, k, sw, su);
+          st4(m + 4 * j, mv[u]);
+          st4(v + 4 * j, vv[u]);
+        }
+      }
+    }
+    scalar_from = nv << 2;
+  }
+  for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
+    float mi = m[i], vi = v[i];
+    lamb1_elem<GT>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
+    m[i] = mi;
+    v[i] = vi;
+  }
+}
+
+template <typename GT>
+__global__ void __launch_bounds__(kThreads)
+    lamb_pass1_kernel(const StepParams p) {
+  __shared__ float red[2][kWarps];
+  __shared__ uint32_t s_next[2];
+  __shared__ int s_last, s_skip;
+  __shared__ LambConsts s_k;
+  if (threadIdx.x == 0) {
+    const bool bc = (p.flags & kFlagBiasCorrection) != 0;
+    const int64_t t = p.d_step ? *p.d_step : int64_t(1);
+    const int skip = (bc && t < 1) ? 1 : 0;
+    float c1 = 1.f, c2 = 1.f;
+    if (bc && !skip) {  // Alg. 2 bias correction, beta^t in fp64
+      c1 = (float)(1.0 / (1.0 - pow(p.beta1, (double)t)));
+      c2 = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
+    }
+    s_k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps};
+    s_skip = skip;
+    if (blockIdx.x == 0) {
+      StepScalars sc{};
+      sc.t = t;
+      sc.c1 = c1;
+      sc.c2 = c2;
+      sc.lr = *p.d_lr;
+      sc.skip = skip;
+      *p.scal = sc;
+      if (skip) atomicOr(p.status, kStatusBadStep);
+    }
+    if (!skip) s_next[0] = atomicAdd(&p.counters[0], 1u);
+  }
+  __syncthreads();
+  if (s_skip) return;
+  const LambConsts k = s_k;
+  int it = 0;
+  uint32_t c = s_next[0];
+  while (c < (uint32_t)p.n_chunks) {
+    if (threadIdx.x == 0) s_next[(it + 1) & 1] = atomicAdd(&p.counters[0], 1u);
+    const ChunkDesc ch = p.chunks[c];
+    const TensorDesc td = p.tensors[ch.tensor];
+    const TensorPtrs tp = p.ptrs[ch.tensor];
+    const float lam = td.decay * p.wd;
+    float sw = 0.f, su = 0.f;
+    lamb1_chunk<GT>(tp, ch, lam, k, sw, su);
+    publish_chunk(p, (int)c, ch, td, sw, su, red, &s_last, 1.0);
+    ++it;
+    c = s_next[it & 1];
+  }
+  retire(p, 0, c);
+}
+
+// ---------------------------------------------------------------------------
+// LAMB pass 2
+// ---------------------------------------------------------------------------
+template <bool kCopy>
+__device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
+                                            const ChunkDesc& ch, float lam,
+                                            float s, const LambConsts& k) {
+  float* __restrict__ w = tp.w + ch.offset;
+  const float* __restrict__ m = tp.m + ch.offset;
+  const float* __restrict__ v = tp.v + ch.offset;
+  const int n = ch.len;
+  int scalar_from = 0;
+  if (tp.vec_ok) {
+    const int nv = n >> 2;
+    for (int base = threadIdx.x; base < nv; base += kThreads * kUnroll2) {
+      float4 wv[kUnroll2], mv[kUnroll2], vv[kUnroll2];
+#pragma unroll
+      for (int u = 0; u < kUnroll2; ++u) {
+        const int j = base + u * kThreads;
+        if (j < nv) {
+          mv[u] = ld4_last(m + 4 * j);
+          vv[u] = ld4_last(v + 4 * j);
+          wv[u] = ld4_last(w + 4 * j);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll2; ++u) {
+        const int j = base + u * kThreads;
+        if (j < nv) {
+          float4 o;
+          o.x = __fmaf_rn(-s, lamb_direction(mv[u].x, vv[u].x, wv[u].x, lam, k), wv[u].x);
+          o.y = __fmaf_rn(-s, lamb_direction(mv[u].y, vv[u].y, wv[u].y, lam, k), wv[u].y);
+          o.z = __fmaf_rn(-s, lamb_direction(mv[u].z, vv[u].z, wv[u].z, lam, k), wv[u].z);
+          o.w = __fmaf_rn(-s, lamb_direction(mv[u].w, vv[u].w, wv[u].w, lam, k), wv[u].w);
+          st4_last(w + 4 * j, o);
+          if (kCopy) st_copy4(tp.copy, ch.offset + 4 * j, o);
+        }
+      }
+    }
+    scalar_from = nv << 2;
+  }
+  for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
+    const float wi = w[i];
+    const float o = __fmaf_rn(-s, lamb_direction(m[i], v[i], wi, lam, k), wi);
+    w[i] = o;
+    if (kCopy) st_copy1(tp.copy, ch.offset + i, o);
+  }
+}
+
+template <bool kCopy>
+__global__ void __launch_bounds__(kThreads)
+    lamb_pass2_kernel(const StepParams p) {
+  __shared__ uint32_t s_next[2];
+  const StepScalars sc = *p.scal;
+  if (sc.skip) return;
+  const LambConsts k{p.b1, p.omb1, p.b2, p.omb2, sc.c1, sc.c2, p.eps};
+  if (threadIdx.x == 0) s_next[0] = atomicAdd(&p.counters[1], 1u);
+  __syncthreads();
+  int it = 0;
+  uint32_t c = s_next[0];
+  const int nc = p.n_chunks;
+  while (c < (uint32_t)nc) {
+    if (threadIdx.x == 0) s_next[(it + 1) & 1] = atomicAdd(&p.counters[1], 1u);
+    // reverse order: the chunks pass 1 touched last are still in L2
+    const ChunkDesc ch = p.chunks[nc - 1 - (int)c];
+    const TensorDesc td = p.tensors[ch.tensor];
+    const TensorPtrs tp = p.ptrs[ch.tensor];
+    const float lam = td.decay * p.wd;
+    const float s = __double2float_rn((double)sc.lr * p.ratio[ch.tensor]);
+    lamb2_chunk<kCopy>(tp, ch, lam, s, k);
+    __syncthreads();  // s_next[(it+1)&1] visible; old slot free to reuse
+    ++it;
+    c = s_next[it & 1];
+  }
+  if (retire(p, 1, c) && threadIdx.x == 0 &&
+      (p.flags & kFlagIncrementStep) && p.d_step)
+    *p.d_step = sc.t + 1;
+}
+
+// ---------------------------------------------------------------------------
+// LARS pass 1 / pass 2
+// ---------------------------------------------------------------------------
+template <typename GT>
+__device__ __forceinline__ void lars1_chunk(const TensorPtrs& tp,
+                                            const ChunkDesc& ch, float lam,
+                                            float b1, float omb1, float& sw,
+                                            float& su) {
+  const float* __restrict__ w = tp.w + ch.offset;
+  float* __restrict__ m = tp.m + ch.offset;
+  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + ch.offset;
+  const int n = ch.len;
+  int scalar_from = 0;
+  if (tp.vec_ok) {
+    const int nv = n >> 2;
+    for (int base = threadIdx.x; base < nv; base += kThreads * kUnroll1) {
+      float4 wv[kUnroll1], mv[kUnroll1], gv[kUnroll1];
+#pragma unroll
+      for (int u = 0; u < kUnroll1; ++u) {
+        const int j = base + u * kThreads;
+        if (j < nv) {
+          gv[u] = ld_grad4(g + 4 * j);
+          mv[u] = ld4(m + 4 * j);
+          wv[u] = ld4(w + 4 * j);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll1; ++u) {
+        const int j = base + u * kThreads;
+        if (j < nv) {
+          float4 o;
+          o.x = lars_momentum(gv[u].x, mv[u].x, wv[u].x, lam, b1, omb1);
+          o.y = lars_momentum(gv[u].y, mv[u].y, wv[u].y, lam, b1, omb1);
+          o.z = lars_momentum(gv[u].z, mv[u].z, wv[u].z, lam, b1, omb1);
+          o.w = lars_momentum(gv[u].w, mv[u].w, wv[u].w, lam, b1, omb1);
+          sw = __fmaf_rn(wv[u].x, wv[u].x, sw);
+          sw = __fmaf_rn(wv[u].y, wv[u].y, sw);
+          sw = __fmaf_rn(wv[u].z, wv[u].z, sw);
+          sw = __fmaf_rn(wv[u].w, wv[u].w, sw);
+          su = __fmaf_rn(o.x, o.x, su);
+          su = __fmaf_rn(o.y, o.y, su);
+          su = __fmaf_rn(o.z, o.z, su);
+          su = __fmaf_rn(o.w, o.w, su);
+          st4(m + 4 * j, o);
+        }
+      }
+    }
+    scalar_from = nv << 2;
+  }
+  for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
+    const float wi = w[i];
+    const float o = lars_momentum(ld_grad1(g + i), m[i], wi, lam, b1, omb1);
+    m[i] = o;
+    sw = __fmaf_rn(wi, wi, sw);
+    su = __fmaf_rn(o, o, su);
+  }
+}
+
+template <typename GT>
+__global__ void __launch_bounds__(kThreads)
+    lars_pass1_kernel(const StepParams p) {
+  __shared__ float red[2][kWarps];
+  __shared__ uint32_t s_next[2];
+  __shared__ int s_last;
+  if (threadIdx.x == 0) {
+    if (blockIdx.x == 0) {
+      StepScalars sc{};
+      sc.t = p.d_step ? *p.d_step : int64_t(0);
+      sc.c1 = 1.f;
+      sc.c2 = 1.f;
+      sc.lr = *p.d_lr;
+      sc.skip = 0;
+      *p.scal = sc;
+    }
+    s_next[0] = atomicAdd(&p.counters[0], 1u);
+  }
+  __syncthreads();
+  int it = 0;
+  uint32_t c = s_next[0];
+  while (c < (uint32_t)p.n_chunks) {
+    if (threadIdx.x == 0) s_next[(it + 1) & 1] = atomicAdd(&p.counters[0], 1u);
+    const ChunkDesc ch = p.chunks[c];
+    const TensorDesc td = p.tensors[ch.tensor];
+    const TensorPtrs tp = p.ptrs[ch.tensor];
+    const float lam = td.decay * p.wd;
+    float sw = 0.f, su = 0.f;
+    lars1_chunk<GT>(tp, ch, lam, p.b1, p.omb1, sw, su);
+    publish_chunk(p, (int)c, ch, td, sw, su, red, &s_last, p.trust);
+    ++it;
+    c = s_next[it & 1];
+  }
+  retire(p, 0, c);
+}
+
+template <bool kCopy>
+__device__ __forceinline__ void lars2_chunk(const TensorPtrs& tp,
+                                            const ChunkDesc& ch, float s) {
+  float* __restrict__ w = tp.w + ch.offset;
+  const float* __restrict__ m = tp.m + ch.offset;
+  const int n = ch.len;
+  int scalar_from = 0;
+  if (tp.vec_ok) {
+    const int nv = n >> 2;
+    for (int base = threadIdx.x; base < nv; base += kThreads * kUnroll2) {
+      float4 wv[kUnroll2], mv[kUnroll2];
+#pragma unroll
+      for (int u = 0; u < kUnroll2; ++u) {
+        const int j = base + u * kThreads;
+        if (j < nv) {
+          mv[u] = ld4_last(m + 4 * j);
+          wv[u] = ld4_last(w + 4 * j);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll2; ++u) {
+        const int j = base + u * kThreads;
+        if (j < nv) {
+          float4 o;
+          o.x = __fmaf_rn(-s, mv[u].x, wv[u].x);
+          o.y = __fmaf_rn(-s, mv[u].y, wv[u].y);
+          o.z = __fmaf_rn(-s, mv[u].z, wv[u].z);
+          o.w = __fmaf_rn(-s, mv[u].w, wv[u].w);
+          st4_last(w + 4 * j, o);
+          if (kCopy) st_copy4(tp.copy, ch.offset + 4 * j, o);
+        }
+      }
+    }
+    scalar_from = nv << 2;
+  }
+  for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
+    const float o = __fmaf_rn(-s, m[i], w[i]);
+    w[i] = o;
+    if (kCopy) st_copy1(tp.copy, ch.offset + i, o);
+  }
+}
+
+template <bool kCopy>
+__global__ void __launch_bounds__(kThreads)
+    lars_pass2_kernel(const StepParams p) {
+  __shared__ uint32_t s_next[2];
+  const StepScalars sc = *p.scal;
+  if (threadIdx.x == 0) s_next[0] = atomicAdd(&p.counters[1], 1u);
+  __syncthreads();
+  int it = 0;
+  uint32_t c = s_next[0];
+  const int nc = p.n_chunks;
+  while (c < (uint32_t)nc) {
+    if (threadIdx.x == 0) s_next[(it + 1) & 1] = atomicAdd(&p.counters[1], 1u);
+    const ChunkDesc ch = p.chunks[nc - 1 - (int)c];
+    const TensorPtrs tp = p.ptrs[ch.tensor];
+    const float s = __double2float_rn((double)sc.lr * p.ratio[ch.tensor]);
+    lars2_chunk<kCopy>(tp, ch, s);
+    __syncthreads();
+    ++it;
+    c = s_next[it & 1];
+  }
+  if (retire(p, 1, c) && threadIdx.x == 0 &&
+      (p.flags & kFlagIncrementStep) && p.d_step)
+    *p.d_step = sc.t + 1;
+}
+
+template <typename K>
+int occupancy_of(K kernel, int* blocks) {
+  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, kernel,
+                                                            kThreads, 0);
+}
+
+}  // namespace
+
+int launch_lamb_pass1(const StepParams& p, int grad_bf16, int grid,
+                      void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (grad_bf16)
+    lamb_pass1_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(p);
+  else
+    lamb_pass1_kernel<float><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
+int launch_lamb_pass2(const StepParams& p, int copy_bf16, int grid,
+                      void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (copy_bf16)
+    lamb_pass2_kernel<true><<<grid, kThreads, 0, s>>>(p);
+  else
+    lamb_pass2_kernel<false><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
+int launch_lars_pass1(const StepParams& p, int grad_bf16, int grid,
+                      void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (grad_bf16)
+    lars_pass1_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(p);
+  else
+    lars_pass1_kernel<float><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
+int launch_lars_pass2(const StepParams& p, int copy_bf16, int grid,
+                      void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (copy_bf16)
+    lars_pass2_kernel<true><<<grid, kThreads, 0, s>>>(p);
+  else
+    lars_pass2_kernel<false><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
+int occupancy_lamb_pass1(int grad_bf16, int* blocks) {
+  return grad_bf16 ? occupancy_of(lamb_pass1_kernel<__nv_bfloat16>, blocks)
+                   : occupancy_of(lamb_pass1_kernel<float>, blocks);
+}
+int occupancy_lamb_pass2(int copy_bf16, int* blocks) {
+  return copy_bf16 ? occupancy_of(lamb_pass2_kernel<true>, blocks)
+                   : occupancy_of(lamb_pass2_kernel<false>, blocks);
+}
+int occupancy_lars_pass1(int grad_bf16, int* blocks) {
+  return grad_bf16 ? occupancy_of(lars_pass1_kernel<__nv_bfloat16>, blocks)
+                   : occupancy_of(lars_pass1_kernel<float>, blocks);
+}
+int occupancy_lars_pass2(int copy_bf16, int* blocks) {
+  return copy_bf16 ? occupancy_of(lars_pass2_kernel<true>, blocks)
+                   : occupancy_of(lars_pass2_kernel<false>, blocks);
+}
+
+}  // namespace lamb
