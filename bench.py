@@ -1,0 +1,480 @@
+#!/usr/bin/env python3
+"""Benchmark of the LAMB optimizer step on the BERT-large parameter layout.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Workload: BERT-large (24 layers, hidden 1024, FFN 4096, vocab 30522): 391
+tensors, 335,141,888 parameters; bf16 gradients, fp32 master weights and Adam
+moments, a bf16 weight copy written every step; beta1 0.9, beta2 0.999,
+eps 1e-6, lambda 0.01 (biases / LayerNorm masked), phi = clip[0, 10],
+eta = 2e-3, measured from step t = 1000 on (the step counter lives on the
+device and is advanced by the kernels).  Inputs are seeded synthetic arrays
+(workloads.bert_large_layout); the W warm-up steps run t = 1..W from m = v = 0
+(W >= 3 gives the configured three warm-up steps).  All state (5.4 GB) is far
+larger than L2, so no explicit L2 flush is needed between steps.
+
+One JSON line is printed by rank 0:
+  value     parameters/s of the whole job, state resident in HBM, timed with
+            CUDA events on the launching stream over K steps
+  e2e       the same metric through the same C-ABI call, but every step also
+            copies that step's bf16 gradients host->device from pinned memory
+            and reads the step's result (the per-tensor trust ratios) back
+  roofline  the dominant kernel's algorithmic bytes / its event-timed
+            duration, against the measured HBM copy bandwidth
+  cpu_baseline  the fp64 oracle on a bounded sample, on this host's cores
+Multi-GPU (torchrun): every rank runs an independent replica (the step has no
+data-path exchange on one node here); value = all ranks' parameters / the
+slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import datetime as _dt
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = ("LAMB step params/sec and achieved HBM GB/s vs GB300 peak "
+          "(BERT-large layout)")
+UNIT = "params/s"
+FALLBACK_HBM_GBS = 6800.0
+# algorithmic bytes per parameter of each kernel (bf16 g, bf16 copy)
+BYTES_PASS1 = 2 + 4 + 4 + 4 + 4 + 4      # read g,m,v,w ; write m,v = 22
+BYTES_PASS2 = 4 + 4 + 4 + 4 + 2          # read m,v,w ; write w, copy = 18
+BYTES_STEP = BYTES_PASS1 + BYTES_PASS2   # 40
+BYTES_SINGLE_TOUCH = 2 + 12 + 12 + 2     # 28
+KERNEL_NAMES = ["lamb_pass1_kernel<bf16>", "lamb_pass2_kernel<copy>"]
+KERNEL_BYTES = [BYTES_PASS1, BYTES_PASS2]
+PROFILE_FILE = os.path.join(ROOT, "profiles", "lamb_kernels_bert_large.md")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--e2e-steps", type=int, default=None,
+                    help="steps of the end-to-end loop (default: min(K, 50))")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0,
+                    help="wall time of the bounded oracle sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=24,
+                    help="encoder layers of the layout (24 = BERT-large; "
+                         "fewer only for small profiling captures)")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# helpers
+# ---------------------------------------------------------------------------
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for name in ("lamb_kernels.cu", "lamb_internal.h"):
+        with open(os.path.join(ROOT, "paper_1904_00962_gb300", "csrc",
+                               name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel_idx):
+    """Per-launch DRAM bytes from the committed ncu summary, if it was taken
+    on the current kernel source; else None."""
+    try:
+        text = open(PROFILE_FILE).read()
+    except OSError:
+        return None
+    m = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", text)
+    if not m or m.group(1) != kernel_source_hash():
+        return None
+    m = re.search(rf"traffic_bytes_per_launch\[{kernel_idx}\]:\s*([0-9.e+]+)",
+                  text)
+    return float(m.group(1)) if m else None
+
+
+class ClockSampler:
+    """nvidia-smi sampled every 100 ms into a temp file; samples whose
+    timestamps fall inside [start, end] are summarised."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,"
+              "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id=None):
+        self.tmp = tempfile.NamedTemporaryFile("w+", suffix=".csv",
+                                               delete=False)
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}",
+               "--format=csv,noheader,nounits", "-lms", "100"]
+        if gpu_id:
+            cmd.insert(1, f"--id={gpu_id}")
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=self.tmp,
+                                         stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        self.window = None
+
+    def mark(self, start, end):
+        self.window = (start, end)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.tmp.flush()
+        rows = []
+        with open(self.tmp.name) as f:
+            for line in f:
+                p = [x.strip() for x in line.split(",")]
+                if len(p) < 9:
+                    continue
+                try:
+                    ts = _dt.datetime.strptime(p[0], "%Y/%m/%d %H:%M:%S.%f")
+                    rows.append((ts, float(p[1]), float(p[2]), p[3], p[4:]))
+                except ValueError:
+                    continue
+        os.unlink(self.tmp.name)
+        if not rows:
+            return None
+        sel = rows
+        if self.window:
+            a, b = self.window
+            inside = [r for r in rows if a <= r[0] <= b]
+            sel = inside if inside else rows
+        names = ["active", "hw_slowdown", "hw_thermal_slowdown",
+                 "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in sel:
+            for name, val in zip(names[1:], r[4][1:]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r[1] for r in sel),
+                "sm_max_mhz": max(r[2] for r in sel),
+                "samples": len(sel),
+                "reasons": sorted(reasons)}
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def select_params(L, target, pool):
+    """Whole tensors from `pool` (cycled) until `target` parameters."""
+    out, n, i = [], 0, 0
+    while n < target:
+        k = pool[i % len(pool)]
+        out.append(k)
+        n += L.sizes[k]
+        i += 1
+    return out
+
+
+def oracle_sample(L, h, seconds=None, target=None):
+    """Times the fp64 oracle on whole BERT-large encoder-layer tensors.
+    Either for `seconds` of wall time (cycling over the tensors) or over a
+    fixed selection of `target` parameters.  Returns (params, seconds)."""
+    from oracle import lamb_oracle as O
+    pool = [k for k, n in enumerate(L.names) if n.startswith("layer0.")]
+    inputs = {}
+
+    def inp(k):
+        if k not in inputs:
+            m, v = L.state_warm(k)
+            inputs[k] = (L.weights(k), L.grad(k, 1), m, v)
+        return inputs[k]
+
+    kw = dict(t=1000, lr=float(h.lr), beta1=h.beta1, beta2=h.beta2,
+              eps=h.eps, weight_decay=h.weight_decay, phi_kind=h.phi,
+              gamma_l=h.gamma_l, gamma_u=h.gamma_u, g_dtype=L.grad_dtype)
+    done, spent, i = 0, 0.0, 0
+    ks = select_params(L, target, pool) if target else None
+    while True:
+        if ks is not None:
+            if i >= len(ks):
+                break
+            k = ks[i]
+        else:
+            if spent >= seconds:
+                break
+            k = pool[i % len(pool)]
+        w, g, m, v = inp(k)
+        t0 = time.perf_counter()
+        O.lamb_tensor(w, g, m, v, decay=bool(L.decay[k]), **kw)
+        spent += time.perf_counter() - t0
+        done += L.sizes[k]
+        i += 1
+    return done, spent
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the fp64 oracle on the host cores
+# ---------------------------------------------------------------------------
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_1904_00962_gb300.workloads import bert_large_layout
+    L = bert_large_layout()
+    h = L.hyper
+    # each step: whole layer-0 tensors totalling ~target parameters, sized so
+    # that K + W steps take about 90 s at ~2 Mparam/s
+    target = int(min(max(2.0e6 * 90.0 / max(args.steps + args.warmup, 1),
+                         4096), 12.6e6))
+    for _ in range(args.warmup):
+        oracle_sample(L, h, target=target)
+    done, spent = 0, 0.0
+    for _ in range(args.steps):
+        d, s = oracle_sample(L, h, target=target)
+        done += d
+        spent += s
+    value = done / spent
+    sample = (f"per step: whole BERT-large layer-0 tensors totalling >= "
+              f"{target} params (fp64 NumPy oracle, one tensor at a time, "
+              f"1 thread)")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * spent / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "bert_large_layout", "n_params": L.n_params,
+                   "n_tensors": L.n_tensors, "grad_dtype": "bf16",
+                   "sample_params_per_step": target},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    from paper_1904_00962_gb300 import binding as B
+    from paper_1904_00962_gb300 import build as build_mod
+    from paper_1904_00962_gb300.state import DeviceState, LambPlan
+    from paper_1904_00962_gb300.workloads import bert_large_layout, bert_layout
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if not os.path.exists(B.LIB_PATH):
+        build_mod.build()
+    B.load()
+
+    if args.layers == 24:
+        L = bert_large_layout()
+        workload = "bert_large_layout"
+    else:
+        L = bert_layout(args.layers, 1024, 4096, name="bert_large",
+                        grad_dtype="bf16", copy_dtype="bf16",
+                        measured_step=1000)
+        workload = f"bert_large_layout_{args.layers}_layers"
+    h = L.hyper
+    P = L.n_params
+    st = DeviceState(L.sizes, grad_dtype="bf16", copy_dtype="bf16",
+                     device=dev)
+    for k in range(L.n_tensors):
+        st.upload("w", k, L.weights(k))
+        st.upload("g", k, L.grad(k, 1))
+    plan = LambPlan(st, L.decay)
+    d_step = torch.ones(1, dtype=torch.int64, device=dev)
+    d_lr = torch.full((1,), float(np.float32(h.lr)), dtype=torch.float32,
+                      device=dev)
+    hyper = B.make_hyper(beta1=h.beta1, beta2=h.beta2, eps=h.eps,
+                         weight_decay=h.weight_decay, phi=h.phi,
+                         gamma_l=h.gamma_l, gamma_u=h.gamma_u,
+                         bias_correction=True, increment_step=True)
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if world > 1:
+            torch.distributed.barrier()
+
+    # warm-up: t = 1..W from m = v = 0, then jump to the measured step
+    for _ in range(args.warmup):
+        plan.lamb_step(hyper, d_step, d_lr)
+    d_step.fill_(1000)
+    barrier()
+
+    gpu_id = None
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        gpu_id = None
+    clocks = ClockSampler(gpu_id) if rank == 0 else None
+    time.sleep(0.3)   # let the sampler start
+
+    # ---- device-resident timed region ----------------------------------
+    B.lamb_plan_set_timing(plan.handle, True)
+    barrier()
+    wall0 = _dt.datetime.now()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        plan.lamb_step(hyper, d_step, d_lr)
+    e1.record(stream)
+    barrier()
+    wall1 = _dt.datetime.now()
+    ms_total = e0.elapsed_time(e1)
+    n_timed, ms_kernels = B.lamb_plan_read_timing(plan.handle, 2)
+    B.lamb_plan_set_timing(plan.handle, False)
+    if clocks:
+        clocks.mark(wall0, wall1)
+    if world > 1:
+        t = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms_total = float(t.item())
+    status = plan.query(clear=True)
+
+    # ---- end to end: pinned host gradients in, trust ratios out ----------
+    k_e2e = args.e2e_steps if args.e2e_steps is not None else min(args.steps, 50)
+    g_host = torch.empty(st.total, dtype=torch.bfloat16).pin_memory()
+    g_host.copy_(st.g.cpu())
+    ratio_host = torch.empty(L.n_tensors, dtype=torch.float64).pin_memory()
+    h2d = L.n_params * 2
+    d2h = L.n_tensors * 8
+    barrier()
+    e2 = torch.cuda.Event(enable_timing=True)
+    e3 = torch.cuda.Event(enable_timing=True)
+    done = torch.cuda.Event()
+    e2.record(stream)
+    for _ in range(k_e2e):
+        st.g.copy_(g_host, non_blocking=True)
+        plan.lamb_step(hyper, d_step, d_lr)
+        B.lamb_plan_copy_trust_ratios(plan.handle, ratio_host.data_ptr(),
+                                      stream=stream.cuda_stream)
+        done.record(stream)
+        done.synchronize()
+    e3.record(stream)
+    barrier()
+    ms_e2e = e2.elapsed_time(e3)
+    if world > 1:
+        t = torch.tensor([ms_e2e], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms_e2e = float(t.item())
+    assert math.isfinite(float(ratio_host[0]))
+    clk = clocks.stop() if clocks else None
+
+    if rank != 0:
+        plan.destroy()
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return 0
+
+    # ---- roofline of the dominant kernel --------------------------------
+    peak, peak_src = load_peaks()
+    per_launch_ms = [ms / max(n_timed, 1) for ms in ms_kernels]
+    dom = int(np.argmax(per_launch_ms))
+    alg_bytes = KERNEL_BYTES[dom] * P
+    achieved = alg_bytes / (per_launch_ms[dom] * 1e-3) / 1e9
+    traffic = profiled_traffic(dom)
+    ms_step = ms_total / args.steps
+    step_gbs = BYTES_STEP * P / (ms_step * 1e-3) / 1e9
+
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        done_p, spent = oracle_sample(L, h, seconds=args.cpu_seconds)
+        cpu = {"value": done_p / spent, "unit": UNIT, "cores": 1,
+               "kind": "oracle",
+               "sample": (f"{done_p} params: whole BERT-large layer-0 tensors "
+                          f"cycled for ~{args.cpu_seconds:.0f} s, fp64 NumPy "
+                          f"oracle, 1 thread")}
+
+    line = {
+        "metric": METRIC,
+        "value": P * world * args.steps / (ms_total * 1e-3),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": workload, "n_params": P,
+                   "n_tensors": L.n_tensors, "grad_dtype": "bf16",
+                   "master_dtype": "f32", "copy_dtype": "bf16",
+                   "step_t": 1000, "lr": float(h.lr), "phi": "clip[0,10]",
+                   "l2": "inputs larger than L2 (5.4 GB state)",
+                   "parallelism": f"replicas{world}" if world > 1 else "1gpu"},
+        "hbm_gbs_step": step_gbs,
+        "frac_of_peak_step_40B": step_gbs / peak,
+        "frac_of_peak_single_touch_28B": BYTES_SINGLE_TOUCH * P /
+        (ms_step * 1e-3) / 1e9 / peak,
+        "kernels": {KERNEL_NAMES[i]: {"ms_per_launch": per_launch_ms[i],
+                                      "alg_bytes_per_param": KERNEL_BYTES[i]}
+                    for i in range(2)},
+        "roofline": {"bound": "hbm", "kernel": KERNEL_NAMES[dom],
+                     "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_source": f"{peak_src} (MEASURED_PEAKS hbm_gbs)"
+                     if peak_src == "measured" else "fallback 6800 GB/s"},
+        "e2e": {"value": P * world * k_e2e / (ms_e2e * 1e-3), "unit": UNIT,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "steps": k_e2e},
+        "gpu_launches": 2 * args.steps,
+        "device_status": status,
+        "clocks": clk,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line))
+    plan.destroy()
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())
