@@ -7,6 +7,10 @@ Tolerances (per element, |gpu - ref| <= tol * scale):
      along a chain also the element's oracle path sum_t |w_t - w_{t-1}|:
      each step's error is relative to that step's update, so near a zero
      crossing |w| alone says nothing about the accumulated error
+     and the update's size built from its operands' magnitudes,
+     lr*rho*(c1*(beta1|m_old| + (1-beta1)|g|)/(sqrt(v_hat)+eps) + lambda|w|)
+     (LARS: lr*rho*(beta1|m_old| + (1-beta1)(|g| + lambda|w|))): when m
+     cancels and w is 0 the update's error follows its operands
   m: scale = max(|ref|, |beta1 m_old| + |(1-beta1) g|  [+ lambda |w| LARS])
      fp32 error follows the operands, not a cancelled result
   v: scale = |ref|                     (a sum of non-negative terms)
@@ -67,15 +71,23 @@ def rel_max(err, scale):
 
 
 def compare_lamb(got_w, got_m, got_v, ref, w_old, m_old, g64, beta1, tol,
-                 w_path=None):
-    """Returns dict of max scaled errors; raises AssertionError on failure."""
+                 w_path=None, upd=None):
+    """Returns dict of max scaled errors; raises AssertionError on failure.
+    upd = (hyper, t, lr, lam) enables the update-operand floor of w."""
     got_w = got_w.astype(np.float64)
     got_m = got_m.astype(np.float64)
+    m_op = beta1 * np.abs(m_old) + (1 - beta1) * np.abs(g64)
     sw = np.maximum(np.abs(ref.w), np.abs(w_old))
     if w_path is not None:
         sw = np.maximum(sw, w_path)
-    sm = np.maximum(np.abs(ref.m), beta1 * np.abs(m_old) +
-                    (1 - beta1) * np.abs(g64))
+    if upd is not None:
+        h, t, lr, lam = upd
+        c1 = 1 / (1 - h.beta1 ** t) if h.bias_correction else 1.0
+        c2 = 1 / (1 - h.beta2 ** t) if h.bias_correction else 1.0
+        u_op = c1 * m_op / (np.sqrt(ref.v * c2) + h.eps) + lam * np.abs(w_old)
+        if np.isfinite(ref.ratio):
+            sw = np.maximum(sw, lr * ref.ratio * u_op)
+    sm = np.maximum(np.abs(ref.m), m_op)
     ew, em = np.abs(got_w - ref.w), np.abs(got_m - ref.m)
     assert _nan_aware_ok(ew, tol * sw, got_w, ref.w), f"w err {rel_max(ew, sw)}"
     assert _nan_aware_ok(em, tol * sm, got_m, ref.m), f"m err {rel_max(em, sm)}"
@@ -89,14 +101,18 @@ def compare_lamb(got_w, got_m, got_v, ref, w_old, m_old, g64, beta1, tol,
 
 
 def compare_lars(got_w, got_m, ref, w_old, m_old, g64, beta1, lam, tol,
-                 w_path=None):
+                 w_path=None, lr=None):
+    """lr enables the update-operand floor of w."""
     got_w = got_w.astype(np.float64)
     got_m = got_m.astype(np.float64)
+    m_op = beta1 * np.abs(m_old) + (1 - beta1) * (np.abs(g64) +
+                                                  lam * np.abs(w_old))
     sw = np.maximum(np.abs(ref.w), np.abs(w_old))
     if w_path is not None:
         sw = np.maximum(sw, w_path)
-    sm = np.maximum(np.abs(ref.m), beta1 * np.abs(m_old) + (1 - beta1) *
-                    (np.abs(g64) + lam * np.abs(w_old)))
+    if lr is not None and np.isfinite(ref.ratio):
+        sw = np.maximum(sw, lr * ref.ratio * m_op)
+    sm = np.maximum(np.abs(ref.m), m_op)
     ew, em = np.abs(got_w - ref.w), np.abs(got_m - ref.m)
     assert _nan_aware_ok(ew, tol * sw, got_w, ref.w), f"w err {rel_max(ew, sw)}"
     assert _nan_aware_ok(em, tol * sm, got_m, ref.m), f"m err {rel_max(em, sm)}"

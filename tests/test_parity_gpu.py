@@ -68,7 +68,8 @@ def test_mlp_chained_lamb(n_steps, bias_correction):
             e = compare_lamb(G.download("w", k), G.download("m", k),
                              G.download("v", k), ref, w0, m0,
                              g.astype(np.float64), h.beta1, tol,
-                             w_path=path[k])
+                             w_path=path[k],
+                             upd=(h, t, lr, h.weight_decay * L.decay[k]))
             worst = max(worst, *e.values())
             rt = TOL_RATIO if t == 1 else TOL_CHAIN
             assert ratio_ok(ratio[k], ref.ratio, rt), (t, k, ratio[k], ref.ratio)
@@ -100,7 +101,8 @@ def test_mlp_chained_lars_100():
             path[k] += np.abs(ref.w - w0)
             compare_lars(G.download("w", k), G.download("m", k), ref, w0, m0,
                          g.astype(np.float64), h.beta1,
-                         h.weight_decay * L.decay[k], tol, w_path=path[k])
+                         h.weight_decay * L.decay[k], tol, w_path=path[k],
+                         lr=lr)
             assert ratio_ok(ratio[k], ref.ratio,
                             TOL_RATIO if t == 1 else TOL_CHAIN)
             state[k] = (ref.w, ref.m)
@@ -136,12 +138,13 @@ def test_full_layout_one_step_every_tensor(name, lars):
             ref = _oracle_lars(L, k, w, g, m, lr, h)
             e = compare_lars(G.download("w", k), G.download("m", k), ref, w,
                              m, g64, h.beta1, h.weight_decay * L.decay[k],
-                             TOL_STEP)
+                             TOL_STEP, lr=lr)
         else:
             ref = _oracle_lamb(L, k, w, g, m, v, t, lr, h)
             e = compare_lamb(G.download("w", k), G.download("m", k),
                              G.download("v", k), ref, w, m, g64, h.beta1,
-                             TOL_STEP)
+                             TOL_STEP,
+                             upd=(h, t, lr, h.weight_decay * L.decay[k]))
         if L.copy_dtype:
             check_copy(G.download("copy", k), G.download("w", k), ref.w)
         assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
@@ -203,11 +206,12 @@ def test_full_layout_warm_trajectory(name, lars):
         if lars:
             compare_lars(G.download("w", k), G.download("m", k), ref, w0, m0,
                          g64, h.beta1, h.weight_decay * L.decay[k], TOL_STEP,
-                         w_path=path[k])
+                         w_path=path[k], lr=lr)
         else:
             compare_lamb(G.download("w", k), G.download("m", k),
                          G.download("v", k), ref, w0, m0, g64, h.beta1,
-                         TOL_STEP, w_path=path[k])
+                         TOL_STEP, w_path=path[k],
+                         upd=(h, ts[-1], lr, h.weight_decay * L.decay[k]))
         if L.copy_dtype:
             check_copy(G.download("copy", k), G.download("w", k), ref.w)
         assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
@@ -252,7 +256,8 @@ def test_ragged_full_size():
         ref = _oracle_lamb(L, k, w, g, z, z, 1, lr, h)
         compare_lamb(G.download("w", k), G.download("m", k),
                      G.download("v", k), ref, w, z, g.astype(np.float64),
-                     h.beta1, TOL_STEP)
+                     h.beta1, TOL_STEP,
+                     upd=(h, 1, lr, h.weight_decay * L.decay[k]))
         assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
         assert ratio_ok(wn[k], ref.wnorm) and ratio_ok(un[k], ref.unorm)
     oracle_map(check, ks)
@@ -327,7 +332,8 @@ def test_edge_layout(grad_dtype, copy_dtype, chunk, bps, misalign):
         ref = _oracle_lamb(L, k, w, g, m, v, 2, lr, h)
         compare_lamb(G.download("w", k), G.download("m", k),
                      G.download("v", k), ref, w, m, O.to_f64(g, grad_dtype),
-                     h.beta1, TOL_STEP)
+                     h.beta1, TOL_STEP,
+                     upd=(h, 2, lr, h.weight_decay * L.decay[k]))
         if copy_dtype:
             check_copy(G.download("copy", k), G.download("w", k), ref.w)
         assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
@@ -359,12 +365,13 @@ def test_edge_layout_phi_and_lars(phi, gl, gu):
                 ref = _oracle_lars(L, k, w, g, m, lr, h)
                 compare_lars(G.download("w", k), G.download("m", k), ref, w,
                              m, g.astype(np.float64), h.beta1,
-                             h.weight_decay * L.decay[k], TOL_STEP)
+                             h.weight_decay * L.decay[k], TOL_STEP, lr=lr)
             else:
                 ref = _oracle_lamb(L, k, w, g, m, v, 3, lr, h)
                 compare_lamb(G.download("w", k), G.download("m", k),
                              G.download("v", k), ref, w, m,
-                             g.astype(np.float64), h.beta1, TOL_STEP)
+                             g.astype(np.float64), h.beta1, TOL_STEP,
+                             upd=(h, 3, lr, h.weight_decay * L.decay[k]))
             assert ratio_ok(ratio[k], ref.ratio), (lars, k)
         G.close()
 
@@ -543,7 +550,8 @@ def test_nonfinite_gradient_propagates_and_is_flagged():
         ref = _oracle_lamb(L, k, w, g, z, z, 1, lr, L.hyper)
         compare_lamb(G.download("w", k), G.download("m", k),
                      G.download("v", k), ref, w, z, g.astype(np.float64),
-                     L.hyper.beta1, TOL_STEP)
+                     L.hyper.beta1, TOL_STEP,
+                     upd=(L.hyper, 1, lr, L.hyper.weight_decay * L.decay[k]))
         assert ratio_ok(ratio[k], ref.ratio)
     assert np.isnan(G.download("w", bad)).all()
     G.close()
