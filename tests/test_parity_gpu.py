@@ -9,7 +9,7 @@ import torch
 
 from gpu_util import (TOL_CHAIN, TOL_RATIO, TOL_STEP, GpuLayout, c_hyper,
                       check_copy, compare_lamb, compare_lars, f32,
-                      hyper_kwargs, oracle_map, ratio_ok)
+                      hyper_kwargs, oracle_map, ratio_ok, worst_of)
 from oracle import lamb_oracle as O
 from paper_1904_00962_gb300 import binding as B
 from paper_1904_00962_gb300 import build as build_mod
@@ -70,7 +70,7 @@ def test_mlp_chained_lamb(n_steps, bias_correction):
                              g.astype(np.float64), h.beta1, tol,
                              w_path=path[k],
                              upd=(h, t, lr, h.weight_decay * L.decay[k]))
-            worst = max(worst, *e.values())
+            worst = max(worst, worst_of(e))
             rt = TOL_RATIO if t == 1 else TOL_CHAIN
             assert ratio_ok(ratio[k], ref.ratio, rt), (t, k, ratio[k], ref.ratio)
             state[k] = (ref.w, ref.m, ref.v)
@@ -146,7 +146,8 @@ def test_full_layout_one_step_every_tensor(name, lars):
                              TOL_STEP,
                              upd=(h, t, lr, h.weight_decay * L.decay[k]))
         if L.copy_dtype:
-            check_copy(G.download("copy", k), G.download("w", k), ref.w)
+            check_copy(G.download("copy", k), G.download("w", k), ref.w,
+                       sw=e["_sw"])
         assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
         assert ratio_ok(wn[k], ref.wnorm) and ratio_ok(un[k], ref.unorm), k
         return abs(ratio[k] - ref.ratio) / max(abs(ref.ratio), 1e-300)
@@ -204,16 +205,17 @@ def test_full_layout_warm_trajectory(name, lars):
         w0, m0, v0, ref, g = final[k]
         g64 = O.to_f64(g, L.grad_dtype)
         if lars:
-            compare_lars(G.download("w", k), G.download("m", k), ref, w0, m0,
-                         g64, h.beta1, h.weight_decay * L.decay[k], TOL_STEP,
-                         w_path=path[k], lr=lr)
+            e = compare_lars(G.download("w", k), G.download("m", k), ref, w0,
+                             m0, g64, h.beta1, h.weight_decay * L.decay[k],
+                             TOL_STEP, w_path=path[k], lr=lr)
         else:
-            compare_lamb(G.download("w", k), G.download("m", k),
-                         G.download("v", k), ref, w0, m0, g64, h.beta1,
-                         TOL_STEP, w_path=path[k],
-                         upd=(h, ts[-1], lr, h.weight_decay * L.decay[k]))
+            e = compare_lamb(G.download("w", k), G.download("m", k),
+                             G.download("v", k), ref, w0, m0, g64, h.beta1,
+                             TOL_STEP, w_path=path[k],
+                             upd=(h, ts[-1], lr, h.weight_decay * L.decay[k]))
         if L.copy_dtype:
-            check_copy(G.download("copy", k), G.download("w", k), ref.w)
+            check_copy(G.download("copy", k), G.download("w", k), ref.w,
+                       sw=e["_sw"])
         assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
     G.close()
 
@@ -330,12 +332,13 @@ def test_edge_layout(grad_dtype, copy_dtype, chunk, bps, misalign):
         w, g = L.weights(k), L.grad(k, 2)
         m, v = L.state_warm(k)
         ref = _oracle_lamb(L, k, w, g, m, v, 2, lr, h)
-        compare_lamb(G.download("w", k), G.download("m", k),
-                     G.download("v", k), ref, w, m, O.to_f64(g, grad_dtype),
-                     h.beta1, TOL_STEP,
-                     upd=(h, 2, lr, h.weight_decay * L.decay[k]))
+        e = compare_lamb(G.download("w", k), G.download("m", k),
+                         G.download("v", k), ref, w, m,
+                         O.to_f64(g, grad_dtype), h.beta1, TOL_STEP,
+                         upd=(h, 2, lr, h.weight_decay * L.decay[k]))
         if copy_dtype:
-            check_copy(G.download("copy", k), G.download("w", k), ref.w)
+            check_copy(G.download("copy", k), G.download("w", k), ref.w,
+                       sw=e["_sw"])
         assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
         if L.sizes[k] == 0:
             assert ratio[k] == 1.0 and wn[k] == 0.0 and un[k] == 0.0
