@@ -12,7 +12,9 @@ Tolerances (per element, |gpu - ref| <= tol * scale):
      (LARS: lr*rho*(beta1|m_old| + (1-beta1)(|g| + lambda|w|))): when m
      cancels and w is 0 the update's error follows its operands
   m: scale = max(|ref|, |beta1 m_old| + |(1-beta1) g|  [+ lambda |w| LARS])
-     fp32 error follows the operands, not a cancelled result
+     fp32 error follows the operands, not a cancelled result; along a chain
+     the running operand size M_t = beta1 M_{t-1} + (1-beta1)|g_t| [+...]
+     (earlier steps' rounding is carried forward with factor beta1)
   v: scale = |ref|                     (a sum of non-negative terms)
   trust ratio: relative 1e-6
 tol = 1e-5 after one step, 1e-4 along chained runs.
@@ -71,7 +73,7 @@ def rel_max(err, scale):
 
 
 def compare_lamb(got_w, got_m, got_v, ref, w_old, m_old, g64, beta1, tol,
-                 w_path=None, upd=None):
+                 w_path=None, upd=None, m_path=None):
     """Returns dict of max scaled errors; raises AssertionError on failure.
     upd = (hyper, t, lr, lam) enables the update-operand floor of w."""
     got_w = got_w.astype(np.float64)
@@ -88,6 +90,8 @@ def compare_lamb(got_w, got_m, got_v, ref, w_old, m_old, g64, beta1, tol,
         if np.isfinite(ref.ratio):
             sw = np.maximum(sw, lr * ref.ratio * u_op)
     sm = np.maximum(np.abs(ref.m), m_op)
+    if m_path is not None:
+        sm = np.maximum(sm, m_path)
     ew, em = np.abs(got_w - ref.w), np.abs(got_m - ref.m)
     assert _nan_aware_ok(ew, tol * sw, got_w, ref.w), f"w err {rel_max(ew, sw)}"
     assert _nan_aware_ok(em, tol * sm, got_m, ref.m), f"m err {rel_max(em, sm)}"
@@ -101,7 +105,7 @@ def compare_lamb(got_w, got_m, got_v, ref, w_old, m_old, g64, beta1, tol,
 
 
 def compare_lars(got_w, got_m, ref, w_old, m_old, g64, beta1, lam, tol,
-                 w_path=None, lr=None):
+                 w_path=None, lr=None, m_path=None):
     """lr enables the update-operand floor of w."""
     got_w = got_w.astype(np.float64)
     got_m = got_m.astype(np.float64)
@@ -113,6 +117,8 @@ def compare_lars(got_w, got_m, ref, w_old, m_old, g64, beta1, lam, tol,
     if lr is not None and np.isfinite(ref.ratio):
         sw = np.maximum(sw, lr * ref.ratio * m_op)
     sm = np.maximum(np.abs(ref.m), m_op)
+    if m_path is not None:
+        sm = np.maximum(sm, m_path)
     ew, em = np.abs(got_w - ref.w), np.abs(got_m - ref.m)
     assert _nan_aware_ok(ew, tol * sw, got_w, ref.w), f"w err {rel_max(ew, sw)}"
     assert _nan_aware_ok(em, tol * sm, got_m, ref.m), f"m err {rel_max(em, sm)}"

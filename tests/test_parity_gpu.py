@@ -55,6 +55,7 @@ def test_mlp_chained_lamb(n_steps, bias_correction):
     hyp = c_hyper(h)
     worst = 0.0
     path = [np.zeros(s) for s in L.sizes]
+    mpath = [np.zeros(s) for s in L.sizes]
     for t in range(1, n_steps + 1):
         G.load_grads(t)
         G.step(t, lr, hyp)
@@ -65,10 +66,11 @@ def test_mlp_chained_lamb(n_steps, bias_correction):
             g = L.grad(k, t)
             ref = _oracle_lamb(L, k, w0, g, m0, v0, t, lr, h)
             path[k] += np.abs(ref.w - w0)
+            mpath[k] = h.beta1 * mpath[k] + (1 - h.beta1) * np.abs(g)
             e = compare_lamb(G.download("w", k), G.download("m", k),
                              G.download("v", k), ref, w0, m0,
                              g.astype(np.float64), h.beta1, tol,
-                             w_path=path[k],
+                             w_path=path[k], m_path=mpath[k],
                              upd=(h, t, lr, h.weight_decay * L.decay[k]))
             worst = max(worst, worst_of(e))
             rt = TOL_RATIO if t == 1 else TOL_CHAIN
@@ -89,6 +91,7 @@ def test_mlp_chained_lars_100():
              for k in range(L.n_tensors)]
     hyp = c_hyper(h, lars=True)
     path = [np.zeros(s) for s in L.sizes]
+    mpath = [np.zeros(s) for s in L.sizes]
     for t in range(1, 101):
         G.load_grads(t)
         G.step(t, lr, hyp, lars=True)
@@ -98,11 +101,13 @@ def test_mlp_chained_lars_100():
             w0, m0 = state[k]
             g = L.grad(k, t)
             ref = _oracle_lars(L, k, w0, g, m0, lr, h)
+            lam = h.weight_decay * L.decay[k]
             path[k] += np.abs(ref.w - w0)
+            mpath[k] = h.beta1 * mpath[k] + (1 - h.beta1) * (
+                np.abs(g) + lam * np.abs(w0))
             compare_lars(G.download("w", k), G.download("m", k), ref, w0, m0,
-                         g.astype(np.float64), h.beta1,
-                         h.weight_decay * L.decay[k], tol, w_path=path[k],
-                         lr=lr)
+                         g.astype(np.float64), h.beta1, lam, tol,
+                         w_path=path[k], lr=lr, m_path=mpath[k])
             assert ratio_ok(ratio[k], ref.ratio,
                             TOL_RATIO if t == 1 else TOL_CHAIN)
             state[k] = (ref.w, ref.m)
@@ -126,7 +131,7 @@ def test_full_layout_one_step_every_tensor(name, lars):
     G.load_warm_state()
     G.load_grads(t)
     lr = f32(h.lr)
-    G.step(t, lr, c_hyper(h, lars=lars))
+    G.step(t, lr, c_hyper(h, lars=lars), lars=lars)
     ratio, wn, un = G.results()
 
     def check(k):
@@ -187,16 +192,22 @@ def test_full_layout_warm_trajectory(name, lars):
     hyp = c_hyper(h, lars=lars)
     final = {}
     path = {k: np.zeros(L.sizes[k]) for k in ks}
+    mpath = {k: np.zeros(L.sizes[k]) for k in ks}
     for i, t in enumerate(ts):
         G.load_grads(i + 1)
         G.step(t, lr, hyp, lars=lars)
         for k in ks:
             w0, m0, v0 = state[k]
             g = L.grad(k, i + 1)
+            g64 = O.to_f64(g, L.grad_dtype)
+            lam = h.weight_decay * L.decay[k]
             if lars:
                 r = _oracle_lars(L, k, w0, g, m0, lr, h)
+                mpath[k] = h.beta1 * mpath[k] + (1 - h.beta1) * (
+                    np.abs(g64) + lam * np.abs(w0))
             else:
                 r = _oracle_lamb(L, k, w0, g, m0, v0, t, lr, h)
+                mpath[k] = h.beta1 * mpath[k] + (1 - h.beta1) * np.abs(g64)
             path[k] += np.abs(r.w - w0)
             final[k] = (w0, m0, v0, r, g)
             state[k] = (r.w, r.m, None if lars else r.v)
@@ -207,11 +218,12 @@ def test_full_layout_warm_trajectory(name, lars):
         if lars:
             e = compare_lars(G.download("w", k), G.download("m", k), ref, w0,
                              m0, g64, h.beta1, h.weight_decay * L.decay[k],
-                             TOL_STEP, w_path=path[k], lr=lr)
+                             TOL_STEP, w_path=path[k], lr=lr,
+                             m_path=mpath[k])
         else:
             e = compare_lamb(G.download("w", k), G.download("m", k),
                              G.download("v", k), ref, w0, m0, g64, h.beta1,
-                             TOL_STEP, w_path=path[k],
+                             TOL_STEP, w_path=path[k], m_path=mpath[k],
                              upd=(h, ts[-1], lr, h.weight_decay * L.decay[k]))
         if L.copy_dtype:
             check_copy(G.download("copy", k), G.download("w", k), ref.w,
