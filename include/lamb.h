@@ -234,6 +234,46 @@ LAMB_API lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensor
                                  int64_t* chunk_offset, int32_t* chunk_len,
                                  int32_t capacity, int32_t* n_chunks);
 
+/* One LAMB step (the same two kernels and numerics as lamb_step with the
+ * default 16384-element chunks) for callers that may not allocate device
+ * memory: code that runs under an allocator owning all GPU memory (a
+ * framework's caching allocator or a fixed pool), code that must not pay the
+ * device-wide synchronisation cudaMalloc/cudaFree can cause, or a plug-in
+ * that is handed a stream and buffers but no right to allocate.  It needs no
+ * plan: every table, partial sum and counter lives in one fixed 4 MiB device
+ * array built into the library, which each GPU that loads the library holds
+ * until the process exits.  (The paper has no counterpart of this entry
+ * point; it is a deployment convenience.)
+ *
+ *   sizes, decay_mask   host arrays [n_tensors] as in lamb_plan_create
+ *                       (decay_mask may be NULL = all decayed)
+ *   w, g, m, v, w_copy  host arrays [n_tensors] of DEVICE pointers as in
+ *                       lamb_plan_bind; v is required; w_copy iff copy_dtype
+ *                       is LAMB_BF16
+ *   hyper, d_step, d_lr as in lamb_step
+ *   d_ratio             NULL or a DEVICE array [n_tensors] of doubles that
+ *                       receives the trust ratios of this step
+ * Limits: n_tensors <= 4096 and at most 131072 chunks of 16384 elements
+ * (2^31 parameters); larger inputs are rejected with LAMB_ERR_INVALID_ARG
+ * before any device work.  Calls no cudaMalloc, cudaFree or other
+ * allocating routine.  The caller's host arrays are copied into the device
+ * array with cudaMemcpyAsync on `stream` and may be reused when the call
+ * returns.  The first call on each device (the current device) looks up the
+ * array's device address and the launch sizes; make that first call before
+ * any stream capture.  All calls share the one array: calls that may overlap
+ * on the GPU (other streams, other host threads) race and must be ordered by
+ * the caller.  Each call rebuilds the tables and clears the counters it
+ * needs, so it does not depend on what the previous call left there.
+ * Device-side conditions (a step count < 1: the step is skipped; non-finite
+ * norms: NaN/Inf propagate) behave as in lamb_step; there is no status
+ * query for this entry point. */
+LAMB_API lamb_status_t lamb_step_noalloc(
+    const int64_t* sizes, int32_t n_tensors, const uint8_t* decay_mask,
+    int32_t grad_dtype, int32_t copy_dtype, void* const* w,
+    const void* const* g, void* const* m, void* const* v,
+    void* const* w_copy, const lamb_hyper_t* hyper, int64_t* d_step,
+    const float* d_lr, double* d_ratio, cudaStream_t stream);
+
 /* Message of the last failed call on this host thread ("" if none). */
 LAMB_API const char* lamb_last_error(void);
 

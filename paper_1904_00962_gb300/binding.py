@@ -45,7 +45,7 @@ EXPORTED = ["lamb_plan_create", "lamb_plan_bind", "lamb_step", "lars_step",
             "lamb_plan_query", "lamb_plan_get_info",
             "lamb_plan_set_timing", "lamb_plan_read_timing",
             "lamb_plan_destroy", "lamb_layout_chunks", "lamb_last_error",
-            "lamb_abi_version"]
+            "lamb_abi_version", "lamb_step_noalloc"]
 
 
 class LambError(RuntimeError):
@@ -115,6 +115,11 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                        POINTER(c_int32), POINTER(c_int64),
                                        POINTER(c_int32), c_int32,
                                        POINTER(c_int32)]
+    lib.lamb_step_noalloc.argtypes = [POINTER(c_int64), c_int32,
+                                      POINTER(c_uint8), c_int32, c_int32,
+                                      POINTER(vp), POINTER(vp), POINTER(vp),
+                                      POINTER(vp), POINTER(vp),
+                                      POINTER(lamb_hyper_t), vp, vp, vp, vp]
     for name in EXPORTED:
         if name in ("lamb_last_error", "lamb_abi_version"):
             continue
@@ -235,6 +240,23 @@ def lamb_plan_read_timing(plan, n_kernels=2):
 def lamb_plan_destroy(plan) -> None:
     if plan:
         _check(load().lamb_plan_destroy(c_void_p(plan)))
+
+
+def lamb_step_noalloc(sizes, decay_mask, grad_dtype, copy_dtype, w, g, m, v,
+                      w_copy, hyper: lamb_hyper_t, d_step, d_lr, d_ratio=0,
+                      stream=0) -> None:
+    """Allocation-free LAMB step (see include/lamb.h): pointer lists as in
+    lamb_plan_bind, d_ratio an optional device float64 array."""
+    n = len(sizes)
+    sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
+    mask = None
+    if decay_mask is not None:
+        mask = (c_uint8 * max(n, 1))(*[1 if d else 0 for d in decay_mask])
+    _check(load().lamb_step_noalloc(
+        sz, n, mask, int(grad_dtype), int(copy_dtype), _ptr_array(w),
+        _ptr_array(g), _ptr_array(m), _ptr_array(v), _ptr_array(w_copy),
+        byref(hyper), c_void_p(d_step or None), c_void_p(d_lr or None),
+        c_void_p(d_ratio or None), c_void_p(stream or None)))
 
 
 def lamb_layout_chunks(sizes, chunk_elems=0):

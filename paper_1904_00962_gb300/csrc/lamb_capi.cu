@@ -34,6 +34,14 @@ lamb_status_t cuda_fail(cudaError_t e, const char* what) {
               (int)e);
 }
 
+}  // namespace
+
+void lamb::set_last_error(const char* msg) {
+  snprintf(g_err, sizeof(g_err), "%s", msg);
+}
+
+namespace {
+
 constexpr int kMaxTimedSteps = 4096;
 constexpr int kKernelsPerStep = 2;
 

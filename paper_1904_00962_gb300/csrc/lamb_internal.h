@@ -97,6 +97,9 @@ int occupancy_lamb_pass2(int copy_bf16, int* blocks);
 int occupancy_lars_pass1(int grad_bf16, int* blocks);
 int occupancy_lars_pass2(int copy_bf16, int* blocks);
 
+// Sets the thread-local message returned by lamb_last_error() (lamb_capi.cu).
+void set_last_error(const char* msg);
+
 // Host planner (planner.cpp).  Returns 0 on success, else writes a message.
 int plan_chunks(const int64_t* sizes, int32_t n, int32_t chunk_elems,
                 ChunkDesc* chunks, int64_t capacity, int64_t* n_chunks,
