@@ -53,9 +53,18 @@ BYTES_PASS1 = 2 + 4 + 4 + 4 + 4 + 4      # read g,m,v,w ; write m,v = 22
 BYTES_PASS2 = 4 + 4 + 4 + 4 + 2          # read m,v,w ; write w, copy = 18
 BYTES_STEP = BYTES_PASS1 + BYTES_PASS2   # 40
 BYTES_SINGLE_TOUCH = 2 + 12 + 12 + 2     # 28
-KERNEL_NAMES = ["lamb_pass1_kernel<bf16>", "lamb_pass2_kernel<copy>"]
-KERNEL_BYTES = [BYTES_PASS1, BYTES_PASS2]
-PROFILE_FILE = os.path.join(ROOT, "profiles", "lamb_kernels_bert_large.md")
+# per algorithm: kernels of one step, their algorithmic bytes per parameter,
+# and the committed ncu summary holding their measured DRAM traffic
+ALGO_CODES = {"auto": 0, "two_pass": 1, "single_touch": 2}
+KERNELS = {
+    1: (["lamb_pass1_kernel<bf16>", "lamb_pass2_kernel<copy>"],
+        [BYTES_PASS1, BYTES_PASS2],
+        os.path.join(ROOT, "profiles", "lamb_kernels_bert_large.md")),
+    # the single-touch kernel is held to the 28 B/param single-touch model
+    # (the embedding, too large for L2, really moves 40 B/param)
+    2: (["fused_step_kernel<lamb,bf16,copy>"], [BYTES_SINGLE_TOUCH],
+        os.path.join(ROOT, "profiles", "lamb_fused_bert_large.md")),
+}
 
 
 def parse_args():
@@ -69,6 +78,12 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=10.0,
                     help="wall time of the bounded oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--algo", choices=list(ALGO_CODES), default="auto",
+                    help="step algorithm of the plan (auto = library default)")
+    ap.add_argument("--lag-items", type=int, default=0,
+                    help="single-touch schedule lag (0 = library default)")
+    ap.add_argument("--l2-budget-mb", type=int, default=0,
+                    help="single-touch L2 budget (0 = library default)")
     ap.add_argument("--layers", type=int, default=24,
                     help="encoder layers of the layout (24 = BERT-large; "
                          "fewer only for small profiling captures)")
@@ -98,11 +113,11 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(kernel_idx):
+def profiled_traffic(profile_file, kernel_idx):
     """Per-launch DRAM bytes from the committed ncu summary, if it was taken
     on the current kernel source; else None."""
     try:
-        text = open(PROFILE_FILE).read()
+        text = open(profile_file).read()
     except OSError:
         return None
     m = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", text)
@@ -317,7 +332,10 @@ def run_ours(args):
     for k in range(L.n_tensors):
         st.upload("w", k, L.weights(k))
         st.upload("g", k, L.grad(k, 1))
-    plan = LambPlan(st, L.decay)
+    plan = LambPlan(st, L.decay, algorithm=ALGO_CODES[args.algo],
+                    lag_items=args.lag_items, l2_budget_mb=args.l2_budget_mb)
+    algo = plan.info()["algorithm"]
+    kernel_names, kernel_bytes, profile_file = KERNELS[algo]
     d_step = torch.ones(1, dtype=torch.int64, device=dev)
     d_lr = torch.full((1,), float(np.float32(h.lr)), dtype=torch.float32,
                       device=dev)
@@ -406,11 +424,12 @@ def run_ours(args):
 
     # ---- roofline of the dominant kernel --------------------------------
     peak, peak_src = load_peaks()
-    per_launch_ms = [ms / max(n_timed, 1) for ms in ms_kernels]
+    per_launch_ms = [ms / max(n_timed, 1)
+                     for ms in ms_kernels[:len(kernel_names)]]
     dom = int(np.argmax(per_launch_ms))
-    alg_bytes = KERNEL_BYTES[dom] * P
+    alg_bytes = kernel_bytes[dom] * P
     achieved = alg_bytes / (per_launch_ms[dom] * 1e-3) / 1e9
-    traffic = profiled_traffic(dom)
+    traffic = profiled_traffic(profile_file, dom)
     ms_step = ms_total / args.steps
     step_gbs = BYTES_STEP * P / (ms_step * 1e-3) / 1e9
 
@@ -446,10 +465,11 @@ def run_ours(args):
         "frac_of_peak_step_40B": step_gbs / peak,
         "frac_of_peak_single_touch_28B": BYTES_SINGLE_TOUCH * P /
         (ms_step * 1e-3) / 1e9 / peak,
-        "kernels": {KERNEL_NAMES[i]: {"ms_per_launch": per_launch_ms[i],
-                                      "alg_bytes_per_param": KERNEL_BYTES[i]}
-                    for i in range(2)},
-        "roofline": {"bound": "hbm", "kernel": KERNEL_NAMES[dom],
+        "algorithm": {1: "two_pass", 2: "single_touch"}[algo],
+        "kernels": {kernel_names[i]: {"ms_per_launch": per_launch_ms[i],
+                                      "alg_bytes_per_param": kernel_bytes[i]}
+                    for i in range(len(kernel_names))},
+        "roofline": {"bound": "hbm", "kernel": kernel_names[dom],
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_source": f"{peak_src} (MEASURED_PEAKS hbm_gbs)"
@@ -457,7 +477,7 @@ def run_ours(args):
         "e2e": {"value": P * world * k_e2e / (ms_e2e * 1e-3), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": k_e2e},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": len(kernel_names) * args.steps,
         "device_status": status,
         "clocks": clk,
         "cpu_baseline": cpu,

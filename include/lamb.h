@@ -92,6 +92,12 @@ typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
 #define LAMB_STATUS_BAD_STEP  0x2u      /* *d_step < 1 with bias correction:
                                            the step was skipped, nothing was
                                            written                          */
+#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* single-touch: a pass-2 item waited
+                                           ~0.5 s for its tensor's norms and
+                                           gave up; the rest of that launch's
+                                           pass-2 items then gave up too, so
+                                           w was not (fully) updated; never
+                                           expected                         */
 
 /* Hyperparameters.  Doubles on purpose: (1 - beta) is formed in double and
  * rounded once to float, so e.g. beta2 = 0.999 gives 1-beta2 = 0.001 to
@@ -109,12 +115,29 @@ typedef struct {
   uint32_t flags;        /* LAMB_FLAG_*                                     */
 } lamb_hyper_t;
 
+/* lamb_plan_options_t.algorithm */
+#define LAMB_ALGO_AUTO 0          /* the library's default (single-touch)    */
+#define LAMB_ALGO_TWO_PASS 1      /* two streaming kernels per step: 40 B of
+                                     HBM traffic per parameter (bf16 g/copy) */
+#define LAMB_ALGO_SINGLE_TOUCH 2  /* one kernel per step; pass 2 of a tensor
+                                     follows its pass 1 closely enough to read
+                                     m, v, w back from L2: ~28 B/parameter
+                                     for tensors whose state fits the L2
+                                     budget                                  */
+
 /* Optional plan-creation knobs (pass NULL for defaults). */
 typedef struct {
-  int32_t chunk_elems;   /* elements per chunk, multiple of 1024 in
+  int32_t chunk_elems;   /* two-pass: elements per chunk, multiple of 1024 in
                             [1024, 1<<24]; 0 = default (16384)             */
   int32_t blocks_per_sm; /* resident CTAs per SM for the persistent grid;
                             0 = as many as the occupancy calculator allows */
+  int32_t algorithm;     /* LAMB_ALGO_*                                     */
+  int32_t l2_budget_mb;  /* single-touch: tensors whose w, m, v take at most
+                            this many MiB keep them in L2 between the
+                            passes; 0 = half the device's L2               */
+  int32_t lag_items;     /* single-touch: work items between a tensor's last
+                            pass-1 item and its pass-2 block; 0 = one item
+                            per resident warp of the grid                  */
 } lamb_plan_options_t;
 
 typedef struct {
@@ -131,6 +154,11 @@ typedef struct {
   int32_t bound;             /* 1 after a successful lamb_plan_bind         */
   int32_t n_vector_tensors;  /* tensors on the vectorised path (after bind) */
   int64_t device_bytes;      /* device memory owned by the plan             */
+  int32_t algorithm;         /* LAMB_ALGO_TWO_PASS or LAMB_ALGO_SINGLE_TOUCH */
+  int32_t n_resident_tensors;/* single-touch: tensors kept in L2            */
+  int64_t n_items;           /* single-touch: work items per step           */
+  int64_t lag_items;         /* single-touch: schedule lag                  */
+  int64_t l2_budget_bytes;   /* single-touch: residency budget              */
 } lamb_plan_info_t;
 
 typedef struct lamb_plan* lamb_plan_t;
@@ -215,8 +243,9 @@ LAMB_API lamb_status_t lamb_plan_get_info(lamb_plan_t plan, lamb_plan_info_t* in
  * stream around every kernel it launches (up to 4096 steps are kept).
  * lamb_plan_read_timing waits for those events, returns the number of steps
  * recorded and the summed device time of each kernel in milliseconds
- * (ms_per_kernel[0..n_kernels-1]; a LAMB or LARS step launches 2 kernels),
- * and clears the record. */
+ * (ms_per_kernel[0..n_kernels-1]; a two-pass step launches 2 kernels, a
+ * single-touch step 1; entries past the step's kernels are 0), and clears
+ * the record. */
 LAMB_API lamb_status_t lamb_plan_set_timing(lamb_plan_t plan, int32_t enable);
 LAMB_API lamb_status_t lamb_plan_read_timing(lamb_plan_t plan, int32_t* n_steps,
                                     double* ms_per_kernel, int32_t n_kernels);
@@ -273,6 +302,21 @@ LAMB_API lamb_status_t lamb_step_noalloc(
     const void* const* g, void* const* m, void* const* v,
     void* const* w_copy, const lamb_hyper_t* hyper, int64_t* d_step,
     const float* d_lr, double* d_ratio, cudaStream_t stream);
+
+/* Host-only planner, no device needed: the work-item order a single-touch
+ * plan would use.  Each item is (fused chunk index << 1) | is_pass2; fused
+ * chunks hold 1024 elements, numbered in tensor order.  l2_budget_bytes and
+ * lag_items as in lamb_plan_options_t (both required, > 0).  Writes up to
+ * `capacity` items, the total into *n_items and, if `resident` is not NULL,
+ * one residency flag per tensor.  INVALID_ARG on bad input or capacity too
+ * small (n_items is still written). */
+LAMB_API lamb_status_t lamb_layout_schedule(const int64_t* sizes,
+                                            int32_t n_tensors,
+                                            int64_t l2_budget_bytes,
+                                            int64_t lag_items,
+                                            uint32_t* items, int64_t capacity,
+                                            int64_t* n_items,
+                                            uint8_t* resident);
 
 /* Message of the last failed call on this host thread ("" if none). */
 LAMB_API const char* lamb_last_error(void);

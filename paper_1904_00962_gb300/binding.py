@@ -45,7 +45,7 @@ EXPORTED = ["lamb_plan_create", "lamb_plan_bind", "lamb_step", "lars_step",
             "lamb_plan_query", "lamb_plan_get_info",
             "lamb_plan_set_timing", "lamb_plan_read_timing",
             "lamb_plan_destroy", "lamb_layout_chunks", "lamb_last_error",
-            "lamb_abi_version", "lamb_step_noalloc"]
+            "lamb_abi_version", "lamb_step_noalloc", "lamb_layout_schedule"]
 
 
 class LambError(RuntimeError):
@@ -65,8 +65,16 @@ class lamb_hyper_t(Structure):
                 ("phi", c_int32), ("flags", c_uint32)]
 
 
+LAMB_ALGO_AUTO = 0
+LAMB_ALGO_TWO_PASS = 1
+LAMB_ALGO_SINGLE_TOUCH = 2
+LAMB_STATUS_WAIT_TIMEOUT = 0x4
+
+
 class lamb_plan_options_t(Structure):
-    _fields_ = [("chunk_elems", c_int32), ("blocks_per_sm", c_int32)]
+    _fields_ = [("chunk_elems", c_int32), ("blocks_per_sm", c_int32),
+                ("algorithm", c_int32), ("l2_budget_mb", c_int32),
+                ("lag_items", c_int32)]
 
 
 class lamb_plan_info_t(Structure):
@@ -76,7 +84,9 @@ class lamb_plan_info_t(Structure):
                 ("num_sms", c_int32), ("device", c_int32),
                 ("grad_dtype", c_int32), ("copy_dtype", c_int32),
                 ("bound", c_int32), ("n_vector_tensors", c_int32),
-                ("device_bytes", c_int64)]
+                ("device_bytes", c_int64), ("algorithm", c_int32),
+                ("n_resident_tensors", c_int32), ("n_items", c_int64),
+                ("lag_items", c_int64), ("l2_budget_bytes", c_int64)]
 
 
 _lib = None
@@ -115,6 +125,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                        POINTER(c_int32), POINTER(c_int64),
                                        POINTER(c_int32), c_int32,
                                        POINTER(c_int32)]
+    lib.lamb_layout_schedule.argtypes = [POINTER(c_int64), c_int32, c_int64,
+                                         c_int64, POINTER(c_uint32), c_int64,
+                                         POINTER(c_int64), POINTER(c_uint8)]
     lib.lamb_step_noalloc.argtypes = [POINTER(c_int64), c_int32,
                                       POINTER(c_uint8), c_int32, c_int32,
                                       POINTER(vp), POINTER(vp), POINTER(vp),
@@ -165,14 +178,17 @@ def make_hyper(*, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01,
 
 def lamb_plan_create(sizes, decay_mask=None, grad_dtype=LAMB_F32,
                      copy_dtype=LAMB_DTYPE_NONE, device=0, chunk_elems=0,
-                     blocks_per_sm=0) -> int:
+                     blocks_per_sm=0, algorithm=LAMB_ALGO_AUTO,
+                     l2_budget_mb=0, lag_items=0) -> int:
     lib = load()
     n = len(sizes)
     sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
     mask = None
     if decay_mask is not None:
         mask = (c_uint8 * max(n, 1))(*[1 if d else 0 for d in decay_mask])
-    opts = lamb_plan_options_t(int(chunk_elems), int(blocks_per_sm))
+    opts = lamb_plan_options_t(int(chunk_elems), int(blocks_per_sm),
+                               int(algorithm), int(l2_budget_mb),
+                               int(lag_items))
     out = c_void_p()
     _check(lib.lamb_plan_create(sz, n, mask, int(grad_dtype), int(copy_dtype),
                                 int(device), byref(opts), byref(out)))
@@ -257,6 +273,25 @@ def lamb_step_noalloc(sizes, decay_mask, grad_dtype, copy_dtype, w, g, m, v,
         _ptr_array(g), _ptr_array(m), _ptr_array(v), _ptr_array(w_copy),
         byref(hyper), c_void_p(d_step or None), c_void_p(d_lr or None),
         c_void_p(d_ratio or None), c_void_p(stream or None)))
+
+
+def lamb_layout_schedule(sizes, l2_budget_bytes, lag_items):
+    """Host-only: (items uint32 array, resident uint8 array) of the
+    single-touch schedule."""
+    lib = load()
+    n = len(sizes)
+    sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
+    count = c_int64()
+    res = np.zeros(max(n, 1), dtype=np.uint8)
+    _check(lib.lamb_layout_schedule(sz, n, int(l2_budget_bytes),
+                                    int(lag_items), None, 0, byref(count),
+                                    res.ctypes.data_as(POINTER(c_uint8))))
+    items = np.zeros(max(count.value, 1), dtype=np.uint32)
+    _check(lib.lamb_layout_schedule(sz, n, int(l2_budget_bytes),
+                                    int(lag_items),
+                                    items.ctypes.data_as(POINTER(c_uint32)),
+                                    count.value, byref(count), None))
+    return items[:count.value], res[:n]
 
 
 def lamb_layout_chunks(sizes, chunk_elems=0):

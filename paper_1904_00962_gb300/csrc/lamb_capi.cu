@@ -75,6 +75,10 @@ struct lamb_plan {
   int num_sms = 0;
   int blocks_per_sm_opt = 0;
   int grid[4] = {0, 0, 0, 0};  // lamb p1, lamb p2, lars p1, lars p2
+  int grid_fused[2] = {0, 0};  // single-touch lamb, lars
+  int algorithm = LAMB_ALGO_TWO_PASS;
+  int64_t n_items = 0, n_groups = 0, lag = 0, l2_budget = 0;
+  int n_resident = 0;
   bool bound = false;
   bool has_v = false;
   int n_vec = 0;
@@ -93,6 +97,15 @@ struct lamb_plan {
   StepScalars* scal = nullptr;
   uint32_t* status = nullptr;
   uint32_t* counters = nullptr;
+  // single-touch tables
+  uint32_t* items = nullptr;
+  FusedChunk* fchunks = nullptr;
+  FusedTensor* ftensors = nullptr;
+  float2* fslots = nullptr;
+  double2* gslots = nullptr;
+  uint32_t* gtickets = nullptr;
+  uint32_t* ftickets = nullptr;
+  uint32_t* ready = nullptr;
 
   bool timing = false;
   int timed_steps = 0;
@@ -138,6 +151,46 @@ lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
   return LAMB_OK;
 }
 
+lamb_status_t lamb_layout_schedule(const int64_t* sizes, int32_t n_tensors,
+                                   int64_t l2_budget_bytes, int64_t lag_items,
+                                   uint32_t* items, int64_t capacity,
+                                   int64_t* n_items, uint8_t* resident) {
+  if (!n_items) return fail(LAMB_ERR_INVALID_ARG, "n_items is NULL");
+  if (n_tensors < 1 || !sizes)
+    return fail(LAMB_ERR_INVALID_ARG, "need n_tensors >= 1 and sizes");
+  if (l2_budget_bytes < 1 || lag_items < 1 || capacity < 0 ||
+      (capacity > 0 && !items))
+    return fail(LAMB_ERR_INVALID_ARG, "bad budget, lag or output buffer");
+  char err[256] = "";
+  int64_t total = 0;
+  for (int32_t k = 0; k < n_tensors; ++k) {
+    if (sizes[k] < 0)
+      return fail(LAMB_ERR_INVALID_ARG, "sizes[%d] is negative", k);
+    if (sizes[k] > (int64_t(1) << 62) - total)
+      return fail(LAMB_ERR_INVALID_ARG, "total element count exceeds 2^62");
+    total += sizes[k];
+  }
+  std::vector<FusedChunk> fc;
+  std::vector<FusedTensor> ft;
+  std::vector<uint32_t> it;
+  int64_t ng = 0;
+  try {
+    if (plan_fused(sizes, n_tensors, nullptr, 12, l2_budget_bytes, lag_items,
+                   &fc, &ft, &it, &ng, err, sizeof(err)))
+      return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  } catch (const std::bad_alloc&) {
+    return fail(LAMB_ERR_OOM, "host allocation failed");
+  }
+  *n_items = (int64_t)it.size();
+  if (resident)
+    for (int32_t k = 0; k < n_tensors; ++k) resident[k] = (uint8_t)ft[k].resident;
+  if ((int64_t)it.size() > capacity)
+    return capacity == 0 ? LAMB_OK
+                         : fail(LAMB_ERR_INVALID_ARG, "capacity too small");
+  std::memcpy(items, it.data(), it.size() * sizeof(uint32_t));
+  return LAMB_OK;
+}
+
 lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
                                const uint8_t* decay_mask, int32_t grad_dtype,
                                int32_t copy_dtype, int32_t device,
@@ -151,13 +204,22 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   if (copy_dtype != LAMB_DTYPE_NONE && copy_dtype != LAMB_BF16)
     return fail(LAMB_ERR_UNSUPPORTED_DTYPE,
                 "copy_dtype %d unsupported (NONE or BF16)", copy_dtype);
-  int chunk = kDefaultChunk, bps = 0;
+  int chunk = kDefaultChunk, bps = 0, algo = LAMB_ALGO_AUTO;
+  int64_t budget_mb = 0, lag_opt = 0;
   if (opts) {
     if (opts->chunk_elems) chunk = opts->chunk_elems;
     if (opts->blocks_per_sm < 0)
       return fail(LAMB_ERR_INVALID_ARG, "blocks_per_sm < 0");
     bps = opts->blocks_per_sm;
+    algo = opts->algorithm;
+    if (algo < LAMB_ALGO_AUTO || algo > LAMB_ALGO_SINGLE_TOUCH)
+      return fail(LAMB_ERR_INVALID_ARG, "unknown algorithm %d", algo);
+    if (opts->l2_budget_mb < 0 || opts->lag_items < 0)
+      return fail(LAMB_ERR_INVALID_ARG, "l2_budget_mb and lag_items >= 0");
+    budget_mb = opts->l2_budget_mb;
+    lag_opt = opts->lag_items;
   }
+  if (algo == LAMB_ALGO_AUTO) algo = LAMB_ALGO_TWO_PASS;
   if (device < 0) return fail(LAMB_ERR_INVALID_ARG, "device < 0");
 
   lamb_plan* p = new (std::nothrow) lamb_plan();
@@ -168,6 +230,7 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   p->grad_bf16 = grad_dtype == LAMB_BF16;
   p->copy_bf16 = copy_dtype == LAMB_BF16;
   p->blocks_per_sm_opt = bps;
+  p->algorithm = algo;
 
   // ---- host planning ----------------------------------------------------
   char err[256] = "";
@@ -222,6 +285,44 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
     if (g < 1) g = 1;
     p->grid[i] = (int)g;
   }
+  // single-touch schedule
+  std::vector<FusedChunk> h_fchunks;
+  std::vector<FusedTensor> h_ftensors;
+  std::vector<uint32_t> h_items;
+  {
+    int focc[2] = {0, 0};
+    rc = occupancy_fused(0, p->grad_bf16, p->copy_bf16, &focc[0]);
+    if (!rc) rc = occupancy_fused(1, p->grad_bf16, p->copy_bf16, &focc[1]);
+    if (rc) {
+      delete p;
+      return cuda_fail((cudaError_t)rc, "occupancy query");
+    }
+    for (int i = 0; i < 2; ++i) {
+      int b = focc[i] < 1 ? 1 : focc[i];
+      if (bps > 0 && bps < b) b = bps;
+      p->grid_fused[i] = p->num_sms * b;
+    }
+    int l2 = 0;
+    e = cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, device);
+    if (e != cudaSuccess) {
+      delete p;
+      return cuda_fail(e, "cudaDeviceGetAttribute(L2)");
+    }
+    p->l2_budget = budget_mb ? budget_mb << 20 : (int64_t)l2 / 2;
+    // one item per warp of the larger grid (8 warps per CTA)
+    p->lag = lag_opt ? lag_opt
+                     : (int64_t)8 * (p->grid_fused[0] > p->grid_fused[1]
+                                         ? p->grid_fused[0]
+                                         : p->grid_fused[1]);
+    if (plan_fused(sizes, n_tensors, decay_mask, 12, p->l2_budget, p->lag,
+                   &h_fchunks, &h_ftensors, &h_items, &p->n_groups, err,
+                   sizeof(err))) {
+      delete p;
+      return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+    }
+    p->n_items = (int64_t)h_items.size();
+    for (const FusedTensor& t : h_ftensors) p->n_resident += t.resident ? 1 : 0;
+  }
 
   const size_t n = (size_t)n_tensors, c = (size_t)nch;
   size_t off = 0;
@@ -240,7 +341,16 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   const size_t o_unorm = carve(n * sizeof(double));
   const size_t o_scal = carve(sizeof(StepScalars));
   const size_t o_status = carve(sizeof(uint32_t));
-  const size_t o_counters = carve(4 * sizeof(uint32_t));
+  const size_t o_counters = carve(8 * sizeof(uint32_t));
+  const size_t nf = h_fchunks.size(), ng = (size_t)p->n_groups;
+  const size_t o_items = carve(h_items.size() * sizeof(uint32_t));
+  const size_t o_fchunks = carve(nf * sizeof(FusedChunk));
+  const size_t o_ftensors = carve(n * sizeof(FusedTensor));
+  const size_t o_fslots = carve(nf * sizeof(float2));
+  const size_t o_gslots = carve(ng * sizeof(double2));
+  const size_t o_gtickets = carve(ng * sizeof(uint32_t));
+  const size_t o_ftickets = carve(n * sizeof(uint32_t));
+  const size_t o_ready = carve(n * sizeof(uint32_t));
   p->arena_bytes = off;
   e = cudaMalloc(&p->arena, p->arena_bytes);
   if (e != cudaSuccess) {
@@ -259,6 +369,14 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   p->scal = reinterpret_cast<StepScalars*>(base + o_scal);
   p->status = reinterpret_cast<uint32_t*>(base + o_status);
   p->counters = reinterpret_cast<uint32_t*>(base + o_counters);
+  p->items = reinterpret_cast<uint32_t*>(base + o_items);
+  p->fchunks = reinterpret_cast<FusedChunk*>(base + o_fchunks);
+  p->ftensors = reinterpret_cast<FusedTensor*>(base + o_ftensors);
+  p->fslots = reinterpret_cast<float2*>(base + o_fslots);
+  p->gslots = reinterpret_cast<double2*>(base + o_gslots);
+  p->gtickets = reinterpret_cast<uint32_t*>(base + o_gtickets);
+  p->ftickets = reinterpret_cast<uint32_t*>(base + o_ftickets);
+  p->ready = reinterpret_cast<uint32_t*>(base + o_ready);
 
   // zero everything (tickets, counters, status, results, pointer table)
   e = cudaMemset(p->arena, 0, p->arena_bytes);
@@ -268,6 +386,19 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   if (e == cudaSuccess)
     e = cudaMemcpy(p->tensors, p->h_tensors.data(), n * sizeof(TensorDesc),
                    cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !h_items.empty())
+    e = cudaMemcpy(p->items, h_items.data(), h_items.size() * sizeof(uint32_t),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && nf)
+    e = cudaMemcpy(p->fchunks, h_fchunks.data(), nf * sizeof(FusedChunk),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(p->ftensors, h_ftensors.data(), n * sizeof(FusedTensor),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) {  // fused launch epoch starts at 1 (ready[] = 0)
+    const uint32_t one = 1u;
+    e = cudaMemcpy(p->counters + 3, &one, sizeof(one), cudaMemcpyHostToDevice);
+  }
   if (e == cudaSuccess) {
     // trust ratio 1 for every tensor until a step computes it (0-element
     // tensors keep it: Q6 zero-norm rule)
@@ -420,6 +551,25 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
   cudaError_t e = cudaSuccess;
   if (timed) e = cudaEventRecord(ev[0], stream);
   int rc = (int)e;
+  if (plan->algorithm == LAMB_ALGO_SINGLE_TOUCH) {
+    FusedParams fp;
+    fp.items = plan->items;
+    fp.fchunks = plan->fchunks;
+    fp.ftensors = plan->ftensors;
+    fp.fslots = plan->fslots;
+    fp.gslots = plan->gslots;
+    fp.gtickets = plan->gtickets;
+    fp.tickets = plan->ftickets;
+    fp.ready = plan->ready;
+    fp.n_items = (int32_t)plan->n_items;
+    if (!rc)
+      rc = launch_fused(sp, fp, lamb ? 0 : 1, plan->grad_bf16, plan->copy_bf16,
+                        plan->grid_fused[lamb ? 0 : 1], stream);
+    if (!rc && timed) rc = (int)cudaEventRecord(ev[1], stream);
+    if (rc) return cuda_fail((cudaError_t)rc, lamb ? "lamb_step" : "lars_step");
+    if (timed) ++plan->timed_steps;
+    return LAMB_OK;
+  }
   if (!rc)
     rc = lamb ? launch_lamb_pass1(sp, plan->grad_bf16, plan->grid[0], stream)
               : launch_lars_pass1(sp, plan->grad_bf16, plan->grid[2], stream);
@@ -506,6 +656,13 @@ lamb_status_t lamb_plan_get_info(lamb_plan_t plan, lamb_plan_info_t* info) {
   info->bound = plan->bound ? 1 : 0;
   info->n_vector_tensors = plan->n_vec;
   info->device_bytes = (int64_t)plan->arena_bytes;
+  info->algorithm = plan->algorithm;
+  info->n_resident_tensors = plan->n_resident;
+  info->n_items = plan->n_items;
+  info->lag_items = plan->lag;
+  info->l2_budget_bytes = plan->l2_budget;
+  if (plan->algorithm == LAMB_ALGO_SINGLE_TOUCH)
+    info->grid_blocks = plan->grid_fused[0];
   return LAMB_OK;
 }
 
@@ -532,11 +689,13 @@ lamb_status_t lamb_plan_read_timing(lamb_plan_t plan, int32_t* n_steps,
   DeviceGuard guard(plan->device);
   if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
   for (int j = 0; j < n_kernels; ++j) ms_per_kernel[j] = 0.0;
+  const int per_step =
+      plan->algorithm == LAMB_ALGO_SINGLE_TOUCH ? 1 : kKernelsPerStep;
   for (int s = 0; s < plan->timed_steps; ++s) {
     cudaEvent_t* ev = &plan->events[(size_t)s * (kKernelsPerStep + 1)];
-    cudaError_t e = cudaEventSynchronize(ev[kKernelsPerStep]);
+    cudaError_t e = cudaEventSynchronize(ev[per_step]);
     if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
-    for (int j = 0; j < kKernelsPerStep && j < n_kernels; ++j) {
+    for (int j = 0; j < per_step && j < n_kernels; ++j) {
       float ms = 0.f;
       e = cudaEventElapsedTime(&ms, ev[j], ev[j + 1]);
       if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");

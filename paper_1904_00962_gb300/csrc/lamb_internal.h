@@ -13,6 +13,8 @@
 #pragma once
 #include <stdint.h>
 
+#include <vector>
+
 namespace lamb {
 
 constexpr int kDefaultChunk = 16384;
@@ -55,7 +57,8 @@ struct __align__(16) StepScalars {
   int32_t pad[2];
 };
 
-enum : uint32_t { kStatusNonfinite = 1u, kStatusBadStep = 2u };
+enum : uint32_t { kStatusNonfinite = 1u, kStatusBadStep = 2u,
+                  kStatusWaitTimeout = 4u };
 enum : uint32_t { kFlagBiasCorrection = 1u, kFlagIncrementStep = 2u };
 
 struct StepParams {
@@ -64,7 +67,9 @@ struct StepParams {
   const TensorPtrs* ptrs;
   float2* slots;
   uint32_t* tickets;
-  uint32_t* counters;     // [0] pass-1 work counter, [1] pass-2 work counter
+  uint32_t* counters;     // [0] pass-1, [1] pass-2, [2] fused work counter,
+                          // [3] launch epoch of the fused kernel (>= 1),
+                          // [4] epoch of a fused launch whose wait gave up
   double* ratio;
   double* wnorm;
   double* unorm;
@@ -81,6 +86,44 @@ struct StepParams {
   int32_t n_chunks;
 };
 
+// ---------------------------------------------------------------------------
+// Single-touch (fused) step: one persistent kernel whose warps draw items --
+// the pass-1 or pass-2 work on one "fused chunk" of kFusedChunk elements --
+// from a host-built schedule in which the pass-2 items of a tensor follow its
+// pass-1 items by a lag of about one wave, so the m, v, w the pass 1 just
+// touched are still in L2 when the pass 2 reads them.
+// ---------------------------------------------------------------------------
+constexpr int kFusedChunk = 1024;     // elements per fused chunk (one warp item)
+constexpr int kGroup = 32;            // fused chunks per first-level combine
+
+struct __align__(8) FusedChunk {
+  int32_t tensor;   // tensor index k
+  int32_t index;    // chunk index inside the tensor (offset = index*kFusedChunk)
+};
+
+struct __align__(16) FusedTensor {
+  int64_t numel;
+  int32_t first_chunk;   // in the fused chunk table
+  int32_t n_chunks;
+  int32_t first_group;   // in the group tables
+  int32_t n_groups;
+  float decay;           // 1.0f: weight decay applies
+  uint32_t resident;     // 1: keep pass-1 data in L2 (evict_last) for pass 2
+};
+
+struct FusedParams {
+  const uint32_t* items;       // (fused chunk << 1) | is_pass2
+  const FusedChunk* fchunks;
+  const FusedTensor* ftensors;
+  float2* fslots;              // per fused chunk (sum w^2, sum u^2), fp32
+  double2* gslots;             // per group, fp64
+  uint32_t* gtickets;          // per group: chunks of the group finished
+  uint32_t* tickets;           // per tensor: groups finished
+  uint32_t* ready;             // per tensor: epoch of the launch that
+                               // finished its norms
+  int32_t n_items;
+};
+
 // Launchers (lamb_kernels.cu).  grid = number of CTAs of the persistent grid.
 // Return cudaError_t as int to keep this header free of CUDA includes.
 int launch_lamb_pass1(const StepParams& p, int grad_bf16, int grid,
@@ -91,6 +134,9 @@ int launch_lars_pass1(const StepParams& p, int grad_bf16, int grid,
                       void* stream);
 int launch_lars_pass2(const StepParams& p, int copy_bf16, int grid,
                       void* stream);
+int launch_fused(const StepParams& p, const FusedParams& f, int lars,
+                 int grad_bf16, int copy_bf16, int grid, void* stream);
+int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks);
 // Resident CTAs per SM of each kernel instantiation (occupancy calculator).
 int occupancy_lamb_pass1(int grad_bf16, int* blocks);
 int occupancy_lamb_pass2(int copy_bf16, int* blocks);
@@ -99,6 +145,15 @@ int occupancy_lars_pass2(int copy_bf16, int* blocks);
 
 // Sets the thread-local message returned by lamb_last_error() (lamb_capi.cu).
 void set_last_error(const char* msg);
+
+// Schedule of the single-touch step (planner.cpp): fused chunk table, tensor
+// table (with the L2-residency flag) and the ordered work items.
+int plan_fused(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
+               int64_t bytes_per_param, int64_t l2_budget, int64_t lag,
+               std::vector<FusedChunk>* fchunks,
+               std::vector<FusedTensor>* ftensors,
+               std::vector<uint32_t>* items, int64_t* n_groups, char* err,
+               int errlen);
 
 // Host planner (planner.cpp).  Returns 0 on success, else writes a message.
 int plan_chunks(const int64_t* sizes, int32_t n, int32_t chunk_elems,

@@ -563,6 +563,393 @@ __global__ void __launch_bounds__(kThreads)
     *p.d_step = sc.t + 1;
 }
 
+// ---------------------------------------------------------------------------
+// Single-touch fused step (one persistent kernel, warps are the workers)
+//
+// Items are drawn in schedule order from counters[2].  A pass-1 item streams
+// one fused chunk (1024 elements) through Alg. 2's moment and ratio lines,
+// stores the new m, v and publishes the chunk's sums; the warp that completes
+// a group of 32 chunks sums them (fp64, fixed order), and the warp that
+// completes a tensor's last group computes its norms and trust ratio and
+// releases ready[k] = epoch.  A pass-2 item waits (bounded) for ready[k] ==
+// epoch and applies the update.  Pass-2 items of a tensor come after all its
+// pass-1 items in the schedule and items are drawn in order, so the earliest
+// unfinished item never waits on anything unfinished: the kernel cannot
+// deadlock.  The wait still gives up after ~0.5 s, sets a status bit and
+// makes every other waiter of the same launch give up at once.
+//
+// L2 policy: pass-1 loads/stores of m, v, w of "resident" tensors (those
+// whose state fits the L2 budget) are evict_last, so pass 2 -- about one
+// wave later -- finds them in L2; gradients and all pass-2 traffic are
+// evict_first.
+// ---------------------------------------------------------------------------
+constexpr int kFusedThreads = 256;                     // 8 warps per CTA
+// 4-element packets per lane per batch: LARS keeps 4 in flight; LAMB keeps 2
+// (its longer arithmetic needs the registers) and runs twice the batches.
+template <bool kLars> __host__ __device__ constexpr int fused_unroll() {
+  return kLars ? 4 : 2;
+}
+template <bool kLars> __host__ __device__ constexpr int fused_batches() {
+  return kFusedChunk / (32 * 4 * fused_unroll<kLars>());
+}
+static_assert(fused_batches<true>() * 32 * 4 * 4 == kFusedChunk, "shape");
+static_assert(fused_batches<false>() * 32 * 4 * 2 == kFusedChunk, "shape");
+constexpr uint32_t kSpinLimit = 1u << 21;              // x <= 256 ns ~ 0.5 s
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ float4 ldp4(const float* p, uint64_t pol) {
+  float4 r;
+  asm volatile(
+      "ld.global.L1::no_allocate.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %5;"
+      : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
+      : "l"(p), "l"(pol));
+  return r;
+}
+__device__ __forceinline__ void stp4(float* p, float4 v, uint64_t pol) {
+  asm volatile(
+      "st.global.L1::no_allocate.L2::cache_hint.v4.f32 [%0], {%1,%2,%3,%4}, %5;"
+      ::"l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "l"(pol)
+      : "memory");
+}
+__device__ __forceinline__ float4 ldp_grad4(const float* p, uint64_t pol) {
+  return ldp4(p, pol);
+}
+__device__ __forceinline__ float4 ldp_grad4(const __nv_bfloat16* p,
+                                            uint64_t pol) {
+  uint32_t a, b;
+  asm volatile(
+      "ld.global.L1::no_allocate.L2::cache_hint.v2.u32 {%0,%1}, [%2], %3;"
+      : "=r"(a), "=r"(b)
+      : "l"(p), "l"(pol));
+  return make_float4(__uint_as_float(a << 16), __uint_as_float(a & 0xffff0000u),
+                     __uint_as_float(b << 16), __uint_as_float(b & 0xffff0000u));
+}
+__device__ __forceinline__ void stp_copy4(void* base, int64_t i, float4 x,
+                                          uint64_t pol) {
+  const __nv_bfloat162 lo = __floats2bfloat162_rn(x.x, x.y);
+  const __nv_bfloat162 hi = __floats2bfloat162_rn(x.z, x.w);
+  const uint32_t a = *reinterpret_cast<const uint32_t*>(&lo);
+  const uint32_t b = *reinterpret_cast<const uint32_t*>(&hi);
+  asm volatile(
+      "st.global.L1::no_allocate.L2::cache_hint.v2.u32 [%0], {%1,%2}, %3;"
+      ::"l"(static_cast<__nv_bfloat16*>(base) + i), "r"(a), "r"(b), "l"(pol)
+      : "memory");
+}
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v)
+               : "memory");
+}
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;"
+               : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+__device__ __forceinline__ double warp_sum_d(double x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_down_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// Element of the fused pass 1: LAMB (Alg. 2) or LARS (Alg. 1) moment update,
+// then the direction u whose norm the trust ratio needs.
+template <bool kLars>
+__device__ __forceinline__ void fused1_elem(float g, float& m, float& v,
+                                            float w, float lam,
+                                            const LambConsts& k, float& sw,
+                                            float& su) {
+  float u;
+  if (kLars) {
+    m = lars_momentum(g, m, w, lam, k.b1, k.omb1);
+    u = m;
+  } else {
+    lamb_moments(g, m, v, k);
+    u = lamb_direction(m, v, w, lam, k);
+  }
+  sw = __fmaf_rn(w, w, sw);
+  su = __fmaf_rn(u, u, su);
+}
+
+template <bool kLars>
+__device__ __forceinline__ float fused2_dir(float m, float v, float w,
+                                            float lam, const LambConsts& k) {
+  return kLars ? m : lamb_direction(m, v, w, lam, k);
+}
+
+// Warp-level pass 1 of one fused chunk; publishes its sums and, if it is the
+// last chunk of its group / tensor, performs the combine.
+template <bool kLars, typename GT>
+__device__ __forceinline__ void fused_pass1(
+    const StepParams& p, const FusedParams& f, const LambConsts& k,
+    const TensorPtrs& tp, const FusedTensor& ft, const FusedChunk& fc,
+    int chunk, int64_t off, int len, float lam, uint64_t pol_first,
+    uint64_t pol_keep, uint32_t epoch, int lane) {
+  float* __restrict__ w = tp.w + off;
+  float* __restrict__ m = tp.m + off;
+  float* __restrict__ v = kLars ? nullptr : tp.v + off;
+  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + off;
+  constexpr int kFU = fused_unroll<kLars>();
+  float sw = 0.f, su = 0.f;
+  int scalar_from = 0;
+  if (tp.vec_ok) {
+    const int nv = len >> 2;
+#pragma unroll 1
+    for (int b = 0; b < fused_batches<kLars>(); ++b) {
+      const int base = b * 32 * kFU + lane;
+      float4 wv[kFU], mv[kFU], vv[kFU], gv[kFU];
+#pragma unroll
+      for (int u = 0; u < kFU; ++u) {
+        const int j = base + u * 32;
+        if (j < nv) {
+          gv[u] = ldp_grad4(g + 4 * j, pol_first);
+          mv[u] = ldp4(m + 4 * j, pol_keep);
+          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_keep);
+          wv[u] = ldp4(w + 4 * j, pol_keep);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kFU; ++u) {
+        const int j = base + u * 32;
+        if (j < nv) {
+          float4& mm = mv[u];
+          float4& vvv = vv[u];
+          fused1_elem<kLars>(gv[u].x, mm.x, vvv.x, wv[u].x, lam, k, sw, su);
+          fused1_elem<kLars>(gv[u].y, mm.y, vvv.y, wv[u].y, lam, k, sw, su);
+          fused1_elem<kLars>(gv[u].z, mm.z, vvv.z, wv[u].z, lam, k, sw, su);
+          fused1_elem<kLars>(gv[u].w, mm.w, vvv.w, wv[u].w, lam, k, sw, su);
+          stp4(m + 4 * j, mm, pol_keep);
+          if (!kLars) stp4(v + 4 * j, vvv, pol_keep);
+        }
+      }
+    }
+    scalar_from = nv << 2;
+  }
+  for (int i = scalar_from + lane; i < len; i += 32) {
+    float mi = m[i];
+    float vi = kLars ? 0.f : v[i];
+    fused1_elem<kLars>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
+    m[i] = mi;
+    if (!kLars) v[i] = vi;
+  }
+  sw = warp_sum(sw);
+  su = warp_sum(su);
+  __syncwarp();
+  const int gl = fc.index / kGroup;
+  const int group = ft.first_group + gl;
+  const int gsize = min(kGroup, ft.n_chunks - gl * kGroup);
+  uint32_t last = 0;
+  if (lane == 0) {
+    f.fslots[chunk] = make_float2(sw, su);
+    // release: this warp's m, v stores and the slot become visible first
+    last = atom_add_acq_rel(&f.gtickets[group], 1u) + 1u == (uint32_t)gsize;
+  }
+  if (!__shfl_sync(0xffffffffu, last, 0)) return;
+  __syncwarp();
+  // first level: the group's chunk sums, fp64, fixed order
+  double aw = 0.0, au = 0.0;
+  if (lane < gsize) {
+    const float2 s = __ldcg(&f.fslots[ft.first_chunk + gl * kGroup + lane]);
+    aw = (double)s.x;
+    au = (double)s.y;
+  }
+  aw = warp_sum_d(aw);
+  au = warp_sum_d(au);
+  if (lane == 0) {
+    f.gslots[group] = make_double2(aw, au);
+    f.gtickets[group] = 0u;
+    last = atom_add_acq_rel(&f.tickets[fc.tensor], 1u) + 1u ==
+           (uint32_t)ft.n_groups;
+  }
+  if (!__shfl_sync(0xffffffffu, last, 0)) return;
+  __syncwarp();
+  // second level: the tensor's group sums -> norms and trust ratio
+  double tw = 0.0, tu = 0.0;
+  for (int i = lane; i < ft.n_groups; i += 32) {
+    const double2 s = __ldcg(&f.gslots[ft.first_group + i]);
+    tw += s.x;
+    tu += s.y;
+  }
+  tw = warp_sum_d(tw);
+  tu = warp_sum_d(tu);
+  if (lane == 0) {
+    const double wn = sqrt(tw), un = sqrt(tu);
+    double rho = 1.0;
+    if (!(wn == 0.0 || un == 0.0))
+      rho = (kLars ? p.trust : 1.0) * phi_of(wn, p) / un;
+    p.ratio[fc.tensor] = rho;
+    p.wnorm[fc.tensor] = wn;
+    p.unorm[fc.tensor] = un;
+    if (!isfinite(tw) || !isfinite(tu)) atomicOr(p.status, kStatusNonfinite);
+    f.tickets[fc.tensor] = 0u;
+    st_release(&f.ready[fc.tensor], epoch);
+  }
+}
+
+// Warp-level pass 2 of one fused chunk.
+template <bool kLars, bool kCopy>
+__device__ __forceinline__ void fused_pass2(
+    const StepParams& p, const FusedParams& f, const LambConsts& k,
+    const TensorPtrs& tp, int tensor, int64_t off, int len, float lam,
+    float lr, uint64_t pol_first, uint32_t epoch, int lane) {
+  uint32_t ok = 1;
+  if (lane == 0) {
+    uint32_t spins = 0, ns = 32;
+    while (ld_acquire(&f.ready[tensor]) != epoch) {
+      // give up after ~0.5 s, or at once if another warp of this launch
+      // already gave up (counters[4] holds the epoch of an aborted launch)
+      if (++spins > kSpinLimit ||
+          *reinterpret_cast<volatile uint32_t*>(&p.counters[4]) == epoch) {
+        ok = 0;
+        atomicOr(p.status, kStatusWaitTimeout);
+        atomicExch(&p.counters[4], epoch);
+        break;
+      }
+      __nanosleep(ns);
+      if (ns < 256) ns <<= 1;
+    }
+  }
+  if (!__shfl_sync(0xffffffffu, ok, 0)) return;   // gave up: leave w as is
+  __syncwarp();
+  (void)ld_acquire(&f.ready[tensor]);               // per-lane acquire
+  const float s = __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]));
+  float* __restrict__ w = tp.w + off;
+  const float* __restrict__ m = tp.m + off;
+  const float* __restrict__ v = kLars ? nullptr : tp.v + off;
+  constexpr int kFU = fused_unroll<kLars>();
+  int scalar_from = 0;
+  if (tp.vec_ok) {
+    const int nv = len >> 2;
+#pragma unroll 1
+    for (int b = 0; b < fused_batches<kLars>(); ++b) {
+      const int base = b * 32 * kFU + lane;
+      float4 wv[kFU], mv[kFU], vv[kFU];
+#pragma unroll
+      for (int u = 0; u < kFU; ++u) {
+        const int j = base + u * 32;
+        if (j < nv) {
+          mv[u] = ldp4(m + 4 * j, pol_first);
+          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_first);
+          wv[u] = ldp4(w + 4 * j, pol_first);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kFU; ++u) {
+        const int j = base + u * 32;
+        if (j < nv) {
+          float4 o;
+          o.x = __fmaf_rn(-s, fused2_dir<kLars>(mv[u].x, vv[u].x, wv[u].x, lam, k), wv[u].x);
+          o.y = __fmaf_rn(-s, fused2_dir<kLars>(mv[u].y, vv[u].y, wv[u].y, lam, k), wv[u].y);
+          o.z = __fmaf_rn(-s, fused2_dir<kLars>(mv[u].z, vv[u].z, wv[u].z, lam, k), wv[u].z);
+          o.w = __fmaf_rn(-s, fused2_dir<kLars>(mv[u].w, vv[u].w, wv[u].w, lam, k), wv[u].w);
+          stp4(w + 4 * j, o, pol_first);
+          if (kCopy) stp_copy4(tp.copy, off + 4 * j, o, pol_first);
+        }
+      }
+    }
+    scalar_from = nv << 2;
+  }
+  for (int i = scalar_from + lane; i < len; i += 32) {
+    const float wi = w[i];
+    const float o = __fmaf_rn(
+        -s, fused2_dir<kLars>(m[i], kLars ? 0.f : v[i], wi, lam, k), wi);
+    w[i] = o;
+    if (kCopy) st_copy1(tp.copy, off + i, o);
+  }
+}
+
+template <bool kLars, typename GT, bool kCopy>
+__global__ void __launch_bounds__(kFusedThreads, 2)
+    fused_step_kernel(const StepParams p, const FusedParams f) {
+  __shared__ LambConsts s_k;
+  __shared__ float s_lr;
+  __shared__ int s_skip;
+  __shared__ uint32_t s_epoch;
+  __shared__ int64_t s_t;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    const bool bc = !kLars && (p.flags & kFlagBiasCorrection) != 0;
+    const int64_t t = p.d_step ? *p.d_step : int64_t(1);
+    const int skip = (bc && t < 1) ? 1 : 0;
+    float c1 = 1.f, c2 = 1.f;
+    if (bc && !skip) {  // Alg. 2 bias correction, beta^t in fp64
+      c1 = (float)(1.0 / (1.0 - pow(p.beta1, (double)t)));
+      c2 = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
+    }
+    s_k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps};
+    s_lr = *p.d_lr;
+    s_skip = skip;
+    s_t = t;
+    s_epoch = *reinterpret_cast<volatile uint32_t*>(&p.counters[3]);
+    if (blockIdx.x == 0) {
+      StepScalars sc{};
+      sc.t = t;
+      sc.c1 = c1;
+      sc.c2 = c2;
+      sc.lr = s_lr;
+      sc.skip = skip;
+      *p.scal = sc;
+      if (skip) atomicOr(p.status, kStatusBadStep);
+    }
+  }
+  __syncthreads();
+  if (s_skip) return;
+  const LambConsts k = s_k;
+  const float lr = s_lr;
+  const uint32_t epoch = s_epoch;
+  const uint64_t pol_first = policy_evict_first();
+  const uint64_t pol_last = policy_evict_last();
+  const uint32_t n_items = (uint32_t)f.n_items;
+  uint32_t next = 0;
+  if (lane == 0) next = atomicAdd(&p.counters[2], 1u);
+  next = __shfl_sync(0xffffffffu, next, 0);
+  while (next < n_items) {
+    const uint32_t item = next;
+    uint32_t pre = 0;
+    if (lane == 0) pre = atomicAdd(&p.counters[2], 1u);  // draw ahead
+    const uint32_t code = __ldg(&f.items[item]);
+    const int chunk = (int)(code >> 1);
+    const FusedChunk fc = f.fchunks[chunk];
+    const FusedTensor ft = f.ftensors[fc.tensor];
+    const TensorPtrs tp = p.ptrs[fc.tensor];
+    const int64_t off = (int64_t)fc.index * kFusedChunk;
+    const int64_t rem = ft.numel - off;
+    const int len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
+    const float lam = ft.decay * p.wd;
+    if ((code & 1u) == 0u)
+      fused_pass1<kLars, GT>(p, f, k, tp, ft, fc, chunk, off, len, lam,
+                             pol_first, ft.resident ? pol_last : pol_first,
+                             epoch, lane);
+    else
+      fused_pass2<kLars, kCopy>(p, f, k, tp, fc.tensor, off, len, lam, lr,
+                                pol_first, epoch, lane);
+    next = __shfl_sync(0xffffffffu, pre, 0);
+  }
+  // Every warp draws exactly one index >= n_items; the warp that draws the
+  // last of them is the last to draw and closes the launch.
+  const uint32_t warps = gridDim.x * (kFusedThreads / 32);
+  if (lane == 0 && next == n_items + warps - 1u) {
+    atomicExch(&p.counters[2], 0u);
+    const uint32_t ne = epoch + 1u == 0u ? 1u : epoch + 1u;
+    atomicExch(&p.counters[3], ne);
+    if ((p.flags & kFlagIncrementStep) && p.d_step) *p.d_step = s_t + 1;
+  }
+}
+
 template <typename K>
 int occupancy_of(K kernel, int* blocks) {
   return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, kernel,
@@ -609,6 +996,41 @@ int launch_lars_pass2(const StepParams& p, int copy_bf16, int grid,
   else
     lars_pass2_kernel<false><<<grid, kThreads, 0, s>>>(p);
   return (int)cudaGetLastError();
+}
+
+int launch_fused(const StepParams& p, const FusedParams& f, int lars,
+                 int grad_bf16, int copy_bf16, int grid, void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int sel = (lars ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0);
+  switch (sel) {
+    case 0: fused_step_kernel<false, float, false><<<grid, kFusedThreads, 0, s>>>(p, f); break;
+    case 1: fused_step_kernel<false, float, true><<<grid, kFusedThreads, 0, s>>>(p, f); break;
+    case 2: fused_step_kernel<false, __nv_bfloat16, false><<<grid, kFusedThreads, 0, s>>>(p, f); break;
+    case 3: fused_step_kernel<false, __nv_bfloat16, true><<<grid, kFusedThreads, 0, s>>>(p, f); break;
+    case 4: fused_step_kernel<true, float, false><<<grid, kFusedThreads, 0, s>>>(p, f); break;
+    case 5: fused_step_kernel<true, float, true><<<grid, kFusedThreads, 0, s>>>(p, f); break;
+    case 6: fused_step_kernel<true, __nv_bfloat16, false><<<grid, kFusedThreads, 0, s>>>(p, f); break;
+    default: fused_step_kernel<true, __nv_bfloat16, true><<<grid, kFusedThreads, 0, s>>>(p, f); break;
+  }
+  return (int)cudaGetLastError();
+}
+
+int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks) {
+  const int sel = (lars ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0);
+  auto q = [&](auto kern) {
+    return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        blocks, kern, kFusedThreads, 0);
+  };
+  switch (sel) {
+    case 0: return q(fused_step_kernel<false, float, false>);
+    case 1: return q(fused_step_kernel<false, float, true>);
+    case 2: return q(fused_step_kernel<false, __nv_bfloat16, false>);
+    case 3: return q(fused_step_kernel<false, __nv_bfloat16, true>);
+    case 4: return q(fused_step_kernel<true, float, false>);
+    case 5: return q(fused_step_kernel<true, float, true>);
+    case 6: return q(fused_step_kernel<true, __nv_bfloat16, false>);
+    default: return q(fused_step_kernel<true, __nv_bfloat16, true>);
+  }
 }
 
 int occupancy_lamb_pass1(int grad_bf16, int* blocks) {

@@ -86,13 +86,14 @@ class LambPlan:
     """A C-library plan bound to a DeviceState."""
 
     def __init__(self, state: DeviceState, decay_mask=None, *, device=None,
-                 chunk_elems=0, blocks_per_sm=0):
+                 chunk_elems=0, blocks_per_sm=0, algorithm=0, l2_budget_mb=0,
+                 lag_items=0):
         self.state = state
         dev = state.device.index if device is None else device
         self.handle = B.lamb_plan_create(
             state.sizes, decay_mask, _dtype_code(state.grad_dtype),
             _dtype_code(state.copy_dtype), dev or 0, chunk_elems,
-            blocks_per_sm)
+            blocks_per_sm, algorithm, l2_budget_mb, lag_items)
         self.n = len(state.sizes)
         self.bind()
 

@@ -7,7 +7,8 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_util import (TOL_CHAIN, TOL_RATIO, TOL_STEP, GpuLayout, c_hyper,
+from gpu_util import (ALGO_IDS, ALGOS, TOL_CHAIN, TOL_RATIO, TOL_STEP,
+                      GpuLayout, c_hyper,
                       check_copy, compare_lamb, compare_lars, f32,
                       hyper_kwargs, oracle_map, ratio_ok, worst_of)
 from oracle import lamb_oracle as O
@@ -17,6 +18,8 @@ from paper_1904_00962_gb300 import workloads as W
 from paper_1904_00962_gb300.state import DeviceState, LambPlan
 
 pytestmark = pytest.mark.gpu
+
+algos = pytest.mark.parametrize("algo", ALGOS, ids=lambda a: ALGO_IDS[a])
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -43,11 +46,12 @@ def _oracle_lars(L, k, w, g, m, lr, h):
 
 @pytest.mark.parametrize("n_steps", [10, 100])
 @pytest.mark.parametrize("bias_correction", [True, False])
-def test_mlp_chained_lamb(n_steps, bias_correction):
+@algos
+def test_mlp_chained_lamb(n_steps, bias_correction, algo):
     L = W.mlp_layout()
     h = L.hyper
     h.bias_correction = bias_correction
-    G = GpuLayout(L)
+    G = GpuLayout(L, algorithm=algo)
     G.load_weights()
     lr = f32(h.lr)
     state = [(L.weights(k).astype(np.float64), np.zeros(L.sizes[k]),
@@ -80,11 +84,12 @@ def test_mlp_chained_lamb(n_steps, bias_correction):
     print(f"mlp {n_steps} steps worst scaled err {worst:.3e}")
 
 
-def test_mlp_chained_lars_100():
+@algos
+def test_mlp_chained_lars_100(algo):
     L = W.mlp_layout()
     h = W.Hyper(lr=1.0, beta1=0.9, weight_decay=1e-4, trust_coef=1e-3,
                 phi="identity", bias_correction=False)
-    G = GpuLayout(L, with_v=False)
+    G = GpuLayout(L, with_v=False, algorithm=algo)
     G.load_weights()
     lr = f32(h.lr)
     state = [(L.weights(k).astype(np.float64), np.zeros(L.sizes[k]))
@@ -122,11 +127,12 @@ def test_mlp_chained_lars_100():
                                        ("bert_large", False),
                                        ("resnet50", False),
                                        ("resnet50", True)])
-def test_full_layout_one_step_every_tensor(name, lars):
+@algos
+def test_full_layout_one_step_every_tensor(name, lars, algo):
     L = W.get_layout(name)
     h = L.lars_hyper if lars else L.hyper
     t = h.measured_step or (h.warm_steps + 1)
-    G = GpuLayout(L, with_v=not lars)
+    G = GpuLayout(L, with_v=not lars, algorithm=algo)
     G.load_weights()
     G.load_warm_state()
     G.load_grads(t)
@@ -178,12 +184,13 @@ def _sample(L, big=6):
                                        ("bert_large", False),
                                        ("resnet50", False),
                                        ("resnet50", True)])
-def test_full_layout_warm_trajectory(name, lars):
+@algos
+def test_full_layout_warm_trajectory(name, lars, algo):
     L = W.get_layout(name)
     h = L.lars_hyper if lars else L.hyper
     ts = list(range(1, h.warm_steps + 1)) + [h.measured_step or
                                                h.warm_steps + 1]
-    G = GpuLayout(L, with_v=not lars)
+    G = GpuLayout(L, with_v=not lars, algorithm=algo)
     G.load_weights()
     lr = f32(h.lr)
     ks = _sample(L)
@@ -236,10 +243,11 @@ def test_full_layout_warm_trajectory(name, lars):
 # Ragged stress layout at full size (10,000 tensors, ~2.7e9 parameters)
 # ---------------------------------------------------------------------------
 
-def test_ragged_full_size():
+@algos
+def test_ragged_full_size(algo):
     L = W.ragged_layout()
     h = L.hyper
-    G = GpuLayout(L)
+    G = GpuLayout(L, algorithm=algo)
     st = G.st
     gen = torch.Generator(device="cuda:0")
     gen.manual_seed(20200101)
@@ -360,13 +368,14 @@ def test_edge_layout(grad_dtype, copy_dtype, chunk, bps, misalign):
 @pytest.mark.parametrize("phi,gl,gu", [("identity", 0.0, math.inf),
                                        ("clip", 0.5, 0.6),
                                        ("clip", 0.0, 1e-3)])
-def test_edge_layout_phi_and_lars(phi, gl, gu):
+@algos
+def test_edge_layout_phi_and_lars(phi, gl, gu, algo):
     L = _edge_layout()
     for lars in (False, True):
         h = W.Hyper(lr=0.5 if lars else 2e-3, phi=phi, gamma_l=gl, gamma_u=gu,
                     trust_coef=1e-3 if lars else 1.0, weight_decay=0.01,
                     bias_correction=not lars)
-        G = GpuLayout(L, with_v=not lars)
+        G = GpuLayout(L, with_v=not lars, algorithm=algo)
         G.load_weights()
         G.load_warm_state()
         G.load_grads(3)
@@ -430,7 +439,8 @@ def test_bitwise_deterministic_across_runs_and_grids(lars):
 # CUDA graph capture: replays read eta and t from device memory
 # ---------------------------------------------------------------------------
 
-def test_graph_replay_equals_eager():
+@algos
+def test_graph_replay_equals_eager(algo):
     L = W.bert_layout(2, 128, 512, vocab=1000, positions=64, name="tinybert",
                       grad_dtype="bf16", copy_dtype="bf16")
     h = L.hyper
@@ -438,7 +448,7 @@ def test_graph_replay_equals_eager():
     hyp = c_hyper(h, increment=True)
 
     def fresh():
-        G = GpuLayout(L)
+        G = GpuLayout(L, algorithm=algo)
         G.load_weights()
         G.d_step.fill_(1)
         return G
@@ -477,7 +487,8 @@ def test_graph_replay_equals_eager():
 # Checkpoint / resume: state is caller-owned, the plan is stateless
 # ---------------------------------------------------------------------------
 
-def test_split_run_resume_is_bitwise_equal():
+@algos
+def test_split_run_resume_is_bitwise_equal(algo):
     L = W.bert_layout(1, 64, 256, vocab=500, positions=32, name="resume")
     h = L.hyper
     hyp = c_hyper(h, increment=True)
@@ -488,17 +499,17 @@ def test_split_run_resume_is_bitwise_equal():
             G.d_lr.fill_(f32(h.lr))
             G.plan.lamb_step(hyp, G.d_step, G.d_lr)
 
-    full = GpuLayout(L)
+    full = GpuLayout(L, algorithm=algo)
     full.load_weights()
     run(full, range(1, 13))
-    a = GpuLayout(L)
+    a = GpuLayout(L, algorithm=algo)
     a.load_weights()
     run(a, range(1, 7))
     torch.cuda.synchronize()
     ckpt = {n: getattr(a.st, n).cpu() for n in ("w", "m", "v")}
     step = a.d_step.cpu()
     a.close()
-    b = GpuLayout(L)
+    b = GpuLayout(L, algorithm=algo)
     for n, t in ckpt.items():
         getattr(b.st, n).copy_(t)
     b.d_step.copy_(step)
@@ -515,9 +526,10 @@ def test_split_run_resume_is_bitwise_equal():
 # Device-side status and argument handling
 # ---------------------------------------------------------------------------
 
-def test_bad_step_count_skips_step_and_sets_status():
+@algos
+def test_bad_step_count_skips_step_and_sets_status(algo):
     L = W.mlp_layout()
-    G = GpuLayout(L)
+    G = GpuLayout(L, algorithm=algo)
     G.load_weights()
     G.load_grads(1)
     before = _snapshot(G)[:3]
@@ -545,9 +557,10 @@ def test_bad_step_count_skips_step_and_sets_status():
     G.close()
 
 
-def test_nonfinite_gradient_propagates_and_is_flagged():
+@algos
+def test_nonfinite_gradient_propagates_and_is_flagged(algo):
     L = _edge_layout()
-    G = GpuLayout(L)
+    G = GpuLayout(L, algorithm=algo)
     G.load_weights()
     G.load_grads(1)
     bad = 9
@@ -572,10 +585,11 @@ def test_nonfinite_gradient_propagates_and_is_flagged():
     G.close()
 
 
-def test_increment_step_matches_oracle_chain():
+@algos
+def test_increment_step_matches_oracle_chain(algo):
     L = W.mlp_layout()
     h = L.hyper
-    G = GpuLayout(L)
+    G = GpuLayout(L, algorithm=algo)
     G.load_weights()
     G.d_step.fill_(1)
     G.d_lr.fill_(f32(h.lr))
@@ -659,14 +673,104 @@ def test_non_default_stream_and_rebind():
     A.close()
 
 
-def test_timing_hook_records_both_kernels():
+@algos
+def test_timing_hook_records_both_kernels(algo):
     L = W.resnet50_layout()
-    G = GpuLayout(L)
+    G = GpuLayout(L, algorithm=algo)
     G.load_weights(); G.load_grads(1)
     B.lamb_plan_set_timing(G.plan.handle, True)
     for t in range(1, 4):
         G.step(t, f32(1e-3), c_hyper(L.hyper))
     n, ms = B.lamb_plan_read_timing(G.plan.handle, 2)
-    assert n == 3 and all(x > 0 for x in ms)
+    assert n == 3 and ms[0] > 0
+    assert (ms[1] > 0) if algo == 1 else (ms[1] == 0)
+    assert G.plan.info()["algorithm"] == algo
     B.lamb_plan_set_timing(G.plan.handle, False)
     G.close()
+
+
+# ---------------------------------------------------------------------------
+# Single-touch specifics: edge layouts, schedule knobs, determinism
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("grad_dtype,copy_dtype", [("f32", None),
+                                                    ("bf16", "bf16")])
+@pytest.mark.parametrize("misalign", [False, True])
+@pytest.mark.parametrize("budget_mb,lag", [(0, 0), (1, 1), (1024, 100000)])
+def test_single_touch_edge_layout(grad_dtype, copy_dtype, misalign, budget_mb,
+                                  lag):
+    L = _edge_layout(grad_dtype, copy_dtype)
+    h = L.hyper
+    G = GpuLayout(L, algorithm=2, l2_budget_mb=budget_mb, lag_items=lag,
+                  misalign={5, 9, 12, 16} if misalign else None)
+    info = G.plan.info()
+    assert info["algorithm"] == 2
+    if budget_mb == 1:        # 1 MiB: only tensors of <= 87381 elements
+        assert info["n_resident_tensors"] == sum(
+            1 for s in L.sizes if s * 12 <= (1 << 20))
+    G.load_weights()
+    G.load_warm_state()
+    G.load_grads(2)
+    lr = f32(h.lr)
+    G.step(2, lr, c_hyper(h))
+    assert G.plan.query(clear=True) == 0
+    ratio, wn, un = G.results()
+    for k in range(L.n_tensors):
+        w, g = L.weights(k), L.grad(k, 2)
+        m, v = L.state_warm(k)
+        ref = _oracle_lamb(L, k, w, g, m, v, 2, lr, h)
+        e = compare_lamb(G.download("w", k), G.download("m", k),
+                         G.download("v", k), ref, w, m,
+                         O.to_f64(g, grad_dtype), h.beta1, TOL_STEP,
+                         upd=(h, 2, lr, h.weight_decay * L.decay[k]))
+        if copy_dtype:
+            check_copy(G.download("copy", k), G.download("w", k), ref.w,
+                       sw=e["_sw"])
+        assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
+    G.close()
+
+
+@pytest.mark.parametrize("lars", [False, True])
+def test_single_touch_bitwise_deterministic_across_schedules(lars):
+    """Chunking is fixed (1024 elements, groups of 32), so neither the grid,
+    the lag nor the L2 budget may change a single bit of the results."""
+    L = W.resnet50_layout()
+    h = L.lars_hyper if lars else L.hyper
+    snaps = []
+    for bps, lag, budget in ((0, 0, 0), (1, 1, 1), (0, 50000, 4096),
+                             (0, 0, 0)):
+        G = GpuLayout(L, with_v=not lars, blocks_per_sm=bps, lag_items=lag,
+                      l2_budget_mb=budget, algorithm=2)
+        G.load_weights()
+        G.load_warm_state()
+        G.load_grads(4)
+        for t in (4, 5, 6):
+            G.step(t, f32(h.lr), c_hyper(h, lars=lars), lars=lars)
+        assert G.plan.query() == 0
+        snaps.append(_snapshot(G))
+        G.close()
+    for other in snaps[1:]:
+        for a, b in zip(snaps[0], other):
+            assert torch.equal(a, b)
+
+
+def test_single_touch_matches_two_pass_within_tolerance():
+    L = W.bert_base_layout()
+    h = L.hyper
+    outs = []
+    for algo in (1, 2):
+        G = GpuLayout(L, algorithm=algo)
+        G.load_weights()
+        G.load_warm_state()
+        G.load_grads(4)
+        G.step(4, f32(h.lr), c_hyper(h))
+        r, _, _ = G.results()
+        outs.append((G.st.w.clone(), G.st.m.clone(), G.st.v.clone(), r))
+        G.close()
+    (w1, m1, v1, r1), (w2, m2, v2, r2) = outs
+    # the moments do not depend on any reduction: bitwise equal
+    assert torch.equal(m1, m2) and torch.equal(v1, v2)
+    np.testing.assert_allclose(r2, r1, rtol=2 * TOL_RATIO, atol=0)
+    d = (w1.double() - w2.double()).abs()
+    assert bool(torch.all(d <= TOL_STEP * w1.double().abs().clamp_min(1e-30)
+                          + 1e-12))
