@@ -136,8 +136,8 @@ typedef struct {
                             this many MiB keep them in L2 between the
                             passes; 0 = half the device's L2               */
   int32_t lag_items;     /* single-touch: work items between a tensor's last
-                            pass-1 item and its pass-2 block; 0 = one item
-                            per resident warp of the grid                  */
+                            pass-1 item and its pass-2 block; 0 = 1.5x the
+                            items the grid holds in flight                 */
 } lamb_plan_options_t;
 
 typedef struct {
@@ -305,7 +305,7 @@ LAMB_API lamb_status_t lamb_step_noalloc(
 
 /* Host-only planner, no device needed: the work-item order a single-touch
  * plan would use.  Each item is (fused chunk index << 1) | is_pass2; fused
- * chunks hold 1024 elements, numbered in tensor order.  l2_budget_bytes and
+ * chunks hold 512 elements, numbered in tensor order.  l2_budget_bytes and
  * lag_items as in lamb_plan_options_t (both required, > 0).  Writes up to
  * `capacity` items, the total into *n_items and, if `resident` is not NULL,
  * one residency flag per tensor.  INVALID_ARG on bad input or capacity too

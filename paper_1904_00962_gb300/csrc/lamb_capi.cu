@@ -309,11 +309,11 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
       return cuda_fail(e, "cudaDeviceGetAttribute(L2)");
     }
     p->l2_budget = budget_mb ? budget_mb << 20 : (int64_t)l2 / 2;
-    // one item per warp of the larger grid (8 warps per CTA)
     p->lag = lag_opt ? lag_opt
-                     : (int64_t)8 * (p->grid_fused[0] > p->grid_fused[1]
-                                         ? p->grid_fused[0]
-                                         : p->grid_fused[1]);
+                     : (int64_t)kFusedLagPerCta *
+                           (p->grid_fused[0] > p->grid_fused[1]
+                                ? p->grid_fused[0]
+                                : p->grid_fused[1]);
     if (plan_fused(sizes, n_tensors, decay_mask, 12, p->l2_budget, p->lag,
                    &h_fchunks, &h_ftensors, &h_items, &p->n_groups, err,
                    sizeof(err))) {

@@ -93,8 +93,11 @@ struct StepParams {
 // pass-1 items by a lag of about one wave, so the m, v, w the pass 1 just
 // touched are still in L2 when the pass 2 reads them.
 // ---------------------------------------------------------------------------
-constexpr int kFusedChunk = 1024;     // elements per fused chunk (one warp item)
+constexpr int kFusedChunk = 512;      // elements per fused chunk (one warp item)
 constexpr int kGroup = 32;            // fused chunks per first-level combine
+// default schedule lag per CTA of the fused grid: 8 warps x 3 prefetch
+// stages hold 24 items in flight; 1.5x that keeps pass-2 waits rare
+constexpr int kFusedLagPerCta = 36;
 
 struct __align__(8) FusedChunk {
   int32_t tensor;   // tensor index k

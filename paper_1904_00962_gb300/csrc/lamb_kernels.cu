@@ -566,17 +566,25 @@ __global__ void __launch_bounds__(kThreads)
 // ---------------------------------------------------------------------------
 // Single-touch fused step (one persistent kernel, warps are the workers)
 //
-// Items are drawn in schedule order from counters[2].  A pass-1 item streams
-// one fused chunk (1024 elements) through Alg. 2's moment and ratio lines,
-// stores the new m, v and publishes the chunk's sums; the warp that completes
-// a group of 32 chunks sums them (fp64, fixed order), and the warp that
-// completes a tensor's last group computes its norms and trust ratio and
-// releases ready[k] = epoch.  A pass-2 item waits (bounded) for ready[k] ==
-// epoch and applies the update.  Pass-2 items of a tensor come after all its
-// pass-1 items in the schedule and items are drawn in order, so the earliest
-// unfinished item never waits on anything unfinished: the kernel cannot
-// deadlock.  The wait still gives up after ~0.5 s, sets a status bit and
-// makes every other waiter of the same launch give up at once.
+// Items are drawn in schedule order from counters[2].  A pass-1 item runs one
+// fused chunk (512 elements) through Alg. 2's moment and ratio lines (Alg. 1
+// for LARS), stores the new m, v and publishes the chunk's sums; the warp that
+// completes a group of 32 chunks sums them (fp64, fixed order), and the warp
+// that completes a tensor's last group computes its norms and trust ratio and
+// releases ready[k] = epoch.  A pass-2 item applies the update once ready[k]
+// == epoch.  Pass-2 items of a tensor come after all its pass-1 items in the
+// schedule and items are drawn in order, so the earliest unfinished item never
+// waits on anything unfinished: the kernel cannot deadlock.  A wait still
+// gives up after ~0.5 s, sets a status bit and makes every other waiter of
+// the same launch give up at once.
+//
+// Memory pipeline: every warp owns a ring of kStages shared-memory stages and
+// prefetches the operands of its next items with cp.async while it computes
+// the current one, so many bytes are in flight without holding registers.  A
+// pass-2 item is prefetched only if its tensor's norms are already final when
+// it is drawn (its m, v come from other warps' pass-1 stores); otherwise, and
+// for tail chunks and unaligned tensors, the item reads global memory
+// directly when its turn comes.
 //
 // L2 policy: pass-1 loads/stores of m, v, w of "resident" tensors (those
 // whose state fits the L2 budget) are evict_last, so pass 2 -- about one
@@ -584,17 +592,29 @@ __global__ void __launch_bounds__(kThreads)
 // evict_first.
 // ---------------------------------------------------------------------------
 constexpr int kFusedThreads = 256;                     // 8 warps per CTA
-// 4-element packets per lane per batch: LARS keeps 4 in flight; LAMB keeps 2
-// (its longer arithmetic needs the registers) and runs twice the batches.
-template <bool kLars> __host__ __device__ constexpr int fused_unroll() {
-  return kLars ? 4 : 2;
-}
-template <bool kLars> __host__ __device__ constexpr int fused_batches() {
-  return kFusedChunk / (32 * 4 * fused_unroll<kLars>());
-}
-static_assert(fused_batches<true>() * 32 * 4 * 4 == kFusedChunk, "shape");
-static_assert(fused_batches<false>() * 32 * 4 * 2 == kFusedChunk, "shape");
+constexpr int kFusedWarps = kFusedThreads / 32;
+constexpr int kStages = 3;                             // prefetch depth per warp
+constexpr int kPktsPerLane = kFusedChunk / 4 / 32;     // 4-element packets
+static_assert(kPktsPerLane * 4 * 32 == kFusedChunk, "fused chunk shape");
 constexpr uint32_t kSpinLimit = 1u << 21;              // x <= 256 ns ~ 0.5 s
+
+// stage layout: m | v (LAMB only) | w | g
+template <bool kLars, typename GT>
+__host__ __device__ constexpr int stage_bytes() {
+  return kFusedChunk * (4 * (kLars ? 2 : 3) + (int)sizeof(GT));
+}
+template <bool kLars, typename GT>
+__host__ __device__ constexpr int fused_smem_bytes() {
+  return kFusedWarps * kStages * stage_bytes<kLars, GT>();
+}
+constexpr int kOffM = 0;
+constexpr int kOffV = 4 * kFusedChunk;
+template <bool kLars> __host__ __device__ constexpr int off_w() {
+  return 4 * kFusedChunk * (kLars ? 1 : 2);
+}
+template <bool kLars> __host__ __device__ constexpr int off_g() {
+  return 4 * kFusedChunk * (kLars ? 2 : 3);
+}
 
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
@@ -623,6 +643,10 @@ __device__ __forceinline__ void stp4(float* p, float4 v, uint64_t pol) {
 __device__ __forceinline__ float4 ldp_grad4(const float* p, uint64_t pol) {
   return ldp4(p, pol);
 }
+__device__ __forceinline__ float4 unpack_bf16x4(uint32_t a, uint32_t b) {
+  return make_float4(__uint_as_float(a << 16), __uint_as_float(a & 0xffff0000u),
+                     __uint_as_float(b << 16), __uint_as_float(b & 0xffff0000u));
+}
 __device__ __forceinline__ float4 ldp_grad4(const __nv_bfloat16* p,
                                             uint64_t pol) {
   uint32_t a, b;
@@ -630,8 +654,17 @@ __device__ __forceinline__ float4 ldp_grad4(const __nv_bfloat16* p,
       "ld.global.L1::no_allocate.L2::cache_hint.v2.u32 {%0,%1}, [%2], %3;"
       : "=r"(a), "=r"(b)
       : "l"(p), "l"(pol));
-  return make_float4(__uint_as_float(a << 16), __uint_as_float(a & 0xffff0000u),
-                     __uint_as_float(b << 16), __uint_as_float(b & 0xffff0000u));
+  return unpack_bf16x4(a, b);
+}
+// gradient packet j of a stage
+__device__ __forceinline__ float4 lds_grad4(const char* gbase, int j,
+                                            const float*) {
+  return *reinterpret_cast<const float4*>(gbase + 16 * j);
+}
+__device__ __forceinline__ float4 lds_grad4(const char* gbase, int j,
+                                            const __nv_bfloat16*) {
+  const uint2 u = *reinterpret_cast<const uint2*>(gbase + 8 * j);
+  return unpack_bf16x4(u.x, u.y);
 }
 __device__ __forceinline__ void stp_copy4(void* base, int64_t i, float4 x,
                                           uint64_t pol) {
@@ -643,6 +676,23 @@ __device__ __forceinline__ void stp_copy4(void* base, int64_t i, float4 x,
       "st.global.L1::no_allocate.L2::cache_hint.v2.u32 [%0], {%1,%2}, %3;"
       ::"l"(static_cast<__nv_bfloat16*>(base) + i), "r"(a), "r"(b), "l"(pol)
       : "memory");
+}
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void cp_async16(uint32_t saddr, const void* g,
+                                           uint64_t pol) {
+  asm volatile(
+      "cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;"
+      ::"r"(saddr), "l"(g), "l"(pol)
+      : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
   uint32_t v;
@@ -691,61 +741,106 @@ __device__ __forceinline__ float fused2_dir(float m, float v, float w,
   return kLars ? m : lamb_direction(m, v, w, lam, k);
 }
 
-// Warp-level pass 1 of one fused chunk; publishes its sums and, if it is the
-// last chunk of its group / tensor, performs the combine.
+template <bool kLars>
+__device__ __forceinline__ void fused1_pkt(float4 gv, float4& mv, float4& vv,
+                                           float4 wv, float lam,
+                                           const LambConsts& k, float& sw,
+                                           float& su) {
+  fused1_elem<kLars>(gv.x, mv.x, vv.x, wv.x, lam, k, sw, su);
+  fused1_elem<kLars>(gv.y, mv.y, vv.y, wv.y, lam, k, sw, su);
+  fused1_elem<kLars>(gv.z, mv.z, vv.z, wv.z, lam, k, sw, su);
+  fused1_elem<kLars>(gv.w, mv.w, vv.w, wv.w, lam, k, sw, su);
+}
+
+template <bool kLars>
+__device__ __forceinline__ float4 fused2_pkt(float4 mv, float4 vv, float4 wv,
+                                             float s, float lam,
+                                             const LambConsts& k) {
+  float4 o;
+  o.x = __fmaf_rn(-s, fused2_dir<kLars>(mv.x, vv.x, wv.x, lam, k), wv.x);
+  o.y = __fmaf_rn(-s, fused2_dir<kLars>(mv.y, vv.y, wv.y, lam, k), wv.y);
+  o.z = __fmaf_rn(-s, fused2_dir<kLars>(mv.z, vv.z, wv.z, lam, k), wv.z);
+  o.w = __fmaf_rn(-s, fused2_dir<kLars>(mv.w, vv.w, wv.w, lam, k), wv.w);
+  return o;
+}
+
+// What one item refers to.
+struct FusedItem {
+  TensorPtrs tp;
+  FusedTensor ft;
+  FusedChunk fc;
+  int chunk;
+  int64_t off;
+  int len;
+  bool pass2;
+};
+
+__device__ __forceinline__ FusedItem fused_item(const StepParams& p,
+                                                const FusedParams& f,
+                                                uint32_t code) {
+  FusedItem it;
+  it.chunk = (int)(code >> 1);
+  it.pass2 = (code & 1u) != 0u;
+  it.fc = f.fchunks[it.chunk];
+  it.ft = f.ftensors[it.fc.tensor];
+  it.tp = p.ptrs[it.fc.tensor];
+  it.off = (int64_t)it.fc.index * kFusedChunk;
+  const int64_t rem = it.ft.numel - it.off;
+  it.len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
+  return it;
+}
+
+// Prefetch the operands of item `code` into `stage` (all lanes).  Returns
+// whether it did: only full chunks of aligned tensors, and pass-2 items only
+// once their tensor's norms are final.
 template <bool kLars, typename GT>
-__device__ __forceinline__ void fused_pass1(
-    const StepParams& p, const FusedParams& f, const LambConsts& k,
-    const TensorPtrs& tp, const FusedTensor& ft, const FusedChunk& fc,
-    int chunk, int64_t off, int len, float lam, uint64_t pol_first,
-    uint64_t pol_keep, uint32_t epoch, int lane) {
-  float* __restrict__ w = tp.w + off;
-  float* __restrict__ m = tp.m + off;
-  float* __restrict__ v = kLars ? nullptr : tp.v + off;
-  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + off;
-  constexpr int kFU = fused_unroll<kLars>();
-  float sw = 0.f, su = 0.f;
-  int scalar_from = 0;
-  if (tp.vec_ok) {
-    const int nv = len >> 2;
-#pragma unroll 1
-    for (int b = 0; b < fused_batches<kLars>(); ++b) {
-      const int base = b * 32 * kFU + lane;
-      float4 wv[kFU], mv[kFU], vv[kFU], gv[kFU];
+__device__ __forceinline__ bool fused_prefetch(const StepParams& p,
+                                               const FusedParams& f,
+                                               uint32_t code, char* stage,
+                                               uint32_t epoch,
+                                               uint64_t pol_first,
+                                               uint64_t pol_last, int lane) {
+  const FusedItem it = fused_item(p, f, code);
+  if (!it.tp.vec_ok || it.len != kFusedChunk) return false;
+  if (it.pass2) {
+    uint32_t ready = 0;
+    if (lane == 0) ready = ld_acquire(&f.ready[it.fc.tensor]) == epoch;
+    if (!__shfl_sync(0xffffffffu, ready, 0)) return false;
+    __syncwarp();
+    (void)ld_acquire(&f.ready[it.fc.tensor]);   // per-lane acquire
+  }
+  const uint64_t pol =
+      (!it.pass2 && it.ft.resident) ? pol_last : pol_first;
+  const uint32_t s = smem_u32(stage);
 #pragma unroll
-      for (int u = 0; u < kFU; ++u) {
-        const int j = base + u * 32;
-        if (j < nv) {
-          gv[u] = ldp_grad4(g + 4 * j, pol_first);
-          mv[u] = ldp4(m + 4 * j, pol_keep);
-          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_keep);
-          wv[u] = ldp4(w + 4 * j, pol_keep);
-        }
-      }
+  for (int u = 0; u < kPktsPerLane; ++u) {
+    const int j = lane + 32 * u;                    // 16-byte piece index
+    cp_async16(s + kOffM + 16 * j, it.tp.m + it.off + 4 * j, pol);
+    if (!kLars) cp_async16(s + kOffV + 16 * j, it.tp.v + it.off + 4 * j, pol);
+    cp_async16(s + off_w<kLars>() + 16 * j, it.tp.w + it.off + 4 * j, pol);
+  }
+  if (!it.pass2) {
+    const GT* g = static_cast<const GT*>(it.tp.g) + it.off;
+    constexpr int kGPieces = kFusedChunk * (int)sizeof(GT) / 16;
 #pragma unroll
-      for (int u = 0; u < kFU; ++u) {
-        const int j = base + u * 32;
-        if (j < nv) {
-          float4& mm = mv[u];
-          float4& vvv = vv[u];
-          fused1_elem<kLars>(gv[u].x, mm.x, vvv.x, wv[u].x, lam, k, sw, su);
-          fused1_elem<kLars>(gv[u].y, mm.y, vvv.y, wv[u].y, lam, k, sw, su);
-          fused1_elem<kLars>(gv[u].z, mm.z, vvv.z, wv[u].z, lam, k, sw, su);
-          fused1_elem<kLars>(gv[u].w, mm.w, vvv.w, wv[u].w, lam, k, sw, su);
-          stp4(m + 4 * j, mm, pol_keep);
-          if (!kLars) stp4(v + 4 * j, vvv, pol_keep);
-        }
-      }
+    for (int u = 0; u < kGPieces / 32; ++u) {
+      const int j = lane + 32 * u;
+      cp_async16(s + off_g<kLars>() + 16 * j,
+                 reinterpret_cast<const char*>(g) + 16 * j, pol_first);
     }
-    scalar_from = nv << 2;
   }
-  for (int i = scalar_from + lane; i < len; i += 32) {
-    float mi = m[i];
-    float vi = kLars ? 0.f : v[i];
-    fused1_elem<kLars>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
-    m[i] = mi;
-    if (!kLars) v[i] = vi;
-  }
+  return true;
+}
+
+// Publish a pass-1 chunk's sums; the last chunk of a group and the last group
+// of a tensor do the fixed-order fp64 combines and release the tensor.
+template <bool kLars>
+__device__ __forceinline__ void fused_publish(const StepParams& p,
+                                           const FusedParams& f,
+                                           const FusedTensor& ft,
+                                           const FusedChunk& fc, int chunk,
+                                           float sw, float su, uint32_t epoch,
+                                           int lane) {
   sw = warp_sum(sw);
   su = warp_sum(su);
   __syncwarp();
@@ -760,7 +855,6 @@ __device__ __forceinline__ void fused_pass1(
   }
   if (!__shfl_sync(0xffffffffu, last, 0)) return;
   __syncwarp();
-  // first level: the group's chunk sums, fp64, fixed order
   double aw = 0.0, au = 0.0;
   if (lane < gsize) {
     const float2 s = __ldcg(&f.fslots[ft.first_chunk + gl * kGroup + lane]);
@@ -777,7 +871,6 @@ __device__ __forceinline__ void fused_pass1(
   }
   if (!__shfl_sync(0xffffffffu, last, 0)) return;
   __syncwarp();
-  // second level: the tensor's group sums -> norms and trust ratio
   double tw = 0.0, tu = 0.0;
   for (int i = lane; i < ft.n_groups; i += 32) {
     const double2 s = __ldcg(&f.gslots[ft.first_group + i]);
@@ -800,12 +893,82 @@ __device__ __forceinline__ void fused_pass1(
   }
 }
 
-// Warp-level pass 2 of one fused chunk.
-template <bool kLars, bool kCopy>
-__device__ __forceinline__ void fused_pass2(
-    const StepParams& p, const FusedParams& f, const LambConsts& k,
-    const TensorPtrs& tp, int tensor, int64_t off, int len, float lam,
-    float lr, uint64_t pol_first, uint32_t epoch, int lane) {
+// Pass 1 of one item, operands from the warp's stage or from global memory.
+template <bool kLars, typename GT>
+__device__ __forceinline__ void fused_pass1(const StepParams& p,
+                                            const FusedParams& f,
+                                            const LambConsts& k,
+                                            const FusedItem& it,
+                                            const char* stage, bool staged,
+                                            uint64_t pol_first,
+                                            uint64_t pol_last, uint32_t epoch,
+                                            int lane) {
+  const TensorPtrs& tp = it.tp;
+  const uint64_t pol_keep = it.ft.resident ? pol_last : pol_first;
+  const float lam = it.ft.decay * p.wd;
+  float* __restrict__ m = tp.m + it.off;
+  float* __restrict__ v = kLars ? nullptr : tp.v + it.off;
+  const float* __restrict__ w = tp.w + it.off;
+  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + it.off;
+  float sw = 0.f, su = 0.f;
+  if (staged) {
+#pragma unroll
+    for (int u = 0; u < kPktsPerLane; ++u) {
+      const int j = lane + 32 * u;
+      float4 mv = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
+      float4 vv = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
+                        : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
+      const float4 wv =
+          *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
+      const float4 gv = lds_grad4(stage + off_g<kLars>(), j, g);
+      fused1_pkt<kLars>(gv, mv, vv, wv, lam, k, sw, su);
+      stp4(m + 4 * j, mv, pol_keep);
+      if (!kLars) stp4(v + 4 * j, vv, pol_keep);
+    }
+  } else {
+    int scalar_from = 0;
+    if (tp.vec_ok) {
+      const int nv = it.len >> 2;
+#pragma unroll 1
+      for (int base = lane; base < nv; base += 64) {
+        float4 wv[2], mv[2], vv[2], gv[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int j = base + 32 * u;
+          if (j < nv) {
+            gv[u] = ldp_grad4(g + 4 * j, pol_first);
+            mv[u] = ldp4(m + 4 * j, pol_keep);
+            if (!kLars) vv[u] = ldp4(v + 4 * j, pol_keep);
+            wv[u] = ldp4(w + 4 * j, pol_keep);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int j = base + 32 * u;
+          if (j < nv) {
+            fused1_pkt<kLars>(gv[u], mv[u], vv[u], wv[u], lam, k, sw, su);
+            stp4(m + 4 * j, mv[u], pol_keep);
+            if (!kLars) stp4(v + 4 * j, vv[u], pol_keep);
+          }
+        }
+      }
+      scalar_from = nv << 2;
+    }
+    for (int i = scalar_from + lane; i < it.len; i += 32) {
+      float mi = m[i];
+      float vi = kLars ? 0.f : v[i];
+      fused1_elem<kLars>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
+      m[i] = mi;
+      if (!kLars) v[i] = vi;
+    }
+  }
+  fused_publish<kLars>(p, f, it.ft, it.fc, it.chunk, sw, su, epoch, lane);
+}
+
+// Bounded wait of a pass-2 item for its tensor's norms (all lanes).
+__device__ __forceinline__ bool fused_wait(const StepParams& p,
+                                           const FusedParams& f, int tensor,
+                                           uint32_t epoch, int lane) {
   uint32_t ok = 1;
   if (lane == 0) {
     uint32_t spins = 0, ns = 32;
@@ -823,24 +986,53 @@ __device__ __forceinline__ void fused_pass2(
       if (ns < 256) ns <<= 1;
     }
   }
-  if (!__shfl_sync(0xffffffffu, ok, 0)) return;   // gave up: leave w as is
+  if (!__shfl_sync(0xffffffffu, ok, 0)) return false;
   __syncwarp();
   (void)ld_acquire(&f.ready[tensor]);               // per-lane acquire
-  const float s = __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]));
-  float* __restrict__ w = tp.w + off;
-  const float* __restrict__ m = tp.m + off;
-  const float* __restrict__ v = kLars ? nullptr : tp.v + off;
-  constexpr int kFU = fused_unroll<kLars>();
+  return true;
+}
+
+// Pass 2 of one item.
+template <bool kLars, bool kCopy>
+__device__ __forceinline__ void fused_pass2(const StepParams& p,
+                                            const FusedParams& f,
+                                            const LambConsts& k,
+                                            const FusedItem& it,
+                                            const char* stage, bool staged,
+                                            float lr, uint64_t pol_first,
+                                            uint32_t epoch, int lane) {
+  if (!staged && !fused_wait(p, f, it.fc.tensor, epoch, lane))
+    return;                                         // gave up: leave w as is
+  const TensorPtrs& tp = it.tp;
+  const float lam = it.ft.decay * p.wd;
+  const float s = __double2float_rn((double)lr * __ldcg(&p.ratio[it.fc.tensor]));
+  float* __restrict__ w = tp.w + it.off;
+  const float* __restrict__ m = tp.m + it.off;
+  const float* __restrict__ v = kLars ? nullptr : tp.v + it.off;
+  if (staged) {
+#pragma unroll
+    for (int u = 0; u < kPktsPerLane; ++u) {
+      const int j = lane + 32 * u;
+      const float4 mv = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
+      const float4 vv = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
+                              : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
+      const float4 wv =
+          *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
+      const float4 o = fused2_pkt<kLars>(mv, vv, wv, s, lam, k);
+      stp4(w + 4 * j, o, pol_first);
+      if (kCopy) stp_copy4(tp.copy, it.off + 4 * j, o, pol_first);
+    }
+    return;
+  }
   int scalar_from = 0;
   if (tp.vec_ok) {
-    const int nv = len >> 2;
+    const int nv = it.len >> 2;
 #pragma unroll 1
-    for (int b = 0; b < fused_batches<kLars>(); ++b) {
-      const int base = b * 32 * kFU + lane;
-      float4 wv[kFU], mv[kFU], vv[kFU];
+    for (int base = lane; base < nv; base += 64) {
+      float4 wv[2], mv[2], vv[2];
 #pragma unroll
-      for (int u = 0; u < kFU; ++u) {
-        const int j = base + u * 32;
+      for (int u = 0; u < 2; ++u) {
+        const int j = base + 32 * u;
         if (j < nv) {
           mv[u] = ldp4(m + 4 * j, pol_first);
           if (!kLars) vv[u] = ldp4(v + 4 * j, pol_first);
@@ -848,39 +1040,37 @@ __device__ __forceinline__ void fused_pass2(
         }
       }
 #pragma unroll
-      for (int u = 0; u < kFU; ++u) {
-        const int j = base + u * 32;
+      for (int u = 0; u < 2; ++u) {
+        const int j = base + 32 * u;
         if (j < nv) {
-          float4 o;
-          o.x = __fmaf_rn(-s, fused2_dir<kLars>(mv[u].x, vv[u].x, wv[u].x, lam, k), wv[u].x);
-          o.y = __fmaf_rn(-s, fused2_dir<kLars>(mv[u].y, vv[u].y, wv[u].y, lam, k), wv[u].y);
-          o.z = __fmaf_rn(-s, fused2_dir<kLars>(mv[u].z, vv[u].z, wv[u].z, lam, k), wv[u].z);
-          o.w = __fmaf_rn(-s, fused2_dir<kLars>(mv[u].w, vv[u].w, wv[u].w, lam, k), wv[u].w);
+          const float4 o = fused2_pkt<kLars>(mv[u], vv[u], wv[u], s, lam, k);
           stp4(w + 4 * j, o, pol_first);
-          if (kCopy) stp_copy4(tp.copy, off + 4 * j, o, pol_first);
+          if (kCopy) stp_copy4(tp.copy, it.off + 4 * j, o, pol_first);
         }
       }
     }
     scalar_from = nv << 2;
   }
-  for (int i = scalar_from + lane; i < len; i += 32) {
+  for (int i = scalar_from + lane; i < it.len; i += 32) {
     const float wi = w[i];
     const float o = __fmaf_rn(
         -s, fused2_dir<kLars>(m[i], kLars ? 0.f : v[i], wi, lam, k), wi);
     w[i] = o;
-    if (kCopy) st_copy1(tp.copy, off + i, o);
+    if (kCopy) st_copy1(tp.copy, it.off + i, o);
   }
 }
 
 template <bool kLars, typename GT, bool kCopy>
-__global__ void __launch_bounds__(kFusedThreads, 2)
+__global__ void __launch_bounds__(kFusedThreads, 1)
     fused_step_kernel(const StepParams p, const FusedParams f) {
+  extern __shared__ __align__(128) char fused_smem[];
   __shared__ LambConsts s_k;
   __shared__ float s_lr;
   __shared__ int s_skip;
   __shared__ uint32_t s_epoch;
   __shared__ int64_t s_t;
   const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
     const bool bc = !kLars && (p.flags & kFlagBiasCorrection) != 0;
     const int64_t t = p.d_step ? *p.d_step : int64_t(1);
@@ -914,35 +1104,67 @@ __global__ void __launch_bounds__(kFusedThreads, 2)
   const uint64_t pol_first = policy_evict_first();
   const uint64_t pol_last = policy_evict_last();
   const uint32_t n_items = (uint32_t)f.n_items;
-  uint32_t next = 0;
-  if (lane == 0) next = atomicAdd(&p.counters[2], 1u);
-  next = __shfl_sync(0xffffffffu, next, 0);
-  while (next < n_items) {
-    const uint32_t item = next;
-    uint32_t pre = 0;
-    if (lane == 0) pre = atomicAdd(&p.counters[2], 1u);  // draw ahead
-    const uint32_t code = __ldg(&f.items[item]);
-    const int chunk = (int)(code >> 1);
-    const FusedChunk fc = f.fchunks[chunk];
-    const FusedTensor ft = f.ftensors[fc.tensor];
-    const TensorPtrs tp = p.ptrs[fc.tensor];
-    const int64_t off = (int64_t)fc.index * kFusedChunk;
-    const int64_t rem = ft.numel - off;
-    const int len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
-    const float lam = ft.decay * p.wd;
-    if ((code & 1u) == 0u)
-      fused_pass1<kLars, GT>(p, f, k, tp, ft, fc, chunk, off, len, lam,
-                             pol_first, ft.resident ? pol_last : pol_first,
-                             epoch, lane);
-    else
-      fused_pass2<kLars, kCopy>(p, f, k, tp, fc.tensor, off, len, lam, lr,
-                                pol_first, epoch, lane);
-    next = __shfl_sync(0xffffffffu, pre, 0);
+  char* ring = fused_smem + warp * kStages * stage_bytes<kLars, GT>();
+
+  // Each warp draws indices until it gets one >= n_items, then stops, so it
+  // draws exactly one such index.
+  uint32_t last_drawn = 0;
+  bool drawing = true;
+  auto draw = [&]() -> uint32_t {
+    if (!drawing) return n_items;
+    uint32_t v = 0;
+    if (lane == 0) v = atomicAdd(&p.counters[2], 1u);
+    v = __shfl_sync(0xffffffffu, v, 0);
+    if (v >= n_items) {
+      drawing = false;
+      last_drawn = v;
+    }
+    return v;
+  };
+
+  uint32_t code[kStages];
+  bool staged[kStages];
+#pragma unroll
+  for (int s = 0; s < kStages; ++s) {
+    const uint32_t i = draw();
+    code[s] = i < n_items ? __ldg(&f.items[i]) : 0xffffffffu;
+    staged[s] = i < n_items &&
+                fused_prefetch<kLars, GT>(p, f, code[s],
+                                          ring + s * stage_bytes<kLars, GT>(),
+                                          epoch, pol_first, pol_last, lane);
+    cp_async_commit();
   }
-  // Every warp draws exactly one index >= n_items; the warp that draws the
-  // last of them is the last to draw and closes the launch.
-  const uint32_t warps = gridDim.x * (kFusedThreads / 32);
-  if (lane == 0 && next == n_items + warps - 1u) {
+  bool done = false;
+  while (!done) {
+#pragma unroll
+    for (int s = 0; s < kStages; ++s) {
+      if (code[s] == 0xffffffffu) {
+        done = true;
+        break;
+      }
+      char* stage = ring + s * stage_bytes<kLars, GT>();
+      cp_async_wait<kStages - 1>();  // this stage's copies have landed
+      __syncwarp();
+      const FusedItem it = fused_item(p, f, code[s]);
+      if (!it.pass2)
+        fused_pass1<kLars, GT>(p, f, k, it, stage, staged[s], pol_first,
+                               pol_last, epoch, lane);
+      else
+        fused_pass2<kLars, kCopy>(p, f, k, it, stage, staged[s], lr,
+                                  pol_first, epoch, lane);
+      __syncwarp();                  // every lane is done with the stage
+      const uint32_t i = draw();
+      code[s] = i < n_items ? __ldg(&f.items[i]) : 0xffffffffu;
+      staged[s] = i < n_items &&
+                  fused_prefetch<kLars, GT>(p, f, code[s], stage, epoch,
+                                            pol_first, pol_last, lane);
+      cp_async_commit();
+    }
+  }
+  cp_async_wait<0>();
+  // The warp that drew the last index >= n_items closes the launch.
+  const uint32_t warps = gridDim.x * kFusedWarps;
+  if (lane == 0 && last_drawn == n_items + warps - 1u) {
     atomicExch(&p.counters[2], 0u);
     const uint32_t ne = epoch + 1u == 0u ? 1u : epoch + 1u;
     atomicExch(&p.counters[3], ne);
@@ -998,38 +1220,53 @@ int launch_lars_pass2(const StepParams& p, int copy_bf16, int grid,
   return (int)cudaGetLastError();
 }
 
-int launch_fused(const StepParams& p, const FusedParams& f, int lars,
-                 int grad_bf16, int copy_bf16, int grid, void* stream) {
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const int sel = (lars ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0);
-  switch (sel) {
-    case 0: fused_step_kernel<false, float, false><<<grid, kFusedThreads, 0, s>>>(p, f); break;
-    case 1: fused_step_kernel<false, float, true><<<grid, kFusedThreads, 0, s>>>(p, f); break;
-    case 2: fused_step_kernel<false, __nv_bfloat16, false><<<grid, kFusedThreads, 0, s>>>(p, f); break;
-    case 3: fused_step_kernel<false, __nv_bfloat16, true><<<grid, kFusedThreads, 0, s>>>(p, f); break;
-    case 4: fused_step_kernel<true, float, false><<<grid, kFusedThreads, 0, s>>>(p, f); break;
-    case 5: fused_step_kernel<true, float, true><<<grid, kFusedThreads, 0, s>>>(p, f); break;
-    case 6: fused_step_kernel<true, __nv_bfloat16, false><<<grid, kFusedThreads, 0, s>>>(p, f); break;
-    default: fused_step_kernel<true, __nv_bfloat16, true><<<grid, kFusedThreads, 0, s>>>(p, f); break;
-  }
+template <bool kLars, typename GT, bool kCopy>
+int launch_fused_t(const StepParams& p, const FusedParams& f, int grid,
+                   cudaStream_t s) {
+  fused_step_kernel<kLars, GT, kCopy>
+      <<<grid, kFusedThreads, fused_smem_bytes<kLars, GT>(), s>>>(p, f);
   return (int)cudaGetLastError();
 }
 
+template <bool kLars, typename GT, bool kCopy>
+int occupancy_fused_t(int* blocks) {
+  // opt in to the dynamic shared memory of the stage rings (a property of
+  // the function, set once; not a device setting)
+  cudaError_t e = cudaFuncSetAttribute(
+      fused_step_kernel<kLars, GT, kCopy>,
+      cudaFuncAttributeMaxDynamicSharedMemorySize,
+      fused_smem_bytes<kLars, GT>());
+  if (e != cudaSuccess) return (int)e;
+  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+      blocks, fused_step_kernel<kLars, GT, kCopy>, kFusedThreads,
+      fused_smem_bytes<kLars, GT>());
+}
+
+int launch_fused(const StepParams& p, const FusedParams& f, int lars,
+                 int grad_bf16, int copy_bf16, int grid, void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch ((lars ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0)) {
+    case 0: return launch_fused_t<false, float, false>(p, f, grid, s);
+    case 1: return launch_fused_t<false, float, true>(p, f, grid, s);
+    case 2: return launch_fused_t<false, __nv_bfloat16, false>(p, f, grid, s);
+    case 3: return launch_fused_t<false, __nv_bfloat16, true>(p, f, grid, s);
+    case 4: return launch_fused_t<true, float, false>(p, f, grid, s);
+    case 5: return launch_fused_t<true, float, true>(p, f, grid, s);
+    case 6: return launch_fused_t<true, __nv_bfloat16, false>(p, f, grid, s);
+    default: return launch_fused_t<true, __nv_bfloat16, true>(p, f, grid, s);
+  }
+}
+
 int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks) {
-  const int sel = (lars ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0);
-  auto q = [&](auto kern) {
-    return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        blocks, kern, kFusedThreads, 0);
-  };
-  switch (sel) {
-    case 0: return q(fused_step_kernel<false, float, false>);
-    case 1: return q(fused_step_kernel<false, float, true>);
-    case 2: return q(fused_step_kernel<false, __nv_bfloat16, false>);
-    case 3: return q(fused_step_kernel<false, __nv_bfloat16, true>);
-    case 4: return q(fused_step_kernel<true, float, false>);
-    case 5: return q(fused_step_kernel<true, float, true>);
-    case 6: return q(fused_step_kernel<true, __nv_bfloat16, false>);
-    default: return q(fused_step_kernel<true, __nv_bfloat16, true>);
+  switch ((lars ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0)) {
+    case 0: return occupancy_fused_t<false, float, false>(blocks);
+    case 1: return occupancy_fused_t<false, float, true>(blocks);
+    case 2: return occupancy_fused_t<false, __nv_bfloat16, false>(blocks);
+    case 3: return occupancy_fused_t<false, __nv_bfloat16, true>(blocks);
+    case 4: return occupancy_fused_t<true, float, false>(blocks);
+    case 5: return occupancy_fused_t<true, float, true>(blocks);
+    case 6: return occupancy_fused_t<true, __nv_bfloat16, false>(blocks);
+    default: return occupancy_fused_t<true, __nv_bfloat16, true>(blocks);
   }
 }
 

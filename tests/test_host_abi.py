@@ -166,7 +166,7 @@ def test_planner_capacity_too_small(lib):
 
 def _check_schedule(sizes, budget, lag):
     items, res = B.lamb_layout_schedule(sizes, budget, lag)
-    nk = [(s + 1023) // 1024 for s in sizes]
+    nk = [(s + 511) // 512 for s in sizes]
     first = np.concatenate([[0], np.cumsum(nk)[:-1]]).astype(np.int64)
     owner = np.repeat(np.arange(len(sizes)), nk)
     chunk = (items >> 1).astype(np.int64)
