@@ -11,6 +11,8 @@ read as one parameter tensor) at a time, following the paper
 (You et al., ICLR 2020):
 
 * ``lamb_tensor``   -- Algorithm 2 (LAMB), steps in the algorithm's order.
+* ``nlamb_tensor``  -- Algorithms 3 and 4 of the appendix (N-LAMB, NN-LAMB:
+                       Nesterov momentum in the first, or both, moments).
 * ``lars_tensor``   -- Algorithm 1 (LARS).
 * ``layerwise_step``-- the general strategy of Section 3: a base update u is
                        normalised per block and rescaled by phi(||x||).
@@ -38,6 +40,16 @@ Q7  LARS takes an extra trust coefficient kappa: ratio = kappa*phi(||x||)/||m||
 Q8  Masked tensors still get the trust ratio; the mask removes decay only.
 Q9  Bias correction uses beta**t in float64 with an integer t >= 1.
 Q15 Non-finite inputs are not masked; NaN/Inf propagate.
+Q12 N-LAMB / NN-LAMB (appendix): the superscripted beta_1^t is the t-th term
+    of a momentum schedule (the input line lists the schedule separately from
+    the constant beta1 of the moment recurrence); it is Dozat's Nadam
+    schedule, which the appendix cites and whose settings it uses:
+    mu_t = beta1 * (1 - 0.5 * 0.96^(t * psi)).  The products prod_{i<=t} mu_i
+    are carried from step to step as optimizer state.  N-LAMB keeps Adam's
+    second moment ("the second moment of Adam was unchanged"), so its
+    v_hat = v_t / (1 - beta2^t); the extra beta2 factor printed in Alg. 3 is
+    read as a typo.  In NN-LAMB the second-moment schedule is constant
+    (beta2), since the algorithm's inputs give none.
 
 Input conventions: arrays may be float32 (or bfloat16 bit patterns given as
 uint16 together with ``g_dtype="bf16"``); they are converted exactly to
@@ -62,6 +74,9 @@ __all__ = [
     "lamb_tensor",
     "lars_tensor",
     "lamb_tensor_scalar",
+    "nadam_mu",
+    "nlamb_tensor",
+    "NLambResult",
     "lamb_step",
     "lars_step",
 ]
@@ -224,6 +239,68 @@ def lars_tensor(w, g, m, *, lr: float, beta1: float = 0.9,
         x, m_t, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u,
         trust_coef=trust_coef)
     return LarsResult(x_new, m_t, ratio, xn, un)
+
+
+def nadam_mu(t: int, beta1: float, psi: float) -> float:
+    """Momentum schedule term mu_t = beta1 * (1 - 0.5 * 0.96^(t psi)) (Dozat's
+    Nadam schedule; reading Q12 of the N-LAMB superscripts)."""
+    return beta1 * (1.0 - 0.5 * 0.96 ** (t * psi))
+
+
+@dataclass
+class NLambResult:
+    w: np.ndarray
+    m: np.ndarray
+    v: np.ndarray
+    mu_product: float   # prod_{i <= t} mu_i, carried to the next step
+    ratio: float
+    wnorm: float
+    unorm: float
+
+
+def nlamb_tensor(w, g, m, v, *, t: int, lr: float, mu_product: float,
+                 beta1: float = 0.975, beta2: float = 0.999, eps: float = 1e-8,
+                 psi: float = 0.004, weight_decay: float = 0.01,
+                 decay: bool = True, nesterov_second_moment: bool = False,
+                 phi_kind: str = "identity", gamma_l: float = 0.0,
+                 gamma_u: float = math.inf, g_dtype: str = "f32") -> NLambResult:
+    """One N-LAMB (Algorithm 3) or, with nesterov_second_moment, NN-LAMB
+    (Algorithm 4) step on one block, in float64.
+
+    mu_product is prod_{i < t} mu_i from the previous steps (1 at t = 1).
+      m_t   = beta1 m + (1-beta1) g
+      m_hat = mu_{t+1} m_t / (1 - prod_{i<=t+1} mu_i)
+              + (1 - mu_t) g / (1 - prod_{i<=t} mu_i)
+      v_t   = beta2 v + (1-beta2) g^2
+      v_hat = v_t / (1 - beta2^t)                                (N-LAMB)
+            = beta2 v_t / (1 - beta2^(t+1)) + (1-beta2) g^2 / (1 - beta2^t)
+                                                                 (NN-LAMB)
+      r = m_hat / (sqrt(v_hat) + eps); then the layerwise step on r + lambda x.
+    """
+    if t < 1:
+        raise ValueError("step count t must be >= 1")
+    x = to_f64(w)
+    gt = to_f64(g, g_dtype)
+    m_prev = to_f64(m)
+    v_prev = to_f64(v)
+    lam = weight_decay if decay else 0.0
+    mu_t = nadam_mu(t, beta1, psi)
+    mu_next = nadam_mu(t + 1, beta1, psi)
+    prod_t = mu_product * mu_t
+    prod_next = prod_t * mu_next
+    m_t = beta1 * m_prev + (1.0 - beta1) * gt
+    m_hat = mu_next * m_t / (1.0 - prod_next) + (1.0 - mu_t) * gt / (1.0 - prod_t)
+    v_t = beta2 * v_prev + (1.0 - beta2) * (gt * gt)
+    if nesterov_second_moment:
+        v_hat = (beta2 * v_t / (1.0 - beta2 ** (t + 1))
+                 + (1.0 - beta2) * (gt * gt) / (1.0 - beta2 ** t))
+    else:
+        v_hat = v_t / (1.0 - beta2 ** t)
+    r_t = m_hat / (np.sqrt(v_hat) + eps)
+    u = r_t + lam * x
+    x_new, ratio, xn, un = layerwise_step(
+        x, u, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u)
+    return NLambResult(x_new, m_t, v_t, prod_t, ratio, xn, un)
 
 
 def lamb_tensor_scalar(w, g, m, v, *, t, lr, beta1=0.9, beta2=0.999, eps=1e-6,
