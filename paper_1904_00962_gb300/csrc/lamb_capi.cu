@@ -98,7 +98,7 @@ struct lamb_plan {
   uint32_t* status = nullptr;
   uint32_t* counters = nullptr;
   // single-touch tables
-  uint32_t* items = nullptr;
+  uint2* items = nullptr;
   FusedChunk* fchunks = nullptr;
   FusedTensor* ftensors = nullptr;
   float2* fslots = nullptr;
@@ -343,7 +343,7 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   const size_t o_status = carve(sizeof(uint32_t));
   const size_t o_counters = carve(8 * sizeof(uint32_t));
   const size_t nf = h_fchunks.size(), ng = (size_t)p->n_groups;
-  const size_t o_items = carve(h_items.size() * sizeof(uint32_t));
+  const size_t o_items = carve(h_items.size() * sizeof(uint2));
   const size_t o_fchunks = carve(nf * sizeof(FusedChunk));
   const size_t o_ftensors = carve(n * sizeof(FusedTensor));
   const size_t o_fslots = carve(nf * sizeof(float2));
@@ -369,7 +369,7 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   p->scal = reinterpret_cast<StepScalars*>(base + o_scal);
   p->status = reinterpret_cast<uint32_t*>(base + o_status);
   p->counters = reinterpret_cast<uint32_t*>(base + o_counters);
-  p->items = reinterpret_cast<uint32_t*>(base + o_items);
+  p->items = reinterpret_cast<uint2*>(base + o_items);
   p->fchunks = reinterpret_cast<FusedChunk*>(base + o_fchunks);
   p->ftensors = reinterpret_cast<FusedTensor*>(base + o_ftensors);
   p->fslots = reinterpret_cast<float2*>(base + o_fslots);
@@ -386,9 +386,17 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   if (e == cudaSuccess)
     e = cudaMemcpy(p->tensors, p->h_tensors.data(), n * sizeof(TensorDesc),
                    cudaMemcpyHostToDevice);
-  if (e == cudaSuccess && !h_items.empty())
-    e = cudaMemcpy(p->items, h_items.data(), h_items.size() * sizeof(uint32_t),
+  if (e == cudaSuccess && !h_items.empty()) {
+    // device items carry the tensor and the chunk index directly
+    std::vector<uint2> dev_items(h_items.size());
+    for (size_t i = 0; i < h_items.size(); ++i) {
+      const FusedChunk& fc = h_fchunks[h_items[i] >> 1];
+      dev_items[i] = make_uint2(((uint32_t)fc.tensor << 1) | (h_items[i] & 1u),
+                                (uint32_t)fc.index);
+    }
+    e = cudaMemcpy(p->items, dev_items.data(), dev_items.size() * sizeof(uint2),
                    cudaMemcpyHostToDevice);
+  }
   if (e == cudaSuccess && nf)
     e = cudaMemcpy(p->fchunks, h_fchunks.data(), nf * sizeof(FusedChunk),
                    cudaMemcpyHostToDevice);

@@ -115,7 +115,8 @@ struct __align__(16) FusedTensor {
 };
 
 struct FusedParams {
-  const uint32_t* items;       // (fused chunk << 1) | is_pass2
+  const uint2* items;          // x = (tensor << 1) | is_pass2, y = index of
+                               // the fused chunk inside the tensor
   const FusedChunk* fchunks;
   const FusedTensor* ftensors;
   float2* fslots;              // per fused chunk (sum w^2, sum u^2), fp32

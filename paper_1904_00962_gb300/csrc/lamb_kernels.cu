@@ -582,9 +582,11 @@ __global__ void __launch_bounds__(kThreads)
 // prefetches the operands of its next items with cp.async while it computes
 // the current one, so many bytes are in flight without holding registers.  A
 // pass-2 item is prefetched only if its tensor's norms are already final when
-// it is drawn (its m, v come from other warps' pass-1 stores); otherwise, and
-// for tail chunks and unaligned tensors, the item reads global memory
-// directly when its turn comes.
+// its stage is filled (its m, v come from other warps' pass-1 stores);
+// otherwise, and for tail chunks and unaligned tensors, the item reads global
+// memory directly when its turn comes.  The control traffic (draws, item
+// descriptors, ready flags, tickets) is pipelined as described at the warp
+// worker below.
 //
 // L2 policy: pass-1 loads/stores of m, v, w of "resident" tensors (those
 // whose state fits the L2 budget) are evict_last, so pass 2 -- about one
@@ -764,97 +766,212 @@ __device__ __forceinline__ float4 fused2_pkt(float4 mv, float4 vv, float4 wv,
   return o;
 }
 
-// What one item refers to.
-struct FusedItem {
-  TensorPtrs tp;
-  FusedTensor ft;
-  FusedChunk fc;
-  int chunk;
-  int64_t off;
-  int len;
-  bool pass2;
-};
-
-__device__ __forceinline__ FusedItem fused_item(const StepParams& p,
-                                                const FusedParams& f,
-                                                uint32_t code) {
-  FusedItem it;
-  it.chunk = (int)(code >> 1);
-  it.pass2 = (code & 1u) != 0u;
-  it.fc = f.fchunks[it.chunk];
-  it.ft = f.ftensors[it.fc.tensor];
-  it.tp = p.ptrs[it.fc.tensor];
-  it.off = (int64_t)it.fc.index * kFusedChunk;
-  const int64_t rem = it.ft.numel - it.off;
-  it.len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
-  return it;
+__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ void fence_acq_rel() {
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
 }
 
-// Prefetch the operands of item `code` into `stage` (all lanes).  Returns
-// whether it did: only full chunks of aligned tensors, and pass-2 items only
-// once their tensor's norms are final.
+// Issue the cp.async copies of one full, aligned chunk into `stage`: m, v
+// (LAMB), w, and for pass 1 the gradient.
 template <bool kLars, typename GT>
-__device__ __forceinline__ bool fused_prefetch(const StepParams& p,
-                                               const FusedParams& f,
-                                               uint32_t code, char* stage,
-                                               uint32_t epoch,
-                                               uint64_t pol_first,
-                                               uint64_t pol_last, int lane) {
-  const FusedItem it = fused_item(p, f, code);
-  if (!it.tp.vec_ok || it.len != kFusedChunk) return false;
-  if (it.pass2) {
-    uint32_t ready = 0;
-    if (lane == 0) ready = ld_acquire(&f.ready[it.fc.tensor]) == epoch;
-    if (!__shfl_sync(0xffffffffu, ready, 0)) return false;
-    __syncwarp();
-    (void)ld_acquire(&f.ready[it.fc.tensor]);   // per-lane acquire
-  }
-  const uint64_t pol =
-      (!it.pass2 && it.ft.resident) ? pol_last : pol_first;
+__device__ __forceinline__ void fused_prefetch_ops(
+    const TensorPtrs& tp, int64_t off, bool pass2, bool resident, char* stage,
+    uint64_t pol_first, uint64_t pol_last, int lane) {
+  const uint64_t pol = (!pass2 && resident) ? pol_last : pol_first;
   const uint32_t s = smem_u32(stage);
 #pragma unroll
   for (int u = 0; u < kPktsPerLane; ++u) {
     const int j = lane + 32 * u;                    // 16-byte piece index
-    cp_async16(s + kOffM + 16 * j, it.tp.m + it.off + 4 * j, pol);
-    if (!kLars) cp_async16(s + kOffV + 16 * j, it.tp.v + it.off + 4 * j, pol);
-    cp_async16(s + off_w<kLars>() + 16 * j, it.tp.w + it.off + 4 * j, pol);
+    cp_async16(s + kOffM + 16 * j, tp.m + off + 4 * j, pol);
+    if (!kLars) cp_async16(s + kOffV + 16 * j, tp.v + off + 4 * j, pol);
+    cp_async16(s + off_w<kLars>() + 16 * j, tp.w + off + 4 * j, pol);
   }
-  if (!it.pass2) {
-    const GT* g = static_cast<const GT*>(it.tp.g) + it.off;
+  if (!pass2) {
+    const char* g = reinterpret_cast<const char*>(
+        static_cast<const GT*>(tp.g) + off);
     constexpr int kGPieces = kFusedChunk * (int)sizeof(GT) / 16;
 #pragma unroll
     for (int u = 0; u < kGPieces / 32; ++u) {
       const int j = lane + 32 * u;
-      cp_async16(s + off_g<kLars>() + 16 * j,
-                 reinterpret_cast<const char*>(g) + 16 * j, pol_first);
+      cp_async16(s + off_g<kLars>() + 16 * j, g + 16 * j, pol_first);
     }
   }
-  return true;
 }
 
-// Publish a pass-1 chunk's sums; the last chunk of a group and the last group
-// of a tensor do the fixed-order fp64 combines and release the tensor.
-template <bool kLars>
-__device__ __forceinline__ void fused_publish(const StepParams& p,
-                                           const FusedParams& f,
-                                           const FusedTensor& ft,
-                                           const FusedChunk& fc, int chunk,
-                                           float sw, float su, uint32_t epoch,
-                                           int lane) {
-  sw = warp_sum(sw);
-  su = warp_sum(su);
-  __syncwarp();
-  const int gl = fc.index / kGroup;
-  const int group = ft.first_group + gl;
-  const int gsize = min(kGroup, ft.n_chunks - gl * kGroup);
-  uint32_t last = 0;
-  if (lane == 0) {
-    f.fslots[chunk] = make_float2(sw, su);
-    // release: this warp's m, v stores and the slot become visible first
-    last = atom_add_acq_rel(&f.gtickets[group], 1u) + 1u == (uint32_t)gsize;
+// Pass 1 of a staged chunk: new m, v into registers, sums of w^2 and u^2.
+template <bool kLars, typename GT>
+__device__ __forceinline__ void fused1_from_stage(const char* stage,
+                                                  float lam,
+                                                  const LambConsts& k,
+                                                  float4* mo, float4* vo,
+                                                  float& sw, float& su,
+                                                  int lane) {
+  const GT* tag = nullptr;
+#pragma unroll
+  for (int u = 0; u < kPktsPerLane; ++u) {
+    const int j = lane + 32 * u;
+    mo[u] = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
+    vo[u] = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
+                  : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
+    const float4 wv =
+        *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
+    const float4 gv = lds_grad4(stage + off_g<kLars>(), j, tag);
+    fused1_pkt<kLars>(gv, mo[u], vo[u], wv, lam, k, sw, su);
   }
-  if (!__shfl_sync(0xffffffffu, last, 0)) return;
+}
+
+template <bool kLars>
+__device__ __forceinline__ void fused1_store(const TensorPtrs& tp,
+                                             int64_t off, const float4* mo,
+                                             const float4* vo,
+                                             uint64_t pol_keep, int lane) {
+#pragma unroll
+  for (int u = 0; u < kPktsPerLane; ++u) {
+    const int j = lane + 32 * u;
+    stp4(tp.m + off + 4 * j, mo[u], pol_keep);
+    if (!kLars) stp4(tp.v + off + 4 * j, vo[u], pol_keep);
+  }
+}
+
+// Pass 1 straight from global memory (tail chunks, unaligned tensors).
+template <bool kLars, typename GT>
+__device__ __forceinline__ void fused1_direct(const TensorPtrs& tp,
+                                              int64_t off, int len, float lam,
+                                              const LambConsts& k, float& sw,
+                                              float& su, uint64_t pol_first,
+                                              uint64_t pol_keep, int lane) {
+  float* __restrict__ m = tp.m + off;
+  float* __restrict__ v = kLars ? nullptr : tp.v + off;
+  const float* __restrict__ w = tp.w + off;
+  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + off;
+  int scalar_from = 0;
+  if (tp.vec_ok) {
+    const int nv = len >> 2;
+#pragma unroll 1
+    for (int base = lane; base < nv; base += 64) {
+      float4 wv[2], mv[2], vv[2], gv[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int j = base + 32 * u;
+        if (j < nv) {
+          gv[u] = ldp_grad4(g + 4 * j, pol_first);
+          mv[u] = ldp4(m + 4 * j, pol_keep);
+          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_keep);
+          wv[u] = ldp4(w + 4 * j, pol_keep);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int j = base + 32 * u;
+        if (j < nv) {
+          fused1_pkt<kLars>(gv[u], mv[u], vv[u], wv[u], lam, k, sw, su);
+          stp4(m + 4 * j, mv[u], pol_keep);
+          if (!kLars) stp4(v + 4 * j, vv[u], pol_keep);
+        }
+      }
+    }
+    scalar_from = nv << 2;
+  }
+  for (int i = scalar_from + lane; i < len; i += 32) {
+    float mi = m[i];
+    float vi = kLars ? 0.f : v[i];
+    fused1_elem<kLars>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
+    m[i] = mi;
+    if (!kLars) v[i] = vi;
+  }
+}
+
+// Pass 2 of a staged chunk: new w into registers.
+template <bool kLars>
+__device__ __forceinline__ void fused2_from_stage(const char* stage, float s,
+                                                  float lam,
+                                                  const LambConsts& k,
+                                                  float4* wo, int lane) {
+#pragma unroll
+  for (int u = 0; u < kPktsPerLane; ++u) {
+    const int j = lane + 32 * u;
+    const float4 mv = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
+    const float4 vv = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
+                            : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
+    const float4 wv =
+        *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
+    wo[u] = fused2_pkt<kLars>(mv, vv, wv, s, lam, k);
+  }
+}
+
+template <bool kCopy>
+__device__ __forceinline__ void fused2_store(const TensorPtrs& tp,
+                                             int64_t off, const float4* wo,
+                                             uint64_t pol_first, int lane) {
+#pragma unroll
+  for (int u = 0; u < kPktsPerLane; ++u) {
+    const int j = lane + 32 * u;
+    stp4(tp.w + off + 4 * j, wo[u], pol_first);
+    if (kCopy) stp_copy4(tp.copy, off + 4 * j, wo[u], pol_first);
+  }
+}
+
+// Pass 2 straight from global memory.
+template <bool kLars, bool kCopy>
+__device__ __forceinline__ void fused2_direct(const TensorPtrs& tp,
+                                              int64_t off, int len, float s,
+                                              float lam, const LambConsts& k,
+                                              uint64_t pol_first, int lane) {
+  float* __restrict__ w = tp.w + off;
+  const float* __restrict__ m = tp.m + off;
+  const float* __restrict__ v = kLars ? nullptr : tp.v + off;
+  int scalar_from = 0;
+  if (tp.vec_ok) {
+    const int nv = len >> 2;
+#pragma unroll 1
+    for (int base = lane; base < nv; base += 64) {
+      float4 wv[2], mv[2], vv[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int j = base + 32 * u;
+        if (j < nv) {
+          mv[u] = ldp4(m + 4 * j, pol_first);
+          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_first);
+          wv[u] = ldp4(w + 4 * j, pol_first);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int j = base + 32 * u;
+        if (j < nv) {
+          const float4 o = fused2_pkt<kLars>(mv[u], vv[u], wv[u], s, lam, k);
+          stp4(w + 4 * j, o, pol_first);
+          if (kCopy) stp_copy4(tp.copy, off + 4 * j, o, pol_first);
+        }
+      }
+    }
+    scalar_from = nv << 2;
+  }
+  for (int i = scalar_from + lane; i < len; i += 32) {
+    const float wi = w[i];
+    const float o = __fmaf_rn(
+        -s, fused2_dir<kLars>(m[i], kLars ? 0.f : v[i], wi, lam, k), wi);
+    w[i] = o;
+    if (kCopy) st_copy1(tp.copy, off + i, o);
+  }
+}
+
+// The warp whose ticket completed group `gl` of tensor `tensor`: fixed-order
+// fp64 sum of the group's chunk sums; the warp that completes the tensor's
+// last group computes its norms and trust ratio and releases ready[tensor].
+template <bool kLars>
+__device__ __forceinline__ void fused_group_combine(const StepParams& p,
+                                                 const FusedParams& f,
+                                                 const FusedTensor& ft,
+                                                 int tensor, int gl, int gsize,
+                                                 uint32_t epoch, int lane) {
   __syncwarp();
+  const int group = ft.first_group + gl;
   double aw = 0.0, au = 0.0;
   if (lane < gsize) {
     const float2 s = __ldcg(&f.fslots[ft.first_chunk + gl * kGroup + lane]);
@@ -863,10 +980,11 @@ __device__ __forceinline__ void fused_publish(const StepParams& p,
   }
   aw = warp_sum_d(aw);
   au = warp_sum_d(au);
+  uint32_t last = 0;
   if (lane == 0) {
     f.gslots[group] = make_double2(aw, au);
     f.gtickets[group] = 0u;
-    last = atom_add_acq_rel(&f.tickets[fc.tensor], 1u) + 1u ==
+    last = atom_add_acq_rel(&f.tickets[tensor], 1u) + 1u ==
            (uint32_t)ft.n_groups;
   }
   if (!__shfl_sync(0xffffffffu, last, 0)) return;
@@ -884,85 +1002,13 @@ __device__ __forceinline__ void fused_publish(const StepParams& p,
     double rho = 1.0;
     if (!(wn == 0.0 || un == 0.0))
       rho = (kLars ? p.trust : 1.0) * phi_of(wn, p) / un;
-    p.ratio[fc.tensor] = rho;
-    p.wnorm[fc.tensor] = wn;
-    p.unorm[fc.tensor] = un;
+    p.ratio[tensor] = rho;
+    p.wnorm[tensor] = wn;
+    p.unorm[tensor] = un;
     if (!isfinite(tw) || !isfinite(tu)) atomicOr(p.status, kStatusNonfinite);
-    f.tickets[fc.tensor] = 0u;
-    st_release(&f.ready[fc.tensor], epoch);
+    f.tickets[tensor] = 0u;
+    st_release(&f.ready[tensor], epoch);
   }
-}
-
-// Pass 1 of one item, operands from the warp's stage or from global memory.
-template <bool kLars, typename GT>
-__device__ __forceinline__ void fused_pass1(const StepParams& p,
-                                            const FusedParams& f,
-                                            const LambConsts& k,
-                                            const FusedItem& it,
-                                            const char* stage, bool staged,
-                                            uint64_t pol_first,
-                                            uint64_t pol_last, uint32_t epoch,
-                                            int lane) {
-  const TensorPtrs& tp = it.tp;
-  const uint64_t pol_keep = it.ft.resident ? pol_last : pol_first;
-  const float lam = it.ft.decay * p.wd;
-  float* __restrict__ m = tp.m + it.off;
-  float* __restrict__ v = kLars ? nullptr : tp.v + it.off;
-  const float* __restrict__ w = tp.w + it.off;
-  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + it.off;
-  float sw = 0.f, su = 0.f;
-  if (staged) {
-#pragma unroll
-    for (int u = 0; u < kPktsPerLane; ++u) {
-      const int j = lane + 32 * u;
-      float4 mv = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
-      float4 vv = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
-                        : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
-      const float4 wv =
-          *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
-      const float4 gv = lds_grad4(stage + off_g<kLars>(), j, g);
-      fused1_pkt<kLars>(gv, mv, vv, wv, lam, k, sw, su);
-      stp4(m + 4 * j, mv, pol_keep);
-      if (!kLars) stp4(v + 4 * j, vv, pol_keep);
-    }
-  } else {
-    int scalar_from = 0;
-    if (tp.vec_ok) {
-      const int nv = it.len >> 2;
-#pragma unroll 1
-      for (int base = lane; base < nv; base += 64) {
-        float4 wv[2], mv[2], vv[2], gv[2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int j = base + 32 * u;
-          if (j < nv) {
-            gv[u] = ldp_grad4(g + 4 * j, pol_first);
-            mv[u] = ldp4(m + 4 * j, pol_keep);
-            if (!kLars) vv[u] = ldp4(v + 4 * j, pol_keep);
-            wv[u] = ldp4(w + 4 * j, pol_keep);
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int j = base + 32 * u;
-          if (j < nv) {
-            fused1_pkt<kLars>(gv[u], mv[u], vv[u], wv[u], lam, k, sw, su);
-            stp4(m + 4 * j, mv[u], pol_keep);
-            if (!kLars) stp4(v + 4 * j, vv[u], pol_keep);
-          }
-        }
-      }
-      scalar_from = nv << 2;
-    }
-    for (int i = scalar_from + lane; i < it.len; i += 32) {
-      float mi = m[i];
-      float vi = kLars ? 0.f : v[i];
-      fused1_elem<kLars>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
-      m[i] = mi;
-      if (!kLars) v[i] = vi;
-    }
-  }
-  fused_publish<kLars>(p, f, it.ft, it.fc, it.chunk, sw, su, epoch, lane);
 }
 
 // Bounded wait of a pass-2 item for its tensor's norms (all lanes).
@@ -992,72 +1038,76 @@ __device__ __forceinline__ bool fused_wait(const StepParams& p,
   return true;
 }
 
-// Pass 2 of one item.
-template <bool kLars, bool kCopy>
-__device__ __forceinline__ void fused_pass2(const StepParams& p,
+// ---------------------------------------------------------------------------
+// The warp worker.  Per warp:
+//   * a data ring of kStages shared-memory stages; the item in a stage had
+//     its operands prefetched with cp.async kStages items earlier;
+//   * a control pipeline one item deep per step: the draw atomic, the item
+//     descriptor load and (pass 2) a relaxed load of the tensor's ready flag
+//     are each issued one item before their results are used;
+//   * a deferred publish: a pass-1 item's ticket is taken one item later (its
+//     stores are long complete, so the release costs little), and the
+//     ticket's answer is looked at one item after that.
+// Before any wait the warp flushes its deferred publishes, so it never waits
+// for work it holds itself.
+// ---------------------------------------------------------------------------
+struct PubState {
+  uint32_t tensor, index;   // pass-1 chunk whose sums are held
+  float sw, su;             // valid in lane 0
+  uint32_t ticket;          // ticket answer (lane 0), for the check step
+  bool pub, chk;            // a publish is pending / a check is pending
+};
+
+__device__ __forceinline__ uint2 invalid_desc() {
+  return make_uint2(0xffffffffu, 0u);
+}
+
+template <bool kLars>
+__device__ __forceinline__ void fused_check(const StepParams& p,
                                             const FusedParams& f,
-                                            const LambConsts& k,
-                                            const FusedItem& it,
-                                            const char* stage, bool staged,
-                                            float lr, uint64_t pol_first,
-                                            uint32_t epoch, int lane) {
-  if (!staged && !fused_wait(p, f, it.fc.tensor, epoch, lane))
-    return;                                         // gave up: leave w as is
-  const TensorPtrs& tp = it.tp;
-  const float lam = it.ft.decay * p.wd;
-  const float s = __double2float_rn((double)lr * __ldcg(&p.ratio[it.fc.tensor]));
-  float* __restrict__ w = tp.w + it.off;
-  const float* __restrict__ m = tp.m + it.off;
-  const float* __restrict__ v = kLars ? nullptr : tp.v + it.off;
-  if (staged) {
-#pragma unroll
-    for (int u = 0; u < kPktsPerLane; ++u) {
-      const int j = lane + 32 * u;
-      const float4 mv = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
-      const float4 vv = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
-                              : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
-      const float4 wv =
-          *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
-      const float4 o = fused2_pkt<kLars>(mv, vv, wv, s, lam, k);
-      stp4(w + 4 * j, o, pol_first);
-      if (kCopy) stp_copy4(tp.copy, it.off + 4 * j, o, pol_first);
-    }
-    return;
+                                            PubState& ps, uint32_t epoch,
+                                            int lane) {
+  if (!ps.chk) return;
+  const FusedTensor ft = f.ftensors[ps.tensor];
+  const int gl = (int)ps.index / kGroup;
+  const int gsize = min(kGroup, ft.n_chunks - gl * kGroup);
+  const uint32_t last =
+      __shfl_sync(0xffffffffu, ps.ticket + 1u == (uint32_t)gsize, 0);
+  ps.chk = false;
+  if (last) fused_group_combine<kLars>(p, f, ft, (int)ps.tensor, gl, gsize,
+                                       epoch, lane);
+}
+
+__device__ __forceinline__ void fused_publish_now(const FusedParams& f,
+                                                  PubState& ps, int lane) {
+  if (!ps.pub) return;
+  if (lane == 0) {
+    const FusedTensor ft = f.ftensors[ps.tensor];
+    f.fslots[ft.first_chunk + ps.index] = make_float2(ps.sw, ps.su);
+    // release: this warp's stores of the chunk's m, v and the slot
+    ps.ticket = atom_add_acq_rel(
+        &f.gtickets[ft.first_group + (int)ps.index / kGroup], 1u);
   }
-  int scalar_from = 0;
-  if (tp.vec_ok) {
-    const int nv = it.len >> 2;
-#pragma unroll 1
-    for (int base = lane; base < nv; base += 64) {
-      float4 wv[2], mv[2], vv[2];
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          mv[u] = ldp4(m + 4 * j, pol_first);
-          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_first);
-          wv[u] = ldp4(w + 4 * j, pol_first);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          const float4 o = fused2_pkt<kLars>(mv[u], vv[u], wv[u], s, lam, k);
-          stp4(w + 4 * j, o, pol_first);
-          if (kCopy) stp_copy4(tp.copy, it.off + 4 * j, o, pol_first);
-        }
-      }
-    }
-    scalar_from = nv << 2;
-  }
-  for (int i = scalar_from + lane; i < it.len; i += 32) {
-    const float wi = w[i];
-    const float o = __fmaf_rn(
-        -s, fused2_dir<kLars>(m[i], kLars ? 0.f : v[i], wi, lam, k), wi);
-    w[i] = o;
-    if (kCopy) st_copy1(tp.copy, it.off + i, o);
-  }
+  ps.pub = false;
+  ps.chk = true;
+}
+
+template <bool kLars>
+__device__ __forceinline__ void fused_publish_step(const StepParams& p,
+                                                   const FusedParams& f,
+                                                   PubState& ps,
+                                                   uint32_t epoch, int lane) {
+  fused_check<kLars>(p, f, ps, epoch, lane);
+  fused_publish_now(f, ps, lane);
+}
+
+template <bool kLars>
+__device__ __forceinline__ void fused_flush(const StepParams& p,
+                                            const FusedParams& f,
+                                            PubState& ps, uint32_t epoch,
+                                            int lane) {
+  fused_publish_step<kLars>(p, f, ps, epoch, lane);
+  fused_check<kLars>(p, f, ps, epoch, lane);
 }
 
 template <bool kLars, typename GT, bool kCopy>
@@ -1104,8 +1154,10 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
   const uint64_t pol_first = policy_evict_first();
   const uint64_t pol_last = policy_evict_last();
   const uint32_t n_items = (uint32_t)f.n_items;
-  char* ring = fused_smem + warp * kStages * stage_bytes<kLars, GT>();
+  constexpr int kSB = stage_bytes<kLars, GT>();
+  char* ring = fused_smem + warp * kStages * kSB;
 
+  // ---- control pipeline --------------------------------------------------
   // Each warp draws indices until it gets one >= n_items, then stops, so it
   // draws exactly one such index.
   uint32_t last_drawn = 0;
@@ -1121,46 +1173,133 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
     }
     return v;
   };
+  auto load_desc = [&](uint32_t i) -> uint2 {
+    return i < n_items ? __ldg(&f.items[i]) : invalid_desc();
+  };
+  auto ready_load = [&](uint2 d) -> uint32_t {
+    if (d.x == 0xffffffffu || (d.x & 1u) == 0u) return 0u;
+    return ld_relaxed(&f.ready[d.x >> 1]);
+  };
+  uint32_t idx_a = draw();
+  uint2 desc_b = load_desc(idx_a);
+  idx_a = draw();
+  uint2 desc_c = desc_b;
+  uint32_t rdy_c = ready_load(desc_c);
+  desc_b = load_desc(idx_a);
+  idx_a = draw();
+  uint32_t synced = 0xffffffffu;   // tensor whose norms this warp acquired
 
-  uint32_t code[kStages];
+  uint2 sd[kStages];
   bool staged[kStages];
-#pragma unroll
-  for (int s = 0; s < kStages; ++s) {
-    const uint32_t i = draw();
-    code[s] = i < n_items ? __ldg(&f.items[i]) : 0xffffffffu;
-    staged[s] = i < n_items &&
-                fused_prefetch<kLars, GT>(p, f, code[s],
-                                          ring + s * stage_bytes<kLars, GT>(),
-                                          epoch, pol_first, pol_last, lane);
+  // fill stage s with desc_c, then advance the control pipeline
+  auto fill_advance = [&](int s) {
+    sd[s] = desc_c;
+    staged[s] = false;
+    if (desc_c.x != 0xffffffffu) {
+      const bool p2 = (desc_c.x & 1u) != 0u;
+      const uint32_t tensor = desc_c.x >> 1;
+      const FusedTensor ft = f.ftensors[tensor];
+      const TensorPtrs tp = p.ptrs[tensor];
+      const int64_t off = (int64_t)desc_c.y * kFusedChunk;
+      bool go = tp.vec_ok && ft.numel - off >= kFusedChunk;
+      if (go && p2) {
+        go = __shfl_sync(0xffffffffu, rdy_c == epoch, 0) != 0;
+        if (go && tensor != synced) {
+          fence_acq_rel();           // acquire: the relaxed load saw the release
+          synced = tensor;
+        }
+      }
+      if (go) {
+        fused_prefetch_ops<kLars, GT>(tp, off, p2, ft.resident != 0u,
+                                      ring + s * kSB, pol_first, pol_last,
+                                      lane);
+        staged[s] = true;
+      }
+    }
     cp_async_commit();
-  }
+    desc_c = desc_b;
+    rdy_c = ready_load(desc_c);
+    desc_b = load_desc(idx_a);
+    idx_a = draw();
+  };
+#pragma unroll
+  for (int s = 0; s < kStages; ++s) fill_advance(s);
+
+  PubState ps;
+  ps.pub = ps.chk = false;
+  ps.tensor = ps.index = 0u;
+  ps.sw = ps.su = 0.f;
+  ps.ticket = 0u;
+
   bool done = false;
   while (!done) {
 #pragma unroll
     for (int s = 0; s < kStages; ++s) {
-      if (code[s] == 0xffffffffu) {
+      const uint2 d = sd[s];
+      if (d.x == 0xffffffffu) {
         done = true;
         break;
       }
-      char* stage = ring + s * stage_bytes<kLars, GT>();
-      cp_async_wait<kStages - 1>();  // this stage's copies have landed
+      char* stage = ring + s * kSB;
+      cp_async_wait<kStages - 1>();   // this stage's copies have landed
       __syncwarp();
-      const FusedItem it = fused_item(p, f, code[s]);
-      if (!it.pass2)
-        fused_pass1<kLars, GT>(p, f, k, it, stage, staged[s], pol_first,
-                               pol_last, epoch, lane);
-      else
-        fused_pass2<kLars, kCopy>(p, f, k, it, stage, staged[s], lr,
-                                  pol_first, epoch, lane);
-      __syncwarp();                  // every lane is done with the stage
-      const uint32_t i = draw();
-      code[s] = i < n_items ? __ldg(&f.items[i]) : 0xffffffffu;
-      staged[s] = i < n_items &&
-                  fused_prefetch<kLars, GT>(p, f, code[s], stage, epoch,
-                                            pol_first, pol_last, lane);
-      cp_async_commit();
+      const bool p2 = (d.x & 1u) != 0u;
+      const uint32_t tensor = d.x >> 1;
+      const FusedTensor ft = f.ftensors[tensor];
+      const TensorPtrs tp = p.ptrs[tensor];
+      const int64_t off = (int64_t)d.y * kFusedChunk;
+      const int64_t rem = ft.numel - off;
+      const int len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
+      const float lam = ft.decay * p.wd;
+      if (!p2) {
+        const uint64_t pol_keep = ft.resident ? pol_last : pol_first;
+        float sw = 0.f, su = 0.f;
+        if (staged[s]) {
+          float4 mo[kPktsPerLane], vo[kPktsPerLane];
+          fused1_from_stage<kLars, GT>(stage, lam, k, mo, vo, sw, su, lane);
+          __syncwarp();               // every lane is done with the stage
+          fill_advance(s);
+          fused_publish_step<kLars>(p, f, ps, epoch, lane);
+          fused1_store<kLars>(tp, off, mo, vo, pol_keep, lane);
+        } else {
+          __syncwarp();
+          fill_advance(s);
+          fused_publish_step<kLars>(p, f, ps, epoch, lane);
+          fused1_direct<kLars, GT>(tp, off, len, lam, k, sw, su, pol_first,
+                                   pol_keep, lane);
+        }
+        ps.sw = warp_sum(sw);
+        ps.su = warp_sum(su);
+        ps.tensor = tensor;
+        ps.index = d.y;
+        ps.pub = true;
+      } else {
+        const float s_upd =
+            staged[s] ? __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]))
+                      : 0.f;
+        if (staged[s]) {
+          float4 wo[kPktsPerLane];
+          fused2_from_stage<kLars>(stage, s_upd, lam, k, wo, lane);
+          __syncwarp();
+          fill_advance(s);
+          fused_publish_step<kLars>(p, f, ps, epoch, lane);
+          fused2_store<kCopy>(tp, off, wo, pol_first, lane);
+        } else {
+          __syncwarp();
+          fill_advance(s);
+          fused_flush<kLars>(p, f, ps, epoch, lane);   // never wait on ourselves
+          if (fused_wait(p, f, (int)tensor, epoch, lane)) {
+            synced = tensor;
+            const float s2 =
+                __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]));
+            fused2_direct<kLars, kCopy>(tp, off, len, s2, lam, k, pol_first,
+                                        lane);
+          }
+        }
+      }
     }
   }
+  fused_flush<kLars>(p, f, ps, epoch, lane);
   cp_async_wait<0>();
   // The warp that drew the last index >= n_items closes the launch.
   const uint32_t warps = gridDim.x * kFusedWarps;
