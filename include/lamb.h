@@ -216,6 +216,32 @@ LAMB_API lamb_status_t lars_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
                         int64_t* d_step, const float* d_lr,
                         cudaStream_t stream);
 
+/* One N-LAMB step (appendix Algorithm 3: Nesterov momentum in the first
+ * moment) or, with nesterov_second_moment = 1, one NN-LAMB step (Algorithm
+ * 4: also in the second moment), over every tensor.  Uses w, g, m, v and
+ * the two-pass kernels (also on a single-touch plan).
+ *   hyper          beta1, beta2, eps, weight_decay, phi as for lamb_step;
+ *                  the bias-correction flag is ignored (the Nesterov forms
+ *                  carry their own corrections); INCREMENT_STEP honoured
+ *   momentum_decay psi of the momentum schedule read from Algorithm 3's
+ *                  inputs: mu_t = beta1 * (1 - 0.5 * 0.96^(t psi)) (Dozat's
+ *                  Nadam schedule; psi = 0.004 is its usual value)
+ *   d_step         DEVICE int64 t >= 1 (required)
+ *   d_lr           DEVICE float eta_t
+ *   d_mu_product   DEVICE double: prod_{i<t} mu_i on entry (1.0 before the
+ *                  first step), replaced by prod_{i<=t} mu_i when the step
+ *                  completes -- optimizer state, like m and v
+ * With u = (mu_{t+1} m_t / (1 - prod_{i<=t+1} mu_i) + (1 - mu_t) g /
+ * (1 - prod_{i<=t} mu_i)) / (sqrt(v_hat) + eps) + lambda_k w, v_hat =
+ * v_t / (1 - beta2^t) (N-LAMB) or beta2 v_t / (1 - beta2^(t+1)) + (1 -
+ * beta2) g^2 / (1 - beta2^t) (NN-LAMB), the update is w <- w - eta
+ * phi(||w||)/||u|| u as in lamb_step.  Capturable like lamb_step. */
+LAMB_API lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                                  double momentum_decay,
+                                  int32_t nesterov_second_moment,
+                                  int64_t* d_step, const float* d_lr,
+                                  double* d_mu_product, cudaStream_t stream);
+
 /* DEVICE arrays [n_tensors] of the last step's trust ratio rho_k, ||w_k||
  * and ||r_k|| (LARS: ||m_k||), in double.  Owned by the plan; valid until
  * destroy; overwritten by the next step.  Any out pointer may be NULL. */

@@ -45,7 +45,8 @@ EXPORTED = ["lamb_plan_create", "lamb_plan_bind", "lamb_step", "lars_step",
             "lamb_plan_query", "lamb_plan_get_info",
             "lamb_plan_set_timing", "lamb_plan_read_timing",
             "lamb_plan_destroy", "lamb_layout_chunks", "lamb_last_error",
-            "lamb_abi_version", "lamb_step_noalloc", "lamb_layout_schedule"]
+            "lamb_abi_version", "lamb_step_noalloc", "lamb_layout_schedule",
+            "nlamb_step"]
 
 
 class LambError(RuntimeError):
@@ -112,6 +113,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                    POINTER(vp), POINTER(vp), vp]
     for name in ("lamb_step", "lars_step"):
         getattr(lib, name).argtypes = [vp, POINTER(lamb_hyper_t), vp, vp, vp]
+    lib.nlamb_step.argtypes = [vp, POINTER(lamb_hyper_t), c_double, c_int32,
+                               vp, vp, vp, vp]
     lib.lamb_plan_trust_ratios.argtypes = [vp, POINTER(vp), POINTER(vp),
                                            POINTER(vp)]
     lib.lamb_plan_copy_trust_ratios.argtypes = [vp, vp, vp, vp, vp]
@@ -211,6 +214,16 @@ def lars_step(plan, hyper: lamb_hyper_t, d_step, d_lr, stream=0) -> None:
     _check(load().lars_step(c_void_p(plan), byref(hyper),
                             c_void_p(d_step or None), c_void_p(d_lr or None),
                             c_void_p(stream or None)))
+
+
+def nlamb_step(plan, hyper: lamb_hyper_t, momentum_decay, nesterov_second_moment,
+               d_step, d_lr, d_mu_product, stream=0) -> None:
+    _check(load().nlamb_step(c_void_p(plan), byref(hyper),
+                             float(momentum_decay),
+                             int(bool(nesterov_second_moment)),
+                             c_void_p(d_step or None), c_void_p(d_lr or None),
+                             c_void_p(d_mu_product or None),
+                             c_void_p(stream or None)))
 
 
 def lamb_plan_trust_ratios(plan):

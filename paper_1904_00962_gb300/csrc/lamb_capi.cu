@@ -603,6 +603,46 @@ lamb_status_t lars_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
   return run_step(plan, hyper, d_step, d_lr, stream, false);
 }
 
+lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                         double momentum_decay, int32_t nesterov_second_moment,
+                         int64_t* d_step, const float* d_lr,
+                         double* d_mu_product, cudaStream_t stream) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  lamb_status_t st = check_hyper(hyper, true);
+  if (st != LAMB_OK) return st;
+  if (!(momentum_decay >= 0.0 && std::isfinite(momentum_decay)))
+    return fail(LAMB_ERR_INVALID_ARG, "momentum_decay must be finite, >= 0");
+  if (nesterov_second_moment != 0 && nesterov_second_moment != 1)
+    return fail(LAMB_ERR_INVALID_ARG, "nesterov_second_moment must be 0 or 1");
+  if (!plan->bound) return fail(LAMB_ERR_NOT_BOUND, "plan is not bound");
+  if (!plan->has_v)
+    return fail(LAMB_ERR_NOT_BOUND, "nlamb_step needs v: bind v pointers");
+  if (!d_step || !d_lr || !d_mu_product)
+    return fail(LAMB_ERR_INVALID_ARG, "d_step, d_lr and d_mu_product are required");
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  StepParams sp;
+  fill_params(plan, hyper, d_step, d_lr, &sp);
+  sp.psi = momentum_decay;
+  sp.d_mu_product = d_mu_product;
+  const int nest = nesterov_second_moment ? 2 : 1;
+  const bool timed = plan->timing && plan->timed_steps < kMaxTimedSteps;
+  cudaEvent_t* ev = timed ? &plan->events[(size_t)plan->timed_steps *
+                                          (kKernelsPerStep + 1)]
+                          : nullptr;
+  int rc = timed ? (int)cudaEventRecord(ev[0], stream) : 0;
+  if (!rc)
+    rc = launch_nlamb_pass1(sp, nest, plan->grad_bf16, plan->grid[0], stream);
+  if (!rc && timed) rc = (int)cudaEventRecord(ev[1], stream);
+  if (!rc)
+    rc = launch_nlamb_pass2(sp, nest, plan->grad_bf16, plan->copy_bf16,
+                            plan->grid[1], stream);
+  if (!rc && timed) rc = (int)cudaEventRecord(ev[2], stream);
+  if (rc) return cuda_fail((cudaError_t)rc, "nlamb_step");
+  if (timed) ++plan->timed_steps;
+  return LAMB_OK;
+}
+
 lamb_status_t lamb_plan_trust_ratios(lamb_plan_t plan, const double** d_ratio,
                                      const double** d_wnorm,
                                      const double** d_unorm) {

@@ -54,7 +54,9 @@ struct __align__(16) StepScalars {
   float c2;         // 1/(1-beta2^t)
   float lr;
   int32_t skip;     // 1: bad step count, nothing is written
-  int32_t pad[2];
+  // N-LAMB / NN-LAMB: m_hat = am*m + ag*g, v_hat = bv*v + bg*g^2
+  float am, ag, bv, bg;
+  double mu_prod;   // prod_{i<=t} mu_i, stored back when the step completes
 };
 
 enum : uint32_t { kStatusNonfinite = 1u, kStatusBadStep = 2u,
@@ -84,6 +86,9 @@ struct StepParams {
   int32_t phi;            // 0 identity, 1 clip
   uint32_t flags;
   int32_t n_chunks;
+  // N-LAMB / NN-LAMB only
+  double psi;             // momentum-schedule decay (Nadam's psi)
+  double* d_mu_product;   // prod_{i<t} mu_i on entry, prod_{i<=t} on exit
 };
 
 // ---------------------------------------------------------------------------
@@ -138,6 +143,11 @@ int launch_lars_pass1(const StepParams& p, int grad_bf16, int grid,
                       void* stream);
 int launch_lars_pass2(const StepParams& p, int copy_bf16, int grid,
                       void* stream);
+// N-LAMB (nest = 1) / NN-LAMB (nest = 2), two-pass.
+int launch_nlamb_pass1(const StepParams& p, int nest, int grad_bf16, int grid,
+                       void* stream);
+int launch_nlamb_pass2(const StepParams& p, int nest, int grad_bf16,
+                       int copy_bf16, int grid, void* stream);
 int launch_fused(const StepParams& p, const FusedParams& f, int lars,
                  int grad_bf16, int copy_bf16, int grid, void* stream);
 int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks);

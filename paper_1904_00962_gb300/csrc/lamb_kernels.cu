@@ -43,6 +43,7 @@ struct LambConsts {
   float b1, omb1, b2, omb2;   // beta1, 1-beta1, beta2, 1-beta2
   float c1, c2;               // 1/(1-beta1^t), 1/(1-beta2^t)
   float eps;
+  float am, ag, bv, bg;       // N-LAMB / NN-LAMB direction coefficients
 };
 
 // Alg. 2: m_t = beta1 m + (1-beta1) g ;  v_t = beta2 v + (1-beta2) g^2
@@ -58,6 +59,23 @@ __device__ __forceinline__ float lamb_direction(float m, float v, float w,
                                                 const LambConsts& k) {
   const float mh = __fmul_rn(m, k.c1);
   const float vh = __fmul_rn(v, k.c2);
+  const float den = __fadd_rn(__fsqrt_rn(vh), k.eps);
+  return __fmaf_rn(lam, w, __fdiv_rn(mh, den));
+}
+
+// Appendix Alg. 3 / 4 (N-LAMB / NN-LAMB):
+//   u = (am m_t + ag g) / (sqrt(bv v_t [+ bg g^2]) + eps) + lambda_k w
+// with am = mu_{t+1}/(1 - prod_{i<=t+1} mu_i), ag = (1 - mu_t)/(1 - prod_{i<=t}
+// mu_i); N-LAMB: bv = 1/(1 - beta2^t); NN-LAMB: bv = beta2/(1 - beta2^(t+1)),
+// bg = (1 - beta2)/(1 - beta2^t).
+template <int kNest>
+__device__ __forceinline__ float nlamb_direction(float m, float v, float g,
+                                                 float w, float lam,
+                                                 const LambConsts& k) {
+  const float mh = __fmaf_rn(k.am, m, __fmul_rn(k.ag, g));
+  const float vh = kNest == 2
+                       ? __fmaf_rn(k.bv, v, __fmul_rn(k.bg, __fmul_rn(g, g)))
+                       : __fmul_rn(v, k.bv);
   const float den = __fadd_rn(__fsqrt_rn(vh), k.eps);
   return __fmaf_rn(lam, w, __fdiv_rn(mh, den));
 }
@@ -214,18 +232,19 @@ __device__ __forceinline__ bool retire(const StepParams& p, int which,
 // ---------------------------------------------------------------------------
 // LAMB pass 1
 // ---------------------------------------------------------------------------
-template <typename GT>
+template <int kNest>
 __device__ __forceinline__ void lamb1_elem(float g, float& m, float& v,
                                            float w, float lam,
                                            const LambConsts& k, float& sw,
                                            float& su) {
   lamb_moments(g, m, v, k);
-  const float u = lamb_direction(m, v, w, lam, k);
+  const float u = kNest ? nlamb_direction<kNest>(m, v, g, w, lam, k)
+                        : lamb_direction(m, v, w, lam, k);
   sw = __fmaf_rn(w, w, sw);
   su = __fmaf_rn(u, u, su);
 }
 
-template <typename GT>
+template <typename GT, int kNest>
 __device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
                                             const ChunkDesc& ch, float lam,
                                             const LambConsts& k, float& sw,
@@ -254,10 +273,10 @@ __device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
       for (int u = 0; u < kUnroll1; ++u) {
         const int j = base + u * kThreads;
         if (j < nv) {
-          lamb1_elem<GT>(gv[u].x, mv[u].x, vv[u].x, wv[u].x, lam, k, sw, su);
-          lamb1_elem<GT>(gv[u].y, mv[u].y, vv[u].y, wv[u].y, lam, k, sw, su);
-          lamb1_elem<GT>(gv[u].z, mv[u].z, vv[u].z, wv[u].z, lam, k, sw, su);
-          lamb1_elem<GT>(gv[u].w, mv[u].w, vv[u].w, wv[u].w, lam, k, sw, su);
+          lamb1_elem<kNest>(gv[u].x, mv[u].x, vv[u].x, wv[u].x, lam, k, sw, su);
+          lamb1_elem<kNest>(gv[u].y, mv[u].y, vv[u].y, wv[u].y, lam, k, sw, su);
+          lamb1_elem<kNest>(gv[u].z, mv[u].z, vv[u].z, wv[u].z, lam, k, sw, su);
+          lamb1_elem<kNest>(gv[u].w, mv[u].w, vv[u].w, wv[u].w, lam, k, sw, su);
           st4(m + 4 * j, mv[u]);
           st4(v + 4 * j, vv[u]);
         }
@@ -267,13 +286,20 @@ __device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
   }
   for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
     float mi = m[i], vi = v[i];
-    lamb1_elem<GT>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
+    lamb1_elem<kNest>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
     m[i] = mi;
     v[i] = vi;
   }
 }
 
-template <typename GT>
+// Nadam momentum schedule term (appendix Alg. 3 inputs): mu_t =
+// beta1 (1 - 0.5 * 0.96^(t psi)); pow is CUDA's, in fp64.
+__device__ __forceinline__ double nadam_mu(double beta1, double psi,
+                                           int64_t t) {
+  return beta1 * (1.0 - 0.5 * pow(0.96, (double)t * psi));
+}
+
+template <typename GT, int kNest>
 __global__ void __launch_bounds__(kThreads)
     lamb_pass1_kernel(const StepParams p) {
   __shared__ float red[2][kWarps];
@@ -281,15 +307,32 @@ __global__ void __launch_bounds__(kThreads)
   __shared__ int s_last, s_skip;
   __shared__ LambConsts s_k;
   if (threadIdx.x == 0) {
-    const bool bc = (p.flags & kFlagBiasCorrection) != 0;
+    const bool bc = kNest != 0 || (p.flags & kFlagBiasCorrection) != 0;
     const int64_t t = p.d_step ? *p.d_step : int64_t(1);
     const int skip = (bc && t < 1) ? 1 : 0;
     float c1 = 1.f, c2 = 1.f;
-    if (bc && !skip) {  // Alg. 2 bias correction, beta^t in fp64
+    if (!kNest && bc && !skip) {  // Alg. 2 bias correction, beta^t in fp64
       c1 = (float)(1.0 / (1.0 - pow(p.beta1, (double)t)));
       c2 = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
     }
-    s_k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps};
+    LambConsts kc{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps,
+                  0.f, 0.f, 0.f, 0.f};
+    double mu_prod = 0.0;
+    if (kNest && !skip) {  // appendix Alg. 3 / 4 coefficients, fp64
+      const double mu_t = nadam_mu(p.beta1, p.psi, t);
+      const double mu_n = nadam_mu(p.beta1, p.psi, t + 1);
+      mu_prod = *p.d_mu_product * mu_t;
+      const double prod_n = mu_prod * mu_n;
+      kc.am = (float)(mu_n / (1.0 - prod_n));
+      kc.ag = (float)((1.0 - mu_t) / (1.0 - mu_prod));
+      if (kNest == 2) {
+        kc.bv = (float)(p.beta2 / (1.0 - pow(p.beta2, (double)(t + 1))));
+        kc.bg = (float)((1.0 - p.beta2) / (1.0 - pow(p.beta2, (double)t)));
+      } else {
+        kc.bv = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
+      }
+    }
+    s_k = kc;
     s_skip = skip;
     if (blockIdx.x == 0) {
       StepScalars sc{};
@@ -298,6 +341,11 @@ __global__ void __launch_bounds__(kThreads)
       sc.c2 = c2;
       sc.lr = *p.d_lr;
       sc.skip = skip;
+      sc.am = kc.am;
+      sc.ag = kc.ag;
+      sc.bv = kc.bv;
+      sc.bg = kc.bg;
+      sc.mu_prod = mu_prod;
       *p.scal = sc;
       if (skip) atomicOr(p.status, kStatusBadStep);
     }
@@ -315,7 +363,7 @@ __global__ void __launch_bounds__(kThreads)
     const TensorPtrs tp = p.ptrs[ch.tensor];
     const float lam = td.decay * p.wd;
     float sw = 0.f, su = 0.f;
-    lamb1_chunk<GT>(tp, ch, lam, k, sw, su);
+    lamb1_chunk<GT, kNest>(tp, ch, lam, k, sw, su);
     publish_chunk(p, (int)c, ch, td, sw, su, red, &s_last, 1.0);
     ++it;
     c = s_next[it & 1];
@@ -326,19 +374,28 @@ __global__ void __launch_bounds__(kThreads)
 // ---------------------------------------------------------------------------
 // LAMB pass 2
 // ---------------------------------------------------------------------------
-template <bool kCopy>
+// Pass-2 direction: LAMB from m, v, w; N-LAMB / NN-LAMB also need g.
+template <int kNest>
+__device__ __forceinline__ float lamb2_dir(float m, float v, float g, float w,
+                                           float lam, const LambConsts& k) {
+  return kNest ? nlamb_direction<kNest>(m, v, g, w, lam, k)
+               : lamb_direction(m, v, w, lam, k);
+}
+
+template <bool kCopy, int kNest, typename GT>
 __device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
                                             const ChunkDesc& ch, float lam,
                                             float s, const LambConsts& k) {
   float* __restrict__ w = tp.w + ch.offset;
   const float* __restrict__ m = tp.m + ch.offset;
   const float* __restrict__ v = tp.v + ch.offset;
+  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + ch.offset;
   const int n = ch.len;
   int scalar_from = 0;
   if (tp.vec_ok) {
     const int nv = n >> 2;
     for (int base = threadIdx.x; base < nv; base += kThreads * kUnroll2) {
-      float4 wv[kUnroll2], mv[kUnroll2], vv[kUnroll2];
+      float4 wv[kUnroll2], mv[kUnroll2], vv[kUnroll2], gv[kUnroll2];
 #pragma unroll
       for (int u = 0; u < kUnroll2; ++u) {
         const int j = base + u * kThreads;
@@ -346,6 +403,7 @@ __device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
           mv[u] = ld4_last(m + 4 * j);
           vv[u] = ld4_last(v + 4 * j);
           wv[u] = ld4_last(w + 4 * j);
+          if (kNest) gv[u] = ld_grad4(g + 4 * j);
         }
       }
 #pragma unroll
@@ -353,10 +411,11 @@ __device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
         const int j = base + u * kThreads;
         if (j < nv) {
           float4 o;
-          o.x = __fmaf_rn(-s, lamb_direction(mv[u].x, vv[u].x, wv[u].x, lam, k), wv[u].x);
-          o.y = __fmaf_rn(-s, lamb_direction(mv[u].y, vv[u].y, wv[u].y, lam, k), wv[u].y);
-          o.z = __fmaf_rn(-s, lamb_direction(mv[u].z, vv[u].z, wv[u].z, lam, k), wv[u].z);
-          o.w = __fmaf_rn(-s, lamb_direction(mv[u].w, vv[u].w, wv[u].w, lam, k), wv[u].w);
+          if (!kNest) gv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+          o.x = __fmaf_rn(-s, lamb2_dir<kNest>(mv[u].x, vv[u].x, gv[u].x, wv[u].x, lam, k), wv[u].x);
+          o.y = __fmaf_rn(-s, lamb2_dir<kNest>(mv[u].y, vv[u].y, gv[u].y, wv[u].y, lam, k), wv[u].y);
+          o.z = __fmaf_rn(-s, lamb2_dir<kNest>(mv[u].z, vv[u].z, gv[u].z, wv[u].z, lam, k), wv[u].z);
+          o.w = __fmaf_rn(-s, lamb2_dir<kNest>(mv[u].w, vv[u].w, gv[u].w, wv[u].w, lam, k), wv[u].w);
           st4_last(w + 4 * j, o);
           if (kCopy) st_copy4(tp.copy, ch.offset + 4 * j, o);
         }
@@ -366,19 +425,22 @@ __device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
   }
   for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
     const float wi = w[i];
-    const float o = __fmaf_rn(-s, lamb_direction(m[i], v[i], wi, lam, k), wi);
+    const float gi = kNest ? ld_grad1(g + i) : 0.f;
+    const float o =
+        __fmaf_rn(-s, lamb2_dir<kNest>(m[i], v[i], gi, wi, lam, k), wi);
     w[i] = o;
     if (kCopy) st_copy1(tp.copy, ch.offset + i, o);
   }
 }
 
-template <bool kCopy>
+template <bool kCopy, int kNest, typename GT>
 __global__ void __launch_bounds__(kThreads)
     lamb_pass2_kernel(const StepParams p) {
   __shared__ uint32_t s_next[2];
   const StepScalars sc = *p.scal;
   if (sc.skip) return;
-  const LambConsts k{p.b1, p.omb1, p.b2, p.omb2, sc.c1, sc.c2, p.eps};
+  const LambConsts k{p.b1, p.omb1, p.b2, p.omb2, sc.c1, sc.c2, p.eps,
+                     sc.am, sc.ag, sc.bv, sc.bg};
   if (threadIdx.x == 0) s_next[0] = atomicAdd(&p.counters[1], 1u);
   __syncthreads();
   int it = 0;
@@ -392,14 +454,15 @@ __global__ void __launch_bounds__(kThreads)
     const TensorPtrs tp = p.ptrs[ch.tensor];
     const float lam = td.decay * p.wd;
     const float s = __double2float_rn((double)sc.lr * p.ratio[ch.tensor]);
-    lamb2_chunk<kCopy>(tp, ch, lam, s, k);
+    lamb2_chunk<kCopy, kNest, GT>(tp, ch, lam, s, k);
     __syncthreads();  // s_next[(it+1)&1] visible; old slot free to reuse
     ++it;
     c = s_next[it & 1];
   }
-  if (retire(p, 1, c) && threadIdx.x == 0 &&
-      (p.flags & kFlagIncrementStep) && p.d_step)
-    *p.d_step = sc.t + 1;
+  if (retire(p, 1, c) && threadIdx.x == 0) {
+    if (kNest && p.d_mu_product) *p.d_mu_product = sc.mu_prod;
+    if ((p.flags & kFlagIncrementStep) && p.d_step) *p.d_step = sc.t + 1;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1052,9 +1115,10 @@ __device__ __forceinline__ bool fused_wait(const StepParams& p,
 // for work it holds itself.
 // ---------------------------------------------------------------------------
 struct PubState {
-  uint32_t tensor, index;   // pass-1 chunk whose sums are held
-  float sw, su;             // valid in lane 0
-  uint32_t ticket;          // ticket answer (lane 0), for the check step
+  uint32_t tensor, index;   // pass-1 chunk whose sums are held (publish)
+  float sw, su;             // its sums, valid in lane 0
+  uint32_t chk_tensor, chk_index;   // chunk whose ticket awaits its check
+  uint32_t ticket;          // that ticket's answer (lane 0)
   bool pub, chk;            // a publish is pending / a check is pending
 };
 
@@ -1068,14 +1132,14 @@ __device__ __forceinline__ void fused_check(const StepParams& p,
                                             PubState& ps, uint32_t epoch,
                                             int lane) {
   if (!ps.chk) return;
-  const FusedTensor ft = f.ftensors[ps.tensor];
-  const int gl = (int)ps.index / kGroup;
+  const FusedTensor ft = f.ftensors[ps.chk_tensor];
+  const int gl = (int)ps.chk_index / kGroup;
   const int gsize = min(kGroup, ft.n_chunks - gl * kGroup);
   const uint32_t last =
       __shfl_sync(0xffffffffu, ps.ticket + 1u == (uint32_t)gsize, 0);
   ps.chk = false;
-  if (last) fused_group_combine<kLars>(p, f, ft, (int)ps.tensor, gl, gsize,
-                                       epoch, lane);
+  if (last) fused_group_combine<kLars>(p, f, ft, (int)ps.chk_tensor, gl,
+                                       gsize, epoch, lane);
 }
 
 __device__ __forceinline__ void fused_publish_now(const FusedParams& f,
@@ -1088,6 +1152,8 @@ __device__ __forceinline__ void fused_publish_now(const FusedParams& f,
     ps.ticket = atom_add_acq_rel(
         &f.gtickets[ft.first_group + (int)ps.index / kGroup], 1u);
   }
+  ps.chk_tensor = ps.tensor;
+  ps.chk_index = ps.index;
   ps.pub = false;
   ps.chk = true;
 }
@@ -1227,7 +1293,7 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
 
   PubState ps;
   ps.pub = ps.chk = false;
-  ps.tensor = ps.index = 0u;
+  ps.tensor = ps.index = ps.chk_tensor = ps.chk_index = 0u;
   ps.sw = ps.su = 0.f;
   ps.ticket = 0u;
 
@@ -1323,9 +1389,37 @@ int launch_lamb_pass1(const StepParams& p, int grad_bf16, int grid,
                       void* stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (grad_bf16)
-    lamb_pass1_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(p);
+    lamb_pass1_kernel<__nv_bfloat16, 0><<<grid, kThreads, 0, s>>>(p);
   else
-    lamb_pass1_kernel<float><<<grid, kThreads, 0, s>>>(p);
+    lamb_pass1_kernel<float, 0><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
+int launch_nlamb_pass1(const StepParams& p, int nest, int grad_bf16, int grid,
+                       void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch ((nest == 2 ? 2 : 0) | (grad_bf16 ? 1 : 0)) {
+    case 0: lamb_pass1_kernel<float, 1><<<grid, kThreads, 0, s>>>(p); break;
+    case 1: lamb_pass1_kernel<__nv_bfloat16, 1><<<grid, kThreads, 0, s>>>(p); break;
+    case 2: lamb_pass1_kernel<float, 2><<<grid, kThreads, 0, s>>>(p); break;
+    default: lamb_pass1_kernel<__nv_bfloat16, 2><<<grid, kThreads, 0, s>>>(p); break;
+  }
+  return (int)cudaGetLastError();
+}
+
+int launch_nlamb_pass2(const StepParams& p, int nest, int grad_bf16,
+                       int copy_bf16, int grid, void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch ((nest == 2 ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0)) {
+    case 0: lamb_pass2_kernel<false, 1, float><<<grid, kThreads, 0, s>>>(p); break;
+    case 1: lamb_pass2_kernel<true, 1, float><<<grid, kThreads, 0, s>>>(p); break;
+    case 2: lamb_pass2_kernel<false, 1, __nv_bfloat16><<<grid, kThreads, 0, s>>>(p); break;
+    case 3: lamb_pass2_kernel<true, 1, __nv_bfloat16><<<grid, kThreads, 0, s>>>(p); break;
+    case 4: lamb_pass2_kernel<false, 2, float><<<grid, kThreads, 0, s>>>(p); break;
+    case 5: lamb_pass2_kernel<true, 2, float><<<grid, kThreads, 0, s>>>(p); break;
+    case 6: lamb_pass2_kernel<false, 2, __nv_bfloat16><<<grid, kThreads, 0, s>>>(p); break;
+    default: lamb_pass2_kernel<true, 2, __nv_bfloat16><<<grid, kThreads, 0, s>>>(p); break;
+  }
   return (int)cudaGetLastError();
 }
 
@@ -1333,9 +1427,9 @@ int launch_lamb_pass2(const StepParams& p, int copy_bf16, int grid,
                       void* stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (copy_bf16)
-    lamb_pass2_kernel<true><<<grid, kThreads, 0, s>>>(p);
+    lamb_pass2_kernel<true, 0, float><<<grid, kThreads, 0, s>>>(p);
   else
-    lamb_pass2_kernel<false><<<grid, kThreads, 0, s>>>(p);
+    lamb_pass2_kernel<false, 0, float><<<grid, kThreads, 0, s>>>(p);
   return (int)cudaGetLastError();
 }
 
@@ -1410,12 +1504,12 @@ int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks) {
 }
 
 int occupancy_lamb_pass1(int grad_bf16, int* blocks) {
-  return grad_bf16 ? occupancy_of(lamb_pass1_kernel<__nv_bfloat16>, blocks)
-                   : occupancy_of(lamb_pass1_kernel<float>, blocks);
+  return grad_bf16 ? occupancy_of(lamb_pass1_kernel<__nv_bfloat16, 0>, blocks)
+                   : occupancy_of(lamb_pass1_kernel<float, 0>, blocks);
 }
 int occupancy_lamb_pass2(int copy_bf16, int* blocks) {
-  return copy_bf16 ? occupancy_of(lamb_pass2_kernel<true>, blocks)
-                   : occupancy_of(lamb_pass2_kernel<false>, blocks);
+  return copy_bf16 ? occupancy_of(lamb_pass2_kernel<true, 0, float>, blocks)
+                   : occupancy_of(lamb_pass2_kernel<false, 0, float>, blocks);
 }
 int occupancy_lars_pass1(int grad_bf16, int* blocks) {
   return grad_bf16 ? occupancy_of(lars_pass1_kernel<__nv_bfloat16>, blocks)

@@ -113,6 +113,14 @@ class LambPlan:
                     d_step.data_ptr() if d_step is not None else 0,
                     d_lr.data_ptr(), _stream(stream))
 
+    def nlamb_step(self, hyper, momentum_decay, nesterov_second_moment,
+                   d_step: torch.Tensor, d_lr: torch.Tensor,
+                   d_mu_product: torch.Tensor, stream=None):
+        B.nlamb_step(self.handle, hyper, momentum_decay,
+                     nesterov_second_moment, d_step.data_ptr(),
+                     d_lr.data_ptr(), d_mu_product.data_ptr(),
+                     _stream(stream))
+
     def results(self, stream=None):
         """(ratio, wnorm, unorm) as new float64 device tensors."""
         dev = self.state.device

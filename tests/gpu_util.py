@@ -129,6 +129,43 @@ def compare_lars(got_w, got_m, ref, w_old, m_old, g64, beta1, lam, tol,
     return {"w": rel_max(ew, sw), "m": rel_max(em, sm), "_sw": sw}
 
 
+def compare_nlamb(got_w, got_m, got_v, ref, w_old, m_old, g64, h, t, lr, lam,
+                  psi, mu_product, nn, tol, w_path=None, m_path=None):
+    """compare_lamb for N-LAMB / NN-LAMB (appendix Algs. 3/4): the same
+    floors, with the update-operand floor built from the Nesterov form."""
+    from oracle import lamb_oracle as O
+    mu_t = O.nadam_mu(t, h.beta1, psi)
+    mu_n = O.nadam_mu(t + 1, h.beta1, psi)
+    p_t = mu_product * mu_t
+    am, ag = mu_n / (1 - p_t * mu_n), (1 - mu_t) / (1 - p_t)
+    if nn:
+        vh = (h.beta2 * ref.v / (1 - h.beta2 ** (t + 1))
+              + (1 - h.beta2) * g64 * g64 / (1 - h.beta2 ** t))
+    else:
+        vh = ref.v / (1 - h.beta2 ** t)
+    m_op = h.beta1 * np.abs(m_old) + (1 - h.beta1) * np.abs(g64)
+    u_op = (am * m_op + ag * np.abs(g64)) / (np.sqrt(vh) + h.eps) + \
+        lam * np.abs(w_old)
+    got_w = got_w.astype(np.float64)
+    got_m = got_m.astype(np.float64)
+    got_v = got_v.astype(np.float64)
+    sw = np.maximum(np.abs(ref.w), np.abs(w_old))
+    if w_path is not None:
+        sw = np.maximum(sw, w_path)
+    if np.isfinite(ref.ratio):
+        sw = np.maximum(sw, lr * ref.ratio * u_op)
+    sm = np.maximum(np.abs(ref.m), m_op)
+    if m_path is not None:
+        sm = np.maximum(sm, m_path)
+    ew, em, ev = (np.abs(got_w - ref.w), np.abs(got_m - ref.m),
+                  np.abs(got_v - ref.v))
+    assert _nan_aware_ok(ew, tol * sw, got_w, ref.w), f"w err {rel_max(ew, sw)}"
+    assert _nan_aware_ok(em, tol * sm, got_m, ref.m), f"m err {rel_max(em, sm)}"
+    assert _nan_aware_ok(ev, tol * np.abs(ref.v), got_v, ref.v), \
+        f"v err {rel_max(ev, np.abs(ref.v))}"
+    return {"w": rel_max(ew, sw), "m": rel_max(em, sm), "_sw": sw}
+
+
 def worst_of(errs):
     return max(v for k, v in errs.items() if not k.startswith("_"))
 
@@ -198,9 +235,15 @@ class GpuLayout:
         else:
             self.plan.lamb_step(hyper, self.d_step, self.d_lr)
 
-    def results(self):
+    def results(self, check_status=True):
+        """Trust ratios and norms of the last step; by default also asserts
+        that the device status word is clear (no non-finite norm, bad step
+        count or abandoned wait)."""
         r, w, u = self.plan.results()
         torch.cuda.synchronize()
+        if check_status:
+            st = self.plan.query()
+            assert st == 0, f"device status 0x{st:x}"
         return r.cpu().numpy(), w.cpu().numpy(), u.cpu().numpy()
 
     def download(self, name, k):

@@ -8,7 +8,7 @@ import pytest
 import torch
 
 from gpu_util import (ALGO_IDS, ALGOS, TOL_CHAIN, TOL_RATIO, TOL_STEP,
-                      GpuLayout, c_hyper,
+                      GpuLayout, c_hyper, compare_nlamb,
                       check_copy, compare_lamb, compare_lars, f32,
                       hyper_kwargs, oracle_map, ratio_ok, worst_of)
 from oracle import lamb_oracle as O
@@ -776,3 +776,115 @@ def test_single_touch_matches_two_pass_within_tolerance():
     d = (w1.double() - w2.double()).abs()
     scale = torch.maximum(w1.double().abs(), w_before.double().abs())
     assert bool(torch.all(d <= TOL_STEP * scale))
+
+
+# ---------------------------------------------------------------------------
+# N-LAMB / NN-LAMB (appendix Algorithms 3 and 4)
+# ---------------------------------------------------------------------------
+
+def _oracle_nlamb(L, k, w, g, m, v, t, lr, h, prod, psi, nn):
+    return O.nlamb_tensor(w, g, m, v, t=t, lr=lr, mu_product=prod,
+                          beta1=h.beta1, beta2=h.beta2, eps=h.eps, psi=psi,
+                          weight_decay=h.weight_decay, decay=bool(L.decay[k]),
+                          nesterov_second_moment=nn, phi_kind=h.phi,
+                          gamma_l=h.gamma_l, gamma_u=h.gamma_u,
+                          g_dtype=L.grad_dtype)
+
+
+@pytest.mark.parametrize("nn", [False, True], ids=["nlamb", "nnlamb"])
+def test_nlamb_chained_mlp_and_edge(nn):
+    """20 chained steps with the step counter and the momentum product
+    advanced on the device, on the MLP and the edge-case layout."""
+    psi = 0.004
+    for L in (W.mlp_layout(), _edge_layout()):
+        h = W.Hyper(lr=1e-3, beta1=0.975, beta2=0.999, eps=1e-8,
+                    weight_decay=0.01, phi="clip", gamma_u=10.0)
+        G = GpuLayout(L)
+        G.load_weights()
+        hyp = c_hyper(h, increment=True)
+        d_prod = torch.ones(1, dtype=torch.float64, device="cuda:0")
+        G.d_step.fill_(1)
+        G.d_lr.fill_(f32(h.lr))
+        lr = f32(h.lr)
+        state = [(L.weights(k).astype(np.float64), np.zeros(s), np.zeros(s))
+                 for k, s in enumerate(L.sizes)]
+        path = [np.zeros(s) for s in L.sizes]
+        mpath = [np.zeros(s) for s in L.sizes]
+        prod = 1.0
+        for t in range(1, 21):
+            G.load_grads(t)
+            G.plan.nlamb_step(hyp, psi, nn, G.d_step, G.d_lr, d_prod)
+            ratio, _, _ = G.results()
+            tol = TOL_STEP if t == 1 else TOL_CHAIN
+            new_prod = None
+            for k in range(L.n_tensors):
+                w0, m0, v0 = state[k]
+                g = L.grad(k, t)
+                ref = _oracle_nlamb(L, k, w0, g, m0, v0, t, lr, h, prod, psi, nn)
+                path[k] += np.abs(ref.w - w0)
+                mpath[k] = h.beta1 * mpath[k] + (1 - h.beta1) * np.abs(g)
+                compare_nlamb(G.download("w", k), G.download("m", k),
+                              G.download("v", k), ref, w0, m0,
+                              g.astype(np.float64), h, t, lr,
+                              h.weight_decay * L.decay[k], psi, prod, nn, tol,
+                              w_path=path[k], m_path=mpath[k])
+                assert ratio_ok(ratio[k], ref.ratio,
+                                TOL_RATIO if t == 1 else TOL_CHAIN), (t, k)
+                state[k] = (ref.w, ref.m, ref.v)
+                new_prod = ref.mu_product
+            prod = new_prod
+            assert math.isclose(float(d_prod.item()), prod, rel_tol=1e-14)
+            assert int(G.d_step.item()) == t + 1
+        G.close()
+
+
+@pytest.mark.parametrize("nn", [False, True], ids=["nlamb", "nnlamb"])
+def test_nlamb_bert_large_one_step_every_tensor(nn):
+    """BERT-large layout (bf16 gradients, bf16 copy) at t = 1000 from a warm
+    state, every tensor against the oracle."""
+    L = W.bert_large_layout()
+    h = W.Hyper(lr=2e-3, beta1=0.975, beta2=0.999, eps=1e-8,
+                weight_decay=0.01, phi="clip", gamma_u=10.0)
+    psi, t = 0.004, 1000
+    prod = math.prod(O.nadam_mu(i, h.beta1, psi) for i in range(1, t))
+    G = GpuLayout(L)
+    G.load_weights()
+    G.load_warm_state()
+    G.load_grads(t)
+    lr = f32(h.lr)
+    d_prod = torch.full((1,), prod, dtype=torch.float64, device="cuda:0")
+    G.d_step.fill_(t)
+    G.d_lr.fill_(lr)
+    G.plan.nlamb_step(c_hyper(h), psi, nn, G.d_step, G.d_lr, d_prod)
+    ratio, wn, un = G.results()
+
+    def check(k):
+        w, g = L.weights(k), L.grad(k, t)
+        m, v = L.state_warm(k)
+        ref = _oracle_nlamb(L, k, w, g, m, v, t, lr, h, prod, psi, nn)
+        e = compare_nlamb(G.download("w", k), G.download("m", k),
+                          G.download("v", k), ref, w, m,
+                          O.to_f64(g, L.grad_dtype), h, t, lr,
+                          h.weight_decay * L.decay[k], psi, prod, nn, TOL_STEP)
+        check_copy(G.download("copy", k), G.download("w", k), ref.w,
+                   sw=e["_sw"])
+        assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
+        assert ratio_ok(wn[k], ref.wnorm) and ratio_ok(un[k], ref.unorm), k
+        return ref.mu_product
+
+    prods = oracle_map(check, range(L.n_tensors))
+    assert math.isclose(float(d_prod.item()), prods[0], rel_tol=1e-14)
+    G.close()
+
+
+def test_nlamb_argument_errors():
+    L = W.mlp_layout()
+    G = GpuLayout(L)
+    d_prod = torch.ones(1, dtype=torch.float64, device="cuda:0")
+    h = c_hyper(L.hyper)
+    with pytest.raises(B.LambError):          # negative momentum decay
+        G.plan.nlamb_step(h, -1.0, False, G.d_step, G.d_lr, d_prod)
+    with pytest.raises(B.LambError):          # product state required
+        B.nlamb_step(G.plan.handle, h, 0.004, 0, G.d_step.data_ptr(),
+                     G.d_lr.data_ptr(), 0)
+    G.close()
