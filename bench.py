@@ -67,6 +67,37 @@ KERNELS = {
 }
 
 
+def two_pass_bytes(opt, gb, cb):
+    """Algorithmic bytes per parameter of a two-pass step (g gb bytes,
+    bf16 copy cb bytes)."""
+    if opt == "lars":
+        return (gb + 8 + 4) + (8 + 4 + cb)
+    if opt in ("nlamb", "nnlamb"):
+        return (gb + 12 + 8) + (12 + gb + 4 + cb)
+    return (gb + 12 + 8) + (12 + 4 + cb)
+
+
+def single_touch_bytes(opt, gb, cb):
+    """Bytes per parameter when every operand is read and written once."""
+    if opt == "lars":
+        return gb + 8 + 4 + 4 + cb
+    return gb + 12 + 8 + 4 + cb
+
+
+def kernel_model(opt, algo, gb, cb):
+    """(kernel names, algorithmic bytes per parameter of each kernel)."""
+    if algo == 2 and opt in ("lamb", "lars"):
+        return ([f"fused_step_kernel<{opt},g{8 * gb},copy{8 * cb}>"],
+                [single_touch_bytes(opt, gb, cb)])
+    if opt == "lars":
+        return (["lars_pass1_kernel", "lars_pass2_kernel"],
+                [gb + 8 + 4, 8 + 4 + cb])
+    nest = opt in ("nlamb", "nnlamb")
+    return ([f"{'n' if nest else ''}lamb_pass1_kernel",
+             f"{'n' if nest else ''}lamb_pass2_kernel"],
+            [gb + 12 + 8, 12 + (gb if nest else 0) + 4 + cb])
+
+
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -84,6 +115,12 @@ def parse_args():
                     help="single-touch schedule lag (0 = library default)")
     ap.add_argument("--l2-budget-mb", type=int, default=0,
                     help="single-touch L2 budget (0 = library default)")
+    ap.add_argument("--layout", default="bert_large",
+                    choices=["bert_large", "bert_base", "resnet50", "ragged",
+                             "mlp"],
+                    help="parameter layout (default: the BERT-large headline)")
+    ap.add_argument("--optimizer", default="lamb",
+                    choices=["lamb", "lars", "nlamb", "nnlamb"])
     ap.add_argument("--layers", type=int, default=24,
                     help="encoder layers of the layout (24 = BERT-large; "
                          "fewer only for small profiling captures)")
@@ -193,6 +230,18 @@ class ClockSampler:
                 "sm_max_mhz": max(r[2] for r in sel),
                 "samples": len(sel),
                 "reasons": sorted(reasons)}
+
+
+def max_over_ranks(value: float, device=None) -> float:
+    """Largest `value` over all ranks (the slowest rank's time); identity
+    without an initialised process group."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
 
 
 def dist_env():
@@ -317,32 +366,56 @@ def run_ours(args):
         build_mod.build()
     B.load()
 
-    if args.layers == 24:
-        L = bert_large_layout()
-        workload = "bert_large_layout"
-    else:
+    from paper_1904_00962_gb300.workloads import get_layout
+    if args.layout == "bert_large" and args.layers != 24:
         L = bert_layout(args.layers, 1024, 4096, name="bert_large",
                         grad_dtype="bf16", copy_dtype="bf16",
                         measured_step=1000)
         workload = f"bert_large_layout_{args.layers}_layers"
-    h = L.hyper
+    else:
+        L = get_layout(args.layout)
+        workload = f"{args.layout}_layout"
+    opt = args.optimizer
+    if opt != "lamb":
+        workload += f"_{opt}"
+    lars = opt == "lars"
+    h = L.lars_hyper if (lars and L.lars_hyper) else L.hyper
+    if lars and not L.lars_hyper:
+        h = type(h)(lr=1.0, beta1=0.9, weight_decay=1e-4, trust_coef=1e-3,
+                    bias_correction=False)
     P = L.n_params
-    st = DeviceState(L.sizes, grad_dtype="bf16", copy_dtype="bf16",
-                     device=dev)
+    st = DeviceState(L.sizes, grad_dtype=L.grad_dtype,
+                     copy_dtype=L.copy_dtype, device=dev, with_v=not lars)
     for k in range(L.n_tensors):
         st.upload("w", k, L.weights(k))
         st.upload("g", k, L.grad(k, 1))
     plan = LambPlan(st, L.decay, algorithm=ALGO_CODES[args.algo],
                     lag_items=args.lag_items, l2_budget_mb=args.l2_budget_mb)
     algo = plan.info()["algorithm"]
-    kernel_names, kernel_bytes, profile_file = KERNELS[algo]
+    kernel_names, kernel_bytes = kernel_model(
+        opt, algo, 2 if L.grad_dtype == "bf16" else 4,
+        2 if L.copy_dtype == "bf16" else 0)
+    profile_file = KERNELS[algo][2] if (
+        args.layout == "bert_large" and opt == "lamb") else None
     d_step = torch.ones(1, dtype=torch.int64, device=dev)
     d_lr = torch.full((1,), float(np.float32(h.lr)), dtype=torch.float32,
                       device=dev)
+    d_prod = torch.ones(1, dtype=torch.float64, device=dev)
     hyper = B.make_hyper(beta1=h.beta1, beta2=h.beta2, eps=h.eps,
                          weight_decay=h.weight_decay, phi=h.phi,
                          gamma_l=h.gamma_l, gamma_u=h.gamma_u,
-                         bias_correction=True, increment_step=True)
+                         trust_coef=h.trust_coef,
+                         bias_correction=not lars, increment_step=True)
+
+    def one_step():
+        if opt == "lamb":
+            plan.lamb_step(hyper, d_step, d_lr)
+        elif opt == "lars":
+            plan.lars_step(hyper, d_step, d_lr)
+        else:
+            plan.nlamb_step(hyper, 0.004, opt == "nnlamb", d_step, d_lr,
+                            d_prod)
+
     stream = torch.cuda.current_stream(dev)
 
     def barrier():
@@ -352,7 +425,7 @@ def run_ours(args):
 
     # warm-up: t = 1..W from m = v = 0, then jump to the measured step
     for _ in range(args.warmup):
-        plan.lamb_step(hyper, d_step, d_lr)
+        one_step()
     d_step.fill_(1000)
     barrier()
 
@@ -372,7 +445,7 @@ def run_ours(args):
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        plan.lamb_step(hyper, d_step, d_lr)
+        one_step()
     e1.record(stream)
     barrier()
     wall1 = _dt.datetime.now()
@@ -381,18 +454,15 @@ def run_ours(args):
     B.lamb_plan_set_timing(plan.handle, False)
     if clocks:
         clocks.mark(wall0, wall1)
-    if world > 1:
-        t = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms_total = float(t.item())
+    ms_total = max_over_ranks(ms_total, dev)
     status = plan.query(clear=True)
 
     # ---- end to end: pinned host gradients in, trust ratios out ----------
     k_e2e = args.e2e_steps if args.e2e_steps is not None else min(args.steps, 50)
-    g_host = torch.empty(st.total, dtype=torch.bfloat16).pin_memory()
+    g_host = torch.empty(st.total, dtype=st.g.dtype).pin_memory()
     g_host.copy_(st.g.cpu())
     ratio_host = torch.empty(L.n_tensors, dtype=torch.float64).pin_memory()
-    h2d = L.n_params * 2
+    h2d = L.n_params * st.g.element_size()
     d2h = L.n_tensors * 8
     barrier()
     e2 = torch.cuda.Event(enable_timing=True)
@@ -401,7 +471,7 @@ def run_ours(args):
     e2.record(stream)
     for _ in range(k_e2e):
         st.g.copy_(g_host, non_blocking=True)
-        plan.lamb_step(hyper, d_step, d_lr)
+        one_step()
         B.lamb_plan_copy_trust_ratios(plan.handle, ratio_host.data_ptr(),
                                       stream=stream.cuda_stream)
         done.record(stream)
@@ -409,10 +479,7 @@ def run_ours(args):
     e3.record(stream)
     barrier()
     ms_e2e = e2.elapsed_time(e3)
-    if world > 1:
-        t = torch.tensor([ms_e2e], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms_e2e = float(t.item())
+    ms_e2e = max_over_ranks(ms_e2e, dev)
     assert math.isfinite(float(ratio_host[0]))
     clk = clocks.stop() if clocks else None
 
@@ -429,9 +496,14 @@ def run_ours(args):
     dom = int(np.argmax(per_launch_ms))
     alg_bytes = kernel_bytes[dom] * P
     achieved = alg_bytes / (per_launch_ms[dom] * 1e-3) / 1e9
-    traffic = profiled_traffic(profile_file, dom)
+    traffic = profiled_traffic(profile_file, dom) if profile_file else None
     ms_step = ms_total / args.steps
-    step_gbs = BYTES_STEP * P / (ms_step * 1e-3) / 1e9
+    step_bytes = sum(kernel_bytes) if algo == 1 or opt in ("nlamb", "nnlamb") \
+        else two_pass_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
+                            2 if L.copy_dtype == "bf16" else 0)
+    single_bytes = single_touch_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
+                                      2 if L.copy_dtype == "bf16" else 0)
+    step_gbs = step_bytes * P / (ms_step * 1e-3) / 1e9
 
     cpu = None
     if not args.no_cpu_baseline and world == 1:
@@ -456,14 +528,19 @@ def run_ours(args):
         "dtype": "f32",
         "data": "synthetic",
         "config": {"workload": workload, "n_params": P,
-                   "n_tensors": L.n_tensors, "grad_dtype": "bf16",
-                   "master_dtype": "f32", "copy_dtype": "bf16",
-                   "step_t": 1000, "lr": float(h.lr), "phi": "clip[0,10]",
-                   "l2": "inputs larger than L2 (5.4 GB state)",
+                   "n_tensors": L.n_tensors, "grad_dtype": L.grad_dtype,
+                   "master_dtype": "f32", "copy_dtype": L.copy_dtype,
+                   "optimizer": opt, "step_t": 1000, "lr": float(h.lr),
+                   "phi": h.phi if h.phi == "identity" else
+                   f"clip[{h.gamma_l:g},{h.gamma_u:g}]",
+                   "l2": "inputs larger than L2" if P * 16 > 130e6 else
+        "state smaller than L2 (no flush; not a bandwidth number)",
                    "parallelism": f"replicas{world}" if world > 1 else "1gpu"},
         "hbm_gbs_step": step_gbs,
-        "frac_of_peak_step_40B": step_gbs / peak,
-        "frac_of_peak_single_touch_28B": BYTES_SINGLE_TOUCH * P /
+        "two_pass_bytes_per_param": step_bytes,
+        "frac_of_peak_two_pass_model": step_gbs / peak,
+        "single_touch_bytes_per_param": single_bytes,
+        "frac_of_peak_single_touch_model": single_bytes * P /
         (ms_step * 1e-3) / 1e9 / peak,
         "algorithm": {1: "two_pass", 2: "single_touch"}[algo],
         "kernels": {kernel_names[i]: {"ms_per_launch": per_launch_ms[i],

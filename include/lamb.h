@@ -85,6 +85,12 @@ typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
                                            the appendix on adam-correction */
 #define LAMB_FLAG_INCREMENT_STEP  0x2u  /* the step writes *d_step = t + 1
                                            on the device when it completes */
+#define LAMB_FLAG_LR_SCHEDULE     0x4u  /* eta_t from t on the device
+                                           (Section 4): eta_0 t / T_w for
+                                           t < T_w, else eta_0 max(0, 1 -
+                                           t / T); d_lr may be NULL, else
+                                           the step writes the eta_t it
+                                           applied there                   */
 
 /* bits of the device status word (lamb_plan_query) */
 #define LAMB_STATUS_NONFINITE 0x1u      /* a tensor's sum of w^2 or of r^2
@@ -113,6 +119,10 @@ typedef struct {
   double trust_coef;     /* LARS kappa (ignored by lamb_step)               */
   int32_t phi;           /* lamb_phi_t                                      */
   uint32_t flags;        /* LAMB_FLAG_*                                     */
+  /* LAMB_FLAG_LR_SCHEDULE only */
+  double lr_base;            /* eta_0 >= 0                                  */
+  int64_t lr_warmup_steps;   /* T_w >= 0 (0: no warmup)                     */
+  int64_t lr_total_steps;    /* T >= 1                                      */
 } lamb_hyper_t;
 
 /* lamb_plan_options_t.algorithm */
@@ -198,7 +208,8 @@ LAMB_API lamb_status_t lamb_plan_bind(lamb_plan_t plan, void* const* w,
  *   d_step  DEVICE int64: t (>= 1 when bias correction is on).  Needed when
  *           LAMB_FLAG_BIAS_CORRECTION or LAMB_FLAG_INCREMENT_STEP is set,
  *           else may be NULL.
- *   d_lr    DEVICE float: eta_t for this step.
+ *   d_lr    DEVICE float: eta_t for this step (with LAMB_FLAG_LR_SCHEDULE:
+ *           NULL, or where the step writes the eta_t it computed).
  * Updates w, m, v in place (and the bf16 copy); g is read only.  Writes the
  * per-tensor norms and trust ratios (lamb_plan_trust_ratios).  No host
  * synchronisation, allocation or pageable copy: capturable in a CUDA graph,

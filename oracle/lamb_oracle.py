@@ -40,6 +40,10 @@ Q7  LARS takes an extra trust coefficient kappa: ratio = kappa*phi(||x||)/||m||
 Q8  Masked tensors still get the trust ratio; the mask removes decay only.
 Q9  Bias correction uses beta**t in float64 with an integer t >= 1.
 Q15 Non-finite inputs are not masked; NaN/Inf propagate.
+Q16 Learning-rate schedule (Section 4: polynomial decay eta_t = eta_0 (1 -
+    t/T) and linear warmup): eta_t = eta_0 t / T_w for t < T_w, else
+    eta_0 max(0, 1 - t/T) -- the decay holds from step 0 and the warmup
+    replaces it during the first T_w steps.
 Q12 N-LAMB / NN-LAMB (appendix): the superscripted beta_1^t is the t-th term
     of a momentum schedule (the input line lists the schedule separately from
     the constant beta1 of the moment recurrence); it is Dozat's Nadam
@@ -75,6 +79,7 @@ __all__ = [
     "lars_tensor",
     "lamb_tensor_scalar",
     "nadam_mu",
+    "lr_schedule",
     "nlamb_tensor",
     "NLambResult",
     "lamb_step",
@@ -239,6 +244,13 @@ def lars_tensor(w, g, m, *, lr: float, beta1: float = 0.9,
         x, m_t, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u,
         trust_coef=trust_coef)
     return LarsResult(x_new, m_t, ratio, xn, un)
+
+
+def lr_schedule(t: int, eta0: float, warmup: int, total: int) -> float:
+    """Section 4 learning rate at step t (reading Q16)."""
+    if warmup > 0 and t < warmup:
+        return eta0 * t / warmup
+    return eta0 * max(0.0, 1.0 - t / total)
 
 
 def nadam_mu(t: int, beta1: float, psi: float) -> float:

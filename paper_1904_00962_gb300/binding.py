@@ -37,6 +37,7 @@ LAMB_PHI_CLIP = 1
 # flags / status bits
 LAMB_FLAG_BIAS_CORRECTION = 0x1
 LAMB_FLAG_INCREMENT_STEP = 0x2
+LAMB_FLAG_LR_SCHEDULE = 0x4
 LAMB_STATUS_NONFINITE = 0x1
 LAMB_STATUS_BAD_STEP = 0x2
 
@@ -63,7 +64,9 @@ class lamb_hyper_t(Structure):
     _fields_ = [("beta1", c_double), ("beta2", c_double), ("eps", c_double),
                 ("weight_decay", c_double), ("gamma_l", c_double),
                 ("gamma_u", c_double), ("trust_coef", c_double),
-                ("phi", c_int32), ("flags", c_uint32)]
+                ("phi", c_int32), ("flags", c_uint32),
+                ("lr_base", c_double), ("lr_warmup_steps", c_int64),
+                ("lr_total_steps", c_int64)]
 
 
 LAMB_ALGO_AUTO = 0
@@ -170,13 +173,18 @@ def lamb_abi_version() -> int:
 
 def make_hyper(*, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01,
                phi="identity", gamma_l=0.0, gamma_u=math.inf, trust_coef=1.0,
-               bias_correction=True, increment_step=False) -> lamb_hyper_t:
-    """Fill a lamb_hyper_t (plain field copy)."""
+               bias_correction=True, increment_step=False, lr_schedule=None
+               ) -> lamb_hyper_t:
+    """Fill a lamb_hyper_t (plain field copy).  lr_schedule: None or
+    (eta_0, warmup_steps, total_steps) for LAMB_FLAG_LR_SCHEDULE."""
     flags = (LAMB_FLAG_BIAS_CORRECTION if bias_correction else 0) | \
-            (LAMB_FLAG_INCREMENT_STEP if increment_step else 0)
+            (LAMB_FLAG_INCREMENT_STEP if increment_step else 0) | \
+            (LAMB_FLAG_LR_SCHEDULE if lr_schedule is not None else 0)
+    base, warm, total = lr_schedule if lr_schedule is not None else (0.0, 0, 1)
     return lamb_hyper_t(beta1, beta2, eps, weight_decay, gamma_l, gamma_u,
                         trust_coef, LAMB_PHI_CLIP if phi == "clip"
-                        else LAMB_PHI_IDENTITY, flags)
+                        else LAMB_PHI_IDENTITY, flags, float(base), int(warm),
+                        int(total))
 
 
 def lamb_plan_create(sizes, decay_mask=None, grad_dtype=LAMB_F32,

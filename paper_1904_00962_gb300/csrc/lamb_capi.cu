@@ -110,6 +110,7 @@ struct lamb_plan {
   bool timing = false;
   int timed_steps = 0;
   std::vector<cudaEvent_t> events;  // kMaxTimedSteps * (kKernelsPerStep + 1)
+  std::vector<uint8_t> timed_kernels;  // kernels each timed step launched
 };
 
 extern "C" {
@@ -494,8 +495,14 @@ static lamb_status_t check_hyper(const lamb_hyper_t* h, bool lamb) {
     return fail(LAMB_ERR_INVALID_ARG, "clip bounds need gamma_l <= gamma_u");
   if (!lamb && !std::isfinite(h->trust_coef))
     return fail(LAMB_ERR_INVALID_ARG, "trust_coef must be finite");
-  if (h->flags & ~(uint32_t)(LAMB_FLAG_BIAS_CORRECTION | LAMB_FLAG_INCREMENT_STEP))
+  if (h->flags & ~(uint32_t)(LAMB_FLAG_BIAS_CORRECTION |
+                             LAMB_FLAG_INCREMENT_STEP | LAMB_FLAG_LR_SCHEDULE))
     return fail(LAMB_ERR_INVALID_ARG, "unknown flag bits 0x%x", h->flags);
+  if ((h->flags & LAMB_FLAG_LR_SCHEDULE) &&
+      !(h->lr_base >= 0.0 && std::isfinite(h->lr_base) &&
+        h->lr_warmup_steps >= 0 && h->lr_total_steps >= 1))
+    return fail(LAMB_ERR_INVALID_ARG,
+                "lr schedule needs lr_base >= 0, warmup >= 0, total >= 1");
   return LAMB_OK;
 }
 
@@ -530,6 +537,12 @@ static void fill_params(lamb_plan* p, const lamb_hyper_t* h, int64_t* d_step,
   sp->phi = h->phi;
   sp->flags = h->flags;
   sp->n_chunks = (int32_t)p->n_chunks;
+  if (h->flags & LAMB_FLAG_LR_SCHEDULE) {
+    sp->lr_base = h->lr_base;
+    sp->lr_warmup = h->lr_warmup_steps;
+    sp->lr_total = h->lr_total_steps;
+    sp->d_lr_out = const_cast<float*>(d_lr);
+  }
 }
 
 static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
@@ -541,9 +554,10 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
   if (!plan->bound) return fail(LAMB_ERR_NOT_BOUND, "plan is not bound");
   if (lamb && !plan->has_v)
     return fail(LAMB_ERR_NOT_BOUND, "lamb_step needs v: bind v pointers");
-  if (!d_lr) return fail(LAMB_ERR_INVALID_ARG, "d_lr is NULL");
+  const bool sched = (hyper->flags & LAMB_FLAG_LR_SCHEDULE) != 0;
+  if (!d_lr && !sched) return fail(LAMB_ERR_INVALID_ARG, "d_lr is NULL");
   const bool needs_step =
-      (hyper->flags & LAMB_FLAG_INCREMENT_STEP) ||
+      (hyper->flags & LAMB_FLAG_INCREMENT_STEP) || sched ||
       (lamb && (hyper->flags & LAMB_FLAG_BIAS_CORRECTION));
   if (needs_step && !d_step)
     return fail(LAMB_ERR_INVALID_ARG, "d_step is NULL but the flags need it");
@@ -575,7 +589,7 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
                         plan->grid_fused[lamb ? 0 : 1], stream);
     if (!rc && timed) rc = (int)cudaEventRecord(ev[1], stream);
     if (rc) return cuda_fail((cudaError_t)rc, lamb ? "lamb_step" : "lars_step");
-    if (timed) ++plan->timed_steps;
+    if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = 1;
     return LAMB_OK;
   }
   if (!rc)
@@ -587,7 +601,7 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
               : launch_lars_pass2(sp, plan->copy_bf16, plan->grid[3], stream);
   if (!rc && timed) rc = (int)cudaEventRecord(ev[2], stream);
   if (rc) return cuda_fail((cudaError_t)rc, lamb ? "lamb_step" : "lars_step");
-  if (timed) ++plan->timed_steps;
+  if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = 2;
   return LAMB_OK;
 }
 
@@ -617,8 +631,10 @@ lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
   if (!plan->bound) return fail(LAMB_ERR_NOT_BOUND, "plan is not bound");
   if (!plan->has_v)
     return fail(LAMB_ERR_NOT_BOUND, "nlamb_step needs v: bind v pointers");
-  if (!d_step || !d_lr || !d_mu_product)
-    return fail(LAMB_ERR_INVALID_ARG, "d_step, d_lr and d_mu_product are required");
+  if (!d_step || !d_mu_product ||
+      (!d_lr && !(hyper->flags & LAMB_FLAG_LR_SCHEDULE)))
+    return fail(LAMB_ERR_INVALID_ARG,
+                "d_step, d_mu_product and d_lr (or a schedule) are required");
   DeviceGuard guard(plan->device);
   if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
   StepParams sp;
@@ -639,7 +655,7 @@ lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
                             plan->grid[1], stream);
   if (!rc && timed) rc = (int)cudaEventRecord(ev[2], stream);
   if (rc) return cuda_fail((cudaError_t)rc, "nlamb_step");
-  if (timed) ++plan->timed_steps;
+  if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = 2;
   return LAMB_OK;
 }
 
@@ -720,6 +736,7 @@ lamb_status_t lamb_plan_set_timing(lamb_plan_t plan, int32_t enable) {
     DeviceGuard guard(plan->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
     plan->events.resize((size_t)kMaxTimedSteps * (kKernelsPerStep + 1));
+    plan->timed_kernels.assign((size_t)kMaxTimedSteps, 0);
     for (auto& ev : plan->events) {
       cudaError_t e = cudaEventCreate(&ev);
       if (e != cudaSuccess) return cuda_fail(e, "cudaEventCreate");
@@ -737,9 +754,8 @@ lamb_status_t lamb_plan_read_timing(lamb_plan_t plan, int32_t* n_steps,
   DeviceGuard guard(plan->device);
   if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
   for (int j = 0; j < n_kernels; ++j) ms_per_kernel[j] = 0.0;
-  const int per_step =
-      plan->algorithm == LAMB_ALGO_SINGLE_TOUCH ? 1 : kKernelsPerStep;
   for (int s = 0; s < plan->timed_steps; ++s) {
+    const int per_step = plan->timed_kernels[(size_t)s];
     cudaEvent_t* ev = &plan->events[(size_t)s * (kKernelsPerStep + 1)];
     cudaError_t e = cudaEventSynchronize(ev[per_step]);
     if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");

@@ -61,7 +61,8 @@ struct __align__(16) StepScalars {
 
 enum : uint32_t { kStatusNonfinite = 1u, kStatusBadStep = 2u,
                   kStatusWaitTimeout = 4u };
-enum : uint32_t { kFlagBiasCorrection = 1u, kFlagIncrementStep = 2u };
+enum : uint32_t { kFlagBiasCorrection = 1u, kFlagIncrementStep = 2u,
+                  kFlagLrSchedule = 4u };
 
 struct StepParams {
   const ChunkDesc* chunks;
@@ -89,6 +90,10 @@ struct StepParams {
   // N-LAMB / NN-LAMB only
   double psi;             // momentum-schedule decay (Nadam's psi)
   double* d_mu_product;   // prod_{i<t} mu_i on entry, prod_{i<=t} on exit
+  // learning-rate schedule (kFlagLrSchedule)
+  double lr_base;
+  int64_t lr_warmup, lr_total;
+  float* d_lr_out;        // where the applied eta_t is written (may be null)
 };
 
 // ---------------------------------------------------------------------------

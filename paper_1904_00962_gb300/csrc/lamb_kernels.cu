@@ -162,6 +162,26 @@ __device__ __forceinline__ float2 cta_sum2(float a, float b,
   return r;
 }
 
+// eta_t: read from device memory, or (kFlagLrSchedule) the Section 4
+// schedule eta_0 t / T_w during warmup, then eta_0 max(0, 1 - t / T).
+__device__ __forceinline__ float step_lr(const StepParams& p, int64_t t) {
+  if (!(p.flags & kFlagLrSchedule)) return *p.d_lr;
+  double lr;
+  if (p.lr_warmup > 0 && t < p.lr_warmup)
+    lr = p.lr_base * (double)t / (double)p.lr_warmup;
+  else
+    lr = p.lr_base * fmax(0.0, 1.0 - (double)t / (double)p.lr_total);
+  return (float)lr;
+}
+
+// The CTA or warp that closes a step: advance the step counter and report
+// the scheduled learning rate.
+__device__ __forceinline__ void close_step(const StepParams& p,
+                                           const StepScalars& sc) {
+  if ((p.flags & kFlagLrSchedule) && p.d_lr_out) *p.d_lr_out = sc.lr;
+  if ((p.flags & kFlagIncrementStep) && p.d_step) *p.d_step = sc.t + 1;
+}
+
 __device__ __forceinline__ double phi_of(double z, const StepParams& p) {
   if (p.phi == 1) {  // clip; comparisons keep NaN as NaN
     if (z < p.gamma_l) return p.gamma_l;
@@ -339,7 +359,7 @@ __global__ void __launch_bounds__(kThreads)
       sc.t = t;
       sc.c1 = c1;
       sc.c2 = c2;
-      sc.lr = *p.d_lr;
+      sc.lr = step_lr(p, t);
       sc.skip = skip;
       sc.am = kc.am;
       sc.ag = kc.ag;
@@ -461,7 +481,7 @@ __global__ void __launch_bounds__(kThreads)
   }
   if (retire(p, 1, c) && threadIdx.x == 0) {
     if (kNest && p.d_mu_product) *p.d_mu_product = sc.mu_prod;
-    if ((p.flags & kFlagIncrementStep) && p.d_step) *p.d_step = sc.t + 1;
+    close_step(p, sc);
   }
 }
 
@@ -535,7 +555,7 @@ __global__ void __launch_bounds__(kThreads)
       sc.t = p.d_step ? *p.d_step : int64_t(0);
       sc.c1 = 1.f;
       sc.c2 = 1.f;
-      sc.lr = *p.d_lr;
+      sc.lr = step_lr(p, sc.t);
       sc.skip = 0;
       *p.scal = sc;
     }
@@ -621,9 +641,7 @@ __global__ void __launch_bounds__(kThreads)
     ++it;
     c = s_next[it & 1];
   }
-  if (retire(p, 1, c) && threadIdx.x == 0 &&
-      (p.flags & kFlagIncrementStep) && p.d_step)
-    *p.d_step = sc.t + 1;
+  if (retire(p, 1, c) && threadIdx.x == 0) close_step(p, sc);
 }
 
 // ---------------------------------------------------------------------------
@@ -1197,7 +1215,7 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
       c2 = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
     }
     s_k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps};
-    s_lr = *p.d_lr;
+    s_lr = step_lr(p, t);
     s_skip = skip;
     s_t = t;
     s_epoch = *reinterpret_cast<volatile uint32_t*>(&p.counters[3]);
@@ -1373,7 +1391,10 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
     atomicExch(&p.counters[2], 0u);
     const uint32_t ne = epoch + 1u == 0u ? 1u : epoch + 1u;
     atomicExch(&p.counters[3], ne);
-    if ((p.flags & kFlagIncrementStep) && p.d_step) *p.d_step = s_t + 1;
+    StepScalars sc{};
+    sc.t = s_t;
+    sc.lr = s_lr;
+    close_step(p, sc);
   }
 }
 

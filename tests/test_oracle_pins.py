@@ -505,3 +505,30 @@ def test_pins_reject_planted_mistake(kind):
 def test_unmutated_oracle_passes_pin_harness():
     for case in _load_cases():
         assert _case_matches(case, _run_case(case)), case["name"]
+
+
+# ---------------------------------------------------------------------------
+# Section 4 learning-rate schedule (reading Q16)
+# ---------------------------------------------------------------------------
+
+def test_lr_schedule_closed_forms():
+    eta0, tw, T = 5e-3, 100, 1000
+    assert O.lr_schedule(50, eta0, tw, T) == pytest.approx(eta0 * 0.5, rel=1e-15)
+    assert O.lr_schedule(1, eta0, tw, T) == pytest.approx(eta0 / 100, rel=1e-15)
+    assert O.lr_schedule(100, eta0, tw, T) == pytest.approx(eta0 * 0.9, rel=1e-15)
+    assert O.lr_schedule(1000, eta0, tw, T) == 0.0
+    assert O.lr_schedule(5000, eta0, tw, T) == 0.0
+    assert O.lr_schedule(10, eta0, 0, T) == pytest.approx(eta0 * 0.99, rel=1e-15)
+
+
+def test_lr_schedule_decay_is_torch_polynomial_lr():
+    """After warmup the decay is torch's PolynomialLR with power 1."""
+    p = torch.zeros(1, requires_grad=True)
+    opt = torch.optim.SGD([p], lr=2e-3)
+    sch = torch.optim.lr_scheduler.PolynomialLR(opt, total_iters=500, power=1.0)
+    for t in range(0, 600):
+        if t >= 1:
+            opt.step()
+            sch.step()
+        assert O.lr_schedule(t, 2e-3, 0, 500) == pytest.approx(
+            opt.param_groups[0]["lr"], rel=1e-12, abs=1e-18), t

@@ -888,3 +888,49 @@ def test_nlamb_argument_errors():
         B.nlamb_step(G.plan.handle, h, 0.004, 0, G.d_step.data_ptr(),
                      G.d_lr.data_ptr(), 0)
     G.close()
+
+
+# ---------------------------------------------------------------------------
+# Section 4 learning-rate schedule computed on the device (reading Q16)
+# ---------------------------------------------------------------------------
+
+@algos
+def test_lr_schedule_on_device(algo):
+    L = W.mlp_layout()
+    h = L.hyper
+    eta0, tw, T = 4e-3, 4, 10
+    G = GpuLayout(L, algorithm=algo)
+    G.load_weights()
+    hyp = B.make_hyper(beta1=h.beta1, beta2=h.beta2, eps=h.eps,
+                       weight_decay=h.weight_decay, phi=h.phi,
+                       increment_step=True, lr_schedule=(eta0, tw, T))
+    G.d_step.fill_(1)
+    state = [(L.weights(k).astype(np.float64), np.zeros(s), np.zeros(s))
+             for k, s in enumerate(L.sizes)]
+    path = [np.zeros(s) for s in L.sizes]
+    for t in range(1, 13):
+        G.load_grads(t)
+        G.plan.lamb_step(hyp, G.d_step, G.d_lr)
+        ratio, _, _ = G.results()
+        lr = f32(O.lr_schedule(t, eta0, tw, T))
+        assert float(G.d_lr.item()) == lr, t          # the eta_t it applied
+        for k in range(L.n_tensors):
+            w0, m0, v0 = state[k]
+            ref = _oracle_lamb(L, k, w0, L.grad(k, t), m0, v0, t, lr, h)
+            path[k] += np.abs(ref.w - w0)
+            got = G.download("w", k).astype(np.float64)
+            scale = np.maximum(np.maximum(np.abs(ref.w), np.abs(w0)), path[k])
+            assert np.all(np.abs(got - ref.w) <= TOL_CHAIN * scale), (t, k)
+            state[k] = (ref.w, ref.m, ref.v)
+    assert int(G.d_step.item()) == 13
+    # after T the schedule is 0: weights stop moving
+    w_before = G.st.w.clone()
+    G.load_grads(99)
+    G.plan.lamb_step(hyp, G.d_step, G.d_lr)
+    torch.cuda.synchronize()
+    assert float(G.d_lr.item()) == 0.0
+    assert torch.equal(w_before, G.st.w)
+    # the schedule may run without any learning-rate buffer
+    B.lamb_step(G.plan.handle, hyp, G.d_step.data_ptr(), 0)
+    torch.cuda.synchronize()
+    G.close()
