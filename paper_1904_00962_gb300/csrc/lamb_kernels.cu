@@ -1309,6 +1309,33 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
 #pragma unroll
   for (int s = 0; s < kStages; ++s) fill_advance(s);
 
+  // pass-2 item of this warp whose tensor was not final when its turn came
+  uint2 parked = invalid_desc();
+  // run a pass-2 item from global memory once its tensor is known final
+  auto run_direct_p2 = [&](uint2 d) {
+    const uint32_t tensor = d.x >> 1;
+    if (tensor != synced) {
+      fence_acq_rel();                 // acquire: the relaxed load saw it
+      synced = tensor;
+    }
+    const FusedTensor ft = f.ftensors[tensor];
+    const TensorPtrs tp = p.ptrs[tensor];
+    const int64_t off = (int64_t)d.y * kFusedChunk;
+    const int64_t rem = ft.numel - off;
+    const int len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
+    const float s2 = __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]));
+    fused2_direct<kLars, kCopy>(tp, off, len, s2, ft.decay * p.wd, k,
+                                pol_first, lane);
+  };
+  // the same after a bounded wait (callers flush their publishes first)
+  auto wait_direct_p2 = [&](uint2 d) {
+    const uint32_t tensor = d.x >> 1;
+    if (fused_wait(p, f, (int)tensor, epoch, lane)) {
+      synced = tensor;
+      run_direct_p2(d);
+    }
+  };
+
   PubState ps;
   ps.pub = ps.chk = false;
   ps.tensor = ps.index = ps.chk_tensor = ps.chk_index = 0u;
@@ -1371,19 +1398,38 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
         } else {
           __syncwarp();
           fill_advance(s);
-          fused_flush<kLars>(p, f, ps, epoch, lane);   // never wait on ourselves
-          if (fused_wait(p, f, (int)tensor, epoch, lane)) {
-            synced = tensor;
-            const float s2 =
-                __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]));
-            fused2_direct<kLars, kCopy>(tp, off, len, s2, lam, k, pol_first,
-                                        lane);
+          fused_publish_step<kLars>(p, f, ps, epoch, lane);
+          // every lane loads the flag itself (one broadcast access) before
+          // its acquire fence; lane 0's value makes the decision uniform
+          const uint32_t r = __shfl_sync(0xffffffffu,
+                                         ld_relaxed(&f.ready[tensor]), 0);
+          if (r == epoch) {               // became final since the fill
+            run_direct_p2(d);
+          } else {
+            // Not final yet: park it instead of waiting, so this warp keeps
+            // working (and publishing) its later pass-1 items.  With the
+            // parking slot taken, finish the parked item first.
+            if (parked.x != 0xffffffffu) {
+              fused_flush<kLars>(p, f, ps, epoch, lane);
+              wait_direct_p2(parked);
+            }
+            parked = d;
           }
+        }
+      }
+      // a parked item whose tensor has become final in the meantime
+      if (parked.x != 0xffffffffu) {
+        const uint32_t r = __shfl_sync(
+            0xffffffffu, ld_relaxed(&f.ready[parked.x >> 1]), 0);
+        if (r == epoch) {
+          run_direct_p2(parked);
+          parked = invalid_desc();
         }
       }
     }
   }
   fused_flush<kLars>(p, f, ps, epoch, lane);
+  if (parked.x != 0xffffffffu) wait_direct_p2(parked);
   cp_async_wait<0>();
   // The warp that drew the last index >= n_items closes the launch.
   const uint32_t warps = gridDim.x * kFusedWarps;
