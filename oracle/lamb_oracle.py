@@ -55,6 +55,16 @@ Q12 N-LAMB / NN-LAMB (appendix): the superscripted beta_1^t is the t-th term
     read as a typo.  In NN-LAMB the second-moment schedule is constant
     (beta2), since the algorithm's inputs give none.
 
+Q17 Gradient norms and the non-finite guard (not in the paper; the
+    training-system checks that accompany a large-batch step): ||g_k|| per
+    block, the global ||g|| = sqrt(sum_k ||g_k||^2) (the norm of the whole
+    gradient viewed as one vector), and a verdict "non-finite" when any
+    element of any g_k is Inf or NaN.  A guarded step with that verdict is
+    not applied: x, m, v and t keep their values.
+Q18 Decoupled weight decay (an ablation of Q4 the paper does not define;
+    the AdamW-style decoupling applied to LAMB): the normalised direction is
+    r alone, ratio = phi(||x||)/||r||, and x <- x - lr*ratio*r - lr*lam*x.
+
 Input conventions: arrays may be float32 (or bfloat16 bit patterns given as
 uint16 together with ``g_dtype="bf16"``); they are converted exactly to
 float64 before any arithmetic.  Hyperparameters are Python floats.
@@ -84,6 +94,8 @@ __all__ = [
     "NLambResult",
     "lamb_step",
     "lars_step",
+    "GradCheck",
+    "grad_check",
 ]
 
 
@@ -193,7 +205,8 @@ def lamb_tensor(w, g, m, v, *, t: int, lr: float, beta1: float = 0.9,
                 weight_decay: float = 0.01, decay: bool = True,
                 phi_kind: str = "identity", gamma_l: float = 0.0,
                 gamma_u: float = math.inf, bias_correction: bool = True,
-                g_dtype: str = "f32") -> LambResult:
+                g_dtype: str = "f32",
+                decoupled_decay: bool = False) -> LambResult:
     """One LAMB step (Algorithm 2) on one block, in float64.
 
     Order of operations follows the algorithm:
@@ -202,6 +215,8 @@ def lamb_tensor(w, g, m, v, *, t: int, lr: float, beta1: float = 0.9,
       m_hat = m_t / (1 - beta1^t),  v_hat = v_t / (1 - beta2^t)
       r_t = m_hat / (sqrt(v_hat) + eps)
       x_{t+1} = x_t - lr * phi(||x_t||) / ||r_t + lam x_t|| * (r_t + lam x_t)
+    With decoupled_decay (reading Q18) the last line becomes
+      x_{t+1} = x_t - lr * phi(||x_t||) / ||r_t|| * r_t - lr * lam * x_t
     """
     if t < 1:
         raise ValueError("step count t must be >= 1")
@@ -219,6 +234,10 @@ def lamb_tensor(w, g, m, v, *, t: int, lr: float, beta1: float = 0.9,
     else:
         m_hat, v_hat = m_t, v_t
     r_t = m_hat / (np.sqrt(v_hat) + eps)
+    if decoupled_decay:
+        x_new, ratio, xn, un = layerwise_step(
+            x, r_t, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u)
+        return LambResult(x_new - lr * lam * x, m_t, v_t, ratio, xn, un)
     u = r_t + lam * x
     x_new, ratio, xn, un = layerwise_step(
         x, u, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u)
@@ -275,7 +294,8 @@ def nlamb_tensor(w, g, m, v, *, t: int, lr: float, mu_product: float,
                  psi: float = 0.004, weight_decay: float = 0.01,
                  decay: bool = True, nesterov_second_moment: bool = False,
                  phi_kind: str = "identity", gamma_l: float = 0.0,
-                 gamma_u: float = math.inf, g_dtype: str = "f32") -> NLambResult:
+                 gamma_u: float = math.inf, g_dtype: str = "f32",
+                 decoupled_decay: bool = False) -> NLambResult:
     """One N-LAMB (Algorithm 3) or, with nesterov_second_moment, NN-LAMB
     (Algorithm 4) step on one block, in float64.
 
@@ -287,7 +307,8 @@ def nlamb_tensor(w, g, m, v, *, t: int, lr: float, mu_product: float,
       v_hat = v_t / (1 - beta2^t)                                (N-LAMB)
             = beta2 v_t / (1 - beta2^(t+1)) + (1-beta2) g^2 / (1 - beta2^t)
                                                                  (NN-LAMB)
-      r = m_hat / (sqrt(v_hat) + eps); then the layerwise step on r + lambda x.
+      r = m_hat / (sqrt(v_hat) + eps); then the layerwise step on r + lambda x
+      (with decoupled_decay, reading Q18: on r, then x -= lr * lambda * x).
     """
     if t < 1:
         raise ValueError("step count t must be >= 1")
@@ -309,6 +330,11 @@ def nlamb_tensor(w, g, m, v, *, t: int, lr: float, mu_product: float,
     else:
         v_hat = v_t / (1.0 - beta2 ** t)
     r_t = m_hat / (np.sqrt(v_hat) + eps)
+    if decoupled_decay:
+        x_new, ratio, xn, un = layerwise_step(
+            x, r_t, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u)
+        return NLambResult(x_new - lr * lam * x, m_t, v_t, prod_t, ratio, xn,
+                           un)
     u = r_t + lam * x
     x_new, ratio, xn, un = layerwise_step(
         x, u, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u)
@@ -358,3 +384,32 @@ def lars_step(ws, gs, ms, decay_mask, *, lr, g_dtype="f32", **hyper):
     return [lars_tensor(w, g, m, lr=lr, decay=bool(d), g_dtype=g_dtype,
                         **hyper)
             for w, g, m, d in zip(ws, gs, ms, decay_mask)]
+
+
+# --------------------------------------------------------------------------
+# Gradient norms and the non-finite guard (reading Q17)
+# --------------------------------------------------------------------------
+
+@dataclass
+class GradCheck:
+    norms: list         # ||g_k|| per block
+    norm: float         # sqrt(sum_k ||g_k||^2)
+    nonfinite: bool     # some element of some g_k is Inf or NaN
+
+
+def grad_check(gs, g_dtype: str = "f32") -> GradCheck:
+    """Per-block l2 norms of the gradient (the norm of Section 2's notation,
+    one block at a time), the l2 norm of the whole gradient, and whether any
+    element is Inf or NaN.  Each square of an fp32 or bf16 value is exact in
+    float64; the per-block sums use NumPy's pairwise reduction and the sum
+    over blocks is exactly rounded (math.fsum).  A non-finite element makes
+    its block's norm Inf or NaN, as the arithmetic gives."""
+    sq = []
+    bad = False
+    for g in gs:
+        x = to_f64(g, g_dtype)
+        if not np.all(np.isfinite(x)):
+            bad = True
+        sq.append(float(np.sum(x * x)))
+    total = math.fsum(sq) if all(math.isfinite(s) for s in sq) else sum(sq)
+    return GradCheck([math.sqrt(s) for s in sq], math.sqrt(total), bad)

@@ -38,6 +38,8 @@ def _run_case(case, lamb_fn=None, lars_fn=None):
                   phi_kind=h["phi"], gamma_l=_ev(h.get("gamma_l", "0")),
                   gamma_u=_ev(h.get("gamma_u", "oo")))
     if case["algorithm"] == "lamb":
+        if h.get("decoupled_decay"):
+            common["decoupled_decay"] = True
         return lamb_fn(arr("w"), arr("g"), arr("m"), arr("v"), t=h["t"],
                        beta2=_ev(h["beta2"]), eps=_ev(h["eps"]),
                        bias_correction=h.get("bias_correction", True),
@@ -483,7 +485,7 @@ def test_pins_reject_planted_mistake(kind):
     mutant = _mutant(kind)
     caught = False
     for case in _load_cases():
-        if case["algorithm"] != "lamb":
+        if case["algorithm"] != "lamb" or case["hyper"].get("decoupled_decay"):
             continue
         if not _case_matches(case, _run_case(case, lamb_fn=mutant)):
             caught = True
