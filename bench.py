@@ -84,18 +84,26 @@ def single_touch_bytes(opt, gb, cb):
     return gb + 12 + 8 + 4 + cb
 
 
-def kernel_model(opt, algo, gb, cb):
-    """(kernel names, algorithmic bytes per parameter of each kernel)."""
-    if algo == 2 and opt in ("lamb", "lars"):
+def kernel_model(opt, algo, gb, cb, variant="plain"):
+    """(kernel names, algorithmic bytes per parameter of each kernel).
+    The skip-on-non-finite variant moves the m, v (LARS: m) writes from
+    pass 1 to pass 2, which then reads g as well."""
+    if algo == 2 and opt in ("lamb", "lars") and variant == "plain":
         return ([f"fused_step_kernel<{opt},g{8 * gb},copy{8 * cb}>"],
                 [single_touch_bytes(opt, gb, cb)])
+    defer = variant == "skip_nonfinite"
     if opt == "lars":
+        if defer:
+            return (["lars_pass1_kernel", "lars_pass2_kernel"],
+                    [gb + 8, gb + 8 + 4 + 4 + cb])
         return (["lars_pass1_kernel", "lars_pass2_kernel"],
                 [gb + 8 + 4, 8 + 4 + cb])
     nest = opt in ("nlamb", "nnlamb")
-    return ([f"{'n' if nest else ''}lamb_pass1_kernel",
-             f"{'n' if nest else ''}lamb_pass2_kernel"],
-            [gb + 12 + 8, 12 + (gb if nest else 0) + 4 + cb])
+    names = [f"{'n' if nest else ''}lamb_pass1_kernel",
+             f"{'n' if nest else ''}lamb_pass2_kernel"]
+    if defer:
+        return names, [gb + 12, gb + 12 + 8 + 4 + cb]
+    return names, [gb + 12 + 8, 12 + (gb if nest else 0) + 4 + cb]
 
 
 def parse_args():
@@ -121,6 +129,11 @@ def parse_args():
                     help="parameter layout (default: the BERT-large headline)")
     ap.add_argument("--optimizer", default="lamb",
                     choices=["lamb", "lars", "nlamb", "nnlamb"])
+    ap.add_argument("--variant", default="plain",
+                    choices=["plain", "grad_norm", "skip_nonfinite",
+                             "decoupled"],
+                    help="optional step flags: the fused gradient check, "
+                         "skip-on-non-finite, or decoupled weight decay")
     ap.add_argument("--layers", type=int, default=24,
                     help="encoder layers of the layout (24 = BERT-large; "
                          "fewer only for small profiling captures)")
@@ -143,7 +156,7 @@ def load_peaks():
 
 def kernel_source_hash():
     h = hashlib.sha256()
-    for name in ("lamb_kernels.cu", "lamb_internal.h"):
+    for name in ("lamb_kernels.cu", "lamb_device.cuh", "lamb_internal.h"):
         with open(os.path.join(ROOT, "paper_1904_00962_gb300", "csrc",
                                name), "rb") as f:
             h.update(f.read())
@@ -378,6 +391,8 @@ def run_ours(args):
     opt = args.optimizer
     if opt != "lamb":
         workload += f"_{opt}"
+    if args.variant != "plain":
+        workload += f"_{args.variant}"
     lars = opt == "lars"
     h = L.lars_hyper if (lars and L.lars_hyper) else L.hyper
     if lars and not L.lars_hyper:
@@ -394,9 +409,10 @@ def run_ours(args):
     algo = plan.info()["algorithm"]
     kernel_names, kernel_bytes = kernel_model(
         opt, algo, 2 if L.grad_dtype == "bf16" else 4,
-        2 if L.copy_dtype == "bf16" else 0)
+        2 if L.copy_dtype == "bf16" else 0, args.variant)
     profile_file = KERNELS[algo][2] if (
-        args.layout == "bert_large" and opt == "lamb") else None
+        args.layout == "bert_large" and opt == "lamb" and
+        args.variant == "plain") else None
     d_step = torch.ones(1, dtype=torch.int64, device=dev)
     d_lr = torch.full((1,), float(np.float32(h.lr)), dtype=torch.float32,
                       device=dev)
@@ -405,7 +421,10 @@ def run_ours(args):
                          weight_decay=h.weight_decay, phi=h.phi,
                          gamma_l=h.gamma_l, gamma_u=h.gamma_u,
                          trust_coef=h.trust_coef,
-                         bias_correction=not lars, increment_step=True)
+                         bias_correction=not lars, increment_step=True,
+                         grad_norm=args.variant == "grad_norm",
+                         skip_nonfinite=args.variant == "skip_nonfinite",
+                         decoupled_decay=args.variant == "decoupled")
 
     def one_step():
         if opt == "lamb":
@@ -498,7 +517,7 @@ def run_ours(args):
     achieved = alg_bytes / (per_launch_ms[dom] * 1e-3) / 1e9
     traffic = profiled_traffic(profile_file, dom) if profile_file else None
     ms_step = ms_total / args.steps
-    step_bytes = sum(kernel_bytes) if algo == 1 or opt in ("nlamb", "nnlamb") \
+    step_bytes = sum(kernel_bytes) if len(kernel_bytes) == 2 \
         else two_pass_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
                             2 if L.copy_dtype == "bf16" else 0)
     single_bytes = single_touch_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
@@ -530,7 +549,8 @@ def run_ours(args):
         "config": {"workload": workload, "n_params": P,
                    "n_tensors": L.n_tensors, "grad_dtype": L.grad_dtype,
                    "master_dtype": "f32", "copy_dtype": L.copy_dtype,
-                   "optimizer": opt, "step_t": 1000, "lr": float(h.lr),
+                   "optimizer": opt, "variant": args.variant,
+                   "step_t": 1000, "lr": float(h.lr),
                    "phi": h.phi if h.phi == "identity" else
                    f"clip[{h.gamma_l:g},{h.gamma_u:g}]",
                    "l2": "inputs larger than L2" if P * 16 > 130e6 else
@@ -542,7 +562,7 @@ def run_ours(args):
         "single_touch_bytes_per_param": single_bytes,
         "frac_of_peak_single_touch_model": single_bytes * P /
         (ms_step * 1e-3) / 1e9 / peak,
-        "algorithm": {1: "two_pass", 2: "single_touch"}[algo],
+        "algorithm": "two_pass" if len(kernel_names) == 2 else "single_touch",
         "kernels": {kernel_names[i]: {"ms_per_launch": per_launch_ms[i],
                                       "alg_bytes_per_param": kernel_bytes[i]}
                     for i in range(len(kernel_names))},

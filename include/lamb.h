@@ -91,6 +91,31 @@ typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
                                            t / T); d_lr may be NULL, else
                                            the step writes the eta_t it
                                            applied there                   */
+#define LAMB_FLAG_GRAD_NORM       0x8u  /* pass 1 also forms ||g_k|| of every
+                                           tensor and the global ||g|| =
+                                           sqrt(sum_k ||g_k||^2), and checks
+                                           every gradient element for Inf /
+                                           NaN (lamb_plan_grad_norms).  The
+                                           sums are fp32 per chunk, fp64
+                                           across chunks: a chunk whose sum
+                                           of g^2 exceeds FLT_MAX reports an
+                                           infinite norm without counting as
+                                           non-finite                       */
+#define LAMB_FLAG_SKIP_NONFINITE  0x10u /* implies GRAD_NORM.  If any element
+                                           of g is Inf or NaN the step writes
+                                           nothing: w, m, v, the bf16 copy,
+                                           *d_step, the scheduled *d_lr and
+                                           the N-LAMB product keep their
+                                           values, and LAMB_STATUS_SKIPPED is
+                                           set.  Pass 2 then forms and writes
+                                           m, v instead of pass 1: one more
+                                           read of g per step              */
+#define LAMB_FLAG_DECOUPLED_DECAY 0x20u /* lamb_step / nlamb_step only: the
+                                           decay term leaves the normalised
+                                           direction, u = r, rho = phi(||w||)
+                                           / ||r||, w <- w - eta rho r - eta
+                                           lambda_k w (an ablation of Alg. 2's
+                                           r + lambda w; not in the paper)  */
 
 /* bits of the device status word (lamb_plan_query) */
 #define LAMB_STATUS_NONFINITE 0x1u      /* a tensor's sum of w^2 or of r^2
@@ -104,6 +129,10 @@ typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
                                            pass-2 items then gave up too, so
                                            w was not (fully) updated; never
                                            expected                         */
+#define LAMB_STATUS_GRAD_NONFINITE 0x8u /* GRAD_NORM: a gradient element was
+                                           Inf or NaN                       */
+#define LAMB_STATUS_SKIPPED   0x10u     /* SKIP_NONFINITE: a step was skipped
+                                           for that reason                  */
 
 /* Hyperparameters.  Doubles on purpose: (1 - beta) is formed in double and
  * rounded once to float, so e.g. beta2 = 0.999 gives 1-beta2 = 0.001 to
@@ -126,7 +155,7 @@ typedef struct {
 } lamb_hyper_t;
 
 /* lamb_plan_options_t.algorithm */
-#define LAMB_ALGO_AUTO 0          /* the library's default (single-touch)    */
+#define LAMB_ALGO_AUTO 0          /* the library's default (two-pass)        */
 #define LAMB_ALGO_TWO_PASS 1      /* two streaming kernels per step: 40 B of
                                      HBM traffic per parameter (bf16 g/copy) */
 #define LAMB_ALGO_SINGLE_TOUCH 2  /* one kernel per step; pass 2 of a tensor
@@ -259,6 +288,30 @@ LAMB_API lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
 LAMB_API lamb_status_t lamb_plan_trust_ratios(lamb_plan_t plan, const double** d_ratio,
                                      const double** d_wnorm,
                                      const double** d_unorm);
+
+/* DEVICE results of the last step's gradient check (LAMB_FLAG_GRAD_NORM or
+ * LAMB_FLAG_SKIP_NONFINITE; the arrays keep their values across steps
+ * without those flags):
+ *   d_gnorm         [n_tensors] ||g_k|| in double (0 for 0-element tensors)
+ *   d_gnorm_global  [1] sqrt(sum_k ||g_k||^2)
+ *   d_nonfinite     [1] 1 if some element of g was Inf or NaN, else 0 (with
+ *                   SKIP_NONFINITE: the step was skipped)
+ * Owned by the plan, valid until destroy.  Any out pointer may be NULL.
+ * A CUDA graph can read them on the device, e.g. to adapt a loss scale. */
+LAMB_API lamb_status_t lamb_plan_grad_norms(lamb_plan_t plan,
+                                            const double** d_gnorm,
+                                            const double** d_gnorm_global,
+                                            const uint32_t** d_nonfinite);
+
+/* Copy the gradient-check results (as lamb_plan_grad_norms) into
+ * caller-owned memory -- device or host, any pointer may be NULL: gnorm
+ * [n_tensors] doubles, gnorm_global [1] double, nonfinite [1] uint32 --
+ * with cudaMemcpyAsync on `stream`.  Does not synchronise. */
+LAMB_API lamb_status_t lamb_plan_copy_grad_norms(lamb_plan_t plan,
+                                                 double* gnorm,
+                                                 double* gnorm_global,
+                                                 uint32_t* nonfinite,
+                                                 cudaStream_t stream);
 
 /* Copy the last step's per-tensor results (as lamb_plan_trust_ratios) into
  * caller-owned arrays of n_tensors doubles -- device or host memory, any of

@@ -38,8 +38,13 @@ LAMB_PHI_CLIP = 1
 LAMB_FLAG_BIAS_CORRECTION = 0x1
 LAMB_FLAG_INCREMENT_STEP = 0x2
 LAMB_FLAG_LR_SCHEDULE = 0x4
+LAMB_FLAG_GRAD_NORM = 0x8
+LAMB_FLAG_SKIP_NONFINITE = 0x10
+LAMB_FLAG_DECOUPLED_DECAY = 0x20
 LAMB_STATUS_NONFINITE = 0x1
 LAMB_STATUS_BAD_STEP = 0x2
+LAMB_STATUS_GRAD_NONFINITE = 0x8
+LAMB_STATUS_SKIPPED = 0x10
 
 EXPORTED = ["lamb_plan_create", "lamb_plan_bind", "lamb_step", "lars_step",
             "lamb_plan_trust_ratios", "lamb_plan_copy_trust_ratios",
@@ -47,7 +52,7 @@ EXPORTED = ["lamb_plan_create", "lamb_plan_bind", "lamb_step", "lars_step",
             "lamb_plan_set_timing", "lamb_plan_read_timing",
             "lamb_plan_destroy", "lamb_layout_chunks", "lamb_last_error",
             "lamb_abi_version", "lamb_step_noalloc", "lamb_layout_schedule",
-            "nlamb_step"]
+            "nlamb_step", "lamb_plan_grad_norms", "lamb_plan_copy_grad_norms"]
 
 
 class LambError(RuntimeError):
@@ -121,6 +126,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.lamb_plan_trust_ratios.argtypes = [vp, POINTER(vp), POINTER(vp),
                                            POINTER(vp)]
     lib.lamb_plan_copy_trust_ratios.argtypes = [vp, vp, vp, vp, vp]
+    lib.lamb_plan_grad_norms.argtypes = [vp, POINTER(vp), POINTER(vp),
+                                         POINTER(vp)]
+    lib.lamb_plan_copy_grad_norms.argtypes = [vp, vp, vp, vp, vp]
     lib.lamb_plan_query.argtypes = [vp, POINTER(c_uint32), c_int32, vp]
     lib.lamb_plan_get_info.argtypes = [vp, POINTER(lamb_plan_info_t)]
     lib.lamb_plan_set_timing.argtypes = [vp, c_int32]
@@ -173,13 +181,17 @@ def lamb_abi_version() -> int:
 
 def make_hyper(*, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01,
                phi="identity", gamma_l=0.0, gamma_u=math.inf, trust_coef=1.0,
-               bias_correction=True, increment_step=False, lr_schedule=None
+               bias_correction=True, increment_step=False, lr_schedule=None,
+               grad_norm=False, skip_nonfinite=False, decoupled_decay=False
                ) -> lamb_hyper_t:
     """Fill a lamb_hyper_t (plain field copy).  lr_schedule: None or
     (eta_0, warmup_steps, total_steps) for LAMB_FLAG_LR_SCHEDULE."""
     flags = (LAMB_FLAG_BIAS_CORRECTION if bias_correction else 0) | \
             (LAMB_FLAG_INCREMENT_STEP if increment_step else 0) | \
-            (LAMB_FLAG_LR_SCHEDULE if lr_schedule is not None else 0)
+            (LAMB_FLAG_LR_SCHEDULE if lr_schedule is not None else 0) | \
+            (LAMB_FLAG_GRAD_NORM if grad_norm else 0) | \
+            (LAMB_FLAG_SKIP_NONFINITE if skip_nonfinite else 0) | \
+            (LAMB_FLAG_DECOUPLED_DECAY if decoupled_decay else 0)
     base, warm, total = lr_schedule if lr_schedule is not None else (0.0, 0, 1)
     return lamb_hyper_t(beta1, beta2, eps, weight_decay, gamma_l, gamma_u,
                         trust_coef, LAMB_PHI_CLIP if phi == "clip"
@@ -239,6 +251,23 @@ def lamb_plan_trust_ratios(plan):
     _check(load().lamb_plan_trust_ratios(c_void_p(plan), byref(r), byref(w),
                                          byref(u)))
     return r.value, w.value, u.value
+
+
+def lamb_plan_grad_norms(plan):
+    """Device addresses of (||g_k|| [n] f64, global ||g|| [1] f64,
+    non-finite flag [1] u32)."""
+    a, b, c = c_void_p(), c_void_p(), c_void_p()
+    _check(load().lamb_plan_grad_norms(c_void_p(plan), byref(a), byref(b),
+                                       byref(c)))
+    return a.value, b.value, c.value
+
+
+def lamb_plan_copy_grad_norms(plan, gnorm=0, gnorm_global=0, nonfinite=0,
+                              stream=0) -> None:
+    """Addresses (device or host) of caller-owned arrays, or 0."""
+    _check(load().lamb_plan_copy_grad_norms(
+        c_void_p(plan), c_void_p(gnorm or None), c_void_p(gnorm_global or None),
+        c_void_p(nonfinite or None), c_void_p(stream or None)))
 
 
 def lamb_plan_copy_trust_ratios(plan, ratio=0, wnorm=0, unorm=0,

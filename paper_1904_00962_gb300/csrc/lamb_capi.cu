@@ -97,6 +97,12 @@ struct lamb_plan {
   StepScalars* scal = nullptr;
   uint32_t* status = nullptr;
   uint32_t* counters = nullptr;
+  // gradient check
+  float2* grad_slots = nullptr;
+  double* grad_sq = nullptr;
+  double* grad_norm = nullptr;
+  GradCheck* grad_check = nullptr;
+  int n_live = 0;               // tensors with at least one chunk
   // single-touch tables
   uint2* items = nullptr;
   FusedChunk* fchunks = nullptr;
@@ -255,7 +261,10 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
     return fail(LAMB_ERR_INVALID_ARG, "%s", err);
   }
   p->n_chunks = nch;
-  for (int k = 0; k < n_tensors; ++k) p->n_params += sizes[k];
+  for (int k = 0; k < n_tensors; ++k) {
+    p->n_params += sizes[k];
+    p->n_live += p->h_tensors[(size_t)k].n_chunks > 0 ? 1 : 0;
+  }
 
   // ---- device ------------------------------------------------------------
   DeviceGuard guard(device);
@@ -343,6 +352,10 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   const size_t o_scal = carve(sizeof(StepScalars));
   const size_t o_status = carve(sizeof(uint32_t));
   const size_t o_counters = carve(8 * sizeof(uint32_t));
+  const size_t o_grad_slots = carve(c * sizeof(float2));
+  const size_t o_grad_sq = carve(n * sizeof(double));
+  const size_t o_grad_norm = carve(n * sizeof(double));
+  const size_t o_grad_check = carve(sizeof(GradCheck));
   const size_t nf = h_fchunks.size(), ng = (size_t)p->n_groups;
   const size_t o_items = carve(h_items.size() * sizeof(uint2));
   const size_t o_fchunks = carve(nf * sizeof(FusedChunk));
@@ -370,6 +383,10 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   p->scal = reinterpret_cast<StepScalars*>(base + o_scal);
   p->status = reinterpret_cast<uint32_t*>(base + o_status);
   p->counters = reinterpret_cast<uint32_t*>(base + o_counters);
+  p->grad_slots = reinterpret_cast<float2*>(base + o_grad_slots);
+  p->grad_sq = reinterpret_cast<double*>(base + o_grad_sq);
+  p->grad_norm = reinterpret_cast<double*>(base + o_grad_norm);
+  p->grad_check = reinterpret_cast<GradCheck*>(base + o_grad_check);
   p->items = reinterpret_cast<uint2*>(base + o_items);
   p->fchunks = reinterpret_cast<FusedChunk*>(base + o_fchunks);
   p->ftensors = reinterpret_cast<FusedTensor*>(base + o_ftensors);
@@ -496,8 +513,14 @@ static lamb_status_t check_hyper(const lamb_hyper_t* h, bool lamb) {
   if (!lamb && !std::isfinite(h->trust_coef))
     return fail(LAMB_ERR_INVALID_ARG, "trust_coef must be finite");
   if (h->flags & ~(uint32_t)(LAMB_FLAG_BIAS_CORRECTION |
-                             LAMB_FLAG_INCREMENT_STEP | LAMB_FLAG_LR_SCHEDULE))
+                             LAMB_FLAG_INCREMENT_STEP | LAMB_FLAG_LR_SCHEDULE |
+                             LAMB_FLAG_GRAD_NORM | LAMB_FLAG_SKIP_NONFINITE |
+                             LAMB_FLAG_DECOUPLED_DECAY))
     return fail(LAMB_ERR_INVALID_ARG, "unknown flag bits 0x%x", h->flags);
+  if (!lamb && (h->flags & LAMB_FLAG_DECOUPLED_DECAY))
+    return fail(LAMB_ERR_INVALID_ARG,
+                "LAMB_FLAG_DECOUPLED_DECAY applies to lamb_step and "
+                "nlamb_step only");
   if ((h->flags & LAMB_FLAG_LR_SCHEDULE) &&
       !(h->lr_base >= 0.0 && std::isfinite(h->lr_base) &&
         h->lr_warmup_steps >= 0 && h->lr_total_steps >= 1))
@@ -537,6 +560,12 @@ static void fill_params(lamb_plan* p, const lamb_hyper_t* h, int64_t* d_step,
   sp->phi = h->phi;
   sp->flags = h->flags;
   sp->n_chunks = (int32_t)p->n_chunks;
+  sp->grad_slots = p->grad_slots;
+  sp->gsq = p->grad_sq;
+  sp->gnorm = p->grad_norm;
+  sp->gcheck = p->grad_check;
+  sp->n_tensors = p->n_tensors;
+  sp->n_live = p->n_live;
   if (h->flags & LAMB_FLAG_LR_SCHEDULE) {
     sp->lr_base = h->lr_base;
     sp->lr_warmup = h->lr_warmup_steps;
@@ -573,7 +602,12 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
   cudaError_t e = cudaSuccess;
   if (timed) e = cudaEventRecord(ev[0], stream);
   int rc = (int)e;
-  if (plan->algorithm == LAMB_ALGO_SINGLE_TOUCH) {
+  // the single-touch kernel implements the plain step; the gradient check,
+  // the skip mode and decoupled decay run on the two-pass kernels
+  const uint32_t two_pass_only = LAMB_FLAG_GRAD_NORM | LAMB_FLAG_SKIP_NONFINITE |
+                                 LAMB_FLAG_DECOUPLED_DECAY;
+  if (plan->algorithm == LAMB_ALGO_SINGLE_TOUCH &&
+      !(hyper->flags & two_pass_only)) {
     FusedParams fp;
     fp.items = plan->items;
     fp.fchunks = plan->fchunks;
@@ -593,12 +627,14 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
     return LAMB_OK;
   }
   if (!rc)
-    rc = lamb ? launch_lamb_pass1(sp, plan->grad_bf16, plan->grid[0], stream)
+    rc = lamb ? launch_lamb_pass1(sp, 0, plan->grad_bf16, plan->grid[0], stream)
               : launch_lars_pass1(sp, plan->grad_bf16, plan->grid[2], stream);
   if (!rc && timed) rc = (int)cudaEventRecord(ev[1], stream);
   if (!rc)
-    rc = lamb ? launch_lamb_pass2(sp, plan->copy_bf16, plan->grid[1], stream)
-              : launch_lars_pass2(sp, plan->copy_bf16, plan->grid[3], stream);
+    rc = lamb ? launch_lamb_pass2(sp, 0, plan->grad_bf16, plan->copy_bf16,
+                                  plan->grid[1], stream)
+              : launch_lars_pass2(sp, plan->grad_bf16, plan->copy_bf16,
+                                  plan->grid[3], stream);
   if (!rc && timed) rc = (int)cudaEventRecord(ev[2], stream);
   if (rc) return cuda_fail((cudaError_t)rc, lamb ? "lamb_step" : "lars_step");
   if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = 2;
@@ -648,11 +684,11 @@ lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
                           : nullptr;
   int rc = timed ? (int)cudaEventRecord(ev[0], stream) : 0;
   if (!rc)
-    rc = launch_nlamb_pass1(sp, nest, plan->grad_bf16, plan->grid[0], stream);
+    rc = launch_lamb_pass1(sp, nest, plan->grad_bf16, plan->grid[0], stream);
   if (!rc && timed) rc = (int)cudaEventRecord(ev[1], stream);
   if (!rc)
-    rc = launch_nlamb_pass2(sp, nest, plan->grad_bf16, plan->copy_bf16,
-                            plan->grid[1], stream);
+    rc = launch_lamb_pass2(sp, nest, plan->grad_bf16, plan->copy_bf16,
+                           plan->grid[1], stream);
   if (!rc && timed) rc = (int)cudaEventRecord(ev[2], stream);
   if (rc) return cuda_fail((cudaError_t)rc, "nlamb_step");
   if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = 2;
@@ -666,6 +702,38 @@ lamb_status_t lamb_plan_trust_ratios(lamb_plan_t plan, const double** d_ratio,
   if (d_ratio) *d_ratio = plan->ratio;
   if (d_wnorm) *d_wnorm = plan->wnorm;
   if (d_unorm) *d_unorm = plan->unorm;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_grad_norms(lamb_plan_t plan, const double** d_gnorm,
+                                   const double** d_gnorm_global,
+                                   const uint32_t** d_nonfinite) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  if (d_gnorm) *d_gnorm = plan->grad_norm;
+  if (d_gnorm_global) *d_gnorm_global = &plan->grad_check->norm;
+  if (d_nonfinite) *d_nonfinite = &plan->grad_check->nonfinite;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_copy_grad_norms(lamb_plan_t plan, double* gnorm,
+                                        double* gnorm_global,
+                                        uint32_t* nonfinite,
+                                        cudaStream_t stream) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  cudaError_t e = cudaSuccess;
+  if (gnorm)
+    e = cudaMemcpyAsync(gnorm, plan->grad_norm,
+                        (size_t)plan->n_tensors * sizeof(double),
+                        cudaMemcpyDefault, stream);
+  if (e == cudaSuccess && gnorm_global)
+    e = cudaMemcpyAsync(gnorm_global, &plan->grad_check->norm, sizeof(double),
+                        cudaMemcpyDefault, stream);
+  if (e == cudaSuccess && nonfinite)
+    e = cudaMemcpyAsync(nonfinite, &plan->grad_check->nonfinite,
+                        sizeof(uint32_t), cudaMemcpyDefault, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "grad norm copy");
   return LAMB_OK;
 }
 

@@ -10,6 +10,10 @@
 //                                       reset to 0 by the last one
 //   double     ratio/wnorm/unorm[n_tensors]  per-tensor results
 //   StepScalars, status word, work counters
+//   float2     grad_slots[n_chunks] 8 B  per-chunk (sum g^2, sum 0*g), pass 1
+//                                       with the gradient check
+//   double     gsq/gnorm[n_tensors]     per-tensor sum g^2 and ||g_k||
+//   GradCheck                           global ||g|| and the step's verdict
 #pragma once
 #include <stdint.h>
 
@@ -60,9 +64,21 @@ struct __align__(16) StepScalars {
 };
 
 enum : uint32_t { kStatusNonfinite = 1u, kStatusBadStep = 2u,
-                  kStatusWaitTimeout = 4u };
+                  kStatusWaitTimeout = 4u, kStatusGradNonfinite = 8u,
+                  kStatusSkipped = 16u };
 enum : uint32_t { kFlagBiasCorrection = 1u, kFlagIncrementStep = 2u,
-                  kFlagLrSchedule = 4u };
+                  kFlagLrSchedule = 4u, kFlagGradNorm = 8u,
+                  kFlagSkipNonfinite = 16u, kFlagDecoupledDecay = 32u };
+
+// Gradient check of one step (kFlagGradNorm / kFlagSkipNonfinite).  Pass 1
+// forms it; pass 2 reads the verdict before it writes anything.
+struct __align__(16) GradCheck {
+  double norm;          // sqrt(sum over all tensors of sum g^2)
+  uint32_t nonfinite;   // 1: some element of g was Inf or NaN
+  uint32_t acc;         // OR of the tensors' flags while pass 1 runs
+  uint32_t done;        // tensors finalised by the running pass 1 (ticket)
+  uint32_t pad;
+};
 
 struct StepParams {
   const ChunkDesc* chunks;
@@ -94,6 +110,14 @@ struct StepParams {
   double lr_base;
   int64_t lr_warmup, lr_total;
   float* d_lr_out;        // where the applied eta_t is written (may be null)
+  // gradient check (kFlagGradNorm / kFlagSkipNonfinite)
+  float2* grad_slots;     // per chunk (sum g^2, sum 0*g); the second is 0,
+                          // or NaN if some element is Inf/NaN
+  double* gsq;            // per tensor sum g^2
+  double* gnorm;          // per tensor ||g_k||
+  GradCheck* gcheck;
+  int32_t n_tensors;
+  int32_t n_live;         // tensors with at least one chunk
 };
 
 // ---------------------------------------------------------------------------
@@ -140,19 +164,16 @@ struct FusedParams {
 
 // Launchers (lamb_kernels.cu).  grid = number of CTAs of the persistent grid.
 // Return cudaError_t as int to keep this header free of CUDA includes.
-int launch_lamb_pass1(const StepParams& p, int grad_bf16, int grid,
+// nest: 0 LAMB, 1 N-LAMB, 2 NN-LAMB.  The gradient-check and deferred-moment
+// variants are chosen from p.flags.
+int launch_lamb_pass1(const StepParams& p, int nest, int grad_bf16, int grid,
                       void* stream);
-int launch_lamb_pass2(const StepParams& p, int copy_bf16, int grid,
-                      void* stream);
+int launch_lamb_pass2(const StepParams& p, int nest, int grad_bf16,
+                      int copy_bf16, int grid, void* stream);
 int launch_lars_pass1(const StepParams& p, int grad_bf16, int grid,
                       void* stream);
-int launch_lars_pass2(const StepParams& p, int copy_bf16, int grid,
-                      void* stream);
-// N-LAMB (nest = 1) / NN-LAMB (nest = 2), two-pass.
-int launch_nlamb_pass1(const StepParams& p, int nest, int grad_bf16, int grid,
-                       void* stream);
-int launch_nlamb_pass2(const StepParams& p, int nest, int grad_bf16,
-                       int copy_bf16, int grid, void* stream);
+int launch_lars_pass2(const StepParams& p, int grad_bf16, int copy_bf16,
+                      int grid, void* stream);
 int launch_fused(const StepParams& p, const FusedParams& f, int lars,
                  int grad_bf16, int copy_bf16, int grid, void* stream);
 int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks);

@@ -17,6 +17,18 @@
 //
 // LARS (Algorithm 1) has the same shape with u = m_t.
 //
+// Optional, chosen per step from the flags:
+//   gradient check  pass 1 also sums g^2 per chunk and 0*g (0, or NaN once
+//                   any element is Inf/NaN); the tensors' finalisers form
+//                   ||g_k||, and the last one the global ||g|| and the
+//                   step's verdict.
+//   skip mode       pass 1 leaves m, v untouched; pass 2 reads the verdict
+//                   first and either writes nothing or forms the moments
+//                   from g itself and writes m, v, w (42 instead of 40 bytes
+//                   per parameter with bf16 g).
+//   decoupled decay lambda_k w leaves u and is applied outside the trust
+//                   ratio: w <- w - eta rho u - eta lambda_k w.
+//
 // Both passes are persistent grids (CTAs = SMs x resident CTAs per SM) that
 // draw chunks from a device work counter, so hundreds of tiny tensors and a
 // 31M-element embedding share one launch.  The grid never waits on itself:
@@ -24,10 +36,10 @@
 // The last CTA to draw from a counter resets it (and the last chunk of a
 // tensor resets its ticket), so the kernels can be replayed from a CUDA
 // graph with no host involvement.
-#include <cuda_runtime.h>
-#include <cuda_bf16.h>
 
-#include "lamb_internal.h"
+#include <type_traits>
+
+#include "lamb_device.cuh"
 
 namespace lamb {
 namespace {
@@ -35,178 +47,77 @@ namespace {
 constexpr int kUnroll1 = 4;   // 4-element packets in flight per thread, pass 1
 constexpr int kUnroll2 = 4;   // same for pass 2
 
-// ---------------------------------------------------------------------------
-// Element arithmetic.  Every operation is an explicit round-to-nearest
-// intrinsic, so the compiler cannot fuse differently in the two passes.
-// ---------------------------------------------------------------------------
-struct LambConsts {
-  float b1, omb1, b2, omb2;   // beta1, 1-beta1, beta2, 1-beta2
-  float c1, c2;               // 1/(1-beta1^t), 1/(1-beta2^t)
-  float eps;
-  float am, ag, bv, bg;       // N-LAMB / NN-LAMB direction coefficients
-};
-
-// Alg. 2: m_t = beta1 m + (1-beta1) g ;  v_t = beta2 v + (1-beta2) g^2
-__device__ __forceinline__ void lamb_moments(float g, float& m, float& v,
-                                             const LambConsts& k) {
-  m = __fmaf_rn(k.b1, m, __fmul_rn(k.omb1, g));
-  v = __fmaf_rn(k.b2, v, __fmul_rn(k.omb2, __fmul_rn(g, g)));
-}
-
-// Alg. 2: u = (m_t c1) / (sqrt(v_t c2) + eps) + lambda_k w
-__device__ __forceinline__ float lamb_direction(float m, float v, float w,
-                                                float lam,
-                                                const LambConsts& k) {
-  const float mh = __fmul_rn(m, k.c1);
-  const float vh = __fmul_rn(v, k.c2);
-  const float den = __fadd_rn(__fsqrt_rn(vh), k.eps);
-  return __fmaf_rn(lam, w, __fdiv_rn(mh, den));
-}
-
-// Appendix Alg. 3 / 4 (N-LAMB / NN-LAMB):
-//   u = (am m_t + ag g) / (sqrt(bv v_t [+ bg g^2]) + eps) + lambda_k w
-// with am = mu_{t+1}/(1 - prod_{i<=t+1} mu_i), ag = (1 - mu_t)/(1 - prod_{i<=t}
-// mu_i); N-LAMB: bv = 1/(1 - beta2^t); NN-LAMB: bv = beta2/(1 - beta2^(t+1)),
-// bg = (1 - beta2)/(1 - beta2^t).
-template <int kNest>
-__device__ __forceinline__ float nlamb_direction(float m, float v, float g,
-                                                 float w, float lam,
-                                                 const LambConsts& k) {
-  const float mh = __fmaf_rn(k.am, m, __fmul_rn(k.ag, g));
-  const float vh = kNest == 2
-                       ? __fmaf_rn(k.bv, v, __fmul_rn(k.bg, __fmul_rn(g, g)))
-                       : __fmul_rn(v, k.bv);
-  const float den = __fadd_rn(__fsqrt_rn(vh), k.eps);
-  return __fmaf_rn(lam, w, __fdiv_rn(mh, den));
-}
-
-// Alg. 1: m_t = beta1 m + (1-beta1) (g + lambda_k w)
-__device__ __forceinline__ float lars_momentum(float g, float m, float w,
-                                               float lam, float b1,
-                                               float omb1) {
-  return __fmaf_rn(b1, m, __fmul_rn(omb1, __fmaf_rn(lam, w, g)));
-}
-
-// ---------------------------------------------------------------------------
-// Memory helpers
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ float4 ld4(const float* p) {
-  return *reinterpret_cast<const float4*>(p);
-}
-__device__ __forceinline__ float4 ld4_last(const float* p) {  // last use
-  return __ldcs(reinterpret_cast<const float4*>(p));
-}
-__device__ __forceinline__ void st4(float* p, float4 x) {
-  *reinterpret_cast<float4*>(p) = x;
-}
-__device__ __forceinline__ void st4_last(float* p, float4 x) {
-  __stcs(reinterpret_cast<float4*>(p), x);
-}
-
-// Gradients are read exactly once: streaming (evict-first) loads.
-__device__ __forceinline__ float4 ld_grad4(const float* p) {
-  return __ldcs(reinterpret_cast<const float4*>(p));
-}
-// bf16 -> f32 widening is exact: the bf16 pattern is the top half of the f32.
-__device__ __forceinline__ float4 ld_grad4(const __nv_bfloat16* p) {
-  const uint2 u = __ldcs(reinterpret_cast<const uint2*>(p));
-  return make_float4(__uint_as_float(u.x << 16),
-                     __uint_as_float(u.x & 0xffff0000u),
-                     __uint_as_float(u.y << 16),
-                     __uint_as_float(u.y & 0xffff0000u));
-}
-__device__ __forceinline__ float ld_grad1(const float* p) { return __ldcs(p); }
-__device__ __forceinline__ float ld_grad1(const __nv_bfloat16* p) {
-  const unsigned short h = __ldcs(reinterpret_cast<const unsigned short*>(p));
-  return __uint_as_float(uint32_t(h) << 16);
-}
-
-__device__ __forceinline__ void st_copy4(void* base, int64_t i, float4 x) {
-  const __nv_bfloat162 lo = __floats2bfloat162_rn(x.x, x.y);  // RNE
-  const __nv_bfloat162 hi = __floats2bfloat162_rn(x.z, x.w);
-  uint2 u;
-  u.x = *reinterpret_cast<const uint32_t*>(&lo);
-  u.y = *reinterpret_cast<const uint32_t*>(&hi);
-  __stcs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(base) + i), u);
-}
-__device__ __forceinline__ void st_copy1(void* base, int64_t i, float x) {
-  static_cast<__nv_bfloat16*>(base)[i] = __float2bfloat16_rn(x);
-}
-
-// ---------------------------------------------------------------------------
-// Reductions: fixed trees, so the result depends only on the data layout.
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ float warp_sum(float x) {
+// Sums of the first N of x[] over the CTA, valid in thread 0 (fixed trees:
+// lanes, then warps).  Contains one barrier; red must hold N rows.
+template <int N>
+__device__ __forceinline__ void cta_sum(float* x, float (*red)[kWarps]) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x += __shfl_down_sync(0xffffffffu, x, o);
-  return x;
-}
-
-// Sum of (a, b) over the CTA, valid in thread 0.  Contains one barrier.
-__device__ __forceinline__ float2 cta_sum2(float a, float b,
-                                           float (*red)[kWarps]) {
-  a = warp_sum(a);
-  b = warp_sum(b);
+  for (int i = 0; i < N; ++i) x[i] = warp_sum(x[i]);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (lane == 0) {
-    red[0][warp] = a;
-    red[1][warp] = b;
+#pragma unroll
+    for (int i = 0; i < N; ++i) red[i][warp] = x[i];
   }
   __syncthreads();
-  float2 r = make_float2(0.f, 0.f);
   if (warp == 0) {
-    a = lane < kWarps ? red[0][lane] : 0.f;
-    b = lane < kWarps ? red[1][lane] : 0.f;
-    r = make_float2(warp_sum(a), warp_sum(b));
+#pragma unroll
+    for (int i = 0; i < N; ++i) x[i] = warp_sum(lane < kWarps ? red[i][lane] : 0.f);
   }
-  return r;
 }
 
-// eta_t: read from device memory, or (kFlagLrSchedule) the Section 4
-// schedule eta_0 t / T_w during warmup, then eta_0 max(0, 1 - t / T).
-__device__ __forceinline__ float step_lr(const StepParams& p, int64_t t) {
-  if (!(p.flags & kFlagLrSchedule)) return *p.d_lr;
-  double lr;
-  if (p.lr_warmup > 0 && t < p.lr_warmup)
-    lr = p.lr_base * (double)t / (double)p.lr_warmup;
-  else
-    lr = p.lr_base * fmax(0.0, 1.0 - (double)t / (double)p.lr_total);
-  return (float)lr;
-}
-
-// The CTA or warp that closes a step: advance the step counter and report
-// the scheduled learning rate.
-__device__ __forceinline__ void close_step(const StepParams& p,
-                                           const StepScalars& sc) {
-  if ((p.flags & kFlagLrSchedule) && p.d_lr_out) *p.d_lr_out = sc.lr;
-  if ((p.flags & kFlagIncrementStep) && p.d_step) *p.d_step = sc.t + 1;
-}
-
-__device__ __forceinline__ double phi_of(double z, const StepParams& p) {
-  if (p.phi == 1) {  // clip; comparisons keep NaN as NaN
-    if (z < p.gamma_l) return p.gamma_l;
-    if (z > p.gamma_u) return p.gamma_u;
+// The tensor that finishes last in pass 1 (gradient check only): the global
+// ||g|| as a fixed-order fp64 sum over the tensors' sum g^2, and the step's
+// verdict, which pass 2 reads before it writes anything.  Warp-wide.
+__device__ __forceinline__ void finalize_grad(const StepParams& p) {
+  __threadfence();
+  const int lane = threadIdx.x & 31;
+  double a = 0.0;
+  for (int k = lane; k < p.n_tensors; k += 32) a += __ldcg(&p.gsq[k]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) a += __shfl_down_sync(0xffffffffu, a, o);
+  if (lane == 0) {
+    const uint32_t bad = atomicExch(&p.gcheck->acc, 0u);
+    p.gcheck->norm = sqrt(a);
+    p.gcheck->nonfinite = bad;
+    if (bad)
+      atomicOr(p.status, kStatusGradNonfinite |
+                             ((p.flags & kFlagSkipNonfinite) ? kStatusSkipped
+                                                             : 0u));
+    p.gcheck->done = 0u;
   }
-  return z;
 }
 
 // Warp 0 of the CTA that finished tensor k's last chunk: fixed-order fp64
 // combine of the chunk slots -> norms and trust ratio.  Resets the ticket.
+// With the gradient check (kGn) it also forms the tensor's sum g^2 and
+// whether any of its elements was Inf/NaN, and counts the tensor done.
+template <bool kGn>
 __device__ __noinline__ void finalize_tensor(const StepParams& p, int k,
                                              int first, int n, double coef) {
   __threadfence();
   const int lane = threadIdx.x & 31;
-  double aw = 0.0, au = 0.0;
+  double aw = 0.0, au = 0.0, ag = 0.0;
+  float az = 0.f;
   for (int i = lane; i < n; i += 32) {
     const float2 s = __ldcg(&p.slots[first + i]);
     aw += (double)s.x;
     au += (double)s.y;
+    if (kGn) {
+      const float2 q = __ldcg(&p.grad_slots[first + i]);
+      ag += (double)q.x;
+      az += q.y;
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     aw += __shfl_down_sync(0xffffffffu, aw, o);
     au += __shfl_down_sync(0xffffffffu, au, o);
+    if (kGn) {
+      ag += __shfl_down_sync(0xffffffffu, ag, o);
+      az += __shfl_down_sync(0xffffffffu, az, o);
+    }
   }
+  int last_tensor = 0;
   if (lane == 0) {
     const double wn = sqrt(aw), un = sqrt(au);
     double rho = 1.0;                                  // zero-norm rule
@@ -215,27 +126,39 @@ __device__ __noinline__ void finalize_tensor(const StepParams& p, int k,
     p.wnorm[k] = wn;
     p.unorm[k] = un;
     if (!isfinite(aw) || !isfinite(au)) atomicOr(p.status, kStatusNonfinite);
+    if (kGn) {
+      p.gsq[k] = ag;
+      p.gnorm[k] = sqrt(ag);
+      if (isnan(az)) atomicOr(&p.gcheck->acc, 1u);
+      __threadfence();
+      last_tensor =
+          atomicAdd(&p.gcheck->done, 1u) + 1u == (uint32_t)p.n_live;
+    }
     p.tickets[k] = 0u;
   }
+  if (kGn && __shfl_sync(0xffffffffu, last_tensor, 0)) finalize_grad(p);
 }
 
-// Chunk epilogue of pass 1: publish the CTA's partial sums, take a ticket,
-// and let the last chunk of the tensor finalise it.
+// Chunk epilogue of pass 1: publish the CTA's partial sums (acc[0] = sum w^2,
+// acc[1] = sum u^2; with kGn also acc[2] = sum g^2, acc[3] = sum 0*g), take a
+// ticket, and let the last chunk of the tensor finalise it.
+template <bool kGn>
 __device__ __forceinline__ void publish_chunk(const StepParams& p, int c,
                                               const ChunkDesc& ch,
-                                              const TensorDesc& td, float sw,
-                                              float su, float (*red)[kWarps],
+                                              const TensorDesc& td, float* acc,
+                                              float (*red)[kWarps],
                                               int* s_last, double coef) {
-  const float2 tot = cta_sum2(sw, su, red);
+  cta_sum<kGn ? 4 : 2>(acc, red);
   if (threadIdx.x == 0) {
-    p.slots[c] = tot;
+    p.slots[c] = make_float2(acc[0], acc[1]);
+    if (kGn) p.grad_slots[c] = make_float2(acc[2], acc[3]);
     __threadfence();
     const uint32_t prev = atomicAdd(&p.tickets[ch.tensor], 1u);
     *s_last = (prev + 1u == (uint32_t)td.n_chunks);
   }
   __syncthreads();
   if (*s_last && threadIdx.x < 32)
-    finalize_tensor(p, ch.tensor, td.first_chunk, td.n_chunks, coef);
+    finalize_tensor<kGn>(p, ch.tensor, td.first_chunk, td.n_chunks, coef);
 }
 
 // Work distribution.  Thread 0 draws chunk indices from counters[which];
@@ -249,26 +172,36 @@ __device__ __forceinline__ bool retire(const StepParams& p, int which,
   return last;
 }
 
+
 // ---------------------------------------------------------------------------
-// LAMB pass 1
+// LAMB pass 1 (also N-LAMB / NN-LAMB: kNest = 1 / 2)
+//
+// acc[] accumulates per thread: sum w^2, sum u^2 and, with the gradient check
+// (kGn), sum g^2 and sum 0*g -- the last is 0 unless some g is Inf or NaN,
+// which makes it NaN whatever the order of the sum.  store = false (the
+// skip-on-non-finite mode) leaves m, v untouched: pass 2 forms and writes
+// them once the step is known to be applied.
 // ---------------------------------------------------------------------------
-template <int kNest>
+template <int kNest, bool kGn>
 __device__ __forceinline__ void lamb1_elem(float g, float& m, float& v,
                                            float w, float lam,
-                                           const LambConsts& k, float& sw,
-                                           float& su) {
+                                           const LambConsts& k, float* acc) {
   lamb_moments(g, m, v, k);
   const float u = kNest ? nlamb_direction<kNest>(m, v, g, w, lam, k)
                         : lamb_direction(m, v, w, lam, k);
-  sw = __fmaf_rn(w, w, sw);
-  su = __fmaf_rn(u, u, su);
+  acc[0] = __fmaf_rn(w, w, acc[0]);
+  acc[1] = __fmaf_rn(u, u, acc[1]);
+  if (kGn) {
+    acc[2] = __fmaf_rn(g, g, acc[2]);
+    acc[3] = __fmaf_rn(g, 0.f, acc[3]);
+  }
 }
 
-template <typename GT, int kNest>
+template <typename GT, int kNest, bool kGn>
 __device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
                                             const ChunkDesc& ch, float lam,
-                                            const LambConsts& k, float& sw,
-                                            float& su) {
+                                            const LambConsts& k, bool store,
+                                            float* acc) {
   float* __restrict__ w = tp.w + ch.offset;
   float* __restrict__ m = tp.m + ch.offset;
   float* __restrict__ v = tp.v + ch.offset;
@@ -293,12 +226,14 @@ __device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
       for (int u = 0; u < kUnroll1; ++u) {
         const int j = base + u * kThreads;
         if (j < nv) {
-          lamb1_elem<kNest>(gv[u].x, mv[u].x, vv[u].x, wv[u].x, lam, k, sw, su);
-          lamb1_elem<kNest>(gv[u].y, mv[u].y, vv[u].y, wv[u].y, lam, k, sw, su);
-          lamb1_elem<kNest>(gv[u].z, mv[u].z, vv[u].z, wv[u].z, lam, k, sw, su);
-          lamb1_elem<kNest>(gv[u].w, mv[u].w, vv[u].w, wv[u].w, lam, k, sw, su);
-          st4(m + 4 * j, mv[u]);
-          st4(v + 4 * j, vv[u]);
+          lamb1_elem<kNest, kGn>(gv[u].x, mv[u].x, vv[u].x, wv[u].x, lam, k, acc);
+          lamb1_elem<kNest, kGn>(gv[u].y, mv[u].y, vv[u].y, wv[u].y, lam, k, acc);
+          lamb1_elem<kNest, kGn>(gv[u].z, mv[u].z, vv[u].z, wv[u].z, lam, k, acc);
+          lamb1_elem<kNest, kGn>(gv[u].w, mv[u].w, vv[u].w, wv[u].w, lam, k, acc);
+          if (store) {
+            st4(m + 4 * j, mv[u]);
+            st4(v + 4 * j, vv[u]);
+          }
         }
       }
     }
@@ -306,9 +241,11 @@ __device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
   }
   for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
     float mi = m[i], vi = v[i];
-    lamb1_elem<kNest>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
-    m[i] = mi;
-    v[i] = vi;
+    lamb1_elem<kNest, kGn>(ld_grad1(g + i), mi, vi, w[i], lam, k, acc);
+    if (store) {
+      m[i] = mi;
+      v[i] = vi;
+    }
   }
 }
 
@@ -319,10 +256,17 @@ __device__ __forceinline__ double nadam_mu(double beta1, double psi,
   return beta1 * (1.0 - 0.5 * pow(0.96, (double)t * psi));
 }
 
-template <typename GT, int kNest>
+// lambda_k inside the normalised direction u (Alg. 2); 0 with decoupled
+// decay, where pass 2 applies lambda_k w outside the trust ratio instead.
+__device__ __forceinline__ float lam_in_u(const StepParams& p,
+                                          const TensorDesc& td) {
+  return (p.flags & kFlagDecoupledDecay) ? 0.f : td.decay * p.wd;
+}
+
+template <typename GT, int kNest, bool kGn>
 __global__ void __launch_bounds__(kThreads)
     lamb_pass1_kernel(const StepParams p) {
-  __shared__ float red[2][kWarps];
+  __shared__ float red[4][kWarps];
   __shared__ uint32_t s_next[2];
   __shared__ int s_last, s_skip;
   __shared__ LambConsts s_k;
@@ -374,6 +318,7 @@ __global__ void __launch_bounds__(kThreads)
   __syncthreads();
   if (s_skip) return;
   const LambConsts k = s_k;
+  const bool store = !(kGn && (p.flags & kFlagSkipNonfinite));
   int it = 0;
   uint32_t c = s_next[0];
   while (c < (uint32_t)p.n_chunks) {
@@ -381,10 +326,9 @@ __global__ void __launch_bounds__(kThreads)
     const ChunkDesc ch = p.chunks[c];
     const TensorDesc td = p.tensors[ch.tensor];
     const TensorPtrs tp = p.ptrs[ch.tensor];
-    const float lam = td.decay * p.wd;
-    float sw = 0.f, su = 0.f;
-    lamb1_chunk<GT, kNest>(tp, ch, lam, k, sw, su);
-    publish_chunk(p, (int)c, ch, td, sw, su, red, &s_last, 1.0);
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    lamb1_chunk<GT, kNest, kGn>(tp, ch, lam_in_u(p, td), k, store, acc);
+    publish_chunk<kGn>(p, (int)c, ch, td, acc, red, &s_last, 1.0);
     ++it;
     c = s_next[it & 1];
   }
@@ -393,8 +337,14 @@ __global__ void __launch_bounds__(kThreads)
 
 // ---------------------------------------------------------------------------
 // LAMB pass 2
+//
+// w <- w - s u with s = eta rho_k, u recomputed bit-identically from the
+// pass-1 operands.  kDefer (skip-on-non-finite mode): m, v still hold the
+// previous step's values, so the moments are formed here from g and written
+// together with w.  Decoupled decay (dd = eta lambda_k != 0): w <- w - s u -
+// dd w; with dd == 0 the extra term is skipped, not added as a zero, so the
+// plain step keeps w - s u bit for bit (signed zeros, Inf - Inf).
 // ---------------------------------------------------------------------------
-// Pass-2 direction: LAMB from m, v, w; N-LAMB / NN-LAMB also need g.
 template <int kNest>
 __device__ __forceinline__ float lamb2_dir(float m, float v, float g, float w,
                                            float lam, const LambConsts& k) {
@@ -402,13 +352,25 @@ __device__ __forceinline__ float lamb2_dir(float m, float v, float g, float w,
                : lamb_direction(m, v, w, lam, k);
 }
 
-template <bool kCopy, int kNest, typename GT>
+template <int kNest, bool kDefer>
+__device__ __forceinline__ float lamb2_elem(float g, float& m, float& v,
+                                            float w, float lam, float s,
+                                            float dd, const LambConsts& k) {
+  if (kDefer) lamb_moments(g, m, v, k);
+  float o = __fmaf_rn(-s, lamb2_dir<kNest>(m, v, g, w, lam, k), w);
+  if (dd != 0.f) o = __fmaf_rn(-dd, w, o);
+  return o;
+}
+
+template <bool kCopy, int kNest, typename GT, bool kDefer>
 __device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
                                             const ChunkDesc& ch, float lam,
-                                            float s, const LambConsts& k) {
+                                            float s, float dd,
+                                            const LambConsts& k) {
+  constexpr bool kG = kNest != 0 || kDefer;   // reads g
   float* __restrict__ w = tp.w + ch.offset;
-  const float* __restrict__ m = tp.m + ch.offset;
-  const float* __restrict__ v = tp.v + ch.offset;
+  float* __restrict__ m = tp.m + ch.offset;
+  float* __restrict__ v = tp.v + ch.offset;
   const GT* __restrict__ g = static_cast<const GT*>(tp.g) + ch.offset;
   const int n = ch.len;
   int scalar_from = 0;
@@ -423,7 +385,7 @@ __device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
           mv[u] = ld4_last(m + 4 * j);
           vv[u] = ld4_last(v + 4 * j);
           wv[u] = ld4_last(w + 4 * j);
-          if (kNest) gv[u] = ld_grad4(g + 4 * j);
+          if (kG) gv[u] = ld_grad4(g + 4 * j);
         }
       }
 #pragma unroll
@@ -431,11 +393,15 @@ __device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
         const int j = base + u * kThreads;
         if (j < nv) {
           float4 o;
-          if (!kNest) gv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-          o.x = __fmaf_rn(-s, lamb2_dir<kNest>(mv[u].x, vv[u].x, gv[u].x, wv[u].x, lam, k), wv[u].x);
-          o.y = __fmaf_rn(-s, lamb2_dir<kNest>(mv[u].y, vv[u].y, gv[u].y, wv[u].y, lam, k), wv[u].y);
-          o.z = __fmaf_rn(-s, lamb2_dir<kNest>(mv[u].z, vv[u].z, gv[u].z, wv[u].z, lam, k), wv[u].z);
-          o.w = __fmaf_rn(-s, lamb2_dir<kNest>(mv[u].w, vv[u].w, gv[u].w, wv[u].w, lam, k), wv[u].w);
+          if (!kG) gv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+          o.x = lamb2_elem<kNest, kDefer>(gv[u].x, mv[u].x, vv[u].x, wv[u].x, lam, s, dd, k);
+          o.y = lamb2_elem<kNest, kDefer>(gv[u].y, mv[u].y, vv[u].y, wv[u].y, lam, s, dd, k);
+          o.z = lamb2_elem<kNest, kDefer>(gv[u].z, mv[u].z, vv[u].z, wv[u].z, lam, s, dd, k);
+          o.w = lamb2_elem<kNest, kDefer>(gv[u].w, mv[u].w, vv[u].w, wv[u].w, lam, s, dd, k);
+          if (kDefer) {
+            st4_last(m + 4 * j, mv[u]);
+            st4_last(v + 4 * j, vv[u]);
+          }
           st4_last(w + 4 * j, o);
           if (kCopy) st_copy4(tp.copy, ch.offset + 4 * j, o);
         }
@@ -444,23 +410,31 @@ __device__ __forceinline__ void lamb2_chunk(const TensorPtrs& tp,
     scalar_from = nv << 2;
   }
   for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
-    const float wi = w[i];
-    const float gi = kNest ? ld_grad1(g + i) : 0.f;
-    const float o =
-        __fmaf_rn(-s, lamb2_dir<kNest>(m[i], v[i], gi, wi, lam, k), wi);
+    float mi = m[i], vi = v[i];
+    const float gi = kG ? ld_grad1(g + i) : 0.f;
+    const float o = lamb2_elem<kNest, kDefer>(gi, mi, vi, w[i], lam, s,
+                                                   dd, k);
+    if (kDefer) {
+      m[i] = mi;
+      v[i] = vi;
+    }
     w[i] = o;
     if (kCopy) st_copy1(tp.copy, ch.offset + i, o);
   }
 }
 
-template <bool kCopy, int kNest, typename GT>
+template <bool kCopy, int kNest, typename GT, bool kDefer>
 __global__ void __launch_bounds__(kThreads)
     lamb_pass2_kernel(const StepParams p) {
   __shared__ uint32_t s_next[2];
   const StepScalars sc = *p.scal;
   if (sc.skip) return;
+  // a step whose gradients held an Inf/NaN writes nothing (and does not
+  // advance t); no CTA draws, so the work counter stays at 0
+  if (kDefer && p.gcheck->nonfinite) return;
   const LambConsts k{p.b1, p.omb1, p.b2, p.omb2, sc.c1, sc.c2, p.eps,
                      sc.am, sc.ag, sc.bv, sc.bg};
+  const bool decoupled = (p.flags & kFlagDecoupledDecay) != 0;
   if (threadIdx.x == 0) s_next[0] = atomicAdd(&p.counters[1], 1u);
   __syncthreads();
   int it = 0;
@@ -472,9 +446,12 @@ __global__ void __launch_bounds__(kThreads)
     const ChunkDesc ch = p.chunks[nc - 1 - (int)c];
     const TensorDesc td = p.tensors[ch.tensor];
     const TensorPtrs tp = p.ptrs[ch.tensor];
-    const float lam = td.decay * p.wd;
+    const float lamk = td.decay * p.wd;
     const float s = __double2float_rn((double)sc.lr * p.ratio[ch.tensor]);
-    lamb2_chunk<kCopy, kNest, GT>(tp, ch, lam, s, k);
+    const float dd =
+        decoupled ? __double2float_rn((double)sc.lr * (double)lamk) : 0.f;
+    lamb2_chunk<kCopy, kNest, GT, kDefer>(tp, ch, decoupled ? 0.f : lamk, s,
+                                          dd, k);
     __syncthreads();  // s_next[(it+1)&1] visible; old slot free to reuse
     ++it;
     c = s_next[it & 1];
@@ -486,13 +463,26 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // ---------------------------------------------------------------------------
-// LARS pass 1 / pass 2
+// LARS pass 1 / pass 2 (u = m_t; same gradient check and deferred mode)
 // ---------------------------------------------------------------------------
-template <typename GT>
+template <bool kGn>
+__device__ __forceinline__ void lars1_elem(float g, float m, float w,
+                                           float lam, float b1, float omb1,
+                                           float* acc, float& o) {
+  o = lars_momentum(g, m, w, lam, b1, omb1);
+  acc[0] = __fmaf_rn(w, w, acc[0]);
+  acc[1] = __fmaf_rn(o, o, acc[1]);
+  if (kGn) {
+    acc[2] = __fmaf_rn(g, g, acc[2]);
+    acc[3] = __fmaf_rn(g, 0.f, acc[3]);
+  }
+}
+
+template <typename GT, bool kGn>
 __device__ __forceinline__ void lars1_chunk(const TensorPtrs& tp,
                                             const ChunkDesc& ch, float lam,
-                                            float b1, float omb1, float& sw,
-                                            float& su) {
+                                            float b1, float omb1, bool store,
+                                            float* acc) {
   const float* __restrict__ w = tp.w + ch.offset;
   float* __restrict__ m = tp.m + ch.offset;
   const GT* __restrict__ g = static_cast<const GT*>(tp.g) + ch.offset;
@@ -516,37 +506,27 @@ __device__ __forceinline__ void lars1_chunk(const TensorPtrs& tp,
         const int j = base + u * kThreads;
         if (j < nv) {
           float4 o;
-          o.x = lars_momentum(gv[u].x, mv[u].x, wv[u].x, lam, b1, omb1);
-          o.y = lars_momentum(gv[u].y, mv[u].y, wv[u].y, lam, b1, omb1);
-          o.z = lars_momentum(gv[u].z, mv[u].z, wv[u].z, lam, b1, omb1);
-          o.w = lars_momentum(gv[u].w, mv[u].w, wv[u].w, lam, b1, omb1);
-          sw = __fmaf_rn(wv[u].x, wv[u].x, sw);
-          sw = __fmaf_rn(wv[u].y, wv[u].y, sw);
-          sw = __fmaf_rn(wv[u].z, wv[u].z, sw);
-          sw = __fmaf_rn(wv[u].w, wv[u].w, sw);
-          su = __fmaf_rn(o.x, o.x, su);
-          su = __fmaf_rn(o.y, o.y, su);
-          su = __fmaf_rn(o.z, o.z, su);
-          su = __fmaf_rn(o.w, o.w, su);
-          st4(m + 4 * j, o);
+          lars1_elem<kGn>(gv[u].x, mv[u].x, wv[u].x, lam, b1, omb1, acc, o.x);
+          lars1_elem<kGn>(gv[u].y, mv[u].y, wv[u].y, lam, b1, omb1, acc, o.y);
+          lars1_elem<kGn>(gv[u].z, mv[u].z, wv[u].z, lam, b1, omb1, acc, o.z);
+          lars1_elem<kGn>(gv[u].w, mv[u].w, wv[u].w, lam, b1, omb1, acc, o.w);
+          if (store) st4(m + 4 * j, o);
         }
       }
     }
     scalar_from = nv << 2;
   }
   for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
-    const float wi = w[i];
-    const float o = lars_momentum(ld_grad1(g + i), m[i], wi, lam, b1, omb1);
-    m[i] = o;
-    sw = __fmaf_rn(wi, wi, sw);
-    su = __fmaf_rn(o, o, su);
+    float o;
+    lars1_elem<kGn>(ld_grad1(g + i), m[i], w[i], lam, b1, omb1, acc, o);
+    if (store) m[i] = o;
   }
 }
 
-template <typename GT>
+template <typename GT, bool kGn>
 __global__ void __launch_bounds__(kThreads)
     lars_pass1_kernel(const StepParams p) {
-  __shared__ float red[2][kWarps];
+  __shared__ float red[4][kWarps];
   __shared__ uint32_t s_next[2];
   __shared__ int s_last;
   if (threadIdx.x == 0) {
@@ -562,6 +542,7 @@ __global__ void __launch_bounds__(kThreads)
     s_next[0] = atomicAdd(&p.counters[0], 1u);
   }
   __syncthreads();
+  const bool store = !(kGn && (p.flags & kFlagSkipNonfinite));
   int it = 0;
   uint32_t c = s_next[0];
   while (c < (uint32_t)p.n_chunks) {
@@ -570,38 +551,49 @@ __global__ void __launch_bounds__(kThreads)
     const TensorDesc td = p.tensors[ch.tensor];
     const TensorPtrs tp = p.ptrs[ch.tensor];
     const float lam = td.decay * p.wd;
-    float sw = 0.f, su = 0.f;
-    lars1_chunk<GT>(tp, ch, lam, p.b1, p.omb1, sw, su);
-    publish_chunk(p, (int)c, ch, td, sw, su, red, &s_last, p.trust);
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    lars1_chunk<GT, kGn>(tp, ch, lam, p.b1, p.omb1, store, acc);
+    publish_chunk<kGn>(p, (int)c, ch, td, acc, red, &s_last, p.trust);
     ++it;
     c = s_next[it & 1];
   }
   retire(p, 0, c);
 }
 
-template <bool kCopy>
+// kDefer: m still holds m_{t-1}; form m_t here (Alg. 1) and write it with w.
+template <bool kCopy, typename GT, bool kDefer>
 __device__ __forceinline__ void lars2_chunk(const TensorPtrs& tp,
-                                            const ChunkDesc& ch, float s) {
+                                            const ChunkDesc& ch, float s,
+                                            float lam, float b1, float omb1) {
   float* __restrict__ w = tp.w + ch.offset;
-  const float* __restrict__ m = tp.m + ch.offset;
+  float* __restrict__ m = tp.m + ch.offset;
+  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + ch.offset;
   const int n = ch.len;
   int scalar_from = 0;
   if (tp.vec_ok) {
     const int nv = n >> 2;
     for (int base = threadIdx.x; base < nv; base += kThreads * kUnroll2) {
-      float4 wv[kUnroll2], mv[kUnroll2];
+      float4 wv[kUnroll2], mv[kUnroll2], gv[kUnroll2];
 #pragma unroll
       for (int u = 0; u < kUnroll2; ++u) {
         const int j = base + u * kThreads;
         if (j < nv) {
           mv[u] = ld4_last(m + 4 * j);
           wv[u] = ld4_last(w + 4 * j);
+          if (kDefer) gv[u] = ld_grad4(g + 4 * j);
         }
       }
 #pragma unroll
       for (int u = 0; u < kUnroll2; ++u) {
         const int j = base + u * kThreads;
         if (j < nv) {
+          if (kDefer) {
+            mv[u].x = lars_momentum(gv[u].x, mv[u].x, wv[u].x, lam, b1, omb1);
+            mv[u].y = lars_momentum(gv[u].y, mv[u].y, wv[u].y, lam, b1, omb1);
+            mv[u].z = lars_momentum(gv[u].z, mv[u].z, wv[u].z, lam, b1, omb1);
+            mv[u].w = lars_momentum(gv[u].w, mv[u].w, wv[u].w, lam, b1, omb1);
+            st4_last(m + 4 * j, mv[u]);
+          }
           float4 o;
           o.x = __fmaf_rn(-s, mv[u].x, wv[u].x);
           o.y = __fmaf_rn(-s, mv[u].y, wv[u].y);
@@ -615,17 +607,24 @@ __device__ __forceinline__ void lars2_chunk(const TensorPtrs& tp,
     scalar_from = nv << 2;
   }
   for (int i = scalar_from + threadIdx.x; i < n; i += kThreads) {
-    const float o = __fmaf_rn(-s, m[i], w[i]);
+    const float wi = w[i];
+    float mi = m[i];
+    if (kDefer) {
+      mi = lars_momentum(ld_grad1(g + i), mi, wi, lam, b1, omb1);
+      m[i] = mi;
+    }
+    const float o = __fmaf_rn(-s, mi, wi);
     w[i] = o;
     if (kCopy) st_copy1(tp.copy, ch.offset + i, o);
   }
 }
 
-template <bool kCopy>
+template <bool kCopy, typename GT, bool kDefer>
 __global__ void __launch_bounds__(kThreads)
     lars_pass2_kernel(const StepParams p) {
   __shared__ uint32_t s_next[2];
   const StepScalars sc = *p.scal;
+  if (kDefer && p.gcheck->nonfinite) return;   // skipped step: no writes
   if (threadIdx.x == 0) s_next[0] = atomicAdd(&p.counters[1], 1u);
   __syncthreads();
   int it = 0;
@@ -636,812 +635,13 @@ __global__ void __launch_bounds__(kThreads)
     const ChunkDesc ch = p.chunks[nc - 1 - (int)c];
     const TensorPtrs tp = p.ptrs[ch.tensor];
     const float s = __double2float_rn((double)sc.lr * p.ratio[ch.tensor]);
-    lars2_chunk<kCopy>(tp, ch, s);
+    const float lam = kDefer ? p.tensors[ch.tensor].decay * p.wd : 0.f;
+    lars2_chunk<kCopy, GT, kDefer>(tp, ch, s, lam, p.b1, p.omb1);
     __syncthreads();
     ++it;
     c = s_next[it & 1];
   }
   if (retire(p, 1, c) && threadIdx.x == 0) close_step(p, sc);
-}
-
-// ---------------------------------------------------------------------------
-// Single-touch fused step (one persistent kernel, warps are the workers)
-//
-// Items are drawn in schedule order from counters[2].  A pass-1 item runs one
-// fused chunk (512 elements) through Alg. 2's moment and ratio lines (Alg. 1
-// for LARS), stores the new m, v and publishes the chunk's sums; the warp that
-// completes a group of 32 chunks sums them (fp64, fixed order), and the warp
-// that completes a tensor's last group computes its norms and trust ratio and
-// releases ready[k] = epoch.  A pass-2 item applies the update once ready[k]
-// == epoch.  Pass-2 items of a tensor come after all its pass-1 items in the
-// schedule and items are drawn in order, so the earliest unfinished item never
-// waits on anything unfinished: the kernel cannot deadlock.  A wait still
-// gives up after ~0.5 s, sets a status bit and makes every other waiter of
-// the same launch give up at once.
-//
-// Memory pipeline: every warp owns a ring of kStages shared-memory stages and
-// prefetches the operands of its next items with cp.async while it computes
-// the current one, so many bytes are in flight without holding registers.  A
-// pass-2 item is prefetched only if its tensor's norms are already final when
-// its stage is filled (its m, v come from other warps' pass-1 stores);
-// otherwise, and for tail chunks and unaligned tensors, the item reads global
-// memory directly when its turn comes.  The control traffic (draws, item
-// descriptors, ready flags, tickets) is pipelined as described at the warp
-// worker below.
-//
-// L2 policy: pass-1 loads/stores of m, v, w of "resident" tensors (those
-// whose state fits the L2 budget) are evict_last, so pass 2 -- about one
-// wave later -- finds them in L2; gradients and all pass-2 traffic are
-// evict_first.
-// ---------------------------------------------------------------------------
-constexpr int kFusedThreads = 256;                     // 8 warps per CTA
-constexpr int kFusedWarps = kFusedThreads / 32;
-constexpr int kStages = 3;                             // prefetch depth per warp
-constexpr int kPktsPerLane = kFusedChunk / 4 / 32;     // 4-element packets
-static_assert(kPktsPerLane * 4 * 32 == kFusedChunk, "fused chunk shape");
-constexpr uint32_t kSpinLimit = 1u << 21;              // x <= 256 ns ~ 0.5 s
-
-// stage layout: m | v (LAMB only) | w | g
-template <bool kLars, typename GT>
-__host__ __device__ constexpr int stage_bytes() {
-  return kFusedChunk * (4 * (kLars ? 2 : 3) + (int)sizeof(GT));
-}
-template <bool kLars, typename GT>
-__host__ __device__ constexpr int fused_smem_bytes() {
-  return kFusedWarps * kStages * stage_bytes<kLars, GT>();
-}
-constexpr int kOffM = 0;
-constexpr int kOffV = 4 * kFusedChunk;
-template <bool kLars> __host__ __device__ constexpr int off_w() {
-  return 4 * kFusedChunk * (kLars ? 1 : 2);
-}
-template <bool kLars> __host__ __device__ constexpr int off_g() {
-  return 4 * kFusedChunk * (kLars ? 2 : 3);
-}
-
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-__device__ __forceinline__ uint64_t policy_evict_last() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-__device__ __forceinline__ float4 ldp4(const float* p, uint64_t pol) {
-  float4 r;
-  asm volatile(
-      "ld.global.L1::no_allocate.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %5;"
-      : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
-      : "l"(p), "l"(pol));
-  return r;
-}
-__device__ __forceinline__ void stp4(float* p, float4 v, uint64_t pol) {
-  asm volatile(
-      "st.global.L1::no_allocate.L2::cache_hint.v4.f32 [%0], {%1,%2,%3,%4}, %5;"
-      ::"l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "l"(pol)
-      : "memory");
-}
-__device__ __forceinline__ float4 ldp_grad4(const float* p, uint64_t pol) {
-  return ldp4(p, pol);
-}
-__device__ __forceinline__ float4 unpack_bf16x4(uint32_t a, uint32_t b) {
-  return make_float4(__uint_as_float(a << 16), __uint_as_float(a & 0xffff0000u),
-                     __uint_as_float(b << 16), __uint_as_float(b & 0xffff0000u));
-}
-__device__ __forceinline__ float4 ldp_grad4(const __nv_bfloat16* p,
-                                            uint64_t pol) {
-  uint32_t a, b;
-  asm volatile(
-      "ld.global.L1::no_allocate.L2::cache_hint.v2.u32 {%0,%1}, [%2], %3;"
-      : "=r"(a), "=r"(b)
-      : "l"(p), "l"(pol));
-  return unpack_bf16x4(a, b);
-}
-// gradient packet j of a stage
-__device__ __forceinline__ float4 lds_grad4(const char* gbase, int j,
-                                            const float*) {
-  return *reinterpret_cast<const float4*>(gbase + 16 * j);
-}
-__device__ __forceinline__ float4 lds_grad4(const char* gbase, int j,
-                                            const __nv_bfloat16*) {
-  const uint2 u = *reinterpret_cast<const uint2*>(gbase + 8 * j);
-  return unpack_bf16x4(u.x, u.y);
-}
-__device__ __forceinline__ void stp_copy4(void* base, int64_t i, float4 x,
-                                          uint64_t pol) {
-  const __nv_bfloat162 lo = __floats2bfloat162_rn(x.x, x.y);
-  const __nv_bfloat162 hi = __floats2bfloat162_rn(x.z, x.w);
-  const uint32_t a = *reinterpret_cast<const uint32_t*>(&lo);
-  const uint32_t b = *reinterpret_cast<const uint32_t*>(&hi);
-  asm volatile(
-      "st.global.L1::no_allocate.L2::cache_hint.v2.u32 [%0], {%1,%2}, %3;"
-      ::"l"(static_cast<__nv_bfloat16*>(base) + i), "r"(a), "r"(b), "l"(pol)
-      : "memory");
-}
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void cp_async16(uint32_t saddr, const void* g,
-                                           uint64_t pol) {
-  asm volatile(
-      "cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;"
-      ::"r"(saddr), "l"(g), "l"(pol)
-      : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p)
-               : "memory");
-  return v;
-}
-__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
-  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v)
-               : "memory");
-}
-__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
-  uint32_t old;
-  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;"
-               : "=r"(old) : "l"(p), "r"(v) : "memory");
-  return old;
-}
-__device__ __forceinline__ double warp_sum_d(double x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x += __shfl_down_sync(0xffffffffu, x, o);
-  return x;
-}
-
-// Element of the fused pass 1: LAMB (Alg. 2) or LARS (Alg. 1) moment update,
-// then the direction u whose norm the trust ratio needs.
-template <bool kLars>
-__device__ __forceinline__ void fused1_elem(float g, float& m, float& v,
-                                            float w, float lam,
-                                            const LambConsts& k, float& sw,
-                                            float& su) {
-  float u;
-  if (kLars) {
-    m = lars_momentum(g, m, w, lam, k.b1, k.omb1);
-    u = m;
-  } else {
-    lamb_moments(g, m, v, k);
-    u = lamb_direction(m, v, w, lam, k);
-  }
-  sw = __fmaf_rn(w, w, sw);
-  su = __fmaf_rn(u, u, su);
-}
-
-template <bool kLars>
-__device__ __forceinline__ float fused2_dir(float m, float v, float w,
-                                            float lam, const LambConsts& k) {
-  return kLars ? m : lamb_direction(m, v, w, lam, k);
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused1_pkt(float4 gv, float4& mv, float4& vv,
-                                           float4 wv, float lam,
-                                           const LambConsts& k, float& sw,
-                                           float& su) {
-  fused1_elem<kLars>(gv.x, mv.x, vv.x, wv.x, lam, k, sw, su);
-  fused1_elem<kLars>(gv.y, mv.y, vv.y, wv.y, lam, k, sw, su);
-  fused1_elem<kLars>(gv.z, mv.z, vv.z, wv.z, lam, k, sw, su);
-  fused1_elem<kLars>(gv.w, mv.w, vv.w, wv.w, lam, k, sw, su);
-}
-
-template <bool kLars>
-__device__ __forceinline__ float4 fused2_pkt(float4 mv, float4 vv, float4 wv,
-                                             float s, float lam,
-                                             const LambConsts& k) {
-  float4 o;
-  o.x = __fmaf_rn(-s, fused2_dir<kLars>(mv.x, vv.x, wv.x, lam, k), wv.x);
-  o.y = __fmaf_rn(-s, fused2_dir<kLars>(mv.y, vv.y, wv.y, lam, k), wv.y);
-  o.z = __fmaf_rn(-s, fused2_dir<kLars>(mv.z, vv.z, wv.z, lam, k), wv.z);
-  o.w = __fmaf_rn(-s, fused2_dir<kLars>(mv.w, vv.w, wv.w, lam, k), wv.w);
-  return o;
-}
-
-__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p)
-               : "memory");
-  return v;
-}
-__device__ __forceinline__ void fence_acq_rel() {
-  asm volatile("fence.acq_rel.gpu;" ::: "memory");
-}
-
-// Issue the cp.async copies of one full, aligned chunk into `stage`: m, v
-// (LAMB), w, and for pass 1 the gradient.
-template <bool kLars, typename GT>
-__device__ __forceinline__ void fused_prefetch_ops(
-    const TensorPtrs& tp, int64_t off, bool pass2, bool resident, char* stage,
-    uint64_t pol_first, uint64_t pol_last, int lane) {
-  const uint64_t pol = (!pass2 && resident) ? pol_last : pol_first;
-  const uint32_t s = smem_u32(stage);
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;                    // 16-byte piece index
-    cp_async16(s + kOffM + 16 * j, tp.m + off + 4 * j, pol);
-    if (!kLars) cp_async16(s + kOffV + 16 * j, tp.v + off + 4 * j, pol);
-    cp_async16(s + off_w<kLars>() + 16 * j, tp.w + off + 4 * j, pol);
-  }
-  if (!pass2) {
-    const char* g = reinterpret_cast<const char*>(
-        static_cast<const GT*>(tp.g) + off);
-    constexpr int kGPieces = kFusedChunk * (int)sizeof(GT) / 16;
-#pragma unroll
-    for (int u = 0; u < kGPieces / 32; ++u) {
-      const int j = lane + 32 * u;
-      cp_async16(s + off_g<kLars>() + 16 * j, g + 16 * j, pol_first);
-    }
-  }
-}
-
-// Pass 1 of a staged chunk: new m, v into registers, sums of w^2 and u^2.
-template <bool kLars, typename GT>
-__device__ __forceinline__ void fused1_from_stage(const char* stage,
-                                                  float lam,
-                                                  const LambConsts& k,
-                                                  float4* mo, float4* vo,
-                                                  float& sw, float& su,
-                                                  int lane) {
-  const GT* tag = nullptr;
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;
-    mo[u] = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
-    vo[u] = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
-                  : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
-    const float4 wv =
-        *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
-    const float4 gv = lds_grad4(stage + off_g<kLars>(), j, tag);
-    fused1_pkt<kLars>(gv, mo[u], vo[u], wv, lam, k, sw, su);
-  }
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused1_store(const TensorPtrs& tp,
-                                             int64_t off, const float4* mo,
-                                             const float4* vo,
-                                             uint64_t pol_keep, int lane) {
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;
-    stp4(tp.m + off + 4 * j, mo[u], pol_keep);
-    if (!kLars) stp4(tp.v + off + 4 * j, vo[u], pol_keep);
-  }
-}
-
-// Pass 1 straight from global memory (tail chunks, unaligned tensors).
-template <bool kLars, typename GT>
-__device__ __forceinline__ void fused1_direct(const TensorPtrs& tp,
-                                              int64_t off, int len, float lam,
-                                              const LambConsts& k, float& sw,
-                                              float& su, uint64_t pol_first,
-                                              uint64_t pol_keep, int lane) {
-  float* __restrict__ m = tp.m + off;
-  float* __restrict__ v = kLars ? nullptr : tp.v + off;
-  const float* __restrict__ w = tp.w + off;
-  const GT* __restrict__ g = static_cast<const GT*>(tp.g) + off;
-  int scalar_from = 0;
-  if (tp.vec_ok) {
-    const int nv = len >> 2;
-#pragma unroll 1
-    for (int base = lane; base < nv; base += 64) {
-      float4 wv[2], mv[2], vv[2], gv[2];
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          gv[u] = ldp_grad4(g + 4 * j, pol_first);
-          mv[u] = ldp4(m + 4 * j, pol_keep);
-          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_keep);
-          wv[u] = ldp4(w + 4 * j, pol_keep);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          fused1_pkt<kLars>(gv[u], mv[u], vv[u], wv[u], lam, k, sw, su);
-          stp4(m + 4 * j, mv[u], pol_keep);
-          if (!kLars) stp4(v + 4 * j, vv[u], pol_keep);
-        }
-      }
-    }
-    scalar_from = nv << 2;
-  }
-  for (int i = scalar_from + lane; i < len; i += 32) {
-    float mi = m[i];
-    float vi = kLars ? 0.f : v[i];
-    fused1_elem<kLars>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
-    m[i] = mi;
-    if (!kLars) v[i] = vi;
-  }
-}
-
-// Pass 2 of a staged chunk: new w into registers.
-template <bool kLars>
-__device__ __forceinline__ void fused2_from_stage(const char* stage, float s,
-                                                  float lam,
-                                                  const LambConsts& k,
-                                                  float4* wo, int lane) {
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;
-    const float4 mv = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
-    const float4 vv = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
-                            : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
-    const float4 wv =
-        *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
-    wo[u] = fused2_pkt<kLars>(mv, vv, wv, s, lam, k);
-  }
-}
-
-template <bool kCopy>
-__device__ __forceinline__ void fused2_store(const TensorPtrs& tp,
-                                             int64_t off, const float4* wo,
-                                             uint64_t pol_first, int lane) {
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;
-    stp4(tp.w + off + 4 * j, wo[u], pol_first);
-    if (kCopy) stp_copy4(tp.copy, off + 4 * j, wo[u], pol_first);
-  }
-}
-
-// Pass 2 straight from global memory.
-template <bool kLars, bool kCopy>
-__device__ __forceinline__ void fused2_direct(const TensorPtrs& tp,
-                                              int64_t off, int len, float s,
-                                              float lam, const LambConsts& k,
-                                              uint64_t pol_first, int lane) {
-  float* __restrict__ w = tp.w + off;
-  const float* __restrict__ m = tp.m + off;
-  const float* __restrict__ v = kLars ? nullptr : tp.v + off;
-  int scalar_from = 0;
-  if (tp.vec_ok) {
-    const int nv = len >> 2;
-#pragma unroll 1
-    for (int base = lane; base < nv; base += 64) {
-      float4 wv[2], mv[2], vv[2];
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          mv[u] = ldp4(m + 4 * j, pol_first);
-          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_first);
-          wv[u] = ldp4(w + 4 * j, pol_first);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          const float4 o = fused2_pkt<kLars>(mv[u], vv[u], wv[u], s, lam, k);
-          stp4(w + 4 * j, o, pol_first);
-          if (kCopy) stp_copy4(tp.copy, off + 4 * j, o, pol_first);
-        }
-      }
-    }
-    scalar_from = nv << 2;
-  }
-  for (int i = scalar_from + lane; i < len; i += 32) {
-    const float wi = w[i];
-    const float o = __fmaf_rn(
-        -s, fused2_dir<kLars>(m[i], kLars ? 0.f : v[i], wi, lam, k), wi);
-    w[i] = o;
-    if (kCopy) st_copy1(tp.copy, off + i, o);
-  }
-}
-
-// The warp whose ticket completed group `gl` of tensor `tensor`: fixed-order
-// fp64 sum of the group's chunk sums; the warp that completes the tensor's
-// last group computes its norms and trust ratio and releases ready[tensor].
-template <bool kLars>
-__device__ __forceinline__ void fused_group_combine(const StepParams& p,
-                                                 const FusedParams& f,
-                                                 const FusedTensor& ft,
-                                                 int tensor, int gl, int gsize,
-                                                 uint32_t epoch, int lane) {
-  __syncwarp();
-  const int group = ft.first_group + gl;
-  double aw = 0.0, au = 0.0;
-  if (lane < gsize) {
-    const float2 s = __ldcg(&f.fslots[ft.first_chunk + gl * kGroup + lane]);
-    aw = (double)s.x;
-    au = (double)s.y;
-  }
-  aw = warp_sum_d(aw);
-  au = warp_sum_d(au);
-  uint32_t last = 0;
-  if (lane == 0) {
-    f.gslots[group] = make_double2(aw, au);
-    f.gtickets[group] = 0u;
-    last = atom_add_acq_rel(&f.tickets[tensor], 1u) + 1u ==
-           (uint32_t)ft.n_groups;
-  }
-  if (!__shfl_sync(0xffffffffu, last, 0)) return;
-  __syncwarp();
-  double tw = 0.0, tu = 0.0;
-  for (int i = lane; i < ft.n_groups; i += 32) {
-    const double2 s = __ldcg(&f.gslots[ft.first_group + i]);
-    tw += s.x;
-    tu += s.y;
-  }
-  tw = warp_sum_d(tw);
-  tu = warp_sum_d(tu);
-  if (lane == 0) {
-    const double wn = sqrt(tw), un = sqrt(tu);
-    double rho = 1.0;
-    if (!(wn == 0.0 || un == 0.0))
-      rho = (kLars ? p.trust : 1.0) * phi_of(wn, p) / un;
-    p.ratio[tensor] = rho;
-    p.wnorm[tensor] = wn;
-    p.unorm[tensor] = un;
-    if (!isfinite(tw) || !isfinite(tu)) atomicOr(p.status, kStatusNonfinite);
-    f.tickets[tensor] = 0u;
-    st_release(&f.ready[tensor], epoch);
-  }
-}
-
-// Bounded wait of a pass-2 item for its tensor's norms (all lanes).
-__device__ __forceinline__ bool fused_wait(const StepParams& p,
-                                           const FusedParams& f, int tensor,
-                                           uint32_t epoch, int lane) {
-  uint32_t ok = 1;
-  if (lane == 0) {
-    uint32_t spins = 0, ns = 32;
-    while (ld_acquire(&f.ready[tensor]) != epoch) {
-      // give up after ~0.5 s, or at once if another warp of this launch
-      // already gave up (counters[4] holds the epoch of an aborted launch)
-      if (++spins > kSpinLimit ||
-          *reinterpret_cast<volatile uint32_t*>(&p.counters[4]) == epoch) {
-        ok = 0;
-        atomicOr(p.status, kStatusWaitTimeout);
-        atomicExch(&p.counters[4], epoch);
-        break;
-      }
-      __nanosleep(ns);
-      if (ns < 256) ns <<= 1;
-    }
-  }
-  if (!__shfl_sync(0xffffffffu, ok, 0)) return false;
-  __syncwarp();
-  (void)ld_acquire(&f.ready[tensor]);               // per-lane acquire
-  return true;
-}
-
-// ---------------------------------------------------------------------------
-// The warp worker.  Per warp:
-//   * a data ring of kStages shared-memory stages; the item in a stage had
-//     its operands prefetched with cp.async kStages items earlier;
-//   * a control pipeline one item deep per step: the draw atomic, the item
-//     descriptor load and (pass 2) a relaxed load of the tensor's ready flag
-//     are each issued one item before their results are used;
-//   * a deferred publish: a pass-1 item's ticket is taken one item later (its
-//     stores are long complete, so the release costs little), and the
-//     ticket's answer is looked at one item after that.
-// Before any wait the warp flushes its deferred publishes, so it never waits
-// for work it holds itself.
-// ---------------------------------------------------------------------------
-struct PubState {
-  uint32_t tensor, index;   // pass-1 chunk whose sums are held (publish)
-  float sw, su;             // its sums, valid in lane 0
-  uint32_t chk_tensor, chk_index;   // chunk whose ticket awaits its check
-  uint32_t ticket;          // that ticket's answer (lane 0)
-  bool pub, chk;            // a publish is pending / a check is pending
-};
-
-__device__ __forceinline__ uint2 invalid_desc() {
-  return make_uint2(0xffffffffu, 0u);
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused_check(const StepParams& p,
-                                            const FusedParams& f,
-                                            PubState& ps, uint32_t epoch,
-                                            int lane) {
-  if (!ps.chk) return;
-  const FusedTensor ft = f.ftensors[ps.chk_tensor];
-  const int gl = (int)ps.chk_index / kGroup;
-  const int gsize = min(kGroup, ft.n_chunks - gl * kGroup);
-  const uint32_t last =
-      __shfl_sync(0xffffffffu, ps.ticket + 1u == (uint32_t)gsize, 0);
-  ps.chk = false;
-  if (last) fused_group_combine<kLars>(p, f, ft, (int)ps.chk_tensor, gl,
-                                       gsize, epoch, lane);
-}
-
-__device__ __forceinline__ void fused_publish_now(const FusedParams& f,
-                                                  PubState& ps, int lane) {
-  if (!ps.pub) return;
-  if (lane == 0) {
-    const FusedTensor ft = f.ftensors[ps.tensor];
-    f.fslots[ft.first_chunk + ps.index] = make_float2(ps.sw, ps.su);
-    // release: this warp's stores of the chunk's m, v and the slot
-    ps.ticket = atom_add_acq_rel(
-        &f.gtickets[ft.first_group + (int)ps.index / kGroup], 1u);
-  }
-  ps.chk_tensor = ps.tensor;
-  ps.chk_index = ps.index;
-  ps.pub = false;
-  ps.chk = true;
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused_publish_step(const StepParams& p,
-                                                   const FusedParams& f,
-                                                   PubState& ps,
-                                                   uint32_t epoch, int lane) {
-  fused_check<kLars>(p, f, ps, epoch, lane);
-  fused_publish_now(f, ps, lane);
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused_flush(const StepParams& p,
-                                            const FusedParams& f,
-                                            PubState& ps, uint32_t epoch,
-                                            int lane) {
-  fused_publish_step<kLars>(p, f, ps, epoch, lane);
-  fused_check<kLars>(p, f, ps, epoch, lane);
-}
-
-template <bool kLars, typename GT, bool kCopy>
-__global__ void __launch_bounds__(kFusedThreads, 1)
-    fused_step_kernel(const StepParams p, const FusedParams f) {
-  extern __shared__ __align__(128) char fused_smem[];
-  __shared__ LambConsts s_k;
-  __shared__ float s_lr;
-  __shared__ int s_skip;
-  __shared__ uint32_t s_epoch;
-  __shared__ int64_t s_t;
-  const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) {
-    const bool bc = !kLars && (p.flags & kFlagBiasCorrection) != 0;
-    const int64_t t = p.d_step ? *p.d_step : int64_t(1);
-    const int skip = (bc && t < 1) ? 1 : 0;
-    float c1 = 1.f, c2 = 1.f;
-    if (bc && !skip) {  // Alg. 2 bias correction, beta^t in fp64
-      c1 = (float)(1.0 / (1.0 - pow(p.beta1, (double)t)));
-      c2 = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
-    }
-    s_k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps};
-    s_lr = step_lr(p, t);
-    s_skip = skip;
-    s_t = t;
-    s_epoch = *reinterpret_cast<volatile uint32_t*>(&p.counters[3]);
-    if (blockIdx.x == 0) {
-      StepScalars sc{};
-      sc.t = t;
-      sc.c1 = c1;
-      sc.c2 = c2;
-      sc.lr = s_lr;
-      sc.skip = skip;
-      *p.scal = sc;
-      if (skip) atomicOr(p.status, kStatusBadStep);
-    }
-  }
-  __syncthreads();
-  if (s_skip) return;
-  const LambConsts k = s_k;
-  const float lr = s_lr;
-  const uint32_t epoch = s_epoch;
-  const uint64_t pol_first = policy_evict_first();
-  const uint64_t pol_last = policy_evict_last();
-  const uint32_t n_items = (uint32_t)f.n_items;
-  constexpr int kSB = stage_bytes<kLars, GT>();
-  char* ring = fused_smem + warp * kStages * kSB;
-
-  // ---- control pipeline --------------------------------------------------
-  // Each warp draws indices until it gets one >= n_items, then stops, so it
-  // draws exactly one such index.
-  uint32_t last_drawn = 0;
-  bool drawing = true;
-  auto draw = [&]() -> uint32_t {
-    if (!drawing) return n_items;
-    uint32_t v = 0;
-    if (lane == 0) v = atomicAdd(&p.counters[2], 1u);
-    v = __shfl_sync(0xffffffffu, v, 0);
-    if (v >= n_items) {
-      drawing = false;
-      last_drawn = v;
-    }
-    return v;
-  };
-  auto load_desc = [&](uint32_t i) -> uint2 {
-    return i < n_items ? __ldg(&f.items[i]) : invalid_desc();
-  };
-  auto ready_load = [&](uint2 d) -> uint32_t {
-    if (d.x == 0xffffffffu || (d.x & 1u) == 0u) return 0u;
-    return ld_relaxed(&f.ready[d.x >> 1]);
-  };
-  uint32_t idx_a = draw();
-  uint2 desc_b = load_desc(idx_a);
-  idx_a = draw();
-  uint2 desc_c = desc_b;
-  uint32_t rdy_c = ready_load(desc_c);
-  desc_b = load_desc(idx_a);
-  idx_a = draw();
-  uint32_t synced = 0xffffffffu;   // tensor whose norms this warp acquired
-
-  uint2 sd[kStages];
-  bool staged[kStages];
-  // fill stage s with desc_c, then advance the control pipeline
-  auto fill_advance = [&](int s) {
-    sd[s] = desc_c;
-    staged[s] = false;
-    if (desc_c.x != 0xffffffffu) {
-      const bool p2 = (desc_c.x & 1u) != 0u;
-      const uint32_t tensor = desc_c.x >> 1;
-      const FusedTensor ft = f.ftensors[tensor];
-      const TensorPtrs tp = p.ptrs[tensor];
-      const int64_t off = (int64_t)desc_c.y * kFusedChunk;
-      bool go = tp.vec_ok && ft.numel - off >= kFusedChunk;
-      if (go && p2) {
-        go = __shfl_sync(0xffffffffu, rdy_c == epoch, 0) != 0;
-        if (go && tensor != synced) {
-          fence_acq_rel();           // acquire: the relaxed load saw the release
-          synced = tensor;
-        }
-      }
-      if (go) {
-        fused_prefetch_ops<kLars, GT>(tp, off, p2, ft.resident != 0u,
-                                      ring + s * kSB, pol_first, pol_last,
-                                      lane);
-        staged[s] = true;
-      }
-    }
-    cp_async_commit();
-    desc_c = desc_b;
-    rdy_c = ready_load(desc_c);
-    desc_b = load_desc(idx_a);
-    idx_a = draw();
-  };
-#pragma unroll
-  for (int s = 0; s < kStages; ++s) fill_advance(s);
-
-  // pass-2 item of this warp whose tensor was not final when its turn came
-  uint2 parked = invalid_desc();
-  // run a pass-2 item from global memory once its tensor is known final
-  auto run_direct_p2 = [&](uint2 d) {
-    const uint32_t tensor = d.x >> 1;
-    if (tensor != synced) {
-      fence_acq_rel();                 // acquire: the relaxed load saw it
-      synced = tensor;
-    }
-    const FusedTensor ft = f.ftensors[tensor];
-    const TensorPtrs tp = p.ptrs[tensor];
-    const int64_t off = (int64_t)d.y * kFusedChunk;
-    const int64_t rem = ft.numel - off;
-    const int len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
-    const float s2 = __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]));
-    fused2_direct<kLars, kCopy>(tp, off, len, s2, ft.decay * p.wd, k,
-                                pol_first, lane);
-  };
-  // the same after a bounded wait (callers flush their publishes first)
-  auto wait_direct_p2 = [&](uint2 d) {
-    const uint32_t tensor = d.x >> 1;
-    if (fused_wait(p, f, (int)tensor, epoch, lane)) {
-      synced = tensor;
-      run_direct_p2(d);
-    }
-  };
-
-  PubState ps;
-  ps.pub = ps.chk = false;
-  ps.tensor = ps.index = ps.chk_tensor = ps.chk_index = 0u;
-  ps.sw = ps.su = 0.f;
-  ps.ticket = 0u;
-
-  bool done = false;
-  while (!done) {
-#pragma unroll
-    for (int s = 0; s < kStages; ++s) {
-      const uint2 d = sd[s];
-      if (d.x == 0xffffffffu) {
-        done = true;
-        break;
-      }
-      char* stage = ring + s * kSB;
-      cp_async_wait<kStages - 1>();   // this stage's copies have landed
-      __syncwarp();
-      const bool p2 = (d.x & 1u) != 0u;
-      const uint32_t tensor = d.x >> 1;
-      const FusedTensor ft = f.ftensors[tensor];
-      const TensorPtrs tp = p.ptrs[tensor];
-      const int64_t off = (int64_t)d.y * kFusedChunk;
-      const int64_t rem = ft.numel - off;
-      const int len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
-      const float lam = ft.decay * p.wd;
-      if (!p2) {
-        const uint64_t pol_keep = ft.resident ? pol_last : pol_first;
-        float sw = 0.f, su = 0.f;
-        if (staged[s]) {
-          float4 mo[kPktsPerLane], vo[kPktsPerLane];
-          fused1_from_stage<kLars, GT>(stage, lam, k, mo, vo, sw, su, lane);
-          __syncwarp();               // every lane is done with the stage
-          fill_advance(s);
-          fused_publish_step<kLars>(p, f, ps, epoch, lane);
-          fused1_store<kLars>(tp, off, mo, vo, pol_keep, lane);
-        } else {
-          __syncwarp();
-          fill_advance(s);
-          fused_publish_step<kLars>(p, f, ps, epoch, lane);
-          fused1_direct<kLars, GT>(tp, off, len, lam, k, sw, su, pol_first,
-                                   pol_keep, lane);
-        }
-        ps.sw = warp_sum(sw);
-        ps.su = warp_sum(su);
-        ps.tensor = tensor;
-        ps.index = d.y;
-        ps.pub = true;
-      } else {
-        const float s_upd =
-            staged[s] ? __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]))
-                      : 0.f;
-        if (staged[s]) {
-          float4 wo[kPktsPerLane];
-          fused2_from_stage<kLars>(stage, s_upd, lam, k, wo, lane);
-          __syncwarp();
-          fill_advance(s);
-          fused_publish_step<kLars>(p, f, ps, epoch, lane);
-          fused2_store<kCopy>(tp, off, wo, pol_first, lane);
-        } else {
-          __syncwarp();
-          fill_advance(s);
-          fused_publish_step<kLars>(p, f, ps, epoch, lane);
-          // every lane loads the flag itself (one broadcast access) before
-          // its acquire fence; lane 0's value makes the decision uniform
-          const uint32_t r = __shfl_sync(0xffffffffu,
-                                         ld_relaxed(&f.ready[tensor]), 0);
-          if (r == epoch) {               // became final since the fill
-            run_direct_p2(d);
-          } else {
-            // Not final yet: park it instead of waiting, so this warp keeps
-            // working (and publishing) its later pass-1 items.  With the
-            // parking slot taken, finish the parked item first.
-            if (parked.x != 0xffffffffu) {
-              fused_flush<kLars>(p, f, ps, epoch, lane);
-              wait_direct_p2(parked);
-            }
-            parked = d;
-          }
-        }
-      }
-      // a parked item whose tensor has become final in the meantime
-      if (parked.x != 0xffffffffu) {
-        const uint32_t r = __shfl_sync(
-            0xffffffffu, ld_relaxed(&f.ready[parked.x >> 1]), 0);
-        if (r == epoch) {
-          run_direct_p2(parked);
-          parked = invalid_desc();
-        }
-      }
-    }
-  }
-  fused_flush<kLars>(p, f, ps, epoch, lane);
-  if (parked.x != 0xffffffffu) wait_direct_p2(parked);
-  cp_async_wait<0>();
-  // The warp that drew the last index >= n_items closes the launch.
-  const uint32_t warps = gridDim.x * kFusedWarps;
-  if (lane == 0 && last_drawn == n_items + warps - 1u) {
-    atomicExch(&p.counters[2], 0u);
-    const uint32_t ne = epoch + 1u == 0u ? 1u : epoch + 1u;
-    atomicExch(&p.counters[3], ne);
-    StepScalars sc{};
-    sc.t = s_t;
-    sc.lr = s_lr;
-    close_step(p, sc);
-  }
 }
 
 template <typename K>
@@ -1450,141 +650,115 @@ int occupancy_of(K kernel, int* blocks) {
                                                             kThreads, 0);
 }
 
+// Variant selection from the step's flags.
+template <typename GT, int kNest>
+int lamb_p1(const StepParams& p, int grid, cudaStream_t s) {
+  if (p.flags & (kFlagGradNorm | kFlagSkipNonfinite))
+    lamb_pass1_kernel<GT, kNest, true><<<grid, kThreads, 0, s>>>(p);
+  else
+    lamb_pass1_kernel<GT, kNest, false><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
+template <bool kCopy, int kNest, typename GT>
+int lamb_p2(const StepParams& p, int grid, cudaStream_t s) {
+  // plain LAMB's pass 2 does not read g: one instantiation for both types
+  using GT2 = typename std::conditional<kNest != 0, GT, float>::type;
+  if (p.flags & kFlagSkipNonfinite)
+    lamb_pass2_kernel<kCopy, kNest, GT, true><<<grid, kThreads, 0, s>>>(p);
+  else
+    lamb_pass2_kernel<kCopy, kNest, GT2, false><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
+template <typename GT>
+int lars_p1(const StepParams& p, int grid, cudaStream_t s) {
+  if (p.flags & (kFlagGradNorm | kFlagSkipNonfinite))
+    lars_pass1_kernel<GT, true><<<grid, kThreads, 0, s>>>(p);
+  else
+    lars_pass1_kernel<GT, false><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
+template <bool kCopy, typename GT>
+int lars_p2(const StepParams& p, int grid, cudaStream_t s) {
+  if (p.flags & kFlagSkipNonfinite)
+    lars_pass2_kernel<kCopy, GT, true><<<grid, kThreads, 0, s>>>(p);
+  else
+    lars_pass2_kernel<kCopy, float, false><<<grid, kThreads, 0, s>>>(p);
+  return (int)cudaGetLastError();
+}
+
 }  // namespace
 
-int launch_lamb_pass1(const StepParams& p, int grad_bf16, int grid,
+int launch_lamb_pass1(const StepParams& p, int nest, int grad_bf16, int grid,
                       void* stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (grad_bf16)
-    lamb_pass1_kernel<__nv_bfloat16, 0><<<grid, kThreads, 0, s>>>(p);
-  else
-    lamb_pass1_kernel<float, 0><<<grid, kThreads, 0, s>>>(p);
-  return (int)cudaGetLastError();
-}
-
-int launch_nlamb_pass1(const StepParams& p, int nest, int grad_bf16, int grid,
-                       void* stream) {
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  switch ((nest == 2 ? 2 : 0) | (grad_bf16 ? 1 : 0)) {
-    case 0: lamb_pass1_kernel<float, 1><<<grid, kThreads, 0, s>>>(p); break;
-    case 1: lamb_pass1_kernel<__nv_bfloat16, 1><<<grid, kThreads, 0, s>>>(p); break;
-    case 2: lamb_pass1_kernel<float, 2><<<grid, kThreads, 0, s>>>(p); break;
-    default: lamb_pass1_kernel<__nv_bfloat16, 2><<<grid, kThreads, 0, s>>>(p); break;
+  switch ((nest == 2 ? 4 : nest == 1 ? 2 : 0) | (grad_bf16 ? 1 : 0)) {
+    case 0: return lamb_p1<float, 0>(p, grid, s);
+    case 1: return lamb_p1<__nv_bfloat16, 0>(p, grid, s);
+    case 2: return lamb_p1<float, 1>(p, grid, s);
+    case 3: return lamb_p1<__nv_bfloat16, 1>(p, grid, s);
+    case 4: return lamb_p1<float, 2>(p, grid, s);
+    default: return lamb_p1<__nv_bfloat16, 2>(p, grid, s);
   }
-  return (int)cudaGetLastError();
 }
 
-int launch_nlamb_pass2(const StepParams& p, int nest, int grad_bf16,
-                       int copy_bf16, int grid, void* stream) {
+int launch_lamb_pass2(const StepParams& p, int nest, int grad_bf16,
+                      int copy_bf16, int grid, void* stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  switch ((nest == 2 ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0)) {
-    case 0: lamb_pass2_kernel<false, 1, float><<<grid, kThreads, 0, s>>>(p); break;
-    case 1: lamb_pass2_kernel<true, 1, float><<<grid, kThreads, 0, s>>>(p); break;
-    case 2: lamb_pass2_kernel<false, 1, __nv_bfloat16><<<grid, kThreads, 0, s>>>(p); break;
-    case 3: lamb_pass2_kernel<true, 1, __nv_bfloat16><<<grid, kThreads, 0, s>>>(p); break;
-    case 4: lamb_pass2_kernel<false, 2, float><<<grid, kThreads, 0, s>>>(p); break;
-    case 5: lamb_pass2_kernel<true, 2, float><<<grid, kThreads, 0, s>>>(p); break;
-    case 6: lamb_pass2_kernel<false, 2, __nv_bfloat16><<<grid, kThreads, 0, s>>>(p); break;
-    default: lamb_pass2_kernel<true, 2, __nv_bfloat16><<<grid, kThreads, 0, s>>>(p); break;
+  switch ((nest == 2 ? 8 : nest == 1 ? 4 : 0) | (grad_bf16 ? 2 : 0) |
+          (copy_bf16 ? 1 : 0)) {
+    case 0: return lamb_p2<false, 0, float>(p, grid, s);
+    case 1: return lamb_p2<true, 0, float>(p, grid, s);
+    case 2: return lamb_p2<false, 0, __nv_bfloat16>(p, grid, s);
+    case 3: return lamb_p2<true, 0, __nv_bfloat16>(p, grid, s);
+    case 4: return lamb_p2<false, 1, float>(p, grid, s);
+    case 5: return lamb_p2<true, 1, float>(p, grid, s);
+    case 6: return lamb_p2<false, 1, __nv_bfloat16>(p, grid, s);
+    case 7: return lamb_p2<true, 1, __nv_bfloat16>(p, grid, s);
+    case 8: return lamb_p2<false, 2, float>(p, grid, s);
+    case 9: return lamb_p2<true, 2, float>(p, grid, s);
+    case 10: return lamb_p2<false, 2, __nv_bfloat16>(p, grid, s);
+    default: return lamb_p2<true, 2, __nv_bfloat16>(p, grid, s);
   }
-  return (int)cudaGetLastError();
-}
-
-int launch_lamb_pass2(const StepParams& p, int copy_bf16, int grid,
-                      void* stream) {
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (copy_bf16)
-    lamb_pass2_kernel<true, 0, float><<<grid, kThreads, 0, s>>>(p);
-  else
-    lamb_pass2_kernel<false, 0, float><<<grid, kThreads, 0, s>>>(p);
-  return (int)cudaGetLastError();
 }
 
 int launch_lars_pass1(const StepParams& p, int grad_bf16, int grid,
                       void* stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (grad_bf16)
-    lars_pass1_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(p);
-  else
-    lars_pass1_kernel<float><<<grid, kThreads, 0, s>>>(p);
-  return (int)cudaGetLastError();
+  return grad_bf16 ? lars_p1<__nv_bfloat16>(p, grid, s)
+                   : lars_p1<float>(p, grid, s);
 }
 
-int launch_lars_pass2(const StepParams& p, int copy_bf16, int grid,
-                      void* stream) {
+int launch_lars_pass2(const StepParams& p, int grad_bf16, int copy_bf16,
+                      int grid, void* stream) {
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (copy_bf16)
-    lars_pass2_kernel<true><<<grid, kThreads, 0, s>>>(p);
-  else
-    lars_pass2_kernel<false><<<grid, kThreads, 0, s>>>(p);
-  return (int)cudaGetLastError();
-}
-
-template <bool kLars, typename GT, bool kCopy>
-int launch_fused_t(const StepParams& p, const FusedParams& f, int grid,
-                   cudaStream_t s) {
-  fused_step_kernel<kLars, GT, kCopy>
-      <<<grid, kFusedThreads, fused_smem_bytes<kLars, GT>(), s>>>(p, f);
-  return (int)cudaGetLastError();
-}
-
-template <bool kLars, typename GT, bool kCopy>
-int occupancy_fused_t(int* blocks) {
-  // opt in to the dynamic shared memory of the stage rings (a property of
-  // the function, set once; not a device setting)
-  cudaError_t e = cudaFuncSetAttribute(
-      fused_step_kernel<kLars, GT, kCopy>,
-      cudaFuncAttributeMaxDynamicSharedMemorySize,
-      fused_smem_bytes<kLars, GT>());
-  if (e != cudaSuccess) return (int)e;
-  return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-      blocks, fused_step_kernel<kLars, GT, kCopy>, kFusedThreads,
-      fused_smem_bytes<kLars, GT>());
-}
-
-int launch_fused(const StepParams& p, const FusedParams& f, int lars,
-                 int grad_bf16, int copy_bf16, int grid, void* stream) {
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  switch ((lars ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0)) {
-    case 0: return launch_fused_t<false, float, false>(p, f, grid, s);
-    case 1: return launch_fused_t<false, float, true>(p, f, grid, s);
-    case 2: return launch_fused_t<false, __nv_bfloat16, false>(p, f, grid, s);
-    case 3: return launch_fused_t<false, __nv_bfloat16, true>(p, f, grid, s);
-    case 4: return launch_fused_t<true, float, false>(p, f, grid, s);
-    case 5: return launch_fused_t<true, float, true>(p, f, grid, s);
-    case 6: return launch_fused_t<true, __nv_bfloat16, false>(p, f, grid, s);
-    default: return launch_fused_t<true, __nv_bfloat16, true>(p, f, grid, s);
-  }
-}
-
-int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks) {
-  switch ((lars ? 4 : 0) | (grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0)) {
-    case 0: return occupancy_fused_t<false, float, false>(blocks);
-    case 1: return occupancy_fused_t<false, float, true>(blocks);
-    case 2: return occupancy_fused_t<false, __nv_bfloat16, false>(blocks);
-    case 3: return occupancy_fused_t<false, __nv_bfloat16, true>(blocks);
-    case 4: return occupancy_fused_t<true, float, false>(blocks);
-    case 5: return occupancy_fused_t<true, float, true>(blocks);
-    case 6: return occupancy_fused_t<true, __nv_bfloat16, false>(blocks);
-    default: return occupancy_fused_t<true, __nv_bfloat16, true>(blocks);
+  switch ((grad_bf16 ? 2 : 0) | (copy_bf16 ? 1 : 0)) {
+    case 0: return lars_p2<false, float>(p, grid, s);
+    case 1: return lars_p2<true, float>(p, grid, s);
+    case 2: return lars_p2<false, __nv_bfloat16>(p, grid, s);
+    default: return lars_p2<true, __nv_bfloat16>(p, grid, s);
   }
 }
 
 int occupancy_lamb_pass1(int grad_bf16, int* blocks) {
-  return grad_bf16 ? occupancy_of(lamb_pass1_kernel<__nv_bfloat16, 0>, blocks)
-                   : occupancy_of(lamb_pass1_kernel<float, 0>, blocks);
+  return grad_bf16
+             ? occupancy_of(lamb_pass1_kernel<__nv_bfloat16, 0, false>, blocks)
+             : occupancy_of(lamb_pass1_kernel<float, 0, false>, blocks);
 }
 int occupancy_lamb_pass2(int copy_bf16, int* blocks) {
-  return copy_bf16 ? occupancy_of(lamb_pass2_kernel<true, 0, float>, blocks)
-                   : occupancy_of(lamb_pass2_kernel<false, 0, float>, blocks);
+  return copy_bf16
+             ? occupancy_of(lamb_pass2_kernel<true, 0, float, false>, blocks)
+             : occupancy_of(lamb_pass2_kernel<false, 0, float, false>, blocks);
 }
 int occupancy_lars_pass1(int grad_bf16, int* blocks) {
-  return grad_bf16 ? occupancy_of(lars_pass1_kernel<__nv_bfloat16>, blocks)
-                   : occupancy_of(lars_pass1_kernel<float>, blocks);
+  return grad_bf16 ? occupancy_of(lars_pass1_kernel<__nv_bfloat16, false>, blocks)
+                   : occupancy_of(lars_pass1_kernel<float, false>, blocks);
 }
 int occupancy_lars_pass2(int copy_bf16, int* blocks) {
-  return copy_bf16 ? occupancy_of(lars_pass2_kernel<true>, blocks)
-                   : occupancy_of(lars_pass2_kernel<false>, blocks);
+  return copy_bf16 ? occupancy_of(lars_pass2_kernel<true, float, false>, blocks)
+                   : occupancy_of(lars_pass2_kernel<false, float, false>, blocks);
 }
 
 }  // namespace lamb

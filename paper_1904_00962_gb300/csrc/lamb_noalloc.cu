@@ -330,10 +330,10 @@ extern "C" LAMB_API lamb_status_t lamb_step_noalloc(
     if (gsz > n_chunks) gsz = n_chunks;
     return (int)(gsz < 1 ? 1 : gsz);
   };
-  int rc = launch_lamb_pass1(sp, gbf, grid_of(nd->occ[gbf]), stream);
+  int rc = launch_lamb_pass1(sp, 0, gbf, grid_of(nd->occ[gbf]), stream);
   if (!rc)
-    rc = launch_lamb_pass2(sp, copy ? 1 : 0, grid_of(nd->occ[2 + (copy ? 1 : 0)]),
-                           stream);
+    rc = launch_lamb_pass2(sp, 0, gbf, copy ? 1 : 0,
+                           grid_of(nd->occ[2 + (copy ? 1 : 0)]), stream);
   if (!rc && d_ratio)
     rc = (int)cudaMemcpyAsync(d_ratio, s + kOffRatio, nb,
                               cudaMemcpyDeviceToDevice, stream);

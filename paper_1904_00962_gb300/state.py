@@ -130,6 +130,17 @@ class LambPlan:
                                       stream=_stream(stream))
         return out
 
+    def grad_norms(self, stream=None):
+        """(||g_k|| [n] f64, global ||g|| [1] f64, non-finite flag [1] i32)
+        of the last step with the gradient check, as new device tensors."""
+        dev = self.state.device
+        out = (torch.empty(self.n, dtype=torch.float64, device=dev),
+               torch.empty(1, dtype=torch.float64, device=dev),
+               torch.empty(1, dtype=torch.int32, device=dev))
+        B.lamb_plan_copy_grad_norms(self.handle, *(t.data_ptr() for t in out),
+                                    stream=_stream(stream))
+        return out
+
     def query(self, clear=False, stream=None) -> int:
         return B.lamb_plan_query(self.handle, clear, _stream(stream))
 
