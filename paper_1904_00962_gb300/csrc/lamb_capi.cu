@@ -554,6 +554,8 @@ static void fill_params(lamb_plan* p, const lamb_hyper_t* h, int64_t* d_step,
   sp->wd = (float)h->weight_decay;
   sp->beta1 = h->beta1;
   sp->beta2 = h->beta2;
+  sp->log2_beta1 = std::log2(h->beta1);   // -inf for beta = 0: beta^t = 0
+  sp->log2_beta2 = std::log2(h->beta2);
   sp->gamma_l = h->gamma_l;
   sp->gamma_u = h->gamma_u;
   sp->trust = h->trust_coef;
@@ -676,6 +678,7 @@ lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
   StepParams sp;
   fill_params(plan, hyper, d_step, d_lr, &sp);
   sp.psi = momentum_decay;
+  sp.log2_mu_decay = momentum_decay * std::log2(0.96);
   sp.d_mu_product = d_mu_product;
   const int nest = nesterov_second_moment ? 2 : 1;
   const bool timed = plan->timing && plan->timed_steps < kMaxTimedSteps;

@@ -138,6 +138,13 @@ __device__ __forceinline__ void close_step(const StepParams& p,
   if ((p.flags & kFlagIncrementStep) && p.d_step) *p.d_step = sc.t + 1;
 }
 
+// b^t for an integer step count t from log2(b): exp2 in fp64 (a power of
+// the bias correction or of a momentum schedule; exact rounding of the
+// exponent product is irrelevant next to the final rounding to float).
+__device__ __forceinline__ double pow_from_log2(double log2_b, double t) {
+  return exp2(t * log2_b);
+}
+
 __device__ __forceinline__ double phi_of(double z, const StepParams& p) {
   if (p.phi == 1) {  // clip; comparisons keep NaN as NaN
     if (z < p.gamma_l) return p.gamma_l;

@@ -566,15 +566,26 @@ __global__ void __launch_bounds__(kFusedThreads, 1)
   __shared__ int64_t s_t;
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) {
-    const bool bc = !kLars && (p.flags & kFlagBiasCorrection) != 0;
+  __shared__ float s_c2;
+  const bool bc = !kLars && (p.flags & kFlagBiasCorrection) != 0;
+  if (threadIdx.x == 32) {  // Alg. 2 bias correction of v, beside c1
     const int64_t t = p.d_step ? *p.d_step : int64_t(1);
-    const int skip = (bc && t < 1) ? 1 : 0;
-    float c1 = 1.f, c2 = 1.f;
-    if (bc && !skip) {  // Alg. 2 bias correction, beta^t in fp64
-      c1 = (float)(1.0 / (1.0 - pow(p.beta1, (double)t)));
-      c2 = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
-    }
+    s_c2 = (bc && t >= 1) ? (float)(1.0 / (1.0 - pow_from_log2(
+                                p.log2_beta2, (double)t)))
+                          : 1.f;
+  }
+  float c1 = 1.f;
+  int64_t t = 1;
+  int skip = 0;
+  if (threadIdx.x == 0) {
+    t = p.d_step ? *p.d_step : int64_t(1);
+    skip = (bc && t < 1) ? 1 : 0;
+    if (bc && !skip)
+      c1 = (float)(1.0 / (1.0 - pow_from_log2(p.log2_beta1, (double)t)));
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const float c2 = s_c2;
     s_k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps};
     s_lr = step_lr(p, t);
     s_skip = skip;

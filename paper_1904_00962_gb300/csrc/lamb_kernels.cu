@@ -250,10 +250,9 @@ __device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
 }
 
 // Nadam momentum schedule term (appendix Alg. 3 inputs): mu_t =
-// beta1 (1 - 0.5 * 0.96^(t psi)); pow is CUDA's, in fp64.
-__device__ __forceinline__ double nadam_mu(double beta1, double psi,
-                                           int64_t t) {
-  return beta1 * (1.0 - 0.5 * pow(0.96, (double)t * psi));
+// beta1 (1 - 0.5 * 0.96^(t psi)).
+__device__ __forceinline__ double nadam_mu(const StepParams& p, int64_t t) {
+  return p.beta1 * (1.0 - 0.5 * pow_from_log2(p.log2_mu_decay, (double)t));
 }
 
 // lambda_k inside the normalised direction u (Alg. 2); 0 with decoupled
@@ -263,46 +262,76 @@ __device__ __forceinline__ float lam_in_u(const StepParams& p,
   return (p.flags & kFlagDecoupledDecay) ? 0.f : td.decay * p.wd;
 }
 
-template <typename GT, int kNest, bool kGn>
-__global__ void __launch_bounds__(kThreads)
-    lamb_pass1_kernel(const StepParams p) {
-  __shared__ float red[4][kWarps];
-  __shared__ uint32_t s_next[2];
-  __shared__ int s_last, s_skip;
-  __shared__ LambConsts s_k;
-  if (threadIdx.x == 0) {
-    const bool bc = kNest != 0 || (p.flags & kFlagBiasCorrection) != 0;
+// Per-launch constants of pass 1.  The fp64 work is spread over the lane 0
+// of warps 0-3 (one power each, with the divisions that need only it) while
+// warp 4 draws the first chunk and warp 5 fetches the N-LAMB product; thread
+// 0 then forms the rest.  The results do not depend on the split.
+template <int kNest>
+__device__ __forceinline__ void pass1_constants(const StepParams& p,
+                                                uint32_t* s_next, int* s_skip,
+                                                LambConsts* s_k) {
+  __shared__ double s_x[3];     // mu_t, mu_{t+1}, prod_{i<t} mu_i
+  __shared__ float s_c[2];      // c1, c2 (LAMB) or bv, bg (N-LAMB)
+  __shared__ int64_t s_t;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool bc = kNest != 0 || (p.flags & kFlagBiasCorrection) != 0;
+  if (lane == 0 && warp < 6) {
     const int64_t t = p.d_step ? *p.d_step : int64_t(1);
-    const int skip = (bc && t < 1) ? 1 : 0;
-    float c1 = 1.f, c2 = 1.f;
-    if (!kNest && bc && !skip) {  // Alg. 2 bias correction, beta^t in fp64
-      c1 = (float)(1.0 / (1.0 - pow(p.beta1, (double)t)));
-      c2 = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
+    const bool skip = bc && t < 1;
+    const double td = (double)t;
+    if (warp == 0) {
+      *s_skip = skip ? 1 : 0;
+      s_t = t;
     }
-    LambConsts kc{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps,
-                  0.f, 0.f, 0.f, 0.f};
-    double mu_prod = 0.0;
-    if (kNest && !skip) {  // appendix Alg. 3 / 4 coefficients, fp64
-      const double mu_t = nadam_mu(p.beta1, p.psi, t);
-      const double mu_n = nadam_mu(p.beta1, p.psi, t + 1);
-      mu_prod = *p.d_mu_product * mu_t;
-      const double prod_n = mu_prod * mu_n;
-      kc.am = (float)(mu_n / (1.0 - prod_n));
-      kc.ag = (float)((1.0 - mu_t) / (1.0 - mu_prod));
-      if (kNest == 2) {
-        kc.bv = (float)(p.beta2 / (1.0 - pow(p.beta2, (double)(t + 1))));
-        kc.bg = (float)((1.0 - p.beta2) / (1.0 - pow(p.beta2, (double)t)));
-      } else {
-        kc.bv = (float)(1.0 / (1.0 - pow(p.beta2, (double)t)));
+    if (!skip) {
+      if (warp == 4) {
+        s_next[0] = atomicAdd(&p.counters[0], 1u);
+      } else if (!kNest) {
+        if (warp < 2)   // Alg. 2 bias correction: 1/(1 - beta^t)
+          s_c[warp] = !bc ? 1.f
+                          : (float)(1.0 / (1.0 - pow_from_log2(
+                                warp == 0 ? p.log2_beta1 : p.log2_beta2, td)));
+      } else if (warp < 2) {           // appendix Alg. 3/4: mu_t, mu_{t+1}
+        s_x[warp] = nadam_mu(p, t + warp);
+      } else if (warp == 2) {          // v_hat's correction at t
+        const double b = pow_from_log2(p.log2_beta2, td);
+        if (kNest == 2) s_c[1] = (float)((1.0 - p.beta2) / (1.0 - b));
+        else s_c[0] = (float)(1.0 / (1.0 - b));
+      } else if (warp == 3) {          // NN-LAMB: beta2 / (1 - beta2^(t+1))
+        if (kNest == 2)
+          s_c[0] = (float)(p.beta2 /
+                           (1.0 - pow_from_log2(p.log2_beta2, td + 1.0)));
+      } else if (kNest) {              // warp 5
+        s_x[2] = *p.d_mu_product;
       }
     }
-    s_k = kc;
-    s_skip = skip;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int64_t t = s_t;
+    const int skip = *s_skip;
+    LambConsts kc{p.b1, p.omb1, p.b2, p.omb2, 1.f, 1.f, p.eps,
+                  0.f, 0.f, 0.f, 0.f};
+    double mu_prod = 0.0;
+    if (!skip) {
+      if (!kNest) {
+        kc.c1 = s_c[0];
+        kc.c2 = s_c[1];
+      } else {
+        const double mu_t = s_x[0], mu_n = s_x[1];
+        mu_prod = s_x[2] * mu_t;
+        kc.am = (float)(mu_n / (1.0 - mu_prod * mu_n));
+        kc.ag = (float)((1.0 - mu_t) / (1.0 - mu_prod));
+        kc.bv = s_c[0];
+        kc.bg = kNest == 2 ? s_c[1] : 0.f;
+      }
+    }
+    *s_k = kc;
     if (blockIdx.x == 0) {
       StepScalars sc{};
       sc.t = t;
-      sc.c1 = c1;
-      sc.c2 = c2;
+      sc.c1 = kc.c1;
+      sc.c2 = kc.c2;
       sc.lr = step_lr(p, t);
       sc.skip = skip;
       sc.am = kc.am;
@@ -313,9 +342,18 @@ __global__ void __launch_bounds__(kThreads)
       *p.scal = sc;
       if (skip) atomicOr(p.status, kStatusBadStep);
     }
-    if (!skip) s_next[0] = atomicAdd(&p.counters[0], 1u);
   }
   __syncthreads();
+}
+
+template <typename GT, int kNest, bool kGn>
+__global__ void __launch_bounds__(kThreads)
+    lamb_pass1_kernel(const StepParams p) {
+  __shared__ float red[4][kWarps];
+  __shared__ uint32_t s_next[2];
+  __shared__ int s_last, s_skip;
+  __shared__ LambConsts s_k;
+  pass1_constants<kNest>(p, s_next, &s_skip, &s_k);
   if (s_skip) return;
   const LambConsts k = s_k;
   const bool store = !(kGn && (p.flags & kFlagSkipNonfinite));

@@ -318,6 +318,8 @@ extern "C" LAMB_API lamb_status_t lamb_step_noalloc(
   sp.wd = (float)h.weight_decay;
   sp.beta1 = h.beta1;
   sp.beta2 = h.beta2;
+  sp.log2_beta1 = std::log2(h.beta1);
+  sp.log2_beta2 = std::log2(h.beta2);
   sp.gamma_l = h.gamma_l;
   sp.gamma_u = h.gamma_u;
   sp.trust = h.trust_coef;
