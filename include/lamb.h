@@ -123,12 +123,14 @@ typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
 #define LAMB_STATUS_BAD_STEP  0x2u      /* *d_step < 1 with bias correction:
                                            the step was skipped, nothing was
                                            written                          */
-#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* single-touch: a pass-2 item waited
-                                           ~0.5 s for its tensor's norms and
-                                           gave up; the rest of that launch's
-                                           pass-2 items then gave up too, so
-                                           w was not (fully) updated; never
-                                           expected                         */
+#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* single-touch: a wait inside the
+                                           kernel (a pass-2 item for its
+                                           tensor's norms, or a stage of the
+                                           operand pipeline) gave up after
+                                           ~0.5 s and the rest of the launch
+                                           gave up with it, so the step is
+                                           incomplete and the plan must be
+                                           destroyed; never expected        */
 #define LAMB_STATUS_GRAD_NONFINITE 0x8u /* GRAD_NORM: a gradient element was
                                            Inf or NaN                       */
 #define LAMB_STATUS_SKIPPED   0x10u     /* SKIP_NONFINITE: a step was skipped
@@ -162,7 +164,11 @@ typedef struct {
                                      follows its pass 1 closely enough to read
                                      m, v, w back from L2: ~28 B/parameter
                                      for tensors whose state fits the L2
-                                     budget                                  */
+                                     budget.  Work items are fused chunks of
+                                     LAMB_FUSED_CHUNK_ELEMS elements.  LAMB
+                                     and LARS only; N-LAMB and the flagged
+                                     variants run two-pass on such a plan  */
+#define LAMB_FUSED_CHUNK_ELEMS 4096
 
 /* Optional plan-creation knobs (pass NULL for defaults). */
 typedef struct {
@@ -175,8 +181,8 @@ typedef struct {
                             this many MiB keep them in L2 between the
                             passes; 0 = half the device's L2               */
   int32_t lag_items;     /* single-touch: work items between a tensor's last
-                            pass-1 item and its pass-2 block; 0 = 1.5x the
-                            items the grid holds in flight                 */
+                            pass-1 item and its pass-2 block; 0 = about the
+                            items the grid holds in flight (8 per CTA)     */
 } lamb_plan_options_t;
 
 typedef struct {
@@ -395,7 +401,7 @@ LAMB_API lamb_status_t lamb_step_noalloc(
 
 /* Host-only planner, no device needed: the work-item order a single-touch
  * plan would use.  Each item is (fused chunk index << 1) | is_pass2; fused
- * chunks hold 512 elements, numbered in tensor order.  l2_budget_bytes and
+ * chunks hold LAMB_FUSED_CHUNK_ELEMS elements, numbered in tensor order.  l2_budget_bytes and
  * lag_items as in lamb_plan_options_t (both required, > 0).  Writes up to
  * `capacity` items, the total into *n_items and, if `resident` is not NULL,
  * one residency flag per tensor.  INVALID_ARG on bad input or capacity too

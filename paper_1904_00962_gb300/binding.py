@@ -77,6 +77,7 @@ class lamb_hyper_t(Structure):
 LAMB_ALGO_AUTO = 0
 LAMB_ALGO_TWO_PASS = 1
 LAMB_ALGO_SINGLE_TOUCH = 2
+LAMB_FUSED_CHUNK_ELEMS = 4096     # work item of a single-touch step
 LAMB_STATUS_WAIT_TIMEOUT = 0x4
 
 

@@ -42,6 +42,8 @@ void lamb::set_last_error(const char* msg) {
 
 namespace {
 
+static_assert(lamb::kFusedChunk == LAMB_FUSED_CHUNK_ELEMS,
+              "the ABI documents the fused chunk size");
 constexpr int kMaxTimedSteps = 4096;
 constexpr int kKernelsPerStep = 2;
 
@@ -77,7 +79,7 @@ struct lamb_plan {
   int grid[4] = {0, 0, 0, 0};  // lamb p1, lamb p2, lars p1, lars p2
   int grid_fused[2] = {0, 0};  // single-touch lamb, lars
   int algorithm = LAMB_ALGO_TWO_PASS;
-  int64_t n_items = 0, n_groups = 0, lag = 0, l2_budget = 0;
+  int64_t n_items = 0, lag = 0, l2_budget = 0;
   int n_resident = 0;
   bool bound = false;
   bool has_v = false;
@@ -105,11 +107,8 @@ struct lamb_plan {
   int n_live = 0;               // tensors with at least one chunk
   // single-touch tables
   uint2* items = nullptr;
-  FusedChunk* fchunks = nullptr;
   FusedTensor* ftensors = nullptr;
   float2* fslots = nullptr;
-  double2* gslots = nullptr;
-  uint32_t* gtickets = nullptr;
   uint32_t* ftickets = nullptr;
   uint32_t* ready = nullptr;
 
@@ -180,10 +179,9 @@ lamb_status_t lamb_layout_schedule(const int64_t* sizes, int32_t n_tensors,
   std::vector<FusedChunk> fc;
   std::vector<FusedTensor> ft;
   std::vector<uint32_t> it;
-  int64_t ng = 0;
   try {
     if (plan_fused(sizes, n_tensors, nullptr, 12, l2_budget_bytes, lag_items,
-                   &fc, &ft, &it, &ng, err, sizeof(err)))
+                   &fc, &ft, &it, err, sizeof(err)))
       return fail(LAMB_ERR_INVALID_ARG, "%s", err);
   } catch (const std::bad_alloc&) {
     return fail(LAMB_ERR_OOM, "host allocation failed");
@@ -325,7 +323,7 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
                                 ? p->grid_fused[0]
                                 : p->grid_fused[1]);
     if (plan_fused(sizes, n_tensors, decay_mask, 12, p->l2_budget, p->lag,
-                   &h_fchunks, &h_ftensors, &h_items, &p->n_groups, err,
+                   &h_fchunks, &h_ftensors, &h_items, err,
                    sizeof(err))) {
       delete p;
       return fail(LAMB_ERR_INVALID_ARG, "%s", err);
@@ -356,13 +354,13 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   const size_t o_grad_sq = carve(n * sizeof(double));
   const size_t o_grad_norm = carve(n * sizeof(double));
   const size_t o_grad_check = carve(sizeof(GradCheck));
-  const size_t nf = h_fchunks.size(), ng = (size_t)p->n_groups;
-  const size_t o_items = carve(h_items.size() * sizeof(uint2));
-  const size_t o_fchunks = carve(nf * sizeof(FusedChunk));
+  const size_t nf = h_fchunks.size();
+  // padded so that a batch of kDrawBatch item records is always readable
+  const size_t n_items_pad =
+      (h_items.size() + kDrawBatch - 1) / kDrawBatch * kDrawBatch;
+  const size_t o_items = carve(n_items_pad * sizeof(uint2));
   const size_t o_ftensors = carve(n * sizeof(FusedTensor));
   const size_t o_fslots = carve(nf * sizeof(float2));
-  const size_t o_gslots = carve(ng * sizeof(double2));
-  const size_t o_gtickets = carve(ng * sizeof(uint32_t));
   const size_t o_ftickets = carve(n * sizeof(uint32_t));
   const size_t o_ready = carve(n * sizeof(uint32_t));
   p->arena_bytes = off;
@@ -388,11 +386,8 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   p->grad_norm = reinterpret_cast<double*>(base + o_grad_norm);
   p->grad_check = reinterpret_cast<GradCheck*>(base + o_grad_check);
   p->items = reinterpret_cast<uint2*>(base + o_items);
-  p->fchunks = reinterpret_cast<FusedChunk*>(base + o_fchunks);
   p->ftensors = reinterpret_cast<FusedTensor*>(base + o_ftensors);
   p->fslots = reinterpret_cast<float2*>(base + o_fslots);
-  p->gslots = reinterpret_cast<double2*>(base + o_gslots);
-  p->gtickets = reinterpret_cast<uint32_t*>(base + o_gtickets);
   p->ftickets = reinterpret_cast<uint32_t*>(base + o_ftickets);
   p->ready = reinterpret_cast<uint32_t*>(base + o_ready);
 
@@ -406,7 +401,7 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
                    cudaMemcpyHostToDevice);
   if (e == cudaSuccess && !h_items.empty()) {
     // device items carry the tensor and the chunk index directly
-    std::vector<uint2> dev_items(h_items.size());
+    std::vector<uint2> dev_items(n_items_pad, make_uint2(0u, 0u));
     for (size_t i = 0; i < h_items.size(); ++i) {
       const FusedChunk& fc = h_fchunks[h_items[i] >> 1];
       dev_items[i] = make_uint2(((uint32_t)fc.tensor << 1) | (h_items[i] & 1u),
@@ -415,9 +410,6 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
     e = cudaMemcpy(p->items, dev_items.data(), dev_items.size() * sizeof(uint2),
                    cudaMemcpyHostToDevice);
   }
-  if (e == cudaSuccess && nf)
-    e = cudaMemcpy(p->fchunks, h_fchunks.data(), nf * sizeof(FusedChunk),
-                   cudaMemcpyHostToDevice);
   if (e == cudaSuccess)
     e = cudaMemcpy(p->ftensors, h_ftensors.data(), n * sizeof(FusedTensor),
                    cudaMemcpyHostToDevice);
@@ -612,11 +604,8 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
       !(hyper->flags & two_pass_only)) {
     FusedParams fp;
     fp.items = plan->items;
-    fp.fchunks = plan->fchunks;
     fp.ftensors = plan->ftensors;
     fp.fslots = plan->fslots;
-    fp.gslots = plan->gslots;
-    fp.gtickets = plan->gtickets;
     fp.tickets = plan->ftickets;
     fp.ready = plan->ready;
     fp.n_items = (int32_t)plan->n_items;

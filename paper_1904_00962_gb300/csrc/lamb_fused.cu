@@ -1,55 +1,86 @@
-// sm_103a kernel of the single-touch LAMB / LARS step (one persistent
-// launch per step; see the comment at the top of the kernel section).
+// sm_103a kernel of the single-touch LAMB / LARS step: one persistent launch
+// per step, in which the pass 2 of a tensor follows its pass 1 closely enough
+// to read m, v, w back from L2 (28 instead of 40 bytes of HBM traffic per
+// parameter for BERT-large's bf16 gradients and bf16 copy).
+//
+// Work items are fused chunks of kFusedChunk elements, pass 1 or pass 2,
+// drawn in the order of a host-built schedule (planner.cpp, plan_fused): the
+// pass-1 items tensor by tensor; the pass-2 block of a tensor whose state fits
+// the L2 budget placed `lag` items after its last pass-1 item; the pass-2
+// blocks of larger tensors at the end.
+//
+// One CTA per SM, warp-specialised:
+//   producer   (warp 16, one lane) draws items in schedule order, keeps the
+//              draws and descriptors of the next items in flight, waits for
+//              a pass-2 item's tensor to be final, and stages each item's
+//              operands in a ring of up to 8 shared-memory stages with TMA
+//              bulk copies (cp.async.bulk) that complete on the stage's
+//              mbarrier;
+//   consumers  (warps 0-15, each walking the stage ring on its own) apply
+//              Alg. 2 (Alg. 1 for LARS) to a staged item and store the
+//              results; for a pass-1 item the last warp to finish it adds
+//              the warps' sums of w^2 and u^2 in warp order and hands the
+//              pair to
+//   publisher  (warp 17), which stores the chunk's sums, takes the tensor's
+//              ticket and, for the tensor's last chunk, combines the chunk
+//              sums in a fixed order in fp64, writes rho_k and releases
+//              ready[k] = epoch.
+// The consumers never wait on a global atomic, and the producer never waits
+// on the consumers' arithmetic except through a free stage.
+//
+// Deadlock freedom: every pass-2 item follows all pass-1 items of its tensor
+// in the schedule, and each CTA takes its items in the order it drew them.
+// The unfinished item with the smallest index therefore sits at the head of
+// its CTA's pipeline with everything it depends on finished, so it always
+// completes; no co-residency of the CTAs is needed.  Every wait is still
+// bounded (~0.5 s): on a timeout the CTA sets LAMB_STATUS_WAIT_TIMEOUT and an
+// abort word that makes every other waiter of the launch give up, waits (also
+// bounded) for its own copies in flight, and returns.
+//
+// Memory ordering: a consumer's m, v stores -> block-scope fence and
+// counter -> the last warp's mbarrier arrive (CTA scope) -> the publisher's
+// acq_rel ticket (GPU scope) -> the
+// finaliser's release of ready[k] -> a producer's acquire of ready[k] ->
+// fence.proxy.async.global -> its TMA reads of m, v (async proxy).
+//
+// Identical arithmetic to the two-pass kernels (lamb_device.cuh); per-chunk
+// fp32 sums and the per-tensor fp64 combine in chunk order make the result
+// independent of which CTA ran which item.
 #include "lamb_device.cuh"
 
 namespace lamb {
 namespace {
 
-// ---------------------------------------------------------------------------
-// Single-touch fused step (one persistent kernel, warps are the workers)
-//
-// Items are drawn in schedule order from counters[2].  A pass-1 item runs one
-// fused chunk (512 elements) through Alg. 2's moment and ratio lines (Alg. 1
-// for LARS), stores the new m, v and publishes the chunk's sums; the warp that
-// completes a group of 32 chunks sums them (fp64, fixed order), and the warp
-// that completes a tensor's last group computes its norms and trust ratio and
-// releases ready[k] = epoch.  A pass-2 item applies the update once ready[k]
-// == epoch.  Pass-2 items of a tensor come after all its pass-1 items in the
-// schedule and items are drawn in order, so the earliest unfinished item never
-// waits on anything unfinished: the kernel cannot deadlock.  A wait still
-// gives up after ~0.5 s, sets a status bit and makes every other waiter of
-// the same launch give up at once.
-//
-// Memory pipeline: every warp owns a ring of kStages shared-memory stages and
-// prefetches the operands of its next items with cp.async while it computes
-// the current one, so many bytes are in flight without holding registers.  A
-// pass-2 item is prefetched only if its tensor's norms are already final when
-// its stage is filled (its m, v come from other warps' pass-1 stores);
-// otherwise, and for tail chunks and unaligned tensors, the item reads global
-// memory directly when its turn comes.  The control traffic (draws, item
-// descriptors, ready flags, tickets) is pipelined as described at the warp
-// worker below.
-//
-// L2 policy: pass-1 loads/stores of m, v, w of "resident" tensors (those
-// whose state fits the L2 budget) are evict_last, so pass 2 -- about one
-// wave later -- finds them in L2; gradients and all pass-2 traffic are
-// evict_first.
-// ---------------------------------------------------------------------------
-constexpr int kFusedThreads = 256;                     // 8 warps per CTA
-constexpr int kFusedWarps = kFusedThreads / 32;
-constexpr int kStages = 3;                             // prefetch depth per warp
-constexpr int kPktsPerLane = kFusedChunk / 4 / 32;     // 4-element packets
-static_assert(kPktsPerLane * 4 * 32 == kFusedChunk, "fused chunk shape");
-constexpr uint32_t kSpinLimit = 1u << 21;              // x <= 256 ns ~ 0.5 s
+constexpr int kConsumerWarps = 16;
+constexpr int kConsumers = kConsumerWarps * 32;           // 512 threads
+constexpr int kProducerWarp = kConsumerWarps;             // warp 16
+constexpr int kPublisherWarp = kConsumerWarps + 1;        // warp 17
+constexpr int kFusedThreads = (kConsumerWarps + 2) * 32;  // 576
+constexpr int kMaxStages = 8;                             // operand ring
+constexpr int kStageBudget = 220 * 1024;                  // dynamic smem
+constexpr int kPubSlots = 16;                             // sums ring
+constexpr int kRedRing = 2 * kMaxStages;                  // partial-sum ring
+constexpr int kPkts = kFusedChunk / 4 / kConsumers;       // float4 per array
+static_assert(kPkts * 4 * kConsumers == kFusedChunk, "fused chunk shape");
+static_assert(kPubSlots <= 32, "the publisher takes up to a warp of entries");
+constexpr uint32_t kSpinLimit = 1u << 21;                 // polls, <= ~0.5 s
 
-// stage layout: m | v (LAMB only) | w | g
+// stage layout: m | v (LAMB) | w | g, each kFusedChunk elements
 template <bool kLars, typename GT>
 __host__ __device__ constexpr int stage_bytes() {
   return kFusedChunk * (4 * (kLars ? 2 : 3) + (int)sizeof(GT));
 }
+// as many stages as fit the budget (7 for LAMB with bf16 g, 6 with fp32 g):
+// the ring must cover the TMA latency of the items behind the one in use
+template <bool kLars, typename GT>
+__host__ __device__ constexpr int n_stages() {
+  return kStageBudget / stage_bytes<kLars, GT>() < kMaxStages
+             ? kStageBudget / stage_bytes<kLars, GT>()
+             : kMaxStages;
+}
 template <bool kLars, typename GT>
 __host__ __device__ constexpr int fused_smem_bytes() {
-  return kFusedWarps * kStages * stage_bytes<kLars, GT>();
+  return n_stages<kLars, GT>() * stage_bytes<kLars, GT>();
 }
 constexpr int kOffM = 0;
 constexpr int kOffV = 4 * kFusedChunk;
@@ -60,6 +91,35 @@ template <bool kLars> __host__ __device__ constexpr int off_g() {
   return 4 * kFusedChunk * (kLars ? 2 : 3);
 }
 
+// item flags in a stage descriptor
+enum : uint32_t { kItemP2 = 1u, kItemDirect = 2u, kItemEnd = 4u,
+                  kItemSkip = 8u, kItemResident = 16u };
+
+struct StageDesc {      // written by the producer, read by the consumers
+  TensorPtrs tp;        // the tensor's arrays (the consumers load nothing
+                        // but the stage and this descriptor)
+  int32_t tensor;
+  int32_t index;        // fused chunk index inside the tensor
+  int32_t len;          // elements in the chunk
+  uint32_t flags;
+  float s;              // pass 2: eta * rho_k
+  float lam;            // lambda_k
+  int32_t first_chunk;  // slot base and chunk count of the tensor
+  int32_t n_chunks;
+};
+
+struct PubEntry {       // a pass-1 chunk's sums, consumers -> publisher
+  int32_t tensor;       // -1: end of the stream
+  int32_t first_chunk;  // the tensor's first fused chunk in the plan
+  int32_t index;        // the chunk's index inside the tensor
+  int32_t n_chunks;
+  float sw, su;
+};
+
+// ---------------------------------------------------------------------------
+// PTX helpers: cache policies, stores with hints, mbarriers, TMA bulk
+// copies, scoped atomics
+// ---------------------------------------------------------------------------
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
@@ -70,37 +130,17 @@ __device__ __forceinline__ uint64_t policy_evict_last() {
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
-__device__ __forceinline__ float4 ldp4(const float* p, uint64_t pol) {
-  float4 r;
-  asm volatile(
-      "ld.global.L1::no_allocate.L2::cache_hint.v4.f32 {%0,%1,%2,%3}, [%4], %5;"
-      : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
-      : "l"(p), "l"(pol));
-  return r;
-}
 __device__ __forceinline__ void stp4(float* p, float4 v, uint64_t pol) {
   asm volatile(
       "st.global.L1::no_allocate.L2::cache_hint.v4.f32 [%0], {%1,%2,%3,%4}, %5;"
       ::"l"(p), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "l"(pol)
       : "memory");
 }
-__device__ __forceinline__ float4 ldp_grad4(const float* p, uint64_t pol) {
-  return ldp4(p, pol);
-}
 __device__ __forceinline__ float4 unpack_bf16x4(uint32_t a, uint32_t b) {
   return make_float4(__uint_as_float(a << 16), __uint_as_float(a & 0xffff0000u),
                      __uint_as_float(b << 16), __uint_as_float(b & 0xffff0000u));
 }
-__device__ __forceinline__ float4 ldp_grad4(const __nv_bfloat16* p,
-                                            uint64_t pol) {
-  uint32_t a, b;
-  asm volatile(
-      "ld.global.L1::no_allocate.L2::cache_hint.v2.u32 {%0,%1}, [%2], %3;"
-      : "=r"(a), "=r"(b)
-      : "l"(p), "l"(pol));
-  return unpack_bf16x4(a, b);
-}
-// gradient packet j of a stage
+// gradient packet j (4 elements) of a stage
 __device__ __forceinline__ float4 lds_grad4(const char* gbase, int j,
                                             const float*) {
   return *reinterpret_cast<const float4*>(gbase + 16 * j);
@@ -124,23 +164,15 @@ __device__ __forceinline__ void stp_copy4(void* base, int64_t i, float4 x,
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-__device__ __forceinline__ void cp_async16(uint32_t saddr, const void* g,
-                                           uint64_t pol) {
-  asm volatile(
-      "cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;"
-      ::"r"(saddr), "l"(g), "l"(pol)
-      : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
   uint32_t v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p)
                : "memory");
   return v;
 }
@@ -154,14 +186,70 @@ __device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
                : "=r"(old) : "l"(p), "r"(v) : "memory");
   return old;
 }
-__device__ __forceinline__ double warp_sum_d(double x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x += __shfl_down_sync(0xffffffffu, x, o);
-  return x;
+// after acquiring another SM's generic-proxy stores: make them visible to
+// this thread's later TMA (async-proxy) reads
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-// Element of the fused pass 1: LAMB (Alg. 2) or LARS (Alg. 1) moment update,
-// then the direction u whose norm the trust ratio needs.
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;"
+               ::"r"(smem_u32(b)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
+  asm volatile("{\n\t.reg .b64 st;\n\t"
+               "mbarrier.arrive.shared::cta.b64 st, [%0];\n\t}"
+               ::"r"(smem_u32(b)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t* b, uint32_t bytes) {
+  asm volatile("{\n\t.reg .b64 st;\n\t"
+               "mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n\t}"
+               ::"r"(smem_u32(b)), "r"(bytes) : "memory");
+}
+// true once the phase of the given parity has completed (non-blocking)
+__device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile("{\n\t.reg .pred p;\n\t"
+               "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+               "selp.u32 %0, 1, 0, p;\n\t}"
+               : "=r"(ok) : "r"(smem_u32(b)), "r"(parity) : "memory");
+  return ok != 0;
+}
+// TMA bulk copy global -> shared; completion counted in bytes on `bar`
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src,
+                                         uint32_t bytes, uint64_t* bar,
+                                         uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1], %2, [%3], %4;"
+      ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(pol)
+      : "memory");
+}
+// A wait that ran out: report it and make every other waiter of this launch
+// (abort word counters[4] == epoch) give up too.
+__device__ __forceinline__ void give_up(uint32_t* status, uint32_t* counters,
+                                        uint32_t epoch) {
+  atomicOr(status, kStatusWaitTimeout);
+  atomicExch(&counters[4], epoch);
+}
+
+// Poll an mbarrier phase with a bounded number of tries; gives up early if
+// another CTA of this launch has aborted.  Returns false on give-up.
+__device__ __noinline__ bool wait_phase(uint64_t* b, uint32_t parity,
+                                        uint32_t* status, uint32_t* counters,
+                                        uint32_t epoch) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if (mbar_test(b, parity)) return true;
+    if ((i & 255) == 255 && ld_relaxed(&counters[4]) == epoch) return false;
+    if (i >= 64) __nanosleep(i >= 4096 ? 256 : 32);
+  }
+  give_up(status, counters, epoch);
+  return false;
+}
+
+// ---------------------------------------------------------------------------
+// Element arithmetic (same functions as the two-pass kernels)
+// ---------------------------------------------------------------------------
 template <bool kLars>
 __device__ __forceinline__ void fused1_elem(float g, float& m, float& v,
                                             float w, float lam,
@@ -180,146 +268,58 @@ __device__ __forceinline__ void fused1_elem(float g, float& m, float& v,
 }
 
 template <bool kLars>
-__device__ __forceinline__ float fused2_dir(float m, float v, float w,
-                                            float lam, const LambConsts& k) {
-  return kLars ? m : lamb_direction(m, v, w, lam, k);
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused1_pkt(float4 gv, float4& mv, float4& vv,
-                                           float4 wv, float lam,
-                                           const LambConsts& k, float& sw,
-                                           float& su) {
-  fused1_elem<kLars>(gv.x, mv.x, vv.x, wv.x, lam, k, sw, su);
-  fused1_elem<kLars>(gv.y, mv.y, vv.y, wv.y, lam, k, sw, su);
-  fused1_elem<kLars>(gv.z, mv.z, vv.z, wv.z, lam, k, sw, su);
-  fused1_elem<kLars>(gv.w, mv.w, vv.w, wv.w, lam, k, sw, su);
-}
-
-template <bool kLars>
-__device__ __forceinline__ float4 fused2_pkt(float4 mv, float4 vv, float4 wv,
+__device__ __forceinline__ float fused2_elem(float m, float v, float w,
                                              float s, float lam,
                                              const LambConsts& k) {
-  float4 o;
-  o.x = __fmaf_rn(-s, fused2_dir<kLars>(mv.x, vv.x, wv.x, lam, k), wv.x);
-  o.y = __fmaf_rn(-s, fused2_dir<kLars>(mv.y, vv.y, wv.y, lam, k), wv.y);
-  o.z = __fmaf_rn(-s, fused2_dir<kLars>(mv.z, vv.z, wv.z, lam, k), wv.z);
-  o.w = __fmaf_rn(-s, fused2_dir<kLars>(mv.w, vv.w, wv.w, lam, k), wv.w);
-  return o;
+  const float u = kLars ? m : lamb_direction(m, v, w, lam, k);
+  return __fmaf_rn(-s, u, w);
 }
 
-__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
-  uint32_t v;
-  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p)
-               : "memory");
-  return v;
-}
-__device__ __forceinline__ void fence_acq_rel() {
-  asm volatile("fence.acq_rel.gpu;" ::: "memory");
-}
-
-// Issue the cp.async copies of one full, aligned chunk into `stage`: m, v
-// (LAMB), w, and for pass 1 the gradient.
+// ---------------------------------------------------------------------------
+// Consumer work on one item
+// ---------------------------------------------------------------------------
+// Pass 1 from a stage (chunk length a multiple of 8): each consumer thread
+// takes packets tid, tid + kConsumers, ...
 template <bool kLars, typename GT>
-__device__ __forceinline__ void fused_prefetch_ops(
-    const TensorPtrs& tp, int64_t off, bool pass2, bool resident, char* stage,
-    uint64_t pol_first, uint64_t pol_last, int lane) {
-  const uint64_t pol = (!pass2 && resident) ? pol_last : pol_first;
-  const uint32_t s = smem_u32(stage);
+__device__ __forceinline__ void c_pass1_staged(const char* st,
+                                               const TensorPtrs& tp,
+                                               int64_t off, int len,
+                                               float lam, const LambConsts& k,
+                                               uint64_t pol_keep, float& sw,
+                                               float& su, int tid) {
+  const GT* tag = nullptr;
+  const int np = len >> 2;
 #pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;                    // 16-byte piece index
-    cp_async16(s + kOffM + 16 * j, tp.m + off + 4 * j, pol);
-    if (!kLars) cp_async16(s + kOffV + 16 * j, tp.v + off + 4 * j, pol);
-    cp_async16(s + off_w<kLars>() + 16 * j, tp.w + off + 4 * j, pol);
-  }
-  if (!pass2) {
-    const char* g = reinterpret_cast<const char*>(
-        static_cast<const GT*>(tp.g) + off);
-    constexpr int kGPieces = kFusedChunk * (int)sizeof(GT) / 16;
-#pragma unroll
-    for (int u = 0; u < kGPieces / 32; ++u) {
-      const int j = lane + 32 * u;
-      cp_async16(s + off_g<kLars>() + 16 * j, g + 16 * j, pol_first);
+  for (int q = 0; q < kPkts; ++q) {
+    const int j = tid + q * kConsumers;
+    if (j < np) {
+      float4 mv = *reinterpret_cast<const float4*>(st + kOffM + 16 * j);
+      float4 vv = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
+                        : *reinterpret_cast<const float4*>(st + kOffV + 16 * j);
+      const float4 wv =
+          *reinterpret_cast<const float4*>(st + off_w<kLars>() + 16 * j);
+      const float4 gv = lds_grad4(st + off_g<kLars>(), j, tag);
+      fused1_elem<kLars>(gv.x, mv.x, vv.x, wv.x, lam, k, sw, su);
+      fused1_elem<kLars>(gv.y, mv.y, vv.y, wv.y, lam, k, sw, su);
+      fused1_elem<kLars>(gv.z, mv.z, vv.z, wv.z, lam, k, sw, su);
+      fused1_elem<kLars>(gv.w, mv.w, vv.w, wv.w, lam, k, sw, su);
+      stp4(tp.m + off + 4 * j, mv, pol_keep);
+      if (!kLars) stp4(tp.v + off + 4 * j, vv, pol_keep);
     }
   }
 }
 
-// Pass 1 of a staged chunk: new m, v into registers, sums of w^2 and u^2.
+// Pass 1 straight from global memory (tail chunks, unaligned tensors)
 template <bool kLars, typename GT>
-__device__ __forceinline__ void fused1_from_stage(const char* stage,
-                                                  float lam,
-                                                  const LambConsts& k,
-                                                  float4* mo, float4* vo,
-                                                  float& sw, float& su,
-                                                  int lane) {
-  const GT* tag = nullptr;
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;
-    mo[u] = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
-    vo[u] = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
-                  : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
-    const float4 wv =
-        *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
-    const float4 gv = lds_grad4(stage + off_g<kLars>(), j, tag);
-    fused1_pkt<kLars>(gv, mo[u], vo[u], wv, lam, k, sw, su);
-  }
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused1_store(const TensorPtrs& tp,
-                                             int64_t off, const float4* mo,
-                                             const float4* vo,
-                                             uint64_t pol_keep, int lane) {
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;
-    stp4(tp.m + off + 4 * j, mo[u], pol_keep);
-    if (!kLars) stp4(tp.v + off + 4 * j, vo[u], pol_keep);
-  }
-}
-
-// Pass 1 straight from global memory (tail chunks, unaligned tensors).
-template <bool kLars, typename GT>
-__device__ __forceinline__ void fused1_direct(const TensorPtrs& tp,
-                                              int64_t off, int len, float lam,
-                                              const LambConsts& k, float& sw,
-                                              float& su, uint64_t pol_first,
-                                              uint64_t pol_keep, int lane) {
+__device__ __forceinline__ void c_pass1_direct(const TensorPtrs& tp,
+                                               int64_t off, int len,
+                                               float lam, const LambConsts& k,
+                                               float& sw, float& su, int tid) {
   float* __restrict__ m = tp.m + off;
   float* __restrict__ v = kLars ? nullptr : tp.v + off;
   const float* __restrict__ w = tp.w + off;
   const GT* __restrict__ g = static_cast<const GT*>(tp.g) + off;
-  int scalar_from = 0;
-  if (tp.vec_ok) {
-    const int nv = len >> 2;
-#pragma unroll 1
-    for (int base = lane; base < nv; base += 64) {
-      float4 wv[2], mv[2], vv[2], gv[2];
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          gv[u] = ldp_grad4(g + 4 * j, pol_first);
-          mv[u] = ldp4(m + 4 * j, pol_keep);
-          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_keep);
-          wv[u] = ldp4(w + 4 * j, pol_keep);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          fused1_pkt<kLars>(gv[u], mv[u], vv[u], wv[u], lam, k, sw, su);
-          stp4(m + 4 * j, mv[u], pol_keep);
-          if (!kLars) stp4(v + 4 * j, vv[u], pol_keep);
-        }
-      }
-    }
-    scalar_from = nv << 2;
-  }
-  for (int i = scalar_from + lane; i < len; i += 32) {
+  for (int i = tid; i < len; i += kConsumers) {
     float mi = m[i];
     float vi = kLars ? 0.f : v[i];
     fused1_elem<kLars>(ld_grad1(g + i), mi, vi, w[i], lam, k, sw, su);
@@ -328,495 +328,489 @@ __device__ __forceinline__ void fused1_direct(const TensorPtrs& tp,
   }
 }
 
-// Pass 2 of a staged chunk: new w into registers.
-template <bool kLars>
-__device__ __forceinline__ void fused2_from_stage(const char* stage, float s,
-                                                  float lam,
-                                                  const LambConsts& k,
-                                                  float4* wo, int lane) {
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;
-    const float4 mv = *reinterpret_cast<const float4*>(stage + kOffM + 16 * j);
-    const float4 vv = kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
-                            : *reinterpret_cast<const float4*>(stage + kOffV + 16 * j);
-    const float4 wv =
-        *reinterpret_cast<const float4*>(stage + off_w<kLars>() + 16 * j);
-    wo[u] = fused2_pkt<kLars>(mv, vv, wv, s, lam, k);
-  }
-}
-
-template <bool kCopy>
-__device__ __forceinline__ void fused2_store(const TensorPtrs& tp,
-                                             int64_t off, const float4* wo,
-                                             uint64_t pol_first, int lane) {
-#pragma unroll
-  for (int u = 0; u < kPktsPerLane; ++u) {
-    const int j = lane + 32 * u;
-    stp4(tp.w + off + 4 * j, wo[u], pol_first);
-    if (kCopy) stp_copy4(tp.copy, off + 4 * j, wo[u], pol_first);
-  }
-}
-
-// Pass 2 straight from global memory.
 template <bool kLars, bool kCopy>
-__device__ __forceinline__ void fused2_direct(const TensorPtrs& tp,
-                                              int64_t off, int len, float s,
-                                              float lam, const LambConsts& k,
-                                              uint64_t pol_first, int lane) {
+__device__ __forceinline__ void c_pass2_staged(const char* st,
+                                               const TensorPtrs& tp,
+                                               int64_t off, int len, float s,
+                                               float lam, const LambConsts& k,
+                                               uint64_t pol_first, int tid) {
+  const int np = len >> 2;
+#pragma unroll
+  for (int q = 0; q < kPkts; ++q) {
+    const int j = tid + q * kConsumers;
+    if (j < np) {
+      const float4 mv = *reinterpret_cast<const float4*>(st + kOffM + 16 * j);
+      const float4 vv =
+          kLars ? make_float4(0.f, 0.f, 0.f, 0.f)
+                : *reinterpret_cast<const float4*>(st + kOffV + 16 * j);
+      const float4 wv =
+          *reinterpret_cast<const float4*>(st + off_w<kLars>() + 16 * j);
+      float4 o;
+      o.x = fused2_elem<kLars>(mv.x, vv.x, wv.x, s, lam, k);
+      o.y = fused2_elem<kLars>(mv.y, vv.y, wv.y, s, lam, k);
+      o.z = fused2_elem<kLars>(mv.z, vv.z, wv.z, s, lam, k);
+      o.w = fused2_elem<kLars>(mv.w, vv.w, wv.w, s, lam, k);
+      stp4(tp.w + off + 4 * j, o, pol_first);
+      if (kCopy) stp_copy4(tp.copy, off + 4 * j, o, pol_first);
+    }
+  }
+}
+
+template <bool kLars, bool kCopy>
+__device__ __forceinline__ void c_pass2_direct(const TensorPtrs& tp,
+                                               int64_t off, int len, float s,
+                                               float lam, const LambConsts& k,
+                                               int tid) {
   float* __restrict__ w = tp.w + off;
   const float* __restrict__ m = tp.m + off;
   const float* __restrict__ v = kLars ? nullptr : tp.v + off;
-  int scalar_from = 0;
-  if (tp.vec_ok) {
-    const int nv = len >> 2;
-#pragma unroll 1
-    for (int base = lane; base < nv; base += 64) {
-      float4 wv[2], mv[2], vv[2];
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          mv[u] = ldp4(m + 4 * j, pol_first);
-          if (!kLars) vv[u] = ldp4(v + 4 * j, pol_first);
-          wv[u] = ldp4(w + 4 * j, pol_first);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 2; ++u) {
-        const int j = base + 32 * u;
-        if (j < nv) {
-          const float4 o = fused2_pkt<kLars>(mv[u], vv[u], wv[u], s, lam, k);
-          stp4(w + 4 * j, o, pol_first);
-          if (kCopy) stp_copy4(tp.copy, off + 4 * j, o, pol_first);
-        }
-      }
-    }
-    scalar_from = nv << 2;
-  }
-  for (int i = scalar_from + lane; i < len; i += 32) {
-    const float wi = w[i];
-    const float o = __fmaf_rn(
-        -s, fused2_dir<kLars>(m[i], kLars ? 0.f : v[i], wi, lam, k), wi);
+  // m, v come from other SMs' pass 1 of this launch: read them from L2
+  for (int i = tid; i < len; i += kConsumers) {
+    const float o = fused2_elem<kLars>(__ldcg(m + i), kLars ? 0.f : __ldcg(v + i),
+                                       w[i], s, lam, k);
     w[i] = o;
     if (kCopy) st_copy1(tp.copy, off + i, o);
   }
 }
 
-// The warp whose ticket completed group `gl` of tensor `tensor`: fixed-order
-// fp64 sum of the group's chunk sums; the warp that completes the tensor's
-// last group computes its norms and trust ratio and releases ready[tensor].
+// ---------------------------------------------------------------------------
+// Publisher: a tensor's last chunk -> norms, trust ratio, ready flag
+// ---------------------------------------------------------------------------
 template <bool kLars>
-__device__ __forceinline__ void fused_group_combine(const StepParams& p,
-                                                 const FusedParams& f,
-                                                 const FusedTensor& ft,
-                                                 int tensor, int gl, int gsize,
-                                                 uint32_t epoch, int lane) {
-  __syncwarp();
-  const int group = ft.first_group + gl;
+__device__ __forceinline__ void finalize_fused(const StepParams& p,
+                                               const FusedParams& f, int k,
+                                               int first, int n,
+                                               uint32_t epoch, int lane) {
+  __threadfence();
   double aw = 0.0, au = 0.0;
-  if (lane < gsize) {
-    const float2 s = __ldcg(&f.fslots[ft.first_chunk + gl * kGroup + lane]);
-    aw = (double)s.x;
-    au = (double)s.y;
+  for (int i = lane; i < n; i += 32) {
+    const float2 s = __ldcg(&f.fslots[first + i]);
+    aw += (double)s.x;
+    au += (double)s.y;
   }
-  aw = warp_sum_d(aw);
-  au = warp_sum_d(au);
-  uint32_t last = 0;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    aw += __shfl_down_sync(0xffffffffu, aw, o);
+    au += __shfl_down_sync(0xffffffffu, au, o);
+  }
   if (lane == 0) {
-    f.gslots[group] = make_double2(aw, au);
-    f.gtickets[group] = 0u;
-    last = atom_add_acq_rel(&f.tickets[tensor], 1u) + 1u ==
-           (uint32_t)ft.n_groups;
-  }
-  if (!__shfl_sync(0xffffffffu, last, 0)) return;
-  __syncwarp();
-  double tw = 0.0, tu = 0.0;
-  for (int i = lane; i < ft.n_groups; i += 32) {
-    const double2 s = __ldcg(&f.gslots[ft.first_group + i]);
-    tw += s.x;
-    tu += s.y;
-  }
-  tw = warp_sum_d(tw);
-  tu = warp_sum_d(tu);
-  if (lane == 0) {
-    const double wn = sqrt(tw), un = sqrt(tu);
-    double rho = 1.0;
+    const double wn = sqrt(aw), un = sqrt(au);
+    double rho = 1.0;                                  // zero-norm rule
     if (!(wn == 0.0 || un == 0.0))
       rho = (kLars ? p.trust : 1.0) * phi_of(wn, p) / un;
-    p.ratio[tensor] = rho;
-    p.wnorm[tensor] = wn;
-    p.unorm[tensor] = un;
-    if (!isfinite(tw) || !isfinite(tu)) atomicOr(p.status, kStatusNonfinite);
-    f.tickets[tensor] = 0u;
-    st_release(&f.ready[tensor], epoch);
+    p.ratio[k] = rho;
+    p.wnorm[k] = wn;
+    p.unorm[k] = un;
+    if (!isfinite(aw) || !isfinite(au)) atomicOr(p.status, kStatusNonfinite);
+    f.tickets[k] = 0u;
+    st_release(&f.ready[k], epoch);
   }
-}
-
-// Bounded wait of a pass-2 item for its tensor's norms (all lanes).
-__device__ __forceinline__ bool fused_wait(const StepParams& p,
-                                           const FusedParams& f, int tensor,
-                                           uint32_t epoch, int lane) {
-  uint32_t ok = 1;
-  if (lane == 0) {
-    uint32_t spins = 0, ns = 32;
-    while (ld_acquire(&f.ready[tensor]) != epoch) {
-      // give up after ~0.5 s, or at once if another warp of this launch
-      // already gave up (counters[4] holds the epoch of an aborted launch)
-      if (++spins > kSpinLimit ||
-          *reinterpret_cast<volatile uint32_t*>(&p.counters[4]) == epoch) {
-        ok = 0;
-        atomicOr(p.status, kStatusWaitTimeout);
-        atomicExch(&p.counters[4], epoch);
-        break;
-      }
-      __nanosleep(ns);
-      if (ns < 256) ns <<= 1;
-    }
-  }
-  if (!__shfl_sync(0xffffffffu, ok, 0)) return false;
   __syncwarp();
-  (void)ld_acquire(&f.ready[tensor]);               // per-lane acquire
-  return true;
 }
 
 // ---------------------------------------------------------------------------
-// The warp worker.  Per warp:
-//   * a data ring of kStages shared-memory stages; the item in a stage had
-//     its operands prefetched with cp.async kStages items earlier;
-//   * a control pipeline one item deep per step: the draw atomic, the item
-//     descriptor load and (pass 2) a relaxed load of the tensor's ready flag
-//     are each issued one item before their results are used;
-//   * a deferred publish: a pass-1 item's ticket is taken one item later (its
-//     stores are long complete, so the release costs little), and the
-//     ticket's answer is looked at one item after that.
-// Before any wait the warp flushes its deferred publishes, so it never waits
-// for work it holds itself.
+// The kernel
 // ---------------------------------------------------------------------------
-struct PubState {
-  uint32_t tensor, index;   // pass-1 chunk whose sums are held (publish)
-  float sw, su;             // its sums, valid in lane 0
-  uint32_t chk_tensor, chk_index;   // chunk whose ticket awaits its check
-  uint32_t ticket;          // that ticket's answer (lane 0)
-  bool pub, chk;            // a publish is pending / a check is pending
-};
-
-__device__ __forceinline__ uint2 invalid_desc() {
-  return make_uint2(0xffffffffu, 0u);
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused_check(const StepParams& p,
-                                            const FusedParams& f,
-                                            PubState& ps, uint32_t epoch,
-                                            int lane) {
-  if (!ps.chk) return;
-  const FusedTensor ft = f.ftensors[ps.chk_tensor];
-  const int gl = (int)ps.chk_index / kGroup;
-  const int gsize = min(kGroup, ft.n_chunks - gl * kGroup);
-  const uint32_t last =
-      __shfl_sync(0xffffffffu, ps.ticket + 1u == (uint32_t)gsize, 0);
-  ps.chk = false;
-  if (last) fused_group_combine<kLars>(p, f, ft, (int)ps.chk_tensor, gl,
-                                       gsize, epoch, lane);
-}
-
-__device__ __forceinline__ void fused_publish_now(const FusedParams& f,
-                                                  PubState& ps, int lane) {
-  if (!ps.pub) return;
-  if (lane == 0) {
-    const FusedTensor ft = f.ftensors[ps.tensor];
-    f.fslots[ft.first_chunk + ps.index] = make_float2(ps.sw, ps.su);
-    // release: this warp's stores of the chunk's m, v and the slot
-    ps.ticket = atom_add_acq_rel(
-        &f.gtickets[ft.first_group + (int)ps.index / kGroup], 1u);
-  }
-  ps.chk_tensor = ps.tensor;
-  ps.chk_index = ps.index;
-  ps.pub = false;
-  ps.chk = true;
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused_publish_step(const StepParams& p,
-                                                   const FusedParams& f,
-                                                   PubState& ps,
-                                                   uint32_t epoch, int lane) {
-  fused_check<kLars>(p, f, ps, epoch, lane);
-  fused_publish_now(f, ps, lane);
-}
-
-template <bool kLars>
-__device__ __forceinline__ void fused_flush(const StepParams& p,
-                                            const FusedParams& f,
-                                            PubState& ps, uint32_t epoch,
-                                            int lane) {
-  fused_publish_step<kLars>(p, f, ps, epoch, lane);
-  fused_check<kLars>(p, f, ps, epoch, lane);
-}
-
 template <bool kLars, typename GT, bool kCopy>
 __global__ void __launch_bounds__(kFusedThreads, 1)
     fused_step_kernel(const StepParams p, const FusedParams f) {
   extern __shared__ __align__(128) char fused_smem[];
+  constexpr int kStages = n_stages<kLars, GT>();
+  __shared__ __align__(8) uint64_t s_full[kStages], s_empty[kStages];
+  __shared__ __align__(8) uint64_t s_pfull[kPubSlots], s_pempty[kPubSlots];
+  __shared__ StageDesc s_desc[kStages];
+  __shared__ PubEntry s_pub[kPubSlots];
+  __shared__ uint32_t s_uses[kStages];   // phases armed on each full barrier
+  __shared__ float s_red[kRedRing][2][kConsumerWarps];
+  __shared__ uint32_t s_redcnt[kRedRing];
+  __shared__ uint32_t s_stopped;
   __shared__ LambConsts s_k;
-  __shared__ float s_lr;
+  __shared__ float s_lr, s_c1, s_c2;
   __shared__ int s_skip;
   __shared__ uint32_t s_epoch;
   __shared__ int64_t s_t;
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  __shared__ float s_c2;
+
+  // ---- per-launch constants (c2 beside c1, in another warp) -------------
   const bool bc = !kLars && (p.flags & kFlagBiasCorrection) != 0;
-  if (threadIdx.x == 32) {  // Alg. 2 bias correction of v, beside c1
+  if (threadIdx.x == 32) {
     const int64_t t = p.d_step ? *p.d_step : int64_t(1);
     s_c2 = (bc && t >= 1) ? (float)(1.0 / (1.0 - pow_from_log2(
                                 p.log2_beta2, (double)t)))
                           : 1.f;
   }
-  float c1 = 1.f;
-  int64_t t = 1;
-  int skip = 0;
   if (threadIdx.x == 0) {
-    t = p.d_step ? *p.d_step : int64_t(1);
-    skip = (bc && t < 1) ? 1 : 0;
-    if (bc && !skip)
-      c1 = (float)(1.0 / (1.0 - pow_from_log2(p.log2_beta1, (double)t)));
+    const int64_t t = p.d_step ? *p.d_step : int64_t(1);
+    const int skip = (bc && t < 1) ? 1 : 0;
+    s_t = t;
+    s_skip = skip;
+    s_c1 = (bc && !skip)
+               ? (float)(1.0 / (1.0 - pow_from_log2(p.log2_beta1, (double)t)))
+               : 1.f;
+    s_lr = step_lr(p, t);
+    s_epoch = *reinterpret_cast<volatile uint32_t*>(&p.counters[3]);
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_empty[i], kConsumerWarps);
+      s_uses[i] = 0u;
+    }
+    for (int i = 0; i < kPubSlots; ++i) {
+      mbar_init(&s_pfull[i], 1);
+      mbar_init(&s_pempty[i], 1);
+    }
+    for (int i = 0; i < kRedRing; ++i) s_redcnt[i] = 0u;
+    s_stopped = 0u;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
   if (threadIdx.x == 0) {
-    const float c2 = s_c2;
-    s_k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps};
-    s_lr = step_lr(p, t);
-    s_skip = skip;
-    s_t = t;
-    s_epoch = *reinterpret_cast<volatile uint32_t*>(&p.counters[3]);
+    const float c1 = s_c1, c2 = s_c2;
+    s_k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, c1, c2, p.eps,
+                     0.f, 0.f, 0.f, 0.f};
     if (blockIdx.x == 0) {
       StepScalars sc{};
-      sc.t = t;
+      sc.t = s_t;
       sc.c1 = c1;
       sc.c2 = c2;
       sc.lr = s_lr;
-      sc.skip = skip;
+      sc.skip = s_skip;
       *p.scal = sc;
-      if (skip) atomicOr(p.status, kStatusBadStep);
+      if (s_skip) atomicOr(p.status, kStatusBadStep);
     }
   }
   __syncthreads();
   if (s_skip) return;
   const LambConsts k = s_k;
-  const float lr = s_lr;
   const uint32_t epoch = s_epoch;
-  const uint64_t pol_first = policy_evict_first();
-  const uint64_t pol_last = policy_evict_last();
-  const uint32_t n_items = (uint32_t)f.n_items;
+  const uint32_t* abort_word = &p.counters[4];
   constexpr int kSB = stage_bytes<kLars, GT>();
-  char* ring = fused_smem + warp * kStages * kSB;
 
-  // ---- control pipeline --------------------------------------------------
-  // Each warp draws indices until it gets one >= n_items, then stops, so it
-  // draws exactly one such index.
-  uint32_t last_drawn = 0;
-  bool drawing = true;
-  auto draw = [&]() -> uint32_t {
-    if (!drawing) return n_items;
-    uint32_t v = 0;
-    if (lane == 0) v = atomicAdd(&p.counters[2], 1u);
-    v = __shfl_sync(0xffffffffu, v, 0);
-    if (v >= n_items) {
-      drawing = false;
-      last_drawn = v;
-    }
-    return v;
-  };
-  auto load_desc = [&](uint32_t i) -> uint2 {
-    return i < n_items ? __ldg(&f.items[i]) : invalid_desc();
-  };
-  auto ready_load = [&](uint2 d) -> uint32_t {
-    if (d.x == 0xffffffffu || (d.x & 1u) == 0u) return 0u;
-    return ld_relaxed(&f.ready[d.x >> 1]);
-  };
-  uint32_t idx_a = draw();
-  uint2 desc_b = load_desc(idx_a);
-  idx_a = draw();
-  uint2 desc_c = desc_b;
-  uint32_t rdy_c = ready_load(desc_c);
-  desc_b = load_desc(idx_a);
-  idx_a = draw();
-  uint32_t synced = 0xffffffffu;   // tensor whose norms this warp acquired
-
-  uint2 sd[kStages];
-  bool staged[kStages];
-  // fill stage s with desc_c, then advance the control pipeline
-  auto fill_advance = [&](int s) {
-    sd[s] = desc_c;
-    staged[s] = false;
-    if (desc_c.x != 0xffffffffu) {
-      const bool p2 = (desc_c.x & 1u) != 0u;
-      const uint32_t tensor = desc_c.x >> 1;
-      const FusedTensor ft = f.ftensors[tensor];
-      const TensorPtrs tp = p.ptrs[tensor];
-      const int64_t off = (int64_t)desc_c.y * kFusedChunk;
-      bool go = tp.vec_ok && ft.numel - off >= kFusedChunk;
-      if (go && p2) {
-        go = __shfl_sync(0xffffffffu, rdy_c == epoch, 0) != 0;
-        if (go && tensor != synced) {
-          fence_acq_rel();           // acquire: the relaxed load saw the release
-          synced = tensor;
+  if (warp == kProducerWarp) {
+    // ======================= producer =====================================
+    if (lane == 0) {
+      const uint32_t n_items = (uint32_t)f.n_items;
+      const uint64_t pol_first = policy_evict_first();
+      const uint64_t pol_last = policy_evict_last();
+      const float lr = s_lr;
+      // Items are drawn in batches of kDrawBatch consecutive schedule items
+      // (one atomic per batch).  Software pipeline, per batch n: the draw of
+      // batch n+3 and the records of batch n+2 are issued, and the tensor
+      // descriptor of batch n+1's first item; each is used one batch later,
+      // so the producer never waits for an atomic or a load it just issued.
+      auto draw = [&]() -> uint32_t {
+        return atomicAdd(&p.counters[2], (uint32_t)kDrawBatch);
+      };
+      // the device item list is padded to a multiple of kDrawBatch
+      auto load_recs = [&](uint32_t b, uint4& ra, uint4& rb) {
+        if (b < n_items) {
+          const uint4* p4 = reinterpret_cast<const uint4*>(f.items + b);
+          ra = p4[0];
+          rb = p4[1];
         }
-      }
-      if (go) {
-        fused_prefetch_ops<kLars, GT>(tp, off, p2, ft.resident != 0u,
-                                      ring + s * kSB, pol_first, pol_last,
-                                      lane);
-        staged[s] = true;
-      }
-    }
-    cp_async_commit();
-    desc_c = desc_b;
-    rdy_c = ready_load(desc_c);
-    desc_b = load_desc(idx_a);
-    idx_a = draw();
-  };
-#pragma unroll
-  for (int s = 0; s < kStages; ++s) fill_advance(s);
-
-  // pass-2 item of this warp whose tensor was not final when its turn came
-  uint2 parked = invalid_desc();
-  // run a pass-2 item from global memory once its tensor is known final
-  auto run_direct_p2 = [&](uint2 d) {
-    const uint32_t tensor = d.x >> 1;
-    if (tensor != synced) {
-      fence_acq_rel();                 // acquire: the relaxed load saw it
-      synced = tensor;
-    }
-    const FusedTensor ft = f.ftensors[tensor];
-    const TensorPtrs tp = p.ptrs[tensor];
-    const int64_t off = (int64_t)d.y * kFusedChunk;
-    const int64_t rem = ft.numel - off;
-    const int len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
-    const float s2 = __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]));
-    fused2_direct<kLars, kCopy>(tp, off, len, s2, ft.decay * p.wd, k,
-                                pol_first, lane);
-  };
-  // the same after a bounded wait (callers flush their publishes first)
-  auto wait_direct_p2 = [&](uint2 d) {
-    const uint32_t tensor = d.x >> 1;
-    if (fused_wait(p, f, (int)tensor, epoch, lane)) {
-      synced = tensor;
-      run_direct_p2(d);
-    }
-  };
-
-  PubState ps;
-  ps.pub = ps.chk = false;
-  ps.tensor = ps.index = ps.chk_tensor = ps.chk_index = 0u;
-  ps.sw = ps.su = 0.f;
-  ps.ticket = 0u;
-
-  bool done = false;
-  while (!done) {
-#pragma unroll
-    for (int s = 0; s < kStages; ++s) {
-      const uint2 d = sd[s];
-      if (d.x == 0xffffffffu) {
-        done = true;
-        break;
-      }
-      char* stage = ring + s * kSB;
-      cp_async_wait<kStages - 1>();   // this stage's copies have landed
-      __syncwarp();
-      const bool p2 = (d.x & 1u) != 0u;
-      const uint32_t tensor = d.x >> 1;
-      const FusedTensor ft = f.ftensors[tensor];
-      const TensorPtrs tp = p.ptrs[tensor];
-      const int64_t off = (int64_t)d.y * kFusedChunk;
-      const int64_t rem = ft.numel - off;
-      const int len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
-      const float lam = ft.decay * p.wd;
-      if (!p2) {
-        const uint64_t pol_keep = ft.resident ? pol_last : pol_first;
-        float sw = 0.f, su = 0.f;
-        if (staged[s]) {
-          float4 mo[kPktsPerLane], vo[kPktsPerLane];
-          fused1_from_stage<kLars, GT>(stage, lam, k, mo, vo, sw, su, lane);
-          __syncwarp();               // every lane is done with the stage
-          fill_advance(s);
-          fused_publish_step<kLars>(p, f, ps, epoch, lane);
-          fused1_store<kLars>(tp, off, mo, vo, pol_keep, lane);
-        } else {
-          __syncwarp();
-          fill_advance(s);
-          fused_publish_step<kLars>(p, f, ps, epoch, lane);
-          fused1_direct<kLars, GT>(tp, off, len, lam, k, sw, su, pol_first,
-                                   pol_keep, lane);
-        }
-        ps.sw = warp_sum(sw);
-        ps.su = warp_sum(su);
-        ps.tensor = tensor;
-        ps.index = d.y;
-        ps.pub = true;
-      } else {
-        const float s_upd =
-            staged[s] ? __double2float_rn((double)lr * __ldcg(&p.ratio[tensor]))
-                      : 0.f;
-        if (staged[s]) {
-          float4 wo[kPktsPerLane];
-          fused2_from_stage<kLars>(stage, s_upd, lam, k, wo, lane);
-          __syncwarp();
-          fill_advance(s);
-          fused_publish_step<kLars>(p, f, ps, epoch, lane);
-          fused2_store<kCopy>(tp, off, wo, pol_first, lane);
-        } else {
-          __syncwarp();
-          fill_advance(s);
-          fused_publish_step<kLars>(p, f, ps, epoch, lane);
-          // every lane loads the flag itself (one broadcast access) before
-          // its acquire fence; lane 0's value makes the decision uniform
-          const uint32_t r = __shfl_sync(0xffffffffu,
-                                         ld_relaxed(&f.ready[tensor]), 0);
-          if (r == epoch) {               // became final since the fill
-            run_direct_p2(d);
-          } else {
-            // Not final yet: park it instead of waiting, so this warp keeps
-            // working (and publishing) its later pass-1 items.  With the
-            // parking slot taken, finish the parked item first.
-            if (parked.x != 0xffffffffu) {
-              fused_flush<kLars>(p, f, ps, epoch, lane);
-              wait_direct_p2(parked);
-            }
-            parked = d;
+      };
+      uint32_t b0 = draw();
+      uint4 a0 = make_uint4(0u, 0u, 0u, 0u), c0 = a0;
+      load_recs(b0, a0, c0);
+      uint32_t b1 = draw();
+      uint4 a1 = make_uint4(0u, 0u, 0u, 0u), c1 = a1;
+      load_recs(b1, a1, c1);
+      uint32_t b2 = draw();
+      int kcur = -1, knext = -1;
+      FusedTensor tcur{}, tnext{};
+      TensorPtrs qcur{}, qnext{};
+      int ready_k = -1;          // tensor whose final norms were acquired
+      float ready_s = 0.f;
+      bool aborted = false, done = false;
+      uint32_t it = 0;
+      while (!done) {
+        // ---- issue the loads used by the next batches ---------------------
+        uint4 a2 = make_uint4(0u, 0u, 0u, 0u), c2 = a2;
+        load_recs(b2, a2, c2);
+        // (b2 was drawn a batch ago; past the end, stop drawing)
+        const uint32_t b3 = b2 < n_items ? draw() : n_items;
+        knext = -1;
+        if (b1 < n_items) {
+          const int kn = (int)(a1.x >> 1);
+          if (kn != kcur) {
+            tnext = f.ftensors[kn];
+            qnext = p.ptrs[kn];
+            knext = kn;
           }
         }
+        // ---- the items of batch b0 ---------------------------------------
+#pragma unroll 1
+        for (int j = 0; j < kDrawBatch; ++j, ++it) {
+          const int s = (int)(it % kStages);
+          const uint32_t use = it / kStages;
+          if (!wait_phase(&s_empty[s], (use & 1u) ^ 1u, p.status, p.counters,
+                          epoch)) {
+            aborted = done = true;
+            break;
+          }
+          s_uses[s] = use + 1u;
+          StageDesc d{};
+          if (b0 + j >= n_items) {
+            d.flags = kItemEnd;
+            s_desc[s] = d;
+            mbar_arrive(&s_full[s]);
+            done = true;
+            break;
+          }
+          const uint4& rr = j < 2 ? a0 : c0;
+          const uint2 r = (j & 1) ? make_uint2(rr.z, rr.w)
+                                  : make_uint2(rr.x, rr.y);
+          const int kt = (int)(r.x >> 1);
+          if (kt != kcur) {
+            if (kt == knext) {
+              tcur = tnext;
+              qcur = qnext;
+            } else {
+              tcur = f.ftensors[kt];
+              qcur = p.ptrs[kt];
+            }
+            kcur = kt;
+          }
+          const bool p2 = (r.x & 1u) != 0;
+          const int64_t off = (int64_t)r.y * kFusedChunk;
+          const int64_t rem = tcur.numel - off;
+          d.tp = qcur;
+          d.tensor = kt;
+          d.index = (int)r.y;
+          d.len = (int)(rem < kFusedChunk ? rem : kFusedChunk);
+          d.lam = tcur.decay * p.wd;
+          d.first_chunk = tcur.first_chunk;
+          d.n_chunks = tcur.n_chunks;
+          const bool resident = tcur.resident != 0;
+          d.flags = (p2 ? kItemP2 : 0u) | (resident ? kItemResident : 0u);
+          // bulk copies need 16-byte aligned addresses and sizes
+          const uintptr_t amask =
+              (uintptr_t)qcur.w | (uintptr_t)qcur.m | (uintptr_t)qcur.g |
+              (kLars ? (uintptr_t)0 : (uintptr_t)qcur.v);
+          const bool direct = (amask & 15u) != 0 || (d.len & 7) != 0;
+          if (direct) d.flags |= kItemDirect;
+          if (p2) {
+            if (kt != ready_k) {
+              bool ok = false;
+              for (uint32_t i = 0; i < kSpinLimit; ++i) {
+                if (ld_acquire(&f.ready[kt]) == epoch) {
+                  ok = true;
+                  break;
+                }
+                if ((i & 255) == 255 && ld_relaxed(abort_word) == epoch) break;
+                __nanosleep(i >= 4096 ? 256 : 32);
+              }
+              if (!ok) {
+                if (ld_relaxed(abort_word) != epoch)
+                  give_up(p.status, p.counters, epoch);
+                d.flags |= kItemSkip;
+                aborted = done = true;
+              } else {
+                fence_proxy_async_global();
+                ready_k = kt;
+                ready_s =
+                    __double2float_rn((double)lr * __ldcg(&p.ratio[kt]));
+              }
+            }
+            d.s = ready_s;
+          }
+          s_desc[s] = d;
+          if (direct || (d.flags & kItemSkip)) {
+            mbar_arrive(&s_full[s]);
+          } else {
+            char* st = fused_smem + s * kSB;
+            const uint32_t nb = (uint32_t)d.len * 4u;
+            const uint32_t gb = p2 ? 0u : (uint32_t)(d.len * (int)sizeof(GT));
+            mbar_arrive_tx(&s_full[s], nb * (kLars ? 2u : 3u) + gb);
+            const uint64_t pol = (!p2 && resident) ? pol_last : pol_first;
+            bulk_g2s(st + kOffM, qcur.m + off, nb, &s_full[s], pol);
+            if (!kLars)
+              bulk_g2s(st + kOffV, qcur.v + off, nb, &s_full[s], pol);
+            bulk_g2s(st + off_w<kLars>(), qcur.w + off, nb, &s_full[s], pol);
+            if (!p2)
+              bulk_g2s(st + off_g<kLars>(),
+                       static_cast<const GT*>(qcur.g) + off, gb, &s_full[s],
+                       pol_first);
+          }
+          if (aborted) break;
+        }
+        b0 = b1;
+        a0 = a1;
+        c0 = c1;
+        b1 = b2;
+        a1 = a2;
+        c1 = c2;
+        b2 = b3;
       }
-      // a parked item whose tensor has become final in the meantime
-      if (parked.x != 0xffffffffu) {
-        const uint32_t r = __shfl_sync(
-            0xffffffffu, ld_relaxed(&f.ready[parked.x >> 1]), 0);
-        if (r == epoch) {
-          run_direct_p2(parked);
-          parked = invalid_desc();
+      // The producer that finishes drawing last closes the launch
+      // (counters[5] counts finished producers): the work counter returns to
+      // 0 and the epoch advances -- the other CTAs cached the epoch and t, so
+      // they are unaffected -- and t advances only if the launch completed.
+      __threadfence();
+      if (atomicAdd(&p.counters[5], 1u) + 1u == gridDim.x) {
+        __threadfence();
+        atomicExch(&p.counters[2], 0u);
+        atomicExch(&p.counters[5], 0u);
+        const uint32_t ne = epoch + 1u == 0u ? 1u : epoch + 1u;
+        atomicExch(&p.counters[3], ne);
+        if (ld_relaxed(abort_word) != epoch) {
+          StepScalars sc{};
+          sc.t = s_t;
+          sc.lr = lr;
+          close_step(p, sc);
+        }
+      }
+    }
+  } else if (warp == kPublisherWarp) {
+    // ======================= publisher ====================================
+    // Lane 0 waits for the next entry; then every entry already pushed
+    // behind it (up to kPubSlots) is taken at once, lane j handling the j-th,
+    // so the ticket atomics of several chunks are in flight together.
+    bool live = true;
+    for (uint32_t q = 0; live;) {
+      int ok = 1;
+      if (lane == 0)
+        ok = wait_phase(&s_pfull[q % kPubSlots], (q / kPubSlots) & 1u,
+                        p.status, p.counters, epoch) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      const uint32_t qj = q + (uint32_t)lane;
+      const int slot = (int)(qj % kPubSlots);
+      const bool full = lane == 0 ||
+                        (lane < kPubSlots &&
+                         mbar_test(&s_pfull[slot], (qj / kPubSlots) & 1u));
+      // entries are taken in order: stop at the first one not yet pushed
+      const uint32_t not_full = __ballot_sync(0xffffffffu, !full);
+      const int cnt = __ffs(not_full) - 1;           // lanes 0 .. cnt-1
+      PubEntry e{};
+      if (lane < cnt) e = s_pub[slot];
+      const uint32_t ends = __ballot_sync(0xffffffffu, lane < cnt && e.tensor < 0);
+      const int take = ends ? __ffs(ends) - 1 : cnt; // entries before the end
+      if (ends) live = false;
+      uint32_t last = 0;
+      if (lane < take) {
+        f.fslots[e.first_chunk + e.index] = make_float2(e.sw, e.su);
+        const uint32_t prev = atom_add_acq_rel(&f.tickets[e.tensor], 1u);
+        last = (prev + 1u == (uint32_t)e.n_chunks) ? 1u : 0u;
+      }
+      if (lane < cnt) mbar_arrive(&s_pempty[slot]);
+      uint32_t lasts = __ballot_sync(0xffffffffu, last != 0u);
+      while (lasts) {                                // tensors completed here
+        const int j = __ffs(lasts) - 1;
+        lasts &= lasts - 1u;
+        const int kt = __shfl_sync(0xffffffffu, e.tensor, j);
+        const int fc = __shfl_sync(0xffffffffu, e.first_chunk, j);
+        const int nc = __shfl_sync(0xffffffffu, e.n_chunks, j);
+        finalize_fused<kLars>(p, f, kt, fc, nc, epoch, lane);
+      }
+      q += (uint32_t)cnt;
+    }
+  } else {
+    // ======================= consumers ====================================
+    // The consumer warps walk the stage ring independently (no barrier among
+    // them).  For a pass-1 item each warp leaves its partial sums in s_red;
+    // the last warp to finish the item (shared-memory counter) adds the 16
+    // partials in warp order and hands them to the publisher, so sums are
+    // pushed in item order.  A warp can run at most kStages items ahead of
+    // the slowest, hence the 2 x kStages rings.
+    const int tid = threadIdx.x;                     // 0 .. kConsumers-1
+    const uint64_t pol_first = policy_evict_first();
+    const uint64_t pol_last = policy_evict_last();
+    uint32_t q = 0;                                  // pass-1 items seen
+    for (uint32_t it = 0;; ++it) {
+      const int s = (int)(it % kStages);
+      const uint32_t use = it / kStages;
+      int ok = 1;
+      if (lane == 0)
+        ok = wait_phase(&s_full[s], use & 1u, p.status, p.counters, epoch) ? 1
+                                                                           : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      __syncwarp();                                  // lane 0 acquired it
+      const StageDesc d = s_desc[s];
+      if (d.flags & kItemEnd) break;
+      if (!(d.flags & kItemSkip)) {
+        const TensorPtrs& tp = d.tp;
+        const int64_t off = (int64_t)d.index * kFusedChunk;
+        const char* st = fused_smem + s * kSB;
+        if (!(d.flags & kItemP2)) {
+          float sw = 0.f, su = 0.f;
+          const uint64_t pol_keep =
+              (d.flags & kItemResident) ? pol_last : pol_first;
+          if (d.flags & kItemDirect)
+            c_pass1_direct<kLars, GT>(tp, off, d.len, d.lam, k, sw, su, tid);
+          else
+            c_pass1_staged<kLars, GT>(st, tp, off, d.len, d.lam, k, pol_keep,
+                                      sw, su, tid);
+          sw = warp_sum(sw);
+          su = warp_sum(su);
+          const int r = (int)(q % kRedRing);
+          if (lane == 0) {
+            s_red[r][0][warp] = sw;
+            s_red[r][1][warp] = su;
+            __threadfence_block();
+            const uint32_t c = atomicAdd(&s_redcnt[r], 1u);
+            if (c + 1u == (uint32_t)kConsumerWarps) {  // last warp of item
+              __threadfence_block();
+              float tw = 0.f, tu = 0.f;
+#pragma unroll
+              for (int i = 0; i < kConsumerWarps; ++i) {
+                tw += s_red[r][0][i];
+                tu += s_red[r][1][i];
+              }
+              s_redcnt[r] = 0u;
+              const int ps = (int)(q % kPubSlots);
+              const uint32_t pph = ((q / kPubSlots) & 1u) ^ 1u;
+              if (wait_phase(&s_pempty[ps], pph, p.status, p.counters,
+                             epoch)) {
+                s_pub[ps] = PubEntry{d.tensor, d.first_chunk, d.index,
+                                     d.n_chunks, tw, tu};
+                mbar_arrive(&s_pfull[ps]);
+              }
+            }
+          }
+          ++q;
+        } else if (d.flags & kItemDirect) {
+          c_pass2_direct<kLars, kCopy>(tp, off, d.len, d.s, d.lam, k, tid);
+        } else {
+          c_pass2_staged<kLars, kCopy>(st, tp, off, d.len, d.s, d.lam, k,
+                                       pol_first, tid);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_empty[s]);
+    }
+    // the last consumer warp to stop ends the sums stream (every push of a
+    // pass-1 item precedes its pusher's stop)
+    if (lane == 0) {
+      __threadfence_block();
+      if (atomicAdd(&s_stopped, 1u) + 1u == (uint32_t)kConsumerWarps) {
+        const int ps = (int)(q % kPubSlots);
+        const uint32_t pph = ((q / kPubSlots) & 1u) ^ 1u;
+        if (wait_phase(&s_pempty[ps], pph, p.status, p.counters, epoch)) {
+          s_pub[ps] = PubEntry{-1, 0, 0, 0, 0.f, 0.f};
+          mbar_arrive(&s_pfull[ps]);
         }
       }
     }
   }
-  fused_flush<kLars>(p, f, ps, epoch, lane);
-  if (parked.x != 0xffffffffu) wait_direct_p2(parked);
-  cp_async_wait<0>();
-  // The warp that drew the last index >= n_items closes the launch.
-  const uint32_t warps = gridDim.x * kFusedWarps;
-  if (lane == 0 && last_drawn == n_items + warps - 1u) {
-    atomicExch(&p.counters[2], 0u);
-    const uint32_t ne = epoch + 1u == 0u ? 1u : epoch + 1u;
-    atomicExch(&p.counters[3], ne);
-    StepScalars sc{};
-    sc.t = s_t;
-    sc.lr = s_lr;
-    close_step(p, sc);
+
+  // ---- no bulk copy may still be writing this CTA's shared memory --------
+  // (after a give-up only: in a completed launch the consumers have taken
+  // every armed phase).  Each armed phase was arrived on by the producer, so
+  // only the bytes of its copies can be outstanding.
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStages; ++i) {
+      const uint32_t u = s_uses[i];
+      if (u == 0u) continue;               // stage never used
+      for (uint32_t n = 0; n < kSpinLimit; ++n) {
+        if (mbar_test(&s_full[i], (u - 1u) & 1u)) break;
+        __nanosleep(64);
+      }
+    }
   }
 }
-
-}  // namespace
 
 template <bool kLars, typename GT, bool kCopy>
 int launch_fused_t(const StepParams& p, const FusedParams& f, int grid,
@@ -828,7 +822,7 @@ int launch_fused_t(const StepParams& p, const FusedParams& f, int grid,
 
 template <bool kLars, typename GT, bool kCopy>
 int occupancy_fused_t(int* blocks) {
-  // opt in to the dynamic shared memory of the stage rings (a property of
+  // opt in to the dynamic shared memory of the stage ring (a property of
   // the function, set once; not a device setting)
   cudaError_t e = cudaFuncSetAttribute(
       fused_step_kernel<kLars, GT, kCopy>,
@@ -839,6 +833,8 @@ int occupancy_fused_t(int* blocks) {
       blocks, fused_step_kernel<kLars, GT, kCopy>, kFusedThreads,
       fused_smem_bytes<kLars, GT>());
 }
+
+}  // namespace
 
 int launch_fused(const StepParams& p, const FusedParams& f, int lars,
                  int grad_bf16, int copy_bf16, int grid, void* stream) {

@@ -88,7 +88,8 @@ struct StepParams {
   uint32_t* tickets;
   uint32_t* counters;     // [0] pass-1, [1] pass-2, [2] fused work counter,
                           // [3] launch epoch of the fused kernel (>= 1),
-                          // [4] epoch of a fused launch whose wait gave up
+                          // [4] epoch of a fused launch whose wait gave up,
+                          // [5] fused producers done drawing this launch
   double* ratio;
   double* wnorm;
   double* unorm;
@@ -127,17 +128,20 @@ struct StepParams {
 };
 
 // ---------------------------------------------------------------------------
-// Single-touch (fused) step: one persistent kernel whose warps draw items --
-// the pass-1 or pass-2 work on one "fused chunk" of kFusedChunk elements --
-// from a host-built schedule in which the pass-2 items of a tensor follow its
-// pass-1 items by a lag of about one wave, so the m, v, w the pass 1 just
-// touched are still in L2 when the pass 2 reads them.
+// Single-touch (fused) step: one persistent kernel (one CTA per SM) that
+// takes work items -- the pass-1 or pass-2 work on one "fused chunk" of
+// kFusedChunk elements -- from a host-built schedule in which the pass-2
+// items of a tensor follow its pass-1 items by a lag of about the items the
+// grid holds in flight, so the m, v, w the pass 1 just touched are still in
+// L2 when the pass 2 reads them.
 // ---------------------------------------------------------------------------
-constexpr int kFusedChunk = 512;      // elements per fused chunk (one warp item)
-constexpr int kGroup = 32;            // fused chunks per first-level combine
-// default schedule lag per CTA of the fused grid: 8 warps x 3 prefetch
-// stages hold 24 items in flight; 1.5x that keeps pass-2 waits rare
-constexpr int kFusedLagPerCta = 36;
+constexpr int kFusedChunk = 4096;     // elements per fused chunk (a CTA item)
+// items a CTA draws at once (one atomic); the device item list is padded to
+// a multiple of it
+constexpr int kDrawBatch = 4;
+// default schedule lag per CTA of the fused grid: a CTA holds up to ~20
+// items (8 stages, 3 batches drawn ahead, 1 in the consumers)
+constexpr int kFusedLagPerCta = 12;
 
 struct __align__(8) FusedChunk {
   int32_t tensor;   // tensor index k
@@ -146,23 +150,19 @@ struct __align__(8) FusedChunk {
 
 struct __align__(16) FusedTensor {
   int64_t numel;
-  int32_t first_chunk;   // in the fused chunk table
+  int32_t first_chunk;   // in the fused chunk table (slot base)
   int32_t n_chunks;
-  int32_t first_group;   // in the group tables
-  int32_t n_groups;
   float decay;           // 1.0f: weight decay applies
   uint32_t resident;     // 1: keep pass-1 data in L2 (evict_last) for pass 2
+  uint32_t pad[2];
 };
 
 struct FusedParams {
   const uint2* items;          // x = (tensor << 1) | is_pass2, y = index of
                                // the fused chunk inside the tensor
-  const FusedChunk* fchunks;
   const FusedTensor* ftensors;
   float2* fslots;              // per fused chunk (sum w^2, sum u^2), fp32
-  double2* gslots;             // per group, fp64
-  uint32_t* gtickets;          // per group: chunks of the group finished
-  uint32_t* tickets;           // per tensor: groups finished
+  uint32_t* tickets;           // per tensor: chunks whose sums are stored
   uint32_t* ready;             // per tensor: epoch of the launch that
                                // finished its norms
   int32_t n_items;
@@ -198,8 +198,7 @@ int plan_fused(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
                int64_t bytes_per_param, int64_t l2_budget, int64_t lag,
                std::vector<FusedChunk>* fchunks,
                std::vector<FusedTensor>* ftensors,
-               std::vector<uint32_t>* items, int64_t* n_groups, char* err,
-               int errlen);
+               std::vector<uint32_t>* items, char* err, int errlen);
 
 // Host planner (planner.cpp).  Returns 0 on success, else writes a message.
 int plan_chunks(const int64_t* sizes, int32_t n, int32_t chunk_elems,

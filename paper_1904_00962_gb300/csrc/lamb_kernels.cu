@@ -44,8 +44,15 @@
 namespace lamb {
 namespace {
 
-constexpr int kUnroll1 = 4;   // 4-element packets in flight per thread, pass 1
-constexpr int kUnroll2 = 4;   // same for pass 2
+// 4-element packets in flight per thread and array.  Pass 1 keeps 2 so that
+// its LAMB kernels fit 80 registers and run 3 CTAs per SM like pass 2: a
+// CTA's chunk epilogue (block reduction, slot, ticket, next descriptors)
+// then leaves two other CTAs streaming on the SM.  Measured on BERT-large:
+// 2 CTAs/SM x 4 packets 1072 us, 3 x 2 1066 us per pass 1 (16,384-element
+// chunks; 1131 vs 1080 us at 8,192).
+constexpr int kUnroll1 = 2;
+constexpr int kUnroll2 = 4;   // pass 2: 80 registers, 3 CTAs per SM
+constexpr int kMinBlocks1 = 3;
 
 // Sums of the first N of x[] over the CTA, valid in thread 0 (fixed trees:
 // lanes, then warps).  Contains one barrier; red must hold N rows.
@@ -347,7 +354,7 @@ __device__ __forceinline__ void pass1_constants(const StepParams& p,
 }
 
 template <typename GT, int kNest, bool kGn>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, kMinBlocks1)
     lamb_pass1_kernel(const StepParams p) {
   __shared__ float red[4][kWarps];
   __shared__ uint32_t s_next[2];

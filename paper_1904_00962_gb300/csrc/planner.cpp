@@ -83,8 +83,8 @@ int plan_chunks(const int64_t* sizes, int32_t n, int32_t chunk_elems,
 // ---------------------------------------------------------------------------
 // Schedule of the single-touch step.
 //
-// Every tensor k of d_k elements becomes ceil(d_k / kFusedChunk) fused chunks
-// and ceil(chunks / kGroup) groups.  Work items are emitted in this order:
+// Every tensor k of d_k elements becomes ceil(d_k / kFusedChunk) fused
+// chunks.  Work items are emitted in this order:
 // the pass-1 items of tensor 0, 1, 2, ... in turn; the pass-2 items of a
 // tensor whose state fits the L2 budget ("resident") are emitted as one block
 // once `lag` further pass-1 items have been emitted after its last pass-1
@@ -100,10 +100,9 @@ int plan_fused(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
                int64_t bytes_per_param, int64_t l2_budget, int64_t lag,
                std::vector<FusedChunk>* fchunks,
                std::vector<FusedTensor>* ftensors,
-               std::vector<uint32_t>* items, int64_t* n_groups, char* err,
-               int errlen) {
+               std::vector<uint32_t>* items, char* err, int errlen) {
   ftensors->assign((size_t)n, FusedTensor{});
-  int64_t nf = 0, ng = 0;
+  int64_t nf = 0;
   for (int32_t k = 0; k < n; ++k) {
     const int64_t d = sizes[k];
     const int64_t nk = (d + kFusedChunk - 1) / kFusedChunk;
@@ -111,12 +110,9 @@ int plan_fused(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
     t.numel = d;
     t.first_chunk = (int32_t)nf;
     t.n_chunks = (int32_t)nk;
-    t.first_group = (int32_t)ng;
-    t.n_groups = (int32_t)((nk + kGroup - 1) / kGroup);
     t.decay = (decay_mask == nullptr || decay_mask[k]) ? 1.0f : 0.0f;
     t.resident = (d <= l2_budget / bytes_per_param) ? 1u : 0u;
     nf += nk;
-    ng += t.n_groups;
     if (nf > (int64_t(1) << 30)) {
       snprintf(err, errlen, "more than 2^30 fused chunks");
       return 1;
@@ -155,7 +151,6 @@ int plan_fused(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
   }
   while (head < pending.size()) emit_pass2(pending[head++].second);
   for (int32_t k : tail) emit_pass2(k);
-  *n_groups = ng;
   return 0;
 }
 

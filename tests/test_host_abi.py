@@ -166,7 +166,8 @@ def test_planner_capacity_too_small(lib):
 
 def _check_schedule(sizes, budget, lag):
     items, res = B.lamb_layout_schedule(sizes, budget, lag)
-    nk = [(s + 511) // 512 for s in sizes]
+    c = B.LAMB_FUSED_CHUNK_ELEMS
+    nk = [(s + c - 1) // c for s in sizes]
     first = np.concatenate([[0], np.cumsum(nk)[:-1]]).astype(np.int64)
     owner = np.repeat(np.arange(len(sizes)), nk)
     chunk = (items >> 1).astype(np.int64)

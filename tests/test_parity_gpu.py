@@ -732,7 +732,7 @@ def test_single_touch_edge_layout(grad_dtype, copy_dtype, misalign, budget_mb,
 
 @pytest.mark.parametrize("lars", [False, True])
 def test_single_touch_bitwise_deterministic_across_schedules(lars):
-    """Chunking is fixed (1024 elements, groups of 32), so neither the grid,
+    """Chunking is fixed (fused chunks of LAMB_FUSED_CHUNK_ELEMS), so neither the grid,
     the lag nor the L2 budget may change a single bit of the results."""
     L = W.resnet50_layout()
     h = L.lars_hyper if lars else L.hyper
