@@ -48,6 +48,23 @@ def test_library_exports_every_declared_symbol(lib):
         assert exported == _declared()
 
 
+def test_binding_constants_match_header_defines():
+    # every #define LAMB_* value the binding mirrors must agree with the ABI
+    hdr = open(os.path.join(ROOT, "include", "lamb.h")).read()
+    defs = dict(re.findall(r"#define\s+(LAMB_[A-Z0-9_]+)\s+(0x[0-9a-fA-F]+|\d+)u?\b",
+                           hdr))
+    checked = 0
+    for name, val in defs.items():
+        if hasattr(B, name):
+            assert getattr(B, name) == int(val, 0), name
+            checked += 1
+    assert checked >= 12
+    for flag in ("LAMB_FLAG_GRAD_NORM", "LAMB_FLAG_SKIP_NONFINITE",
+                 "LAMB_FLAG_DECOUPLED_DECAY", "LAMB_FUSED_CHUNK_ELEMS",
+                 "LAMB_STATUS_SKIPPED"):
+        assert flag in defs and hasattr(B, flag), flag
+
+
 def test_abi_version(lib):
     assert B.lamb_abi_version() == 1
 
