@@ -155,11 +155,17 @@ def load_peaks():
 
 
 def kernel_source_hash():
+    """sha256 (16 hex digits) of the two-pass kernels' code with comments and
+    whitespace removed, so that editing a comment does not invalidate the
+    committed ncu traffic figures while any change of code does."""
     h = hashlib.sha256()
     for name in ("lamb_kernels.cu", "lamb_device.cuh", "lamb_internal.h"):
         with open(os.path.join(ROOT, "paper_1904_00962_gb300", "csrc",
-                               name), "rb") as f:
-            h.update(f.read())
+                               name)) as f:
+            src = f.read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", " ", src)
+        h.update(" ".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 

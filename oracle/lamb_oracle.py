@@ -58,8 +58,8 @@ Q12 N-LAMB / NN-LAMB (appendix): the superscripted beta_1^t is the t-th term
 Q17 Gradient norms and the non-finite guard (not in the paper; the
     training-system checks that accompany a large-batch step): ||g_k|| per
     block, the global ||g|| = sqrt(sum_k ||g_k||^2) (the norm of the whole
-    gradient viewed as one vector), and a verdict "non-finite" when any
-    element of any g_k is Inf or NaN.  A guarded step with that verdict is
+    gradient viewed as one vector), and a decision "non-finite" when any
+    element of any g_k is Inf or NaN.  A guarded step with that decision is
     not applied: x, m, v and t keep their values.
 Q18 Decoupled weight decay (an ablation of Q4 the paper does not define;
     the AdamW-style decoupling applied to LAMB): the normalised direction is

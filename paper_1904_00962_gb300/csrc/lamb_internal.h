@@ -13,7 +13,7 @@
 //   float2     grad_slots[n_chunks] 8 B  per-chunk (sum g^2, sum 0*g), pass 1
 //                                       with the gradient check
 //   double     gsq/gnorm[n_tensors]     per-tensor sum g^2 and ||g_k||
-//   GradCheck                           global ||g|| and the step's verdict
+//   GradCheck                           global ||g|| and the step's decision
 #pragma once
 #include <stdint.h>
 
@@ -71,7 +71,7 @@ enum : uint32_t { kFlagBiasCorrection = 1u, kFlagIncrementStep = 2u,
                   kFlagSkipNonfinite = 16u, kFlagDecoupledDecay = 32u };
 
 // Gradient check of one step (kFlagGradNorm / kFlagSkipNonfinite).  Pass 1
-// forms it; pass 2 reads the verdict before it writes anything.
+// forms it; pass 2 reads the decision before it writes anything.
 struct __align__(16) GradCheck {
   double norm;          // sqrt(sum over all tensors of sum g^2)
   uint32_t nonfinite;   // 1: some element of g was Inf or NaN

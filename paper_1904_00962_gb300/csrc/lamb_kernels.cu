@@ -21,8 +21,8 @@
 //   gradient check  pass 1 also sums g^2 per chunk and 0*g (0, or NaN once
 //                   any element is Inf/NaN); the tensors' finalisers form
 //                   ||g_k||, and the last one the global ||g|| and the
-//                   step's verdict.
-//   skip mode       pass 1 leaves m, v untouched; pass 2 reads the verdict
+//                   step's decision.
+//   skip mode       pass 1 leaves m, v untouched; pass 2 reads the decision
 //                   first and either writes nothing or forms the moments
 //                   from g itself and writes m, v, w (42 instead of 40 bytes
 //                   per parameter with bf16 g).
@@ -74,7 +74,7 @@ __device__ __forceinline__ void cta_sum(float* x, float (*red)[kWarps]) {
 
 // The tensor that finishes last in pass 1 (gradient check only): the global
 // ||g|| as a fixed-order fp64 sum over the tensors' sum g^2, and the step's
-// verdict, which pass 2 reads before it writes anything.  Warp-wide.
+// decision, which pass 2 reads before it writes anything.  Warp-wide.
 __device__ __forceinline__ void finalize_grad(const StepParams& p) {
   __threadfence();
   const int lane = threadIdx.x & 31;

@@ -1,6 +1,6 @@
 """GPU parity of the optional step variants against the fp64 oracle:
 
-* the gradient check (per-tensor and global ||g||, Inf/NaN verdict) fused
+* the gradient check (per-tensor and global ||g||, Inf/NaN decision) fused
   into pass 1 (oracle reading Q17);
 * the skip-on-non-finite mode, in which a step whose gradients hold an Inf
   or NaN writes nothing, and a finite step is bit-identical to the plain one;
