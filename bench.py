@@ -119,6 +119,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--algo", choices=list(ALGO_CODES), default="auto",
                     help="step algorithm of the plan (auto = library default)")
+    ap.add_argument("--chunk-elems", type=int, default=0,
+                    help="two-pass chunk size (0 = library default)")
     ap.add_argument("--lag-items", type=int, default=0,
                     help="single-touch schedule lag (0 = library default)")
     ap.add_argument("--l2-budget-mb", type=int, default=0,
@@ -411,6 +413,7 @@ def run_ours(args):
         st.upload("w", k, L.weights(k))
         st.upload("g", k, L.grad(k, 1))
     plan = LambPlan(st, L.decay, algorithm=ALGO_CODES[args.algo],
+                    chunk_elems=args.chunk_elems,
                     lag_items=args.lag_items, l2_budget_mb=args.l2_budget_mb)
     algo = plan.info()["algorithm"]
     kernel_names, kernel_bytes = kernel_model(
