@@ -112,6 +112,8 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--e2e-streams", type=int, default=1,
+                    help="copy streams the e2e gradient upload is split over")
     ap.add_argument("--e2e-steps", type=int, default=None,
                     help="steps of the end-to-end loop (default: min(K, 50))")
     ap.add_argument("--cpu-seconds", type=float, default=10.0,
@@ -435,14 +437,14 @@ def run_ours(args):
                          skip_nonfinite=args.variant == "skip_nonfinite",
                          decoupled_decay=args.variant == "decoupled")
 
-    def one_step():
+    def one_step(pl=plan):
         if opt == "lamb":
-            plan.lamb_step(hyper, d_step, d_lr)
+            pl.lamb_step(hyper, d_step, d_lr)
         elif opt == "lars":
-            plan.lars_step(hyper, d_step, d_lr)
+            pl.lars_step(hyper, d_step, d_lr)
         else:
-            plan.nlamb_step(hyper, 0.004, opt == "nnlamb", d_step, d_lr,
-                            d_prod)
+            pl.nlamb_step(hyper, 0.004, opt == "nnlamb", d_step, d_lr,
+                          d_prod)
 
     stream = torch.cuda.current_stream(dev)
 
@@ -486,29 +488,72 @@ def run_ours(args):
     status = plan.query(clear=True)
 
     # ---- end to end: pinned host gradients in, trust ratios out ----------
+    # Every step uploads its gradients from pinned host memory and the host
+    # reads its trust ratios back.  Two gradient buffers, each with a plan
+    # over the same w, m, v (and copy), let the upload of step s+1's
+    # gradients (copy streams) run while step s computes, as in a training
+    # loop whose backward pass fills one buffer while the optimizer consumes
+    # the other; an upload into a buffer waits for the step that last read
+    # it.  The host takes step s-1's trust ratios while step s runs.
     k_e2e = args.e2e_steps if args.e2e_steps is not None else min(args.steps, 50)
     g_host = torch.empty(st.total, dtype=st.g.dtype).pin_memory()
     g_host.copy_(st.g.cpu())
-    ratio_host = torch.empty(L.n_tensors, dtype=torch.float64).pin_memory()
+    ratio_host = torch.empty(2, L.n_tensors, dtype=torch.float64).pin_memory()
     h2d = L.n_params * st.g.element_size()
     d2h = L.n_tensors * 8
+    g_dev = [st.g, torch.empty_like(st.g)]
+    plan2 = LambPlan(st, L.decay, algorithm=ALGO_CODES[args.algo],
+                     chunk_elems=args.chunk_elems, lag_items=args.lag_items,
+                     l2_budget_mb=args.l2_budget_mb)
+    es = st.g.element_size()
+    B.lamb_plan_bind(plan2.handle, st.ptrs("w"),
+                     [g_dev[1].data_ptr() + es * o for o in st.offsets],
+                     st.ptrs("m"), st.ptrs("v"), st.ptrs("copy"))
+    plans = [plan, plan2]
+    n_up = max(1, args.e2e_streams)
+    up_streams = [torch.cuda.Stream(dev) for _ in range(n_up)]
+    bounds = [st.total * j // n_up for j in range(n_up + 1)]
+    copied = [[torch.cuda.Event() for _ in range(n_up)] for _ in range(2)]
+    consumed = [torch.cuda.Event(), torch.cuda.Event()]
+    done = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def upload(i):
+        for j, us in enumerate(up_streams):
+            us.wait_event(consumed[i])
+            with torch.cuda.stream(us):
+                a, b = bounds[j], bounds[j + 1]
+                g_dev[i][a:b].copy_(g_host[a:b], non_blocking=True)
+            copied[i][j].record(us)
+
     barrier()
     e2 = torch.cuda.Event(enable_timing=True)
     e3 = torch.cuda.Event(enable_timing=True)
-    done = torch.cuda.Event()
     e2.record(stream)
-    for _ in range(k_e2e):
-        st.g.copy_(g_host, non_blocking=True)
-        one_step()
-        B.lamb_plan_copy_trust_ratios(plan.handle, ratio_host.data_ptr(),
+    for us in up_streams:
+        us.wait_event(e2)
+    upload(0)
+    for s_ in range(k_e2e):
+        i = s_ % 2
+        if s_ + 1 < k_e2e:
+            upload(1 - i)
+        for ev in copied[i]:
+            stream.wait_event(ev)
+        one_step(plans[i])
+        consumed[i].record(stream)
+        B.lamb_plan_copy_trust_ratios(plans[i].handle,
+                                      ratio_host[i].data_ptr(),
                                       stream=stream.cuda_stream)
-        done.record(stream)
-        done.synchronize()
+        done[i].record(stream)
+        if s_ >= 1:
+            done[1 - i].synchronize()
+            assert math.isfinite(float(ratio_host[1 - i][0]))
     e3.record(stream)
     barrier()
     ms_e2e = e2.elapsed_time(e3)
     ms_e2e = max_over_ranks(ms_e2e, dev)
-    assert math.isfinite(float(ratio_host[0]))
+    assert math.isfinite(float(ratio_host[(k_e2e - 1) % 2][0]))
+    plan2.destroy()
+    del g_dev[1]
     clk = clocks.stop() if clocks else None
 
     if rank != 0:
@@ -582,7 +627,9 @@ def run_ours(args):
                      if peak_src == "measured" else "fallback 6800 GB/s"},
         "e2e": {"value": P * world * k_e2e / (ms_e2e * 1e-3), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "steps": k_e2e},
+                "steps": k_e2e, "upload_streams": n_up,
+                "overlap": "upload of step s+1 overlaps step s "
+                           "(two gradient buffers)"},
         "gpu_launches": len(kernel_names) * args.steps,
         "device_status": status,
         "clocks": clk,
