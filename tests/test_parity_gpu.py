@@ -614,6 +614,69 @@ def test_increment_step_matches_oracle_chain(algo):
     G.close()
 
 
+
+@algos
+def test_two_plans_alternating_gradient_buffers(algo):
+    """Double-buffered gradients, the pattern of a training loop that
+    uploads (or computes) step t+1's gradients while step t runs: two plans
+    over the same w, m, v and bf16 copy, each bound to its own gradient
+    buffer, take turns on one stream with one device step counter
+    (INCREMENT_STEP).  Every step must equal, bit for bit, one plan stepping
+    through the same gradients in a single buffer."""
+    L = W.bert_layout(2, 256, 1024, name="bert_small", grad_dtype="bf16",
+                      copy_dtype="bf16")
+    h = L.hyper
+    hyp = c_hyper(h, increment=True)
+    dev = torch.device("cuda:0")
+    gen = torch.Generator(device=dev)
+
+    def grads(t, total):
+        gen.manual_seed(1000 + t)
+        return (torch.randn(total, device=dev, generator=gen) *
+                1e-3).to(torch.bfloat16)
+
+    def fresh():
+        G = GpuLayout(L, algorithm=algo)
+        G.load_weights()
+        G.d_step.fill_(1)
+        G.d_lr.fill_(f32(h.lr))
+        return G
+
+    n_steps = 6
+    # one plan, one buffer
+    A = fresh()
+    ref = []
+    for t in range(1, n_steps + 1):
+        A.st.g.copy_(grads(t, A.st.total))
+        A.plan.lamb_step(hyp, A.d_step, A.d_lr)
+        r, _, _ = A.plan.results()
+        ref.append(r.clone())
+    torch.cuda.synchronize()
+    # two plans, two buffers, alternating
+    Bl = fresh()
+    st = Bl.st
+    g2 = torch.empty_like(st.g)
+    plan2 = LambPlan(st, L.decay, algorithm=algo)
+    es = st.g.element_size()
+    B.lamb_plan_bind(plan2.handle, st.ptrs("w"),
+                     [g2.data_ptr() + es * o for o in st.offsets],
+                     st.ptrs("m"), st.ptrs("v"), st.ptrs("copy"))
+    bufs, plans = [st.g, g2], [Bl.plan, plan2]
+    for t in range(1, n_steps + 1):
+        i = (t - 1) % 2
+        bufs[i].copy_(grads(t, st.total))
+        plans[i].lamb_step(hyp, Bl.d_step, Bl.d_lr)
+        r, _, _ = plans[i].results()
+        assert torch.equal(r, ref[t - 1]), t
+    torch.cuda.synchronize()
+    assert int(Bl.d_step.item()) == n_steps + 1 == int(A.d_step.item())
+    assert plan2.query() == 0 and Bl.plan.query() == 0
+    for name in ("w", "m", "v", "copy"):
+        assert torch.equal(getattr(st, name), getattr(A.st, name)), name
+    plan2.destroy()
+    A.close()
+    Bl.close()
+
 def test_argument_errors_on_device_plans():
     L = W.mlp_layout()
     st = DeviceState(L.sizes, with_v=False)
