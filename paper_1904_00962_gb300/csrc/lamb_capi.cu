@@ -192,15 +192,15 @@ lamb_status_t lamb_layout_schedule(const int64_t* sizes, int32_t n_tensors,
   if ((int64_t)it.size() > capacity)
     return capacity == 0 ? LAMB_OK
                          : fail(LAMB_ERR_INVALID_ARG, "capacity too small");
-  std::memcpy(items, it.data(), it.size() * sizeof(uint32_t));
+  if (!it.empty()) std::memcpy(items, it.data(), it.size() * sizeof(uint32_t));
   return LAMB_OK;
 }
 
-lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
-                               const uint8_t* decay_mask, int32_t grad_dtype,
-                               int32_t copy_dtype, int32_t device,
-                               const lamb_plan_options_t* opts,
-                               lamb_plan_t* out) {
+static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
+                                 const uint8_t* decay_mask, int32_t grad_dtype,
+                                 int32_t copy_dtype, int32_t device,
+                                 const lamb_plan_options_t* opts,
+                                 lamb_plan_t* out) {
   if (out == nullptr) return fail(LAMB_ERR_INVALID_ARG, "out is NULL");
   *out = nullptr;
   if (grad_dtype != LAMB_F32 && grad_dtype != LAMB_BF16)
@@ -229,6 +229,21 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
 
   lamb_plan* p = new (std::nothrow) lamb_plan();
   if (!p) return fail(LAMB_ERR_OOM, "host allocation failed");
+  // Frees the plan (and its device arena, on its own device) on every path
+  // that does not hand it to the caller, a thrown host allocation included.
+  struct Owner {
+    lamb_plan* p;
+    ~Owner() {
+      if (!p) return;
+      if (p->arena) {
+        int cur = -1;
+        const bool got = cudaGetDevice(&cur) == cudaSuccess;
+        if (cudaSetDevice(p->device) == cudaSuccess) cudaFree(p->arena);
+        if (got) cudaSetDevice(cur);
+      }
+      delete p;
+    }
+  } owner{p};
   p->device = device;
   p->n_tensors = n_tensors;
   p->chunk_elems = chunk;
@@ -241,7 +256,6 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   char err[256] = "";
   int64_t nch = 0;
   if (n_tensors < 1 || sizes == nullptr) {
-    delete p;
     return fail(LAMB_ERR_INVALID_ARG, n_tensors < 1
                                           ? "n_tensors must be >= 1"
                                           : "sizes is NULL");
@@ -249,13 +263,11 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   p->h_tensors.resize((size_t)n_tensors);
   if (plan_chunks(sizes, n_tensors, chunk, nullptr, 0, &nch,
                   p->h_tensors.data(), decay_mask, err, sizeof(err))) {
-    delete p;
     return fail(LAMB_ERR_INVALID_ARG, "%s", err);
   }
   std::vector<ChunkDesc> h_chunks((size_t)nch);
   if (plan_chunks(sizes, n_tensors, chunk, h_chunks.data(), nch, &nch,
                   p->h_tensors.data(), decay_mask, err, sizeof(err))) {
-    delete p;
     return fail(LAMB_ERR_INVALID_ARG, "%s", err);
   }
   p->n_chunks = nch;
@@ -267,13 +279,11 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   // ---- device ------------------------------------------------------------
   DeviceGuard guard(device);
   if (guard.err != cudaSuccess) {
-    delete p;
     return cuda_fail(guard.err, "cudaSetDevice");
   }
   cudaError_t e = cudaDeviceGetAttribute(&p->num_sms,
                                          cudaDevAttrMultiProcessorCount, device);
   if (e != cudaSuccess) {
-    delete p;
     return cuda_fail(e, "cudaDeviceGetAttribute");
   }
   int occ[4] = {0, 0, 0, 0};
@@ -282,7 +292,6 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   if (!rc) rc = occupancy_lars_pass1(p->grad_bf16, &occ[2]);
   if (!rc) rc = occupancy_lars_pass2(p->copy_bf16, &occ[3]);
   if (rc) {
-    delete p;
     return cuda_fail((cudaError_t)rc, "occupancy query");
   }
   for (int i = 0; i < 4; ++i) {
@@ -302,7 +311,6 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
     rc = occupancy_fused(0, p->grad_bf16, p->copy_bf16, &focc[0]);
     if (!rc) rc = occupancy_fused(1, p->grad_bf16, p->copy_bf16, &focc[1]);
     if (rc) {
-      delete p;
       return cuda_fail((cudaError_t)rc, "occupancy query");
     }
     for (int i = 0; i < 2; ++i) {
@@ -313,7 +321,6 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
     int l2 = 0;
     e = cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, device);
     if (e != cudaSuccess) {
-      delete p;
       return cuda_fail(e, "cudaDeviceGetAttribute(L2)");
     }
     p->l2_budget = budget_mb ? budget_mb << 20 : (int64_t)l2 / 2;
@@ -325,7 +332,6 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
     if (plan_fused(sizes, n_tensors, decay_mask, 12, p->l2_budget, p->lag,
                    &h_fchunks, &h_ftensors, &h_items, err,
                    sizeof(err))) {
-      delete p;
       return fail(LAMB_ERR_INVALID_ARG, "%s", err);
     }
     p->n_items = (int64_t)h_items.size();
@@ -366,7 +372,6 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
   p->arena_bytes = off;
   e = cudaMalloc(&p->arena, p->arena_bytes);
   if (e != cudaSuccess) {
-    delete p;
     return cuda_fail(e, "cudaMalloc(plan)");
   }
   char* base = static_cast<char*>(p->arena);
@@ -418,19 +423,31 @@ lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
     e = cudaMemcpy(p->counters + 3, &one, sizeof(one), cudaMemcpyHostToDevice);
   }
   if (e == cudaSuccess) {
-    // trust ratio 1 for every tensor until a step computes it (0-element
-    // tensors keep it: Q6 zero-norm rule)
+    // trust ratio 1 for every tensor until a step computes it; a 0-element
+    // tensor keeps it (its norms are 0, and a zero norm gives ratio 1)
     std::vector<double> ones(n, 1.0);
     e = cudaMemcpy(p->ratio, ones.data(), n * sizeof(double),
                    cudaMemcpyHostToDevice);
   }
   if (e != cudaSuccess) {
-    cudaFree(p->arena);
-    delete p;
     return cuda_fail(e, "plan upload");
   }
+  owner.p = nullptr;
   *out = p;
   return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_create(const int64_t* sizes, int32_t n_tensors,
+                               const uint8_t* decay_mask, int32_t grad_dtype,
+                               int32_t copy_dtype, int32_t device,
+                               const lamb_plan_options_t* opts,
+                               lamb_plan_t* out) {
+  try {
+    return plan_create(sizes, n_tensors, decay_mask, grad_dtype, copy_dtype,
+                       device, opts, out);
+  } catch (const std::bad_alloc&) {
+    return fail(LAMB_ERR_OOM, "host allocation failed");
+  }
 }
 
 lamb_status_t lamb_plan_bind(lamb_plan_t plan, void* const* w,
@@ -444,7 +461,12 @@ lamb_status_t lamb_plan_bind(lamb_plan_t plan, void* const* w,
     return fail(LAMB_ERR_INVALID_ARG,
                 "plan writes a bf16 copy: w_copy pointer array is required");
   const int n = plan->n_tensors;
-  std::vector<TensorPtrs> h((size_t)n);
+  std::vector<TensorPtrs> h;
+  try {
+    h.resize((size_t)n);
+  } catch (const std::bad_alloc&) {
+    return fail(LAMB_ERR_OOM, "host allocation failed");
+  }
   int n_vec = 0;
   const uintptr_t ga = plan->grad_bf16 ? 8 : 16;
   for (int k = 0; k < n; ++k) {
@@ -792,14 +814,23 @@ lamb_status_t lamb_plan_get_info(lamb_plan_t plan, lamb_plan_info_t* info) {
 
 lamb_status_t lamb_plan_set_timing(lamb_plan_t plan, int32_t enable) {
   if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
-  if (enable && plan->events.empty()) {
+  const size_t n_events = (size_t)kMaxTimedSteps * (kKernelsPerStep + 1);
+  if (enable && plan->events.size() < n_events) {
     DeviceGuard guard(plan->device);
     if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
-    plan->events.resize((size_t)kMaxTimedSteps * (kKernelsPerStep + 1));
-    plan->timed_kernels.assign((size_t)kMaxTimedSteps, 0);
-    for (auto& ev : plan->events) {
+    try {
+      plan->timed_kernels.assign((size_t)kMaxTimedSteps, 0);
+      plan->events.reserve(n_events);
+    } catch (const std::bad_alloc&) {
+      return fail(LAMB_ERR_OOM, "host allocation failed");
+    }
+    // only created events are kept (destroy releases exactly those); a
+    // failed call leaves timing off and the next one carries on
+    while (plan->events.size() < n_events) {
+      cudaEvent_t ev;
       cudaError_t e = cudaEventCreate(&ev);
       if (e != cudaSuccess) return cuda_fail(e, "cudaEventCreate");
+      plan->events.push_back(ev);
     }
   }
   plan->timing = enable != 0;
