@@ -66,7 +66,7 @@ typedef enum {
   LAMB_ERR_INVALID_ARG = 1,        /* bad size, count, pointer or value   */
   LAMB_ERR_UNSUPPORTED_DTYPE = 2,  /* dtype code not supported here       */
   LAMB_ERR_CUDA = 3,               /* a CUDA runtime call or launch failed */
-  LAMB_ERR_OOM = 4,                /* device allocation failed            */
+  LAMB_ERR_OOM = 4,                /* device or host allocation failed    */
   LAMB_ERR_NOT_BOUND = 5           /* step before lamb_plan_bind, or the
                                       array the step needs was not bound  */
 } lamb_status_t;
@@ -181,8 +181,8 @@ typedef struct {
                             this many MiB keep them in L2 between the
                             passes; 0 = half the device's L2               */
   int32_t lag_items;     /* single-touch: work items between a tensor's last
-                            pass-1 item and its pass-2 block; 0 = about the
-                            items the grid holds in flight (8 per CTA)     */
+                            pass-1 item and its pass-2 block; 0 = 12 per
+                            CTA of the grid, about what it holds in flight */
 } lamb_plan_options_t;
 
 typedef struct {
