@@ -504,6 +504,72 @@ def test_pins_reject_planted_mistake(kind):
     assert caught, f"planted mistake {kind!r} passed every pin"
 
 
+
+def _lars_mutant(kind):
+    """Algorithm 1 with one plausible error planted."""
+    def lars(w, g, m, *, lr, beta1=0.9, weight_decay=0.0, decay=True,
+             trust_coef=1.0, phi_kind="identity", gamma_l=0.0,
+             gamma_u=math.inf, g_dtype="f32"):
+        x = O.to_f64(w); gt = O.to_f64(g, g_dtype); m0 = O.to_f64(m)
+        lam = weight_decay if (decay or kind == "decay_ignores_mask") else 0.0
+        if kind == "no_m_damping":
+            m_t = beta1 * m0 + gt + lam * x
+        elif kind == "decay_outside_momentum":
+            m_t = beta1 * m0 + (1 - beta1) * gt
+        else:
+            m_t = beta1 * m0 + (1 - beta1) * (gt + lam * x)
+        u = m_t + lam * x if kind == "decay_outside_momentum" else m_t
+        xn, un = O.block_norm(x), O.block_norm(u)
+        if kind == "norm_of_g":
+            un = O.block_norm(gt)
+        kappa = 1.0 if kind == "no_trust_coef" else trust_coef
+        if xn == 0 or un == 0:
+            ratio = 0.0 if kind == "zero_rule_zero" else 1.0
+        elif kind == "norms_swapped":
+            ratio = kappa * O.phi(un, phi_kind, gamma_l, gamma_u) / xn
+        else:
+            ratio = kappa * O.phi(xn, phi_kind, gamma_l, gamma_u) / un
+        sign = 1.0 if kind == "update_sign" else -1.0
+        return O.LarsResult(x + sign * lr * ratio * u, m_t, ratio, xn, un)
+    return lars
+
+
+@pytest.mark.parametrize("kind", ["decay_ignores_mask", "no_m_damping",
+                                  "decay_outside_momentum", "norm_of_g",
+                                  "no_trust_coef", "zero_rule_zero",
+                                  "norms_swapped", "update_sign"])
+def test_pins_reject_planted_lars_mistake(kind):
+    mutant = _lars_mutant(kind)
+    caught = False
+    for case in _load_cases():
+        if case["algorithm"] != "lars":
+            continue
+        if not _case_matches(case, _run_case(case, lars_fn=mutant)):
+            caught = True
+    # library pin: torch SGD momentum with dampening beta1 and L2 decay, and
+    # the step-norm closed form with the trust coefficient
+    rng = np.random.default_rng(98)
+    w, g, m, _ = _rand_block(rng, 96)
+    for wd in (0.0, 0.05):
+        p = torch.tensor(w, dtype=torch.float64, requires_grad=True)
+        opt = torch.optim.SGD([p], lr=1.0, momentum=0.9, dampening=0.9,
+                              weight_decay=wd)
+        opt.state[p] = {"momentum_buffer": torch.tensor(m, dtype=torch.float64)}
+        p.grad = torch.tensor(g, dtype=torch.float64)
+        opt.step()
+        buf = opt.state[p]["momentum_buffer"].numpy()
+        res = mutant(w, g, m, lr=0.5, beta1=0.9, weight_decay=wd,
+                     trust_coef=1e-3)
+        want = w - 0.5 * 1e-3 * np.linalg.norm(w) / np.linalg.norm(buf) * buf
+        if not (np.allclose(res.m, buf, rtol=1e-13, atol=1e-20)
+                and np.allclose(res.w, want, rtol=1e-12, atol=1e-20)):
+            caught = True
+    res = mutant(w, g, m, lr=0.1, weight_decay=1e-4, trust_coef=1e-3)
+    if not math.isclose(np.linalg.norm(res.w - w), 0.1 * 1e-3 * np.linalg.norm(w),
+                        rel_tol=1e-9):
+        caught = True
+    assert caught, f"planted LARS mistake {kind!r} passed every pin"
+
 def test_unmutated_oracle_passes_pin_harness():
     for case in _load_cases():
         assert _case_matches(case, _run_case(case)), case["name"]
