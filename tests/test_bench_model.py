@@ -1,0 +1,96 @@
+"""CPU tests of bench.py's measurement model: the algorithmic bytes per
+parameter of every kernel it times, and the rule that ties the committed ncu
+traffic figures to the kernel source they were taken on."""
+import os
+import shutil
+import sys
+
+import pytest
+
+from conftest import ROOT
+
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+# (optimizer, g bytes, copy bytes, variant) -> per-kernel bytes per parameter.
+# Two-pass LAMB: pass 1 reads g, m, v, w and writes m, v; pass 2 reads m, v, w
+# and writes w and the copy.  LARS has no v.  N-LAMB's pass 2 also reads g
+# (the Nesterov term).  The skip mode moves the m, v writes to pass 2, which
+# then re-reads g.
+CASES = [
+    ("lamb", 2, 2, "plain", [22, 18], 40, 28),     # BERT-large
+    ("lamb", 4, 0, "plain", [24, 16], 40, 28),     # fp32 LAMB
+    ("lars", 4, 0, "plain", [16, 12], 28, 20),     # fp32 LARS
+    ("lamb", 2, 2, "skip_nonfinite", [14, 28], 40, 28),
+    ("lars", 4, 0, "skip_nonfinite", [12, 20], 28, 20),
+    ("nlamb", 2, 2, "plain", [22, 20], 42, 28),
+    ("nnlamb", 4, 0, "plain", [24, 20], 44, 28),
+    ("lamb", 2, 2, "grad_norm", [22, 18], 40, 28),
+    ("lamb", 2, 2, "decoupled", [22, 18], 40, 28),
+]
+
+
+@pytest.mark.parametrize("opt,gb,cb,variant,per_kernel,two_pass,single",
+                         CASES)
+def test_kernel_byte_model(opt, gb, cb, variant, per_kernel, two_pass,
+                           single):
+    names, got = bench.kernel_model(opt, 1, gb, cb, variant)
+    assert got == per_kernel and len(names) == 2
+    assert bench.two_pass_bytes(opt, gb, cb) == two_pass
+    assert bench.single_touch_bytes(opt, gb, cb) == single
+    if variant in ("plain", "grad_norm", "decoupled"):
+        assert sum(got) == two_pass
+    if variant == "skip_nonfinite":   # one more read of g per step
+        assert sum(got) == two_pass + gb
+
+
+def test_single_touch_model_is_one_kernel():
+    names, got = bench.kernel_model("lamb", 2, 2, 2)
+    assert len(names) == 1 and got == [28]
+    # the flagged variants run on the two-pass kernels of such a plan
+    names, got = bench.kernel_model("lamb", 2, 2, 2, "grad_norm")
+    assert len(names) == 2 and got == [22, 18]
+
+
+def _tree_copy(tmp_path):
+    dst = tmp_path / "paper_1904_00962_gb300" / "csrc"
+    shutil.copytree(os.path.join(ROOT, "paper_1904_00962_gb300", "csrc"), dst,
+                    ignore=shutil.ignore_patterns("*.o", "*.so"))
+    return dst
+
+
+def test_kernel_hash_ignores_comments_not_code(tmp_path, monkeypatch):
+    base = bench.kernel_source_hash()
+    csrc = _tree_copy(tmp_path)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.kernel_source_hash() == base
+    f = csrc / "lamb_kernels.cu"
+    src = f.read_text()
+    f.write_text("// a new comment line\n/* and a block\n comment */\n" +
+                 src.replace("\n", "\n  ", 5))
+    assert bench.kernel_source_hash() == base
+    f.write_text(src.replace("kUnroll2 = 4", "kUnroll2 = 2", 1))
+    assert bench.kernel_source_hash() != base
+
+
+def test_profiled_traffic_only_for_matching_source(tmp_path):
+    good = tmp_path / "good.md"
+    good.write_text(f"kernel_source_sha256: {bench.kernel_source_hash()}\n"
+                    "traffic_bytes_per_launch[0]: 7.1586e9\n"
+                    "traffic_bytes_per_launch[1]: 5.8486e9\n")
+    assert bench.profiled_traffic(str(good), 0) == 7.1586e9
+    assert bench.profiled_traffic(str(good), 1) == 5.8486e9
+    assert bench.profiled_traffic(str(good), 2) is None
+    stale = tmp_path / "stale.md"
+    stale.write_text("kernel_source_sha256: 0123456789abcdef\n"
+                     "traffic_bytes_per_launch[0]: 7.1586e9\n")
+    assert bench.profiled_traffic(str(stale), 0) is None
+    assert bench.profiled_traffic(str(tmp_path / "missing.md"), 0) is None
+
+
+def test_committed_kernel_profile_has_the_parsed_fields():
+    text = open(bench.KERNELS[1][2]).read()
+    assert "kernel_source_sha256:" in text
+    for i in range(2):
+        assert f"traffic_bytes_per_launch[{i}]:" in text
