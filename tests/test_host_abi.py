@@ -275,6 +275,43 @@ def test_create_validates_before_touching_the_device(lib):
     assert ei.value.status == B.LAMB_ERR_INVALID_ARG
 
 
+
+def test_noalloc_validates_before_touching_the_device(lib):
+    """Every rejection of the allocation-free step happens on the host, before
+    any CUDA call: the pointers below are never dereferenced (no case here is
+    valid, so none reaches the device)."""
+    P = 1 << 20                                   # fake, 16-byte aligned
+    hyp = B.make_hyper()                          # bias correction on
+
+    def call(sizes=(8, 8), grad=B.LAMB_F32, copy=B.LAMB_DTYPE_NONE, ptr=P,
+             w_copy=None, hyper=hyp, d_step=P, d_lr=P):
+        n = len(sizes)
+        B.lamb_step_noalloc(list(sizes), None, grad, copy, [ptr] * n,
+                            [ptr] * n, [ptr] * n, [ptr] * n, w_copy, hyper,
+                            d_step, d_lr)
+
+    cases = [
+        (dict(sizes=()), B.LAMB_ERR_INVALID_ARG, "n_tensors"),
+        (dict(sizes=(1,) * 4097), B.LAMB_ERR_INVALID_ARG, "4096"),
+        (dict(sizes=(8, -1)), B.LAMB_ERR_INVALID_ARG, "negative"),
+        (dict(sizes=((1 << 31) + 1,)), B.LAMB_ERR_INVALID_ARG, "chunks"),
+        (dict(grad=7), B.LAMB_ERR_UNSUPPORTED_DTYPE, "grad_dtype"),
+        (dict(copy=B.LAMB_F32), B.LAMB_ERR_UNSUPPORTED_DTYPE, "copy_dtype"),
+        (dict(copy=B.LAMB_BF16), B.LAMB_ERR_INVALID_ARG, "w_copy"),
+        (dict(hyper=B.make_hyper(beta1=1.0)), B.LAMB_ERR_INVALID_ARG, "hyper"),
+        (dict(hyper=B.make_hyper(grad_norm=True)), B.LAMB_ERR_INVALID_ARG,
+         "hyper"),
+        (dict(d_step=0), B.LAMB_ERR_INVALID_ARG, "d_step"),
+        (dict(d_lr=0), B.LAMB_ERR_INVALID_ARG, "d_lr"),
+        (dict(ptr=0), B.LAMB_ERR_INVALID_ARG, "NULL"),
+        (dict(ptr=P + 2), B.LAMB_ERR_INVALID_ARG, "aligned"),
+    ]
+    for kw, status, word in cases:
+        with pytest.raises(B.LambError) as ei:
+            call(**kw)
+        assert ei.value.status == status, kw
+        assert word in B.lamb_last_error(), (kw, B.lamb_last_error())
+
 @pytest.mark.skipif(cuda_available(), reason="checks the no-GPU error path")
 def test_create_without_gpu_reports_cuda_error(lib):
     with pytest.raises(B.LambError) as ei:
