@@ -10,10 +10,12 @@ read as one parameter tensor) at a time, following the paper
 "Large Batch Optimization for Deep Learning: Training BERT in 76 minutes"
 (You et al., ICLR 2020):
 
-* ``lamb_tensor``   -- Algorithm 2 (LAMB), steps in the algorithm's order.
+* ``lamb_tensor``   -- Algorithm 2 (LAMB), steps in the algorithm's order;
+                       ``lamb_direction`` is its element-wise part.
 * ``nlamb_tensor``  -- Algorithms 3 and 4 of the appendix (N-LAMB, NN-LAMB:
                        Nesterov momentum in the first, or both, moments).
-* ``lars_tensor``   -- Algorithm 1 (LARS).
+* ``lars_tensor``   -- Algorithm 1 (LARS); ``lars_momentum`` is its
+                       element-wise part.
 * ``layerwise_step``-- the general strategy of Section 3: a base update u is
                        normalised per block and rescaled by phi(||x||).
 * ``phi``           -- the scaling function of Section 3,
@@ -200,6 +202,38 @@ class LarsResult:
     unorm: float        # ||m_t||
 
 
+def lamb_direction(w, g, m, v, *, t: int, beta1: float = 0.9,
+                   beta2: float = 0.999, eps: float = 1e-6,
+                   weight_decay: float = 0.01, decay: bool = True,
+                   bias_correction: bool = True, g_dtype: str = "f32",
+                   decoupled_decay: bool = False):
+    """The element-wise part of Algorithm 2 for one block (or any slice of
+    one): (m_t, v_t, u) in float64, u = r_t + lam x_t (r_t alone with
+    decoupled decay, reading Q18).
+
+      m_t = beta1 m_{t-1} + (1-beta1) g_t
+      v_t = beta2 v_{t-1} + (1-beta2) g_t^2
+      m_hat = m_t / (1 - beta1^t),  v_hat = v_t / (1 - beta2^t)
+      r_t = m_hat / (sqrt(v_hat) + eps)
+    """
+    if t < 1:
+        raise ValueError("step count t must be >= 1")
+    x = to_f64(w)
+    gt = to_f64(g, g_dtype)
+    m_prev = to_f64(m)
+    v_prev = to_f64(v)
+    lam = weight_decay if decay else 0.0
+    m_t = beta1 * m_prev + (1.0 - beta1) * gt
+    v_t = beta2 * v_prev + (1.0 - beta2) * (gt * gt)
+    if bias_correction:
+        m_hat = m_t / (1.0 - beta1 ** t)
+        v_hat = v_t / (1.0 - beta2 ** t)
+    else:
+        m_hat, v_hat = m_t, v_t
+    r_t = m_hat / (np.sqrt(v_hat) + eps)
+    return m_t, v_t, (r_t if decoupled_decay else r_t + lam * x)
+
+
 def lamb_tensor(w, g, m, v, *, t: int, lr: float, beta1: float = 0.9,
                 beta2: float = 0.999, eps: float = 1e-6,
                 weight_decay: float = 0.01, decay: bool = True,
@@ -218,29 +252,17 @@ def lamb_tensor(w, g, m, v, *, t: int, lr: float, beta1: float = 0.9,
     With decoupled_decay (reading Q18) the last line becomes
       x_{t+1} = x_t - lr * phi(||x_t||) / ||r_t|| * r_t - lr * lam * x_t
     """
-    if t < 1:
-        raise ValueError("step count t must be >= 1")
     x = to_f64(w)
-    gt = to_f64(g, g_dtype)
-    m_prev = to_f64(m)
-    v_prev = to_f64(v)
     lam = weight_decay if decay else 0.0
-
-    m_t = beta1 * m_prev + (1.0 - beta1) * gt
-    v_t = beta2 * v_prev + (1.0 - beta2) * (gt * gt)
-    if bias_correction:
-        m_hat = m_t / (1.0 - beta1 ** t)
-        v_hat = v_t / (1.0 - beta2 ** t)
-    else:
-        m_hat, v_hat = m_t, v_t
-    r_t = m_hat / (np.sqrt(v_hat) + eps)
-    if decoupled_decay:
-        x_new, ratio, xn, un = layerwise_step(
-            x, r_t, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u)
-        return LambResult(x_new - lr * lam * x, m_t, v_t, ratio, xn, un)
-    u = r_t + lam * x
+    m_t, v_t, u = lamb_direction(
+        w, g, m, v, t=t, beta1=beta1, beta2=beta2, eps=eps,
+        weight_decay=weight_decay, decay=decay,
+        bias_correction=bias_correction, g_dtype=g_dtype,
+        decoupled_decay=decoupled_decay)
     x_new, ratio, xn, un = layerwise_step(
         x, u, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u)
+    if decoupled_decay:
+        return LambResult(x_new - lr * lam * x, m_t, v_t, ratio, xn, un)
     return LambResult(x_new, m_t, v_t, ratio, xn, un)
 
 
@@ -255,14 +277,23 @@ def lars_tensor(w, g, m, *, lr: float, beta1: float = 0.9,
       x_{t+1} = x_t - lr * kappa * phi(||x_t||) / ||m_t|| * m_t
     """
     x = to_f64(w)
-    gt = to_f64(g, g_dtype)
-    m_prev = to_f64(m)
-    lam = weight_decay if decay else 0.0
-    m_t = beta1 * m_prev + (1.0 - beta1) * (gt + lam * x)
+    m_t = lars_momentum(w, g, m, beta1=beta1, weight_decay=weight_decay,
+                        decay=decay, g_dtype=g_dtype)
     x_new, ratio, xn, un = layerwise_step(
         x, m_t, lr, phi_kind=phi_kind, gamma_l=gamma_l, gamma_u=gamma_u,
         trust_coef=trust_coef)
     return LarsResult(x_new, m_t, ratio, xn, un)
+
+
+def lars_momentum(w, g, m, *, beta1: float = 0.9, weight_decay: float = 0.0,
+                  decay: bool = True, g_dtype: str = "f32") -> np.ndarray:
+    """The element-wise part of Algorithm 1 for one block (or any slice of
+    one): m_t = beta1 m_{t-1} + (1-beta1) (g_t + lam x_t), float64."""
+    x = to_f64(w)
+    gt = to_f64(g, g_dtype)
+    m_prev = to_f64(m)
+    lam = weight_decay if decay else 0.0
+    return beta1 * m_prev + (1.0 - beta1) * (gt + lam * x)
 
 
 def lr_schedule(t: int, eta0: float, warmup: int, total: int) -> float:
