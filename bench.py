@@ -55,7 +55,7 @@ BYTES_STEP = BYTES_PASS1 + BYTES_PASS2   # 40
 BYTES_SINGLE_TOUCH = 2 + 12 + 12 + 2     # 28
 # per algorithm: kernels of one step, their algorithmic bytes per parameter,
 # and the committed ncu summary holding their measured DRAM traffic
-ALGO_CODES = {"auto": 0, "two_pass": 1, "single_touch": 2}
+ALGO_CODES = {"auto": 0, "two_pass": 1, "single_touch": 2, "on_chip": 3}
 KERNELS = {
     1: (["lamb_pass1_kernel<bf16>", "lamb_pass2_kernel<copy>"],
         [BYTES_PASS1, BYTES_PASS2],
@@ -84,10 +84,21 @@ def single_touch_bytes(opt, gb, cb):
     return gb + 12 + 8 + 4 + cb
 
 
-def kernel_model(opt, algo, gb, cb, variant="plain"):
+def kernel_model(opt, algo, gb, cb, variant="plain", streamed_frac=0.0):
     """(kernel names, algorithmic bytes per parameter of each kernel).
     The skip-on-non-finite variant moves the m, v (LARS: m) writes from
     pass 1 to pass 2, which then reads g as well."""
+    if algo == 3 and variant in ("plain", "decoupled"):
+        # tensors too large for a round go through the two-pass kernels
+        # first; bytes are per parameter of the whole layout
+        f = streamed_frac
+        on = ([f"onchip_step_kernel<{opt},g{8 * gb},copy{8 * cb}>"],
+              [(1 - f) * single_touch_bytes(opt, gb, cb)])
+        if f == 0:
+            return on
+        names, per = kernel_model(opt, 1, gb, cb, variant)
+        return ([n + "(streamed)" for n in names] + on[0],
+                [b * f for b in per] + on[1])
     if algo == 2 and opt in ("lamb", "lars") and variant == "plain":
         return ([f"fused_step_kernel<{opt},g{8 * gb},copy{8 * cb}>"],
                 [single_touch_bytes(opt, gb, cb)])
@@ -417,11 +428,16 @@ def run_ours(args):
     plan = LambPlan(st, L.decay, algorithm=ALGO_CODES[args.algo],
                     chunk_elems=args.chunk_elems,
                     lag_items=args.lag_items, l2_budget_mb=args.l2_budget_mb)
-    algo = plan.info()["algorithm"]
+    info = plan.info()
+    algo = info["algorithm"]
+    streamed = 0
+    if algo == 3:
+        cap = info["grid_blocks"] * info["rows_per_cta"] * info["row_elems"]
+        streamed = sum(s for s in L.sizes if s > cap)
     kernel_names, kernel_bytes = kernel_model(
         opt, algo, 2 if L.grad_dtype == "bf16" else 4,
-        2 if L.copy_dtype == "bf16" else 0, args.variant)
-    profile_file = KERNELS[algo][2] if (
+        2 if L.copy_dtype == "bf16" else 0, args.variant, streamed / P)
+    profile_file = KERNELS[algo][2] if algo in KERNELS and (
         args.layout == "bert_large" and opt == "lamb" and
         args.variant == "plain") else None
     d_step = torch.ones(1, dtype=torch.int64, device=dev)
@@ -480,7 +496,7 @@ def run_ours(args):
     barrier()
     wall1 = _dt.datetime.now()
     ms_total = e0.elapsed_time(e1)
-    n_timed, ms_kernels = B.lamb_plan_read_timing(plan.handle, 2)
+    n_timed, ms_kernels = B.lamb_plan_read_timing(plan.handle, 3)
     B.lamb_plan_set_timing(plan.handle, False)
     if clocks:
         clocks.mark(wall0, wall1)
@@ -571,11 +587,13 @@ def run_ours(args):
     achieved = alg_bytes / (per_launch_ms[dom] * 1e-3) / 1e9
     traffic = profiled_traffic(profile_file, dom) if profile_file else None
     ms_step = ms_total / args.steps
-    step_bytes = sum(kernel_bytes) if len(kernel_bytes) == 2 \
+    step_bytes = sum(kernel_bytes) if algo != 2 \
         else two_pass_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
                             2 if L.copy_dtype == "bf16" else 0)
     single_bytes = single_touch_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
                                       2 if L.copy_dtype == "bf16" else 0)
+    two_bytes = two_pass_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
+                               2 if L.copy_dtype == "bf16" else 0)
     step_gbs = step_bytes * P / (ms_step * 1e-3) / 1e9
 
     cpu = None
@@ -610,13 +628,18 @@ def run_ours(args):
                    "l2": "inputs larger than L2" if P * 16 > 130e6 else
         "state smaller than L2 (no flush; not a bandwidth number)",
                    "parallelism": f"replicas{world}" if world > 1 else "1gpu"},
+        # the step's own algorithmic bytes (what the chosen kernels must move)
+        "alg_bytes_per_param": step_bytes,
         "hbm_gbs_step": step_gbs,
-        "two_pass_bytes_per_param": step_bytes,
-        "frac_of_peak_two_pass_model": step_gbs / peak,
+        "frac_of_peak_alg": step_gbs / peak,
+        # the same time against the two fixed byte models
+        "two_pass_bytes_per_param": two_bytes,
+        "frac_of_peak_two_pass_model": two_bytes * P / (ms_step * 1e-3) /
+        1e9 / peak,
         "single_touch_bytes_per_param": single_bytes,
         "frac_of_peak_single_touch_model": single_bytes * P /
         (ms_step * 1e-3) / 1e9 / peak,
-        "algorithm": "two_pass" if len(kernel_names) == 2 else "single_touch",
+        "algorithm": {1: "two_pass", 2: "single_touch", 3: "on_chip"}[algo],
         "kernels": {kernel_names[i]: {"ms_per_launch": per_launch_ms[i],
                                       "alg_bytes_per_param": kernel_bytes[i]}
                     for i in range(len(kernel_names))},

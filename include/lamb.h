@@ -52,7 +52,7 @@
 extern "C" {
 #endif
 
-#define LAMB_ABI_VERSION 1
+#define LAMB_ABI_VERSION 2
 
 /* Only the entry points below are exported from liblamb.so. */
 #if defined(__GNUC__)
@@ -123,14 +123,17 @@ typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
 #define LAMB_STATUS_BAD_STEP  0x2u      /* *d_step < 1 with bias correction:
                                            the step was skipped, nothing was
                                            written                          */
-#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* single-touch: a wait inside the
-                                           kernel (a pass-2 item for its
-                                           tensor's norms, or a stage of the
-                                           operand pipeline) gave up after
-                                           ~0.5 s and the rest of the launch
-                                           gave up with it, so the step is
+#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* single-touch or on-chip: a wait
+                                           inside the kernel (single-touch: a
+                                           pass-2 item for its tensor's
+                                           norms, or a stage of the operand
+                                           pipeline, ~0.5 s; on-chip: a grid
+                                           barrier, wait_limit_ms) gave up
+                                           and the rest of the launch gave up
+                                           with it, so the step is
                                            incomplete and the plan must be
-                                           destroyed; never expected        */
+                                           destroyed (its later steps do
+                                           nothing); never expected         */
 #define LAMB_STATUS_GRAD_NONFINITE 0x8u /* GRAD_NORM: a gradient element was
                                            Inf or NaN                       */
 #define LAMB_STATUS_SKIPPED   0x10u     /* SKIP_NONFINITE: a step was skipped
@@ -157,7 +160,11 @@ typedef struct {
 } lamb_hyper_t;
 
 /* lamb_plan_options_t.algorithm */
-#define LAMB_ALGO_AUTO 0          /* the library's default (two-pass)        */
+#define LAMB_ALGO_AUTO 0          /* the library's default: on-chip when the
+                                     whole layout fits one on-chip round (one
+                                     launch, one grid barrier; ~4.2M
+                                     parameters on a GB300), else two-pass
+                                     (lamb_plan_get_info reports the choice) */
 #define LAMB_ALGO_TWO_PASS 1      /* two streaming kernels per step: 40 B of
                                      HBM traffic per parameter (bf16 g/copy) */
 #define LAMB_ALGO_SINGLE_TOUCH 2  /* one kernel per step; pass 2 of a tensor
@@ -168,7 +175,25 @@ typedef struct {
                                      LAMB_FUSED_CHUNK_ELEMS elements.  LAMB
                                      and LARS only; N-LAMB and the flagged
                                      variants run two-pass on such a plan  */
+#define LAMB_ALGO_ON_CHIP 3       /* one cooperative kernel per step (one CTA
+                                     per SM).  Consecutive tensors are taken in
+                                     rounds that fit the grid's shared memory
+                                     (rows of LAMB_ONCHIP_ROW_ELEMS elements,
+                                     ~223 rows per SM: ~4.3M parameters on
+                                     152 SMs): pass 1 reads g, m, v, w once and
+                                     keeps w and the direction on chip across
+                                     a grid barrier, pass 2 writes w from
+                                     there -- 28 B/parameter (bf16 g/copy).  A
+                                     tensor larger than a round ("streamed")
+                                     goes through the two-pass kernels first
+                                     (40 B/parameter; 3 launches per step
+                                     then).  LAMB, LARS, N-LAMB, NN-LAMB,
+                                     decoupled decay and the schedule; the
+                                     gradient check and the skip mode run
+                                     two-pass on such a plan               */
 #define LAMB_FUSED_CHUNK_ELEMS 4096
+#define LAMB_ONCHIP_ROW_ELEMS 128
+#define LAMB_TAIL_CHUNK_ELEMS 2048
 
 /* Optional plan-creation knobs (pass NULL for defaults). */
 typedef struct {
@@ -183,6 +208,34 @@ typedef struct {
   int32_t lag_items;     /* single-touch: work items between a tensor's last
                             pass-1 item and its pass-2 block; 0 = 12 per
                             CTA of the grid, about what it holds in flight */
+  int32_t wait_limit_ms; /* on-chip: a grid-barrier wait gives up after this
+                            long (LAMB_STATUS_WAIT_TIMEOUT); 0 = 1000      */
+  int32_t test_unmet_wait; /* on-chip, for tests of the give-up path only:
+                            nonzero makes every grid barrier wait for one
+                            arrival more than the grid makes, so the first
+                            wait runs out after wait_limit_ms and the launch
+                            returns with LAMB_STATUS_WAIT_TIMEOUT.  0 for
+                            every real use                                 */
+  int32_t onchip_max_ctas; /* on-chip: at most this many CTAs (one per SM);
+                            0 = the SM count                               */
+  int32_t onchip_rows;   /* on-chip: rows of shared memory per CTA, at most
+                            what the device holds; 0 = that maximum.  Fewer
+                            rows make smaller rounds                       */
+  int64_t tail_elems;    /* two-pass: elements at each end of the layout
+                            (the tensors laid end to end) cut into chunks
+                            of LAMB_TAIL_CHUNK_ELEMS, so that the last
+                            chunks a pass draws are short; 0 = none (the
+                            default: measured slower on every layout here,
+                            the short chunks' per-chunk cost outweighs the
+                            shorter tail)                                  */
+  int32_t shard_world;   /* data-parallel shards of the step (0 or 1: the
+                            plan covers every chunk).  With shard_world = W
+                            the plan owns chunk range shard_rank of W
+                            (lamb_layout_shard) and is driven by
+                            lamb_shard_pass1 / lamb_shard_pass2; every rank
+                            must build its plan from the same sizes,
+                            chunk_elems and tail_elems                     */
+  int32_t shard_rank;    /* 0 <= shard_rank < shard_world                  */
 } lamb_plan_options_t;
 
 typedef struct {
@@ -204,6 +257,17 @@ typedef struct {
   int64_t n_items;           /* single-touch: work items per step           */
   int64_t lag_items;         /* single-touch: schedule lag                  */
   int64_t l2_budget_bytes;   /* single-touch: residency budget              */
+  int32_t n_rounds;          /* on-chip: rounds per step                    */
+  int32_t n_streamed_tensors;/* on-chip: tensors too large for a round,
+                                updated by the two-pass kernels            */
+  int32_t rows_per_cta;      /* on-chip: rows of shared memory per CTA      */
+  int32_t row_elems;         /* on-chip: elements per row                   */
+  int64_t tail_elems;        /* two-pass: elements at each end of the layout
+                                in LAMB_TAIL_CHUNK_ELEMS chunks             */
+  int32_t shard_world;       /* 1 if the plan is not sharded                */
+  int32_t shard_rank;
+  int64_t shard_chunk_begin; /* this shard's chunks [begin, end)            */
+  int64_t shard_chunk_end;
 } lamb_plan_info_t;
 
 typedef struct lamb_plan* lamb_plan_t;
@@ -350,48 +414,64 @@ LAMB_API lamb_status_t lamb_plan_read_timing(lamb_plan_t plan, int32_t* n_steps,
 LAMB_API lamb_status_t lamb_plan_destroy(lamb_plan_t plan);
 
 /* Host-only planner, no device needed: the chunk table lamb_plan_create
- * would build.  Writes up to `capacity` rows into the three host arrays
- * (any may be NULL when capacity is 0) and the total row count into
- * *n_chunks.  INVALID_ARG on bad sizes/chunk_elems or capacity too small
- * (n_chunks is still written). */
+ * would build.  Chunks hold chunk_elems elements (0 = 16384), except within
+ * tail_elems of either end of the layout (the tensors laid end to end), where
+ * they hold LAMB_TAIL_CHUNK_ELEMS; a chunk never spans two tensors.  A plan
+ * uses the tail reported by lamb_plan_get_info.  Writes up to `capacity`
+ * rows into the three host arrays (any may be NULL when capacity is 0) and
+ * the total row count into *n_chunks.  INVALID_ARG on bad sizes, chunk_elems
+ * or tail_elems (< 0), or capacity too small (n_chunks is still written). */
 LAMB_API lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
-                                 int32_t chunk_elems, int32_t* chunk_tensor,
-                                 int64_t* chunk_offset, int32_t* chunk_len,
-                                 int32_t capacity, int32_t* n_chunks);
+                                 int32_t chunk_elems, int64_t tail_elems,
+                                 int32_t* chunk_tensor, int64_t* chunk_offset,
+                                 int32_t* chunk_len, int32_t capacity,
+                                 int32_t* n_chunks);
 
-/* One LAMB step (the same two kernels and numerics as lamb_step with the
- * default 16384-element chunks) for callers that may not allocate device
+/* One LAMB step (the same two kernels, chunking and numerics as lamb_step on
+ * a two-pass plan with the default 16384-element chunks and no tail: the
+ * results are bitwise equal) for callers that may not allocate device
  * memory: code that runs under an allocator owning all GPU memory (a
  * framework's caching allocator or a fixed pool), code that must not pay the
  * device-wide synchronisation cudaMalloc/cudaFree can cause, or a plug-in
  * that is handed a stream and buffers but no right to allocate.  It needs no
  * plan: every table, partial sum and counter lives in one fixed 4 MiB device
- * array built into the library, which each GPU that loads the library holds
- * until the process exits.  (The paper has no counterpart of this entry
- * point; it is a deployment convenience.)
+ * array built into the library, which each GPU that uses it holds until the
+ * process exits.  (The paper has no counterpart of this entry point; it is a
+ * deployment convenience.)
  *
  *   sizes, decay_mask   host arrays [n_tensors] as in lamb_plan_create
  *                       (decay_mask may be NULL = all decayed)
  *   w, g, m, v, w_copy  host arrays [n_tensors] of DEVICE pointers as in
  *                       lamb_plan_bind; v is required; w_copy iff copy_dtype
  *                       is LAMB_BF16
- *   hyper, d_step, d_lr as in lamb_step
+ *   hyper, d_step, d_lr as in lamb_step (flags: BIAS_CORRECTION and
+ *                       INCREMENT_STEP only)
  *   d_ratio             NULL or a DEVICE array [n_tensors] of doubles that
  *                       receives the trust ratios of this step
- * Limits: n_tensors <= 4096 and at most 131072 chunks of 16384 elements
- * (2^31 parameters); larger inputs are rejected with LAMB_ERR_INVALID_ARG
- * before any device work.  Calls no cudaMalloc, cudaFree or other
- * allocating routine.  The caller's host arrays are copied into the device
- * array with cudaMemcpyAsync on `stream` and may be reused when the call
- * returns.  The first call on each device (the current device) looks up the
- * array's device address and the launch sizes; make that first call before
- * any stream capture.  All calls share the one array: calls that may overlap
- * on the GPU (other streams, other host threads) race and must be ordered by
- * the caller.  Each call rebuilds the tables and clears the counters it
- * needs, so it does not depend on what the previous call left there.
- * Device-side conditions (a step count < 1: the step is skipped; non-finite
- * norms: NaN/Inf propagate) behave as in lamb_step; there is no status
- * query for this entry point. */
+ * Limits: n_tensors <= 4096, no tensor above 2^31 elements and at most
+ * 131072 chunks of 16384 elements in total (2^31 parameters); larger inputs
+ * are rejected with LAMB_ERR_INVALID_ARG before any device work.  Calls no
+ * cudaMalloc, cudaFree or other allocating routine.
+ * The caller's host arrays (sizes, decay_mask and the five pointer arrays)
+ * are copied into the device array with cudaMemcpyAsync on `stream`.  From
+ * pageable memory those copies have read them when the call returns, so
+ * they may be reused at once; from page-locked (pinned) memory a copy may
+ * still be reading them after the call returns, so keep them unchanged until
+ * `stream` has passed the call (e.g. synchronise it).  Under stream capture
+ * the copies become graph nodes that read the same host arrays at every
+ * replay, which must then stay valid and unchanged for the graph's life.
+ * The first call on each device (the current device) looks up the array's
+ * device address; with CUDA's lazy module loading (the default) that first
+ * use also loads the library's kernels and reserves the 4 MiB there, so make
+ * the first call before any stream capture and before a memory pool claims
+ * all device memory (or load eagerly with CUDA_MODULE_LOADING=EAGER).  All
+ * calls share the one array: calls that may overlap on the GPU (other
+ * streams, other host threads) race and must be ordered by the caller.
+ * Each call rebuilds the tables and clears the counters it needs, so it does
+ * not depend on what the previous call left there.  Device-side conditions
+ * (a step count < 1: the step is skipped; non-finite norms: NaN/Inf
+ * propagate) behave as in lamb_step; there is no status query for this
+ * entry point. */
 LAMB_API lamb_status_t lamb_step_noalloc(
     const int64_t* sizes, int32_t n_tensors, const uint8_t* decay_mask,
     int32_t grad_dtype, int32_t copy_dtype, void* const* w,
@@ -413,6 +493,105 @@ LAMB_API lamb_status_t lamb_layout_schedule(const int64_t* sizes,
                                             uint32_t* items, int64_t capacity,
                                             int64_t* n_items,
                                             uint8_t* resident);
+
+/* Host-only planner, no device needed: the rounds of an on-chip plan
+ * (LAMB_ALGO_ON_CHIP) with `grid` CTAs of rows_per_cta rows (1..224) each.
+ * One output row per piece, in round order, then CTA order: its round, its
+ * CTA, tensor, first element inside the tensor, element count, first row
+ * inside the CTA's slice and row count; then one row per tensor too large
+ * for a round (updated by the two-pass kernels), with round and CTA -1, the
+ * whole tensor as its elements and 0 rows.
+ * Writes up to `capacity` pieces (the output arrays may be NULL when
+ * capacity is 0), the total into *n_pieces and the round count into
+ * *n_rounds.  INVALID_ARG on bad input or capacity too small (the counts are
+ * still written).  lamb_plan_create uses the same planner with the device's
+ * SM count (at most; at least 32 rows per CTA) and shared-memory rows
+ * (lamb_plan_get_info reports both). */
+LAMB_API lamb_status_t lamb_layout_rounds(
+    const int64_t* sizes, int32_t n_tensors, int32_t grid,
+    int32_t rows_per_cta, int32_t* piece_round, int32_t* piece_cta,
+    int32_t* piece_tensor, int64_t* piece_offset, int64_t* piece_len,
+    int32_t* piece_first_row, int32_t* piece_rows, int64_t capacity,
+    int64_t* n_pieces, int32_t* n_rounds);
+
+/* ---------------------------------------------------------------------------
+ * Data-parallel (sharded) step.
+ *
+ * The step shards over chunk ranges: rank r of W updates only the chunks of
+ * its range (lamb_layout_shard), with one exchange per step -- the per-chunk
+ * sums of w^2 and u^2 (u = r + lambda_k w; LARS: m), 2 floats per chunk (165
+ * KB for BERT-large), which every rank needs to form the trust ratios of
+ * the tensors its range touches.  Per step, on each rank:
+ *   lamb_shard_pass1   zeroes the plan's sums array, then reads g, m, v, w
+ *                      of the rank's chunks, writes m, v and the chunks'
+ *                      sums (Alg. 2 moment lines; Alg. 1 for LARS);
+ *   (caller)           all-reduce (sum) of the float array lamb_plan_partials
+ *                      returns, in place, across the ranks -- every entry
+ *                      has one non-zero contributor, so the sum is exact and
+ *                      every rank ends with the same array;
+ *   lamb_shard_pass2   forms every tensor's norms and rho_k from the array
+ *                      with the fixed-order combine of an unsharded step,
+ *                      then updates w (and the bf16 copy) of the rank's
+ *                      chunks; closes the step (INCREMENT_STEP, schedule,
+ *                      N-LAMB product) like lamb_step.
+ * The results on each rank's range, and the trust ratios, are bitwise equal
+ * to one unsharded step of the same layout and tail.  The gradients of the
+ * rank's range must be reduced (e.g. reduce-scattered) before pass 1, and
+ * the new w gathered after pass 2, by the caller.  The kernels touch only
+ * the rank's elements of w, g, m, v and the copy.  Not taken: GRAD_NORM,
+ * SKIP_NONFINITE (INVALID_ARG).  Both halves are capturable; no timing
+ * events are recorded for them.
+ *   optimizer       LAMB_OPT_*; LARS uses trust_coef, the N-LAMB forms
+ *                   momentum_decay and d_mu_product as in nlamb_step (both
+ *                   halves take the same arguments)
+ *   d_step, d_lr    as in lamb_step (N-LAMB: d_step required)
+ * ------------------------------------------------------------------------- */
+#define LAMB_OPT_LAMB 0
+#define LAMB_OPT_LARS 1
+#define LAMB_OPT_NLAMB 2
+#define LAMB_OPT_NNLAMB 3
+
+LAMB_API lamb_status_t lamb_shard_pass1(lamb_plan_t plan,
+                                        const lamb_hyper_t* hyper,
+                                        int32_t optimizer,
+                                        double momentum_decay,
+                                        int64_t* d_step, const float* d_lr,
+                                        double* d_mu_product,
+                                        cudaStream_t stream);
+LAMB_API lamb_status_t lamb_shard_pass2(lamb_plan_t plan,
+                                        const lamb_hyper_t* hyper,
+                                        int32_t optimizer,
+                                        double momentum_decay,
+                                        int64_t* d_step, const float* d_lr,
+                                        double* d_mu_product,
+                                        cudaStream_t stream);
+
+/* DEVICE float array of 2 x n_chunks values (per chunk: sum of w^2, sum of
+ * u^2) that lamb_shard_pass1 writes and lamb_shard_pass2 reads; owned by the
+ * plan, valid until destroy.  *n_floats receives 2 x n_chunks. */
+LAMB_API lamb_status_t lamb_plan_partials(lamb_plan_t plan, float** d_partials,
+                                          int64_t* n_floats);
+
+/* Copies the sums array (2 x n_chunks floats, as lamb_plan_partials) out of
+ * the plan into buf (to_plan = 0) or from buf into the plan (to_plan = 1),
+ * with cudaMemcpyAsync on `stream`; buf is device or host memory.  For a
+ * caller whose all-reduce wants its own buffer (e.g. a framework tensor):
+ * copy out, all-reduce, copy back.  Capturable with a device buffer. */
+LAMB_API lamb_status_t lamb_plan_copy_partials(lamb_plan_t plan, float* buf,
+                                               int32_t to_plan,
+                                               cudaStream_t stream);
+
+/* Host-only: the chunk range [*chunk_begin, *chunk_end) of shard `rank` of
+ * `world` for the chunk table lamb_layout_chunks(sizes, chunk_elems,
+ * tail_elems) gives: the chunks whose first element, counted over the layout
+ * (tensors laid end to end), lies in [total rank / world, total (rank + 1) /
+ * world).  A range may be empty.  INVALID_ARG on bad input. */
+LAMB_API lamb_status_t lamb_layout_shard(const int64_t* sizes,
+                                         int32_t n_tensors,
+                                         int32_t chunk_elems,
+                                         int64_t tail_elems, int32_t world,
+                                         int32_t rank, int64_t* chunk_begin,
+                                         int64_t* chunk_end);
 
 /* Message of the last failed call on this host thread ("" if none). */
 LAMB_API const char* lamb_last_error(void);

@@ -52,7 +52,10 @@ EXPORTED = ["lamb_plan_create", "lamb_plan_bind", "lamb_step", "lars_step",
             "lamb_plan_set_timing", "lamb_plan_read_timing",
             "lamb_plan_destroy", "lamb_layout_chunks", "lamb_last_error",
             "lamb_abi_version", "lamb_step_noalloc", "lamb_layout_schedule",
-            "nlamb_step", "lamb_plan_grad_norms", "lamb_plan_copy_grad_norms"]
+            "nlamb_step", "lamb_plan_grad_norms", "lamb_plan_copy_grad_norms",
+            "lamb_layout_rounds", "lamb_shard_pass1", "lamb_shard_pass2",
+            "lamb_plan_partials", "lamb_layout_shard",
+            "lamb_plan_copy_partials"]
 
 
 class LambError(RuntimeError):
@@ -77,14 +80,24 @@ class lamb_hyper_t(Structure):
 LAMB_ALGO_AUTO = 0
 LAMB_ALGO_TWO_PASS = 1
 LAMB_ALGO_SINGLE_TOUCH = 2
+LAMB_ALGO_ON_CHIP = 3
 LAMB_FUSED_CHUNK_ELEMS = 4096     # work item of a single-touch step
+LAMB_ONCHIP_ROW_ELEMS = 128       # row of an on-chip step
+LAMB_TAIL_CHUNK_ELEMS = 2048      # chunks near the ends of a two-pass layout
+LAMB_OPT_LAMB = 0
+LAMB_OPT_LARS = 1
+LAMB_OPT_NLAMB = 2
+LAMB_OPT_NNLAMB = 3
 LAMB_STATUS_WAIT_TIMEOUT = 0x4
 
 
 class lamb_plan_options_t(Structure):
     _fields_ = [("chunk_elems", c_int32), ("blocks_per_sm", c_int32),
                 ("algorithm", c_int32), ("l2_budget_mb", c_int32),
-                ("lag_items", c_int32)]
+                ("lag_items", c_int32), ("wait_limit_ms", c_int32),
+                ("test_unmet_wait", c_int32), ("onchip_max_ctas", c_int32),
+                ("onchip_rows", c_int32), ("tail_elems", c_int64),
+                ("shard_world", c_int32), ("shard_rank", c_int32)]
 
 
 class lamb_plan_info_t(Structure):
@@ -96,7 +109,12 @@ class lamb_plan_info_t(Structure):
                 ("bound", c_int32), ("n_vector_tensors", c_int32),
                 ("device_bytes", c_int64), ("algorithm", c_int32),
                 ("n_resident_tensors", c_int32), ("n_items", c_int64),
-                ("lag_items", c_int64), ("l2_budget_bytes", c_int64)]
+                ("lag_items", c_int64), ("l2_budget_bytes", c_int64),
+                ("n_rounds", c_int32), ("n_streamed_tensors", c_int32),
+                ("rows_per_cta", c_int32), ("row_elems", c_int32),
+                ("tail_elems", c_int64), ("shard_world", c_int32),
+                ("shard_rank", c_int32), ("shard_chunk_begin", c_int64),
+                ("shard_chunk_end", c_int64)]
 
 
 _lib = None
@@ -137,6 +155,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                           POINTER(c_double), c_int32]
     lib.lamb_plan_destroy.argtypes = [vp]
     lib.lamb_layout_chunks.argtypes = [POINTER(c_int64), c_int32, c_int32,
+                                       c_int64,
                                        POINTER(c_int32), POINTER(c_int64),
                                        POINTER(c_int32), c_int32,
                                        POINTER(c_int32)]
@@ -148,6 +167,17 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                       POINTER(vp), POINTER(vp), POINTER(vp),
                                       POINTER(vp), POINTER(vp),
                                       POINTER(lamb_hyper_t), vp, vp, vp, vp]
+    for name in ("lamb_shard_pass1", "lamb_shard_pass2"):
+        getattr(lib, name).argtypes = [vp, POINTER(lamb_hyper_t), c_int32,
+                                       c_double, vp, vp, vp, vp]
+    lib.lamb_plan_partials.argtypes = [vp, POINTER(vp), POINTER(c_int64)]
+    lib.lamb_plan_copy_partials.argtypes = [vp, vp, c_int32, vp]
+    lib.lamb_layout_shard.argtypes = [POINTER(c_int64), c_int32, c_int32,
+                                      c_int64, c_int32, c_int32,
+                                      POINTER(c_int64), POINTER(c_int64)]
+    lib.lamb_layout_rounds.argtypes = [POINTER(c_int64), c_int32, c_int32,
+                                       c_int32, *([vp] * 7), c_int64,
+                                       POINTER(c_int64), POINTER(c_int32)]
     for name in EXPORTED:
         if name in ("lamb_last_error", "lamb_abi_version"):
             continue
@@ -203,7 +233,10 @@ def make_hyper(*, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01,
 def lamb_plan_create(sizes, decay_mask=None, grad_dtype=LAMB_F32,
                      copy_dtype=LAMB_DTYPE_NONE, device=0, chunk_elems=0,
                      blocks_per_sm=0, algorithm=LAMB_ALGO_AUTO,
-                     l2_budget_mb=0, lag_items=0) -> int:
+                     l2_budget_mb=0, lag_items=0, wait_limit_ms=0,
+                     test_unmet_wait=False, onchip_max_ctas=0,
+                     onchip_rows=0, tail_elems=0, shard_world=0,
+                     shard_rank=0) -> int:
     lib = load()
     n = len(sizes)
     sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
@@ -212,7 +245,11 @@ def lamb_plan_create(sizes, decay_mask=None, grad_dtype=LAMB_F32,
         mask = (c_uint8 * max(n, 1))(*[1 if d else 0 for d in decay_mask])
     opts = lamb_plan_options_t(int(chunk_elems), int(blocks_per_sm),
                                int(algorithm), int(l2_budget_mb),
-                               int(lag_items))
+                               int(lag_items), int(wait_limit_ms),
+                               int(bool(test_unmet_wait)),
+                               int(onchip_max_ctas), int(onchip_rows),
+                               int(tail_elems), int(shard_world),
+                               int(shard_rank))
     out = c_void_p()
     _check(lib.lamb_plan_create(sz, n, mask, int(grad_dtype), int(copy_dtype),
                                 int(device), byref(opts), byref(out)))
@@ -345,13 +382,14 @@ def lamb_layout_schedule(sizes, l2_budget_bytes, lag_items):
     return items[:count.value], res[:n]
 
 
-def lamb_layout_chunks(sizes, chunk_elems=0):
+def lamb_layout_chunks(sizes, chunk_elems=0, tail_elems=0):
     """Host-only planner: returns (tensor, offset, length) int arrays."""
     lib = load()
     n = len(sizes)
     sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
     count = c_int32()
-    st = lib.lamb_layout_chunks(sz, n, int(chunk_elems), None, None, None, 0,
+    st = lib.lamb_layout_chunks(sz, n, int(chunk_elems), int(tail_elems),
+                                None, None, None, 0,
                                 byref(count))
     _check(st)
     cap = count.value
@@ -359,7 +397,82 @@ def lamb_layout_chunks(sizes, chunk_elems=0):
     o = np.zeros(max(cap, 1), dtype=np.int64)
     ln = np.zeros(max(cap, 1), dtype=np.int32)
     _check(lib.lamb_layout_chunks(
-        sz, n, int(chunk_elems), t.ctypes.data_as(POINTER(c_int32)),
+        sz, n, int(chunk_elems), int(tail_elems),
+        t.ctypes.data_as(POINTER(c_int32)),
         o.ctypes.data_as(POINTER(c_int64)), ln.ctypes.data_as(POINTER(c_int32)),
         cap, byref(count)))
     return t[:cap], o[:cap], ln[:cap]
+
+
+def lamb_layout_rounds(sizes, grid, rows_per_cta):
+    """Host-only: the pieces of an on-chip plan as a dict of arrays (round,
+    cta, tensor, offset, len, first_row, rows) and the round count."""
+    lib = load()
+    n = len(sizes)
+    sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
+    count, rounds = c_int64(), c_int32()
+    _check(lib.lamb_layout_rounds(sz, n, int(grid), int(rows_per_cta),
+                                  *([None] * 7), 0, byref(count),
+                                  byref(rounds)))
+    cap = count.value
+    out = {"round": np.zeros(max(cap, 1), np.int32),
+           "cta": np.zeros(max(cap, 1), np.int32),
+           "tensor": np.zeros(max(cap, 1), np.int32),
+           "offset": np.zeros(max(cap, 1), np.int64),
+           "len": np.zeros(max(cap, 1), np.int64),
+           "first_row": np.zeros(max(cap, 1), np.int32),
+           "rows": np.zeros(max(cap, 1), np.int32)}
+    _check(lib.lamb_layout_rounds(
+        sz, n, int(grid), int(rows_per_cta),
+        *[out[k].ctypes.data for k in ("round", "cta", "tensor", "offset",
+                                        "len", "first_row", "rows")],
+        cap, byref(count), byref(rounds)))
+    return {k: v[:cap] for k, v in out.items()}, int(rounds.value)
+
+
+def lamb_shard_pass1(plan, hyper: lamb_hyper_t, optimizer=LAMB_OPT_LAMB,
+                     momentum_decay=0.0, d_step=0, d_lr=0, d_mu_product=0,
+                     stream=0) -> None:
+    _check(load().lamb_shard_pass1(c_void_p(plan), byref(hyper),
+                                   int(optimizer), float(momentum_decay),
+                                   c_void_p(d_step or None),
+                                   c_void_p(d_lr or None),
+                                   c_void_p(d_mu_product or None),
+                                   c_void_p(stream or None)))
+
+
+def lamb_shard_pass2(plan, hyper: lamb_hyper_t, optimizer=LAMB_OPT_LAMB,
+                     momentum_decay=0.0, d_step=0, d_lr=0, d_mu_product=0,
+                     stream=0) -> None:
+    _check(load().lamb_shard_pass2(c_void_p(plan), byref(hyper),
+                                   int(optimizer), float(momentum_decay),
+                                   c_void_p(d_step or None),
+                                   c_void_p(d_lr or None),
+                                   c_void_p(d_mu_product or None),
+                                   c_void_p(stream or None)))
+
+
+def lamb_plan_partials(plan):
+    """(device address of the float sums array, number of floats)."""
+    ptr, n = c_void_p(), c_int64()
+    _check(load().lamb_plan_partials(c_void_p(plan), byref(ptr), byref(n)))
+    return ptr.value, int(n.value)
+
+
+def lamb_layout_shard(sizes, world, rank, chunk_elems=0, tail_elems=0):
+    """Host-only: chunk range (begin, end) of shard `rank` of `world`."""
+    n = len(sizes)
+    sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
+    b, e = c_int64(), c_int64()
+    _check(load().lamb_layout_shard(sz, n, int(chunk_elems), int(tail_elems),
+                                    int(world), int(rank), byref(b),
+                                    byref(e)))
+    return int(b.value), int(e.value)
+
+
+def lamb_plan_copy_partials(plan, buf, to_plan, stream=0) -> None:
+    """Copy the plan's sums array to (to_plan false) or from (true) the
+    device or host address buf."""
+    _check(load().lamb_plan_copy_partials(c_void_p(plan), c_void_p(buf),
+                                          int(bool(to_plan)),
+                                          c_void_p(stream or None)))

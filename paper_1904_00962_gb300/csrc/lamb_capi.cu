@@ -45,7 +45,7 @@ namespace {
 static_assert(lamb::kFusedChunk == LAMB_FUSED_CHUNK_ELEMS,
               "the ABI documents the fused chunk size");
 constexpr int kMaxTimedSteps = 4096;
-constexpr int kKernelsPerStep = 2;
+constexpr int kKernelsPerStep = 3;
 
 // Restores the caller's current device on scope exit.
 struct DeviceGuard {
@@ -72,6 +72,9 @@ struct lamb_plan {
   int64_t n_chunks = 0;
   int64_t n_params = 0;
   int chunk_elems = kDefaultChunk;
+  int64_t tail_elems = 0;       // elements at each end in short chunks
+  int shard_world = 1, shard_rank = 0;
+  int64_t shard_cb = 0, shard_ce = 0;   // this shard's chunk range
   int grad_bf16 = 0;
   int copy_bf16 = 0;
   int num_sms = 0;
@@ -111,12 +114,49 @@ struct lamb_plan {
   float2* fslots = nullptr;
   uint32_t* ftickets = nullptr;
   uint32_t* ready = nullptr;
+  // on-chip single-touch tables
+  int oc_grid = 0;
+  int oc_rows = 0;              // rows of shared memory per CTA
+  int oc_n_rounds = 0;
+  int oc_n_streamed = 0;
+  int64_t oc_n_slots = 0;
+  int64_t oc_wait_ns = 0;
+  int oc_extra = 0;
+  std::vector<OcPiece> h_oc_pieces;   // without pointers (filled by bind)
+  OcSlice* oc_slices = nullptr;
+  OcPiece* oc_pieces = nullptr;
+  float4* oc_slots = nullptr;
+  uint32_t* oc_bar = nullptr;
+  // the streamed tensors' chunk table for the two-pass kernels
+  int64_t oc_n_chunks = 0;
+  int oc_sub_grid[4] = {0, 0, 0, 0};
+  ChunkDesc* oc_chunks = nullptr;
+  TensorDesc* oc_tensors = nullptr;
 
   bool timing = false;
   int timed_steps = 0;
   std::vector<cudaEvent_t> events;  // kMaxTimedSteps * (kKernelsPerStep + 1)
   std::vector<uint8_t> timed_kernels;  // kernels each timed step launched
 };
+
+void lamb::fill_hyper(const lamb_hyper_t& h, StepParams* sp) {
+  // (1 - beta) formed in double and rounded once
+  sp->b1 = (float)h.beta1;
+  sp->omb1 = (float)(1.0 - h.beta1);
+  sp->b2 = (float)h.beta2;
+  sp->omb2 = (float)(1.0 - h.beta2);
+  sp->eps = (float)h.eps;
+  sp->wd = (float)h.weight_decay;
+  sp->beta1 = h.beta1;
+  sp->beta2 = h.beta2;
+  sp->log2_beta1 = std::log2(h.beta1);   // -inf for beta = 0: beta^t = 0
+  sp->log2_beta2 = std::log2(h.beta2);
+  sp->gamma_l = h.gamma_l;
+  sp->gamma_u = h.gamma_u;
+  sp->trust = h.trust_coef;
+  sp->phi = h.phi;
+  sp->flags = h.flags;
+}
 
 extern "C" {
 
@@ -125,9 +165,10 @@ const char* lamb_last_error(void) { return g_err; }
 int32_t lamb_abi_version(void) { return LAMB_ABI_VERSION; }
 
 lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
-                                 int32_t chunk_elems, int32_t* chunk_tensor,
-                                 int64_t* chunk_offset, int32_t* chunk_len,
-                                 int32_t capacity, int32_t* n_chunks) {
+                                 int32_t chunk_elems, int64_t tail_elems,
+                                 int32_t* chunk_tensor, int64_t* chunk_offset,
+                                 int32_t* chunk_len, int32_t capacity,
+                                 int32_t* n_chunks) {
   if (n_chunks == nullptr) return fail(LAMB_ERR_INVALID_ARG, "n_chunks is NULL");
   if (capacity < 0) return fail(LAMB_ERR_INVALID_ARG, "capacity < 0");
   if (capacity > 0 && (!chunk_tensor || !chunk_offset || !chunk_len))
@@ -141,9 +182,11 @@ lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
   }
   int64_t count = 0;
   char err[256] = "";
+  if (tail_elems < 0) return fail(LAMB_ERR_INVALID_ARG, "tail_elems < 0");
   const int rc = plan_chunks(sizes, n_tensors, chunk_elems,
                              capacity ? rows.data() : nullptr, capacity,
-                             &count, nullptr, nullptr, err, sizeof(err));
+                             &count, nullptr, nullptr, err, sizeof(err),
+                             tail_elems, kTailChunk);
   *n_chunks = (int32_t)(count > INT32_MAX ? INT32_MAX : count);
   if (rc) return fail(LAMB_ERR_INVALID_ARG, "%s", err);
   if (count > capacity && capacity > 0)
@@ -154,6 +197,34 @@ lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
     chunk_offset[i] = rows[i].offset;
     chunk_len[i] = rows[i].len;
   }
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_layout_shard(const int64_t* sizes, int32_t n_tensors,
+                                int32_t chunk_elems, int64_t tail_elems,
+                                int32_t world, int32_t rank,
+                                int64_t* chunk_begin, int64_t* chunk_end) {
+  if (!chunk_begin || !chunk_end)
+    return fail(LAMB_ERR_INVALID_ARG, "chunk_begin and chunk_end are required");
+  if (world < 1 || rank < 0 || rank >= world)
+    return fail(LAMB_ERR_INVALID_ARG, "need 0 <= rank < world");
+  if (tail_elems < 0) return fail(LAMB_ERR_INVALID_ARG, "tail_elems < 0");
+  if (chunk_elems == 0) chunk_elems = kDefaultChunk;
+  char err[256] = "";
+  int64_t count = 0;
+  if (plan_chunks(sizes, n_tensors, chunk_elems, nullptr, 0, &count, nullptr,
+                  nullptr, err, sizeof(err), tail_elems, kTailChunk))
+    return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  std::vector<ChunkDesc> rows;
+  try {
+    rows.resize((size_t)count);
+  } catch (const std::bad_alloc&) {
+    return fail(LAMB_ERR_OOM, "host allocation failed");
+  }
+  if (plan_chunks(sizes, n_tensors, chunk_elems, rows.data(), count, &count,
+                  nullptr, nullptr, err, sizeof(err), tail_elems, kTailChunk))
+    return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  shard_range(rows.data(), count, world, rank, chunk_begin, chunk_end);
   return LAMB_OK;
 }
 
@@ -196,6 +267,79 @@ lamb_status_t lamb_layout_schedule(const int64_t* sizes, int32_t n_tensors,
   return LAMB_OK;
 }
 
+lamb_status_t lamb_layout_rounds(const int64_t* sizes, int32_t n_tensors,
+                                 int32_t grid, int32_t rows_per_cta,
+                                 int32_t* piece_round, int32_t* piece_cta,
+                                 int32_t* piece_tensor, int64_t* piece_offset,
+                                 int64_t* piece_len, int32_t* piece_first_row,
+                                 int32_t* piece_rows, int64_t capacity,
+                                 int64_t* n_pieces, int32_t* n_rounds) {
+  if (!n_pieces || !n_rounds)
+    return fail(LAMB_ERR_INVALID_ARG, "n_pieces and n_rounds are required");
+  if (n_tensors < 1 || !sizes)
+    return fail(LAMB_ERR_INVALID_ARG, "need n_tensors >= 1 and sizes");
+  if (capacity < 0 ||
+      (capacity > 0 && (!piece_round || !piece_cta || !piece_tensor ||
+                        !piece_offset || !piece_len || !piece_first_row ||
+                        !piece_rows)))
+    return fail(LAMB_ERR_INVALID_ARG, "bad capacity or output arrays");
+  int64_t total = 0;
+  for (int32_t k = 0; k < n_tensors; ++k) {
+    if (sizes[k] < 0)
+      return fail(LAMB_ERR_INVALID_ARG, "sizes[%d] is negative", k);
+    if (sizes[k] > (int64_t(1) << 62) - total)
+      return fail(LAMB_ERR_INVALID_ARG, "total element count exceeds 2^62");
+    total += sizes[k];
+  }
+  std::vector<OcSlice> slices;
+  std::vector<OcPiece> pieces;
+  std::vector<int32_t> streamed;
+  int64_t n_slots = 0;
+  int32_t rounds = 0;
+  char err[256] = "";
+  try {
+    if (plan_onchip(sizes, n_tensors, nullptr, grid, rows_per_cta, &rounds,
+                    &slices, &pieces, &streamed, &n_slots, err, sizeof(err)))
+      return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  } catch (const std::bad_alloc&) {
+    return fail(LAMB_ERR_OOM, "host allocation failed");
+  }
+  const int64_t total_pieces = (int64_t)(pieces.size() + streamed.size());
+  *n_pieces = total_pieces;
+  *n_rounds = rounds;
+  if (total_pieces > capacity)
+    return capacity == 0 ? LAMB_OK
+                         : fail(LAMB_ERR_INVALID_ARG, "capacity too small");
+  int64_t i = 0;
+  for (int32_t r = 0; r < rounds; ++r) {
+    for (int32_t c = 0; c < grid; ++c) {
+      const OcSlice& sl = slices[(size_t)r * (size_t)grid + (size_t)c];
+      for (int j = 0; j < sl.n_pieces; ++j) {
+        const OcPiece& pc = pieces[(size_t)sl.piece_begin + (size_t)j];
+        piece_round[i] = r;
+        piece_cta[i] = c;
+        piece_tensor[i] = pc.tensor;
+        piece_offset[i] = pc.offset;
+        piece_len[i] = pc.len;
+        piece_first_row[i] = pc.first_row;
+        piece_rows[i] = pc.n_rows;
+        ++i;
+      }
+    }
+  }
+  for (int32_t k : streamed) {
+    piece_round[i] = -1;
+    piece_cta[i] = -1;
+    piece_tensor[i] = k;
+    piece_offset[i] = 0;
+    piece_len[i] = sizes[k];
+    piece_first_row[i] = 0;
+    piece_rows[i] = 0;
+    ++i;
+  }
+  return LAMB_OK;
+}
+
 static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
                                  const uint8_t* decay_mask, int32_t grad_dtype,
                                  int32_t copy_dtype, int32_t device,
@@ -210,21 +354,44 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
     return fail(LAMB_ERR_UNSUPPORTED_DTYPE,
                 "copy_dtype %d unsupported (NONE or BF16)", copy_dtype);
   int chunk = kDefaultChunk, bps = 0, algo = LAMB_ALGO_AUTO;
-  int64_t budget_mb = 0, lag_opt = 0;
+  int64_t budget_mb = 0, lag_opt = 0, wait_ms = 1000;
+  int unmet_wait = 0, oc_max_ctas = 0, oc_rows_opt = 0;
+  int64_t tail_opt = 0;
+  int sh_world = 1, sh_rank = 0;
   if (opts) {
     if (opts->chunk_elems) chunk = opts->chunk_elems;
     if (opts->blocks_per_sm < 0)
       return fail(LAMB_ERR_INVALID_ARG, "blocks_per_sm < 0");
     bps = opts->blocks_per_sm;
     algo = opts->algorithm;
-    if (algo < LAMB_ALGO_AUTO || algo > LAMB_ALGO_SINGLE_TOUCH)
+    if (algo < LAMB_ALGO_AUTO || algo > LAMB_ALGO_ON_CHIP)
       return fail(LAMB_ERR_INVALID_ARG, "unknown algorithm %d", algo);
     if (opts->l2_budget_mb < 0 || opts->lag_items < 0)
       return fail(LAMB_ERR_INVALID_ARG, "l2_budget_mb and lag_items >= 0");
     budget_mb = opts->l2_budget_mb;
     lag_opt = opts->lag_items;
+    if (opts->wait_limit_ms < 0)
+      return fail(LAMB_ERR_INVALID_ARG, "wait_limit_ms >= 0");
+    if (opts->wait_limit_ms) wait_ms = opts->wait_limit_ms;
+    unmet_wait = opts->test_unmet_wait != 0;
+    if (opts->onchip_max_ctas < 0 || opts->onchip_rows < 0)
+      return fail(LAMB_ERR_INVALID_ARG, "onchip_max_ctas, onchip_rows >= 0");
+    oc_max_ctas = opts->onchip_max_ctas;
+    oc_rows_opt = opts->onchip_rows;
+    if (opts->tail_elems < 0)
+      return fail(LAMB_ERR_INVALID_ARG, "tail_elems must be >= 0");
+    tail_opt = opts->tail_elems;
+    if (opts->shard_world < 0 || opts->shard_rank < 0 ||
+        (opts->shard_world > 0 && opts->shard_rank >= opts->shard_world) ||
+        (opts->shard_world == 0 && opts->shard_rank != 0))
+      return fail(LAMB_ERR_INVALID_ARG,
+                  "need 0 <= shard_rank < shard_world (or both 0)");
+    if (opts->shard_world > 0) {
+      sh_world = opts->shard_world;
+      sh_rank = opts->shard_rank;
+    }
   }
-  if (algo == LAMB_ALGO_AUTO) algo = LAMB_ALGO_TWO_PASS;
+  const bool auto_algo = algo == LAMB_ALGO_AUTO;
   if (device < 0) return fail(LAMB_ERR_INVALID_ARG, "device < 0");
 
   lamb_plan* p = new (std::nothrow) lamb_plan();
@@ -261,20 +428,12 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
                                           : "sizes is NULL");
   }
   p->h_tensors.resize((size_t)n_tensors);
+  // validates the sizes before the device is touched
   if (plan_chunks(sizes, n_tensors, chunk, nullptr, 0, &nch,
                   p->h_tensors.data(), decay_mask, err, sizeof(err))) {
     return fail(LAMB_ERR_INVALID_ARG, "%s", err);
   }
-  std::vector<ChunkDesc> h_chunks((size_t)nch);
-  if (plan_chunks(sizes, n_tensors, chunk, h_chunks.data(), nch, &nch,
-                  p->h_tensors.data(), decay_mask, err, sizeof(err))) {
-    return fail(LAMB_ERR_INVALID_ARG, "%s", err);
-  }
-  p->n_chunks = nch;
-  for (int k = 0; k < n_tensors; ++k) {
-    p->n_params += sizes[k];
-    p->n_live += p->h_tensors[(size_t)k].n_chunks > 0 ? 1 : 0;
-  }
+  for (int k = 0; k < n_tensors; ++k) p->n_params += sizes[k];
 
   // ---- device ------------------------------------------------------------
   DeviceGuard guard(device);
@@ -286,6 +445,27 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   if (e != cudaSuccess) {
     return cuda_fail(e, "cudaDeviceGetAttribute");
   }
+  // the chunk table, optionally with short chunks at both ends of the layout
+  // (the last chunks each pass draws)
+  p->tail_elems = tail_opt;
+  if (plan_chunks(sizes, n_tensors, chunk, nullptr, 0, &nch,
+                  p->h_tensors.data(), decay_mask, err, sizeof(err),
+                  p->tail_elems, kTailChunk)) {
+    return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  }
+  std::vector<ChunkDesc> h_chunks((size_t)nch);
+  if (plan_chunks(sizes, n_tensors, chunk, h_chunks.data(), nch, &nch,
+                  p->h_tensors.data(), decay_mask, err, sizeof(err),
+                  p->tail_elems, kTailChunk)) {
+    return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+  }
+  p->n_chunks = nch;
+  for (int k = 0; k < n_tensors; ++k)
+    p->n_live += p->h_tensors[(size_t)k].n_chunks > 0 ? 1 : 0;
+  p->shard_world = sh_world;
+  p->shard_rank = sh_rank;
+  shard_range(h_chunks.data(), nch, sh_world, sh_rank, &p->shard_cb,
+              &p->shard_ce);
   int occ[4] = {0, 0, 0, 0};
   int rc = occupancy_lamb_pass1(p->grad_bf16, &occ[0]);
   if (!rc) rc = occupancy_lamb_pass2(p->copy_bf16, &occ[1]);
@@ -338,6 +518,77 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
     for (const FusedTensor& t : h_ftensors) p->n_resident += t.resident ? 1 : 0;
   }
 
+  // on-chip rounds
+  std::vector<OcSlice> h_slices;
+  std::vector<ChunkDesc> h_sub_chunks;
+  std::vector<TensorDesc> h_sub_tensors;
+  if (algo == LAMB_ALGO_ON_CHIP || auto_algo) {
+    rc = onchip_prepare(device, &p->oc_rows);
+    if (rc) {
+      return cuda_fail((cudaError_t)rc, "on-chip kernel set-up");
+    }
+    if (oc_rows_opt > 0) {
+      if (oc_rows_opt > p->oc_rows)
+        return fail(LAMB_ERR_INVALID_ARG,
+                    "onchip_rows %d exceeds the %d rows a CTA holds",
+                    oc_rows_opt, p->oc_rows);
+      p->oc_rows = oc_rows_opt;
+    }
+    int64_t total_rows = 0;
+    for (int k = 0; k < n_tensors; ++k)
+      total_rows += (sizes[k] + kOcRow - 1) / kOcRow;
+    int ctas = p->num_sms;
+    if (oc_max_ctas > 0 && oc_max_ctas < ctas) ctas = oc_max_ctas;
+    p->oc_grid = onchip_grid(total_rows, ctas);
+    std::vector<int32_t> streamed;
+    if (plan_onchip(sizes, n_tensors, decay_mask, p->oc_grid, p->oc_rows,
+                    &p->oc_n_rounds, &h_slices, &p->h_oc_pieces, &streamed,
+                    &p->oc_n_slots, err, sizeof(err))) {
+      return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+    }
+    p->oc_n_streamed = (int)streamed.size();
+    if (p->oc_n_rounds == 0) p->oc_grid = 1;   // nothing to do but close
+    // AUTO: the on-chip step when the whole layout is one round (one grid
+    // barrier, one launch, 28 B/parameter); with more rounds the per-round
+    // barrier and ratio time make the two-pass step the faster one
+    if (auto_algo) {
+      const bool one_round = p->oc_n_rounds <= 1 && streamed.empty();
+      algo = one_round ? LAMB_ALGO_ON_CHIP : LAMB_ALGO_TWO_PASS;
+      p->algorithm = algo;
+      if (!one_round) {
+        h_slices.clear();
+        p->h_oc_pieces.clear();
+        streamed.clear();
+        p->oc_n_rounds = 0;
+        p->oc_n_streamed = 0;
+        p->oc_n_slots = 0;
+      }
+    }
+    if (!streamed.empty()) {
+      // chunk table of the streamed tensors only (the others count as empty)
+      std::vector<int64_t> sub((size_t)n_tensors, 0);
+      for (int32_t k : streamed) sub[(size_t)k] = sizes[k];
+      h_sub_tensors.resize((size_t)n_tensors);
+      const int64_t sub_tail = tail_opt;
+      if (plan_chunks(sub.data(), n_tensors, chunk, nullptr, 0,
+                      &p->oc_n_chunks, h_sub_tensors.data(), decay_mask, err,
+                      sizeof(err), sub_tail, kTailChunk)) {
+        return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+      }
+      h_sub_chunks.resize((size_t)p->oc_n_chunks);
+      if (plan_chunks(sub.data(), n_tensors, chunk, h_sub_chunks.data(),
+                      p->oc_n_chunks, &p->oc_n_chunks, h_sub_tensors.data(),
+                      decay_mask, err, sizeof(err), sub_tail, kTailChunk)) {
+        return fail(LAMB_ERR_INVALID_ARG, "%s", err);
+      }
+      for (int i = 0; i < 4; ++i)
+        p->oc_sub_grid[i] = (int)(p->oc_n_chunks < p->grid[i]
+                                      ? p->oc_n_chunks : p->grid[i]);
+    }
+    p->oc_wait_ns = wait_ms * 1000000;
+    p->oc_extra = unmet_wait;
+  }
+
   const size_t n = (size_t)n_tensors, c = (size_t)nch;
   size_t off = 0;
   auto carve = [&](size_t bytes) {
@@ -369,6 +620,12 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   const size_t o_fslots = carve(nf * sizeof(float2));
   const size_t o_ftickets = carve(n * sizeof(uint32_t));
   const size_t o_ready = carve(n * sizeof(uint32_t));
+  const size_t o_oc_chunks = carve(h_sub_chunks.size() * sizeof(ChunkDesc));
+  const size_t o_oc_tensors = carve(h_sub_tensors.size() * sizeof(TensorDesc));
+  const size_t o_oc_slices = carve(h_slices.size() * sizeof(OcSlice));
+  const size_t o_oc_pieces = carve(p->h_oc_pieces.size() * sizeof(OcPiece));
+  const size_t o_oc_slots = carve((size_t)p->oc_n_slots * sizeof(float4));
+  const size_t o_oc_bar = carve(kBarWords * sizeof(uint32_t));
   p->arena_bytes = off;
   e = cudaMalloc(&p->arena, p->arena_bytes);
   if (e != cudaSuccess) {
@@ -395,6 +652,12 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   p->fslots = reinterpret_cast<float2*>(base + o_fslots);
   p->ftickets = reinterpret_cast<uint32_t*>(base + o_ftickets);
   p->ready = reinterpret_cast<uint32_t*>(base + o_ready);
+  p->oc_chunks = reinterpret_cast<ChunkDesc*>(base + o_oc_chunks);
+  p->oc_tensors = reinterpret_cast<TensorDesc*>(base + o_oc_tensors);
+  p->oc_slices = reinterpret_cast<OcSlice*>(base + o_oc_slices);
+  p->oc_pieces = reinterpret_cast<OcPiece*>(base + o_oc_pieces);
+  p->oc_slots = reinterpret_cast<float4*>(base + o_oc_slots);
+  p->oc_bar = reinterpret_cast<uint32_t*>(base + o_oc_bar);
 
   // zero everything (tickets, counters, status, results, pointer table)
   e = cudaMemset(p->arena, 0, p->arena_bytes);
@@ -418,6 +681,17 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   if (e == cudaSuccess)
     e = cudaMemcpy(p->ftensors, h_ftensors.data(), n * sizeof(FusedTensor),
                    cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !h_sub_chunks.empty())
+    e = cudaMemcpy(p->oc_chunks, h_sub_chunks.data(),
+                   h_sub_chunks.size() * sizeof(ChunkDesc),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !h_sub_tensors.empty())
+    e = cudaMemcpy(p->oc_tensors, h_sub_tensors.data(),
+                   h_sub_tensors.size() * sizeof(TensorDesc),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !h_slices.empty())
+    e = cudaMemcpy(p->oc_slices, h_slices.data(),
+                   h_slices.size() * sizeof(OcSlice), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) {  // fused launch epoch starts at 1 (ready[] = 0)
     const uint32_t one = 1u;
     e = cudaMemcpy(p->counters + 3, &one, sizeof(one), cudaMemcpyHostToDevice);
@@ -497,11 +771,30 @@ lamb_status_t lamb_plan_bind(lamb_plan_t plan, void* const* w,
     t.vec_ok = ok ? 1u : 0u;
     n_vec += ok;
   }
+  // on-chip pieces carry their tensor's pointers
+  std::vector<OcPiece> oc;
+  try {
+    oc = plan->h_oc_pieces;
+  } catch (const std::bad_alloc&) {
+    return fail(LAMB_ERR_OOM, "host allocation failed");
+  }
+  for (OcPiece& pc : oc) {
+    const TensorPtrs& t = h[(size_t)pc.tensor];
+    pc.w = t.w;
+    pc.g = t.g;
+    pc.m = t.m;
+    pc.v = t.v;
+    pc.copy = t.copy;
+    pc.flags = (pc.flags & ~kOcVec) | (t.vec_ok ? kOcVec : 0u);
+  }
   DeviceGuard guard(plan->device);
   if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
   cudaError_t e = cudaMemcpyAsync(plan->ptrs, h.data(),
                                   (size_t)n * sizeof(TensorPtrs),
                                   cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess && !oc.empty())
+    e = cudaMemcpyAsync(plan->oc_pieces, oc.data(), oc.size() * sizeof(OcPiece),
+                        cudaMemcpyHostToDevice, stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cuda_fail(e, "pointer table upload");
   plan->bound = true;
@@ -546,6 +839,7 @@ static lamb_status_t check_hyper(const lamb_hyper_t* h, bool lamb) {
 static void fill_params(lamb_plan* p, const lamb_hyper_t* h, int64_t* d_step,
                         const float* d_lr, StepParams* sp) {
   std::memset(sp, 0, sizeof(*sp));
+  fill_hyper(*h, sp);
   sp->chunks = p->chunks;
   sp->tensors = p->tensors;
   sp->ptrs = p->ptrs;
@@ -559,22 +853,6 @@ static void fill_params(lamb_plan* p, const lamb_hyper_t* h, int64_t* d_step,
   sp->status = p->status;
   sp->d_step = d_step;
   sp->d_lr = d_lr;
-  // (1 - beta) formed in double and rounded once
-  sp->b1 = (float)h->beta1;
-  sp->omb1 = (float)(1.0 - h->beta1);
-  sp->b2 = (float)h->beta2;
-  sp->omb2 = (float)(1.0 - h->beta2);
-  sp->eps = (float)h->eps;
-  sp->wd = (float)h->weight_decay;
-  sp->beta1 = h->beta1;
-  sp->beta2 = h->beta2;
-  sp->log2_beta1 = std::log2(h->beta1);   // -inf for beta = 0: beta^t = 0
-  sp->log2_beta2 = std::log2(h->beta2);
-  sp->gamma_l = h->gamma_l;
-  sp->gamma_u = h->gamma_u;
-  sp->trust = h->trust_coef;
-  sp->phi = h->phi;
-  sp->flags = h->flags;
   sp->n_chunks = (int32_t)p->n_chunks;
   sp->grad_slots = p->grad_slots;
   sp->gsq = p->grad_sq;
@@ -590,12 +868,66 @@ static void fill_params(lamb_plan* p, const lamb_hyper_t* h, int64_t* d_step,
   }
 }
 
+// The on-chip kernel runs every step but those with the gradient check or the
+// skip mode (their decision needs all of g before anything is written).
+static bool onchip_takes(const lamb_plan* p, uint32_t flags) {
+  return p->algorithm == LAMB_ALGO_ON_CHIP &&
+         !(flags & (LAMB_FLAG_GRAD_NORM | LAMB_FLAG_SKIP_NONFINITE));
+}
+
+// An on-chip step: the streamed tensors (if any) through the two-pass kernels
+// over their own chunk table, with the closing writes (t + 1, the scheduled
+// eta, the N-LAMB product) left to the on-chip kernel, which runs last.
+// Records an event after each kernel when ev is not NULL; returns the number
+// of kernels launched, or a negated CUDA error.
+static int launch_onchip_step(const lamb_plan* p, const StepParams& sp,
+                              int opt, cudaStream_t stream, cudaEvent_t* ev) {
+  int n = 0, rc = 0;
+  if (p->oc_n_chunks > 0) {
+    StepParams sub = sp;
+    sub.chunks = p->oc_chunks;
+    sub.tensors = p->oc_tensors;
+    sub.n_chunks = (int32_t)p->oc_n_chunks;
+    sub.flags |= kFlagNoClose;
+    const bool lars = opt == 3;
+    rc = lars ? launch_lars_pass1(sub, p->grad_bf16, p->oc_sub_grid[2], stream)
+              : launch_lamb_pass1(sub, opt, p->grad_bf16, p->oc_sub_grid[0],
+                                  stream);
+    if (!rc && ev) rc = (int)cudaEventRecord(ev[++n], stream);
+    else if (!rc) ++n;
+    if (!rc)
+      rc = lars ? launch_lars_pass2(sub, p->grad_bf16, p->copy_bf16,
+                                    p->oc_sub_grid[3], stream)
+                : launch_lamb_pass2(sub, opt, p->grad_bf16, p->copy_bf16,
+                                    p->oc_sub_grid[1], stream);
+    if (!rc && ev) rc = (int)cudaEventRecord(ev[++n], stream);
+    else if (!rc) ++n;
+    if (rc) return -rc;
+  }
+  OcParams q;
+  q.slices = p->oc_slices;
+  q.pieces = p->oc_pieces;
+  q.slots = p->oc_slots;
+  q.bar = p->oc_bar;
+  q.n_rounds = p->oc_n_rounds;
+  q.extra_arrivals = p->oc_extra;
+  q.wait_limit_ns = p->oc_wait_ns;
+  rc = launch_onchip(sp, q, opt, p->grad_bf16, p->copy_bf16, p->oc_grid,
+                     p->oc_rows, stream);
+  if (!rc && ev) rc = (int)cudaEventRecord(ev[++n], stream);
+  else if (!rc) ++n;
+  return rc ? -rc : n;
+}
+
 static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
                               int64_t* d_step, const float* d_lr,
                               cudaStream_t stream, bool lamb) {
   if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
   lamb_status_t st = check_hyper(hyper, lamb);
   if (st != LAMB_OK) return st;
+  if (plan->shard_world > 1)
+    return fail(LAMB_ERR_INVALID_ARG,
+                "a sharded plan steps with lamb_shard_pass1/lamb_shard_pass2");
   if (!plan->bound) return fail(LAMB_ERR_NOT_BOUND, "plan is not bound");
   if (lamb && !plan->has_v)
     return fail(LAMB_ERR_NOT_BOUND, "lamb_step needs v: bind v pointers");
@@ -618,6 +950,13 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
   cudaError_t e = cudaSuccess;
   if (timed) e = cudaEventRecord(ev[0], stream);
   int rc = (int)e;
+  if (onchip_takes(plan, hyper->flags)) {
+    const int n = rc ? -rc : launch_onchip_step(plan, sp, lamb ? 0 : 3, stream,
+                                                 ev);
+    if (n < 0) return cuda_fail((cudaError_t)-n, lamb ? "lamb_step" : "lars_step");
+    if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = (uint8_t)n;
+    return LAMB_OK;
+  }
   // the single-touch kernel implements the plain step; the gradient check,
   // the skip mode and decoupled decay run on the two-pass kernels
   const uint32_t two_pass_only = LAMB_FLAG_GRAD_NORM | LAMB_FLAG_SKIP_NONFINITE |
@@ -677,6 +1016,9 @@ lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
     return fail(LAMB_ERR_INVALID_ARG, "momentum_decay must be finite, >= 0");
   if (nesterov_second_moment != 0 && nesterov_second_moment != 1)
     return fail(LAMB_ERR_INVALID_ARG, "nesterov_second_moment must be 0 or 1");
+  if (plan->shard_world > 1)
+    return fail(LAMB_ERR_INVALID_ARG,
+                "a sharded plan steps with lamb_shard_pass1/lamb_shard_pass2");
   if (!plan->bound) return fail(LAMB_ERR_NOT_BOUND, "plan is not bound");
   if (!plan->has_v)
     return fail(LAMB_ERR_NOT_BOUND, "nlamb_step needs v: bind v pointers");
@@ -697,6 +1039,12 @@ lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
                                           (kKernelsPerStep + 1)]
                           : nullptr;
   int rc = timed ? (int)cudaEventRecord(ev[0], stream) : 0;
+  if (onchip_takes(plan, hyper->flags)) {
+    const int n = rc ? -rc : launch_onchip_step(plan, sp, nest, stream, ev);
+    if (n < 0) return cuda_fail((cudaError_t)-n, "nlamb_step");
+    if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = (uint8_t)n;
+    return LAMB_OK;
+  }
   if (!rc)
     rc = launch_lamb_pass1(sp, nest, plan->grad_bf16, plan->grid[0], stream);
   if (!rc && timed) rc = (int)cudaEventRecord(ev[1], stream);
@@ -706,6 +1054,132 @@ lamb_status_t nlamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
   if (!rc && timed) rc = (int)cudaEventRecord(ev[2], stream);
   if (rc) return cuda_fail((cudaError_t)rc, "nlamb_step");
   if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = 2;
+  return LAMB_OK;
+}
+
+// Shared checks and parameters of the two halves of a sharded step.
+static lamb_status_t shard_params(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                                  int32_t optimizer, double momentum_decay,
+                                  int64_t* d_step, const float* d_lr,
+                                  double* d_mu_product, StepParams* sp) {
+  if (!plan) return fail(LAMB_ERR_INVALID_ARG, "plan is NULL");
+  if (optimizer < LAMB_OPT_LAMB || optimizer > LAMB_OPT_NNLAMB)
+    return fail(LAMB_ERR_INVALID_ARG, "unknown optimizer %d", optimizer);
+  const bool lars = optimizer == LAMB_OPT_LARS;
+  const bool nest = optimizer >= LAMB_OPT_NLAMB;
+  lamb_status_t st = check_hyper(hyper, !lars);
+  if (st != LAMB_OK) return st;
+  if (hyper->flags & (LAMB_FLAG_GRAD_NORM | LAMB_FLAG_SKIP_NONFINITE))
+    return fail(LAMB_ERR_INVALID_ARG,
+                "a sharded step takes neither GRAD_NORM nor SKIP_NONFINITE");
+  if (!plan->bound) return fail(LAMB_ERR_NOT_BOUND, "plan is not bound");
+  if (!lars && !plan->has_v)
+    return fail(LAMB_ERR_NOT_BOUND, "this optimizer needs v: bind v pointers");
+  const bool sched = (hyper->flags & LAMB_FLAG_LR_SCHEDULE) != 0;
+  if (!d_lr && !sched) return fail(LAMB_ERR_INVALID_ARG, "d_lr is NULL");
+  const bool needs_step =
+      (hyper->flags & LAMB_FLAG_INCREMENT_STEP) || sched || nest ||
+      (!lars && (hyper->flags & LAMB_FLAG_BIAS_CORRECTION));
+  if (needs_step && !d_step)
+    return fail(LAMB_ERR_INVALID_ARG, "d_step is NULL but the step needs it");
+  if (nest && !(momentum_decay >= 0.0 && std::isfinite(momentum_decay)))
+    return fail(LAMB_ERR_INVALID_ARG, "momentum_decay must be finite, >= 0");
+  if (nest && !d_mu_product)
+    return fail(LAMB_ERR_INVALID_ARG, "N-LAMB needs d_mu_product");
+  fill_params(plan, hyper, d_step, d_lr, sp);
+  if (nest) {
+    sp->psi = momentum_decay;
+    sp->log2_mu_decay = momentum_decay * std::log2(0.96);
+    sp->d_mu_product = d_mu_product;
+  }
+  // this shard's chunks; the slots keep their global chunk index
+  sp->chunks = plan->chunks + plan->shard_cb;
+  sp->slots = plan->slots + plan->shard_cb;
+  sp->n_chunks = (int32_t)(plan->shard_ce - plan->shard_cb);
+  return LAMB_OK;
+}
+
+static int shard_grid(const lamb_plan* p, int which) {
+  const int64_t n = p->shard_ce - p->shard_cb;
+  const int g = p->grid[which];
+  return n < 1 ? 1 : (n < g ? (int)n : g);
+}
+
+lamb_status_t lamb_shard_pass1(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                               int32_t optimizer, double momentum_decay,
+                               int64_t* d_step, const float* d_lr,
+                               double* d_mu_product, cudaStream_t stream) {
+  StepParams sp;
+  lamb_status_t st = shard_params(plan, hyper, optimizer, momentum_decay,
+                                  d_step, d_lr, d_mu_product, &sp);
+  if (st != LAMB_OK) return st;
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  sp.flags |= kFlagNoFinalize;
+  // every slot starts at zero, so that a sum over the ranks' arrays is exact
+  cudaError_t e = cudaMemsetAsync(plan->slots, 0,
+                                  (size_t)plan->n_chunks * sizeof(float2),
+                                  stream);
+  int rc = (int)e;
+  if (!rc)
+    rc = optimizer == LAMB_OPT_LARS
+             ? launch_lars_pass1(sp, plan->grad_bf16, shard_grid(plan, 2),
+                                 stream)
+             : launch_lamb_pass1(sp, optimizer - (optimizer >= 2 ? 1 : 0),
+                                 plan->grad_bf16, shard_grid(plan, 0), stream);
+  if (rc) return cuda_fail((cudaError_t)rc, "lamb_shard_pass1");
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_shard_pass2(lamb_plan_t plan, const lamb_hyper_t* hyper,
+                               int32_t optimizer, double momentum_decay,
+                               int64_t* d_step, const float* d_lr,
+                               double* d_mu_product, cudaStream_t stream) {
+  StepParams sp;
+  lamb_status_t st = shard_params(plan, hyper, optimizer, momentum_decay,
+                                  d_step, d_lr, d_mu_product, &sp);
+  if (st != LAMB_OK) return st;
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  const bool lars = optimizer == LAMB_OPT_LARS;
+  StepParams all = sp;   // the finaliser reads every tensor's slots
+  all.chunks = plan->chunks;
+  all.slots = plan->slots;
+  all.n_chunks = (int32_t)plan->n_chunks;
+  int rc = launch_finalize_all(all, lars ? hyper->trust_coef : 1.0, stream);
+  if (!rc)
+    rc = lars ? launch_lars_pass2(sp, plan->grad_bf16, plan->copy_bf16,
+                                  shard_grid(plan, 3), stream)
+              : launch_lamb_pass2(sp, optimizer - (optimizer >= 2 ? 1 : 0),
+                                  plan->grad_bf16, plan->copy_bf16,
+                                  shard_grid(plan, 1), stream);
+  if (rc) return cuda_fail((cudaError_t)rc, "lamb_shard_pass2");
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_partials(lamb_plan_t plan, float** d_partials,
+                                 int64_t* n_floats) {
+  if (!plan || !d_partials || !n_floats)
+    return fail(LAMB_ERR_INVALID_ARG, "NULL argument");
+  *d_partials = reinterpret_cast<float*>(plan->slots);
+  *n_floats = 2 * plan->n_chunks;
+  return LAMB_OK;
+}
+
+lamb_status_t lamb_plan_copy_partials(lamb_plan_t plan, float* buf,
+                                      int32_t to_plan, cudaStream_t stream) {
+  if (!plan || !buf) return fail(LAMB_ERR_INVALID_ARG, "NULL argument");
+  if (to_plan != 0 && to_plan != 1)
+    return fail(LAMB_ERR_INVALID_ARG, "to_plan must be 0 or 1");
+  DeviceGuard guard(plan->device);
+  if (guard.err != cudaSuccess) return cuda_fail(guard.err, "cudaSetDevice");
+  const size_t bytes = (size_t)plan->n_chunks * sizeof(float2);
+  const cudaError_t e =
+      to_plan ? cudaMemcpyAsync(plan->slots, buf, bytes, cudaMemcpyDefault,
+                                stream)
+              : cudaMemcpyAsync(buf, plan->slots, bytes, cudaMemcpyDefault,
+                                stream);
+  if (e != cudaSuccess) return cuda_fail(e, "partials copy");
   return LAMB_OK;
 }
 
@@ -809,6 +1283,19 @@ lamb_status_t lamb_plan_get_info(lamb_plan_t plan, lamb_plan_info_t* info) {
   info->l2_budget_bytes = plan->l2_budget;
   if (plan->algorithm == LAMB_ALGO_SINGLE_TOUCH)
     info->grid_blocks = plan->grid_fused[0];
+  if (plan->algorithm == LAMB_ALGO_ON_CHIP) {
+    info->grid_blocks = plan->oc_grid;
+    info->threads_per_block = kOcThreads;
+  }
+  info->n_rounds = plan->oc_n_rounds;
+  info->n_streamed_tensors = plan->oc_n_streamed;
+  info->rows_per_cta = plan->oc_rows;
+  info->tail_elems = plan->tail_elems;
+  info->shard_world = plan->shard_world;
+  info->shard_rank = plan->shard_rank;
+  info->shard_chunk_begin = plan->shard_cb;
+  info->shard_chunk_end = plan->shard_ce;
+  info->row_elems = kOcRow;
   return LAMB_OK;
 }
 

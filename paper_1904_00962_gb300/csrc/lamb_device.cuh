@@ -134,6 +134,7 @@ __device__ __forceinline__ float step_lr(const StepParams& p, int64_t t) {
 // the scheduled learning rate.
 __device__ __forceinline__ void close_step(const StepParams& p,
                                            const StepScalars& sc) {
+  if (p.flags & kFlagNoClose) return;
   if ((p.flags & kFlagLrSchedule) && p.d_lr_out) *p.d_lr_out = sc.lr;
   if ((p.flags & kFlagIncrementStep) && p.d_step) *p.d_step = sc.t + 1;
 }
@@ -151,6 +152,101 @@ __device__ __forceinline__ double phi_of(double z, const StepParams& p) {
     if (z > p.gamma_u) return p.gamma_u;
   }
   return z;
+}
+
+// Nadam momentum schedule term (appendix Alg. 3 inputs): mu_t =
+// beta1 (1 - 0.5 * 0.96^(t psi)).
+__device__ __forceinline__ double nadam_mu(const StepParams& p, int64_t t) {
+  return p.beta1 * (1.0 - 0.5 * pow_from_log2(p.log2_mu_decay, (double)t));
+}
+
+// Per-launch constants of a LAMB / N-LAMB step (Alg. 2 bias correction, the
+// appendix Algs. 3/4 momentum schedule).  The fp64 work is spread over the
+// lane 0 of warps 0-3 (one power each, with the divisions that need only it)
+// while warp 4 draws the first chunk (kDraw: a pass 1 that takes work from
+// counters[0]) and warp 5 fetches the N-LAMB product; thread 0 then forms the
+// rest.  The results do not depend on the split.  CTA 0 stores them in
+// *p.scal; s_t (optional) receives the step count t.
+template <int kNest, bool kDraw>
+__device__ __forceinline__ void step_constants(const StepParams& p,
+                                               uint32_t* s_next, int* s_skip,
+                                               LambConsts* s_k,
+                                               int64_t* s_t_out) {
+  __shared__ double s_x[3];     // mu_t, mu_{t+1}, prod_{i<t} mu_i
+  __shared__ float s_c[2];      // c1, c2 (LAMB) or bv, bg (N-LAMB)
+  __shared__ int64_t s_t;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool bc = kNest != 0 || (p.flags & kFlagBiasCorrection) != 0;
+  if (lane == 0 && warp < 6) {
+    const int64_t t = p.d_step ? *p.d_step : int64_t(1);
+    const bool skip = bc && t < 1;
+    const double td = (double)t;
+    if (warp == 0) {
+      *s_skip = skip ? 1 : 0;
+      s_t = t;
+    }
+    if (!skip) {
+      if (warp == 4) {
+        if (kDraw) s_next[0] = atomicAdd(&p.counters[0], 1u);
+      } else if (!kNest) {
+        if (warp < 2)   // Alg. 2 bias correction: 1/(1 - beta^t)
+          s_c[warp] = !bc ? 1.f
+                          : (float)(1.0 / (1.0 - pow_from_log2(
+                                warp == 0 ? p.log2_beta1 : p.log2_beta2, td)));
+      } else if (warp < 2) {           // appendix Alg. 3/4: mu_t, mu_{t+1}
+        s_x[warp] = nadam_mu(p, t + warp);
+      } else if (warp == 2) {          // v_hat's correction at t
+        const double b = pow_from_log2(p.log2_beta2, td);
+        if (kNest == 2) s_c[1] = (float)((1.0 - p.beta2) / (1.0 - b));
+        else s_c[0] = (float)(1.0 / (1.0 - b));
+      } else if (warp == 3) {          // NN-LAMB: beta2 / (1 - beta2^(t+1))
+        if (kNest == 2)
+          s_c[0] = (float)(p.beta2 /
+                           (1.0 - pow_from_log2(p.log2_beta2, td + 1.0)));
+      } else if (kNest) {              // warp 5
+        s_x[2] = *p.d_mu_product;
+      }
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int64_t t = s_t;
+    const int skip = *s_skip;
+    LambConsts kc{p.b1, p.omb1, p.b2, p.omb2, 1.f, 1.f, p.eps,
+                  0.f, 0.f, 0.f, 0.f};
+    double mu_prod = 0.0;
+    if (!skip) {
+      if (!kNest) {
+        kc.c1 = s_c[0];
+        kc.c2 = s_c[1];
+      } else {
+        const double mu_t = s_x[0], mu_n = s_x[1];
+        mu_prod = s_x[2] * mu_t;
+        kc.am = (float)(mu_n / (1.0 - mu_prod * mu_n));
+        kc.ag = (float)((1.0 - mu_t) / (1.0 - mu_prod));
+        kc.bv = s_c[0];
+        kc.bg = kNest == 2 ? s_c[1] : 0.f;
+      }
+    }
+    *s_k = kc;
+    if (s_t_out) *s_t_out = t;
+    if (blockIdx.x == 0) {
+      StepScalars sc{};
+      sc.t = t;
+      sc.c1 = kc.c1;
+      sc.c2 = kc.c2;
+      sc.lr = step_lr(p, t);
+      sc.skip = skip;
+      sc.am = kc.am;
+      sc.ag = kc.ag;
+      sc.bv = kc.bv;
+      sc.bg = kc.bg;
+      sc.mu_prod = mu_prod;
+      *p.scal = sc;
+      if (skip) atomicOr(p.status, kStatusBadStep);
+    }
+  }
+  __syncthreads();
 }
 
 }  // namespace

@@ -19,6 +19,8 @@
 
 #include <vector>
 
+#include "lamb.h"
+
 namespace lamb {
 
 constexpr int kDefaultChunk = 16384;
@@ -68,7 +70,13 @@ enum : uint32_t { kStatusNonfinite = 1u, kStatusBadStep = 2u,
                   kStatusSkipped = 16u };
 enum : uint32_t { kFlagBiasCorrection = 1u, kFlagIncrementStep = 2u,
                   kFlagLrSchedule = 4u, kFlagGradNorm = 8u,
-                  kFlagSkipNonfinite = 16u, kFlagDecoupledDecay = 32u };
+                  kFlagSkipNonfinite = 16u, kFlagDecoupledDecay = 32u,
+                  // internal: a launch that is not the step's last leaves
+                  // t, the scheduled eta and the N-LAMB product alone
+                  kFlagNoClose = 1u << 30,
+                  // internal: pass 1 of a shard stores its chunk sums and
+                  // finalises nothing (the sums are exchanged first)
+                  kFlagNoFinalize = 1u << 29 };
 
 // Gradient check of one step (kFlagGradNorm / kFlagSkipNonfinite).  Pass 1
 // forms it; pass 2 reads the decision before it writes anything.
@@ -168,6 +176,90 @@ struct FusedParams {
   int32_t n_items;
 };
 
+// ---------------------------------------------------------------------------
+// On-chip single-touch step (lamb_onchip.cu): one cooperative launch per step,
+// one CTA per SM.  The tensors are cut into rounds: runs of whole tensors whose
+// elements fit the grid's shared memory.  Every CTA owns a fixed slice of a
+// round's rows (kOcRow elements each), keeps w and the update direction of its
+// rows in shared memory across a grid barrier, and writes the new w from
+// there.  A tensor too large for one round is "streamed": the two-pass kernels
+// take it, over a chunk table of such tensors only, before the on-chip launch.
+// ---------------------------------------------------------------------------
+constexpr int kOcThreads = 768;
+constexpr int kOcWarps = kOcThreads / 32;
+constexpr int kOcRow = 128;          // elements per row: one float4 per lane
+constexpr int kOcMaxPieces = 16;     // pieces per CTA and round
+constexpr int kOcMaxRows = 224;      // rows per CTA (the plan may use fewer)
+constexpr int kOcRowBytes = 2 * kOcRow * 4;   // w and u of a row, fp32
+
+enum : uint32_t { kOcVec = 1u,       // arrays aligned for 4-element access
+                  kOcExport = 2u };  // this piece's CTA writes rho_k, norms
+
+// A piece: the rows of one tensor inside one CTA's slice of a round.  Pointers
+// are filled in by bind.
+struct __align__(16) OcPiece {
+  float* w;
+  const void* g;
+  float* m;
+  float* v;
+  void* copy;
+  int64_t offset;     // element of the tensor at the piece's first row
+  int32_t len;        // elements of the piece
+  int32_t tensor;
+  int32_t slot;       // this piece's partial-sum slot
+  int32_t t_slot;     // the tensor's first slot
+  int32_t t_nslots;   // the tensor's slots, combined in this order
+  int16_t first_row;  // CTA-local row where the piece starts
+  int16_t n_rows;
+  float decay;        // 1.0f: weight decay applies
+  uint32_t flags;     // kOcVec | kOcExport
+};
+static_assert(sizeof(OcPiece) == 80, "OcPiece layout");
+
+struct __align__(8) OcSlice {   // one CTA's part of a resident round
+  int32_t piece_begin;
+  int16_t n_pieces;
+  int16_t n_rows;
+};
+
+// Words of the plan's barrier block (uint32 indices; each group on its own
+// 128-byte line)
+constexpr int kBarCount = 0;     // arrivals at the current grid barrier
+constexpr int kBarGen = 32;      // barrier generation
+constexpr int kBarAbort = 33;    // a wait gave up: the plan is unusable
+constexpr int kBarWords = 64;
+
+struct OcParams {
+  const OcSlice* slices;  // [n_rounds][grid]
+  const OcPiece* pieces;
+  float4* slots;          // per piece: sum w^2 and sum u^2, each as a
+                          // two-float value (hi, lo)
+  uint32_t* bar;          // kBarWords words, see kBar*
+  int32_t n_rounds;
+  int32_t extra_arrivals; // > 0 only in tests of the give-up path
+  int64_t wait_limit_ns;  // a barrier wait gives up after this long
+};
+
+// Host planner of the on-chip step (planner.cpp).  grid CTAs, rows_per_cta
+// rows of shared memory each.  Pieces come back without pointers; streamed
+// receives the tensors too large for a round, in order.
+int plan_onchip(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
+                int32_t grid, int32_t rows_per_cta, int32_t* n_rounds,
+                std::vector<OcSlice>* slices, std::vector<OcPiece>* pieces,
+                std::vector<int32_t>* streamed, int64_t* n_slots, char* err,
+                int errlen);
+// CTAs of the on-chip grid for a layout of total_rows rows (at least 32 rows
+// per CTA, at most num_sms).
+int32_t onchip_grid(int64_t total_rows, int32_t num_sms);
+
+// Launcher (lamb_onchip.cu): opt 0 LAMB, 1 N-LAMB, 2 NN-LAMB, 3 LARS.
+int launch_onchip(const StepParams& p, const OcParams& q, int opt,
+                  int grad_bf16, int copy_bf16, int grid, int rows_per_cta,
+                  void* stream);
+// Rows of shared memory a CTA can hold on `device`, after the kernels' static
+// shared memory; also raises the kernels' dynamic shared-memory limit.
+int onchip_prepare(int device, int* rows_per_cta);
+
 // Launchers (lamb_kernels.cu).  grid = number of CTAs of the persistent grid.
 // Return cudaError_t as int to keep this header free of CUDA includes.
 // nest: 0 LAMB, 1 N-LAMB, 2 NN-LAMB.  The gradient-check and deferred-moment
@@ -180,6 +272,14 @@ int launch_lars_pass1(const StepParams& p, int grad_bf16, int grid,
                       void* stream);
 int launch_lars_pass2(const StepParams& p, int grad_bf16, int copy_bf16,
                       int grid, void* stream);
+// Every tensor's rho_k and norms from the complete chunk slots (coef: 1 for
+// LAMB, kappa for LARS).
+int launch_finalize_all(const StepParams& p, double coef, void* stream);
+// Chunk range [*begin, *end) of shard `rank` of `world`: contiguous ranges
+// of the chunk table with about equal elements, cut at chunk boundaries
+// (planner.cpp).
+void shard_range(const ChunkDesc* chunks, int64_t n_chunks, int32_t world,
+                 int32_t rank, int64_t* begin, int64_t* end);
 int launch_fused(const StepParams& p, const FusedParams& f, int lars,
                  int grad_bf16, int copy_bf16, int grid, void* stream);
 int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks);
@@ -188,6 +288,10 @@ int occupancy_lamb_pass1(int grad_bf16, int* blocks);
 int occupancy_lamb_pass2(int copy_bf16, int* blocks);
 int occupancy_lars_pass1(int grad_bf16, int* blocks);
 int occupancy_lars_pass2(int copy_bf16, int* blocks);
+
+// The hyperparameter-derived fields of a StepParams (lamb_capi.cu): betas,
+// their complements and log2s, eps, lambda, phi and its bounds, kappa, flags.
+void fill_hyper(const lamb_hyper_t& h, StepParams* sp);
 
 // Sets the thread-local message returned by lamb_last_error() (lamb_capi.cu).
 void set_last_error(const char* msg);
@@ -201,9 +305,12 @@ int plan_fused(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
                std::vector<uint32_t>* items, char* err, int errlen);
 
 // Host planner (planner.cpp).  Returns 0 on success, else writes a message.
+// Within tail_elems of either end of the layout the chunks hold tail_chunk
+// elements (0: no tail).
 int plan_chunks(const int64_t* sizes, int32_t n, int32_t chunk_elems,
                 ChunkDesc* chunks, int64_t capacity, int64_t* n_chunks,
                 TensorDesc* tensors, const uint8_t* decay_mask, char* err,
-                int errlen);
+                int errlen, int64_t tail_elems = 0, int32_t tail_chunk = 0);
+constexpr int kTailChunk = 2048;   // elements per chunk near the layout's ends
 
 }  // namespace lamb

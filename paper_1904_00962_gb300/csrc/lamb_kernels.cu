@@ -159,9 +159,13 @@ __device__ __forceinline__ void publish_chunk(const StepParams& p, int c,
   if (threadIdx.x == 0) {
     p.slots[c] = make_float2(acc[0], acc[1]);
     if (kGn) p.grad_slots[c] = make_float2(acc[2], acc[3]);
-    __threadfence();
-    const uint32_t prev = atomicAdd(&p.tickets[ch.tensor], 1u);
-    *s_last = (prev + 1u == (uint32_t)td.n_chunks);
+    if (p.flags & kFlagNoFinalize) {   // a shard: the sums are exchanged first
+      *s_last = 0;
+    } else {
+      __threadfence();
+      const uint32_t prev = atomicAdd(&p.tickets[ch.tensor], 1u);
+      *s_last = (prev + 1u == (uint32_t)td.n_chunks);
+    }
   }
   __syncthreads();
   if (*s_last && threadIdx.x < 32)
@@ -256,101 +260,11 @@ __device__ __forceinline__ void lamb1_chunk(const TensorPtrs& tp,
   }
 }
 
-// Nadam momentum schedule term (appendix Alg. 3 inputs): mu_t =
-// beta1 (1 - 0.5 * 0.96^(t psi)).
-__device__ __forceinline__ double nadam_mu(const StepParams& p, int64_t t) {
-  return p.beta1 * (1.0 - 0.5 * pow_from_log2(p.log2_mu_decay, (double)t));
-}
-
 // lambda_k inside the normalised direction u (Alg. 2); 0 with decoupled
 // decay, where pass 2 applies lambda_k w outside the trust ratio instead.
 __device__ __forceinline__ float lam_in_u(const StepParams& p,
                                           const TensorDesc& td) {
   return (p.flags & kFlagDecoupledDecay) ? 0.f : td.decay * p.wd;
-}
-
-// Per-launch constants of pass 1.  The fp64 work is spread over the lane 0
-// of warps 0-3 (one power each, with the divisions that need only it) while
-// warp 4 draws the first chunk and warp 5 fetches the N-LAMB product; thread
-// 0 then forms the rest.  The results do not depend on the split.
-template <int kNest>
-__device__ __forceinline__ void pass1_constants(const StepParams& p,
-                                                uint32_t* s_next, int* s_skip,
-                                                LambConsts* s_k) {
-  __shared__ double s_x[3];     // mu_t, mu_{t+1}, prod_{i<t} mu_i
-  __shared__ float s_c[2];      // c1, c2 (LAMB) or bv, bg (N-LAMB)
-  __shared__ int64_t s_t;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool bc = kNest != 0 || (p.flags & kFlagBiasCorrection) != 0;
-  if (lane == 0 && warp < 6) {
-    const int64_t t = p.d_step ? *p.d_step : int64_t(1);
-    const bool skip = bc && t < 1;
-    const double td = (double)t;
-    if (warp == 0) {
-      *s_skip = skip ? 1 : 0;
-      s_t = t;
-    }
-    if (!skip) {
-      if (warp == 4) {
-        s_next[0] = atomicAdd(&p.counters[0], 1u);
-      } else if (!kNest) {
-        if (warp < 2)   // Alg. 2 bias correction: 1/(1 - beta^t)
-          s_c[warp] = !bc ? 1.f
-                          : (float)(1.0 / (1.0 - pow_from_log2(
-                                warp == 0 ? p.log2_beta1 : p.log2_beta2, td)));
-      } else if (warp < 2) {           // appendix Alg. 3/4: mu_t, mu_{t+1}
-        s_x[warp] = nadam_mu(p, t + warp);
-      } else if (warp == 2) {          // v_hat's correction at t
-        const double b = pow_from_log2(p.log2_beta2, td);
-        if (kNest == 2) s_c[1] = (float)((1.0 - p.beta2) / (1.0 - b));
-        else s_c[0] = (float)(1.0 / (1.0 - b));
-      } else if (warp == 3) {          // NN-LAMB: beta2 / (1 - beta2^(t+1))
-        if (kNest == 2)
-          s_c[0] = (float)(p.beta2 /
-                           (1.0 - pow_from_log2(p.log2_beta2, td + 1.0)));
-      } else if (kNest) {              // warp 5
-        s_x[2] = *p.d_mu_product;
-      }
-    }
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const int64_t t = s_t;
-    const int skip = *s_skip;
-    LambConsts kc{p.b1, p.omb1, p.b2, p.omb2, 1.f, 1.f, p.eps,
-                  0.f, 0.f, 0.f, 0.f};
-    double mu_prod = 0.0;
-    if (!skip) {
-      if (!kNest) {
-        kc.c1 = s_c[0];
-        kc.c2 = s_c[1];
-      } else {
-        const double mu_t = s_x[0], mu_n = s_x[1];
-        mu_prod = s_x[2] * mu_t;
-        kc.am = (float)(mu_n / (1.0 - mu_prod * mu_n));
-        kc.ag = (float)((1.0 - mu_t) / (1.0 - mu_prod));
-        kc.bv = s_c[0];
-        kc.bg = kNest == 2 ? s_c[1] : 0.f;
-      }
-    }
-    *s_k = kc;
-    if (blockIdx.x == 0) {
-      StepScalars sc{};
-      sc.t = t;
-      sc.c1 = kc.c1;
-      sc.c2 = kc.c2;
-      sc.lr = step_lr(p, t);
-      sc.skip = skip;
-      sc.am = kc.am;
-      sc.ag = kc.ag;
-      sc.bv = kc.bv;
-      sc.bg = kc.bg;
-      sc.mu_prod = mu_prod;
-      *p.scal = sc;
-      if (skip) atomicOr(p.status, kStatusBadStep);
-    }
-  }
-  __syncthreads();
 }
 
 template <typename GT, int kNest, bool kGn>
@@ -360,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks1)
   __shared__ uint32_t s_next[2];
   __shared__ int s_last, s_skip;
   __shared__ LambConsts s_k;
-  pass1_constants<kNest>(p, s_next, &s_skip, &s_k);
+  step_constants<kNest, true>(p, s_next, &s_skip, &s_k, nullptr);
   if (s_skip) return;
   const LambConsts k = s_k;
   const bool store = !(kGn && (p.flags & kFlagSkipNonfinite));
@@ -502,7 +416,8 @@ __global__ void __launch_bounds__(kThreads)
     c = s_next[it & 1];
   }
   if (retire(p, 1, c) && threadIdx.x == 0) {
-    if (kNest && p.d_mu_product) *p.d_mu_product = sc.mu_prod;
+    if (kNest && p.d_mu_product && !(p.flags & kFlagNoClose))
+      *p.d_mu_product = sc.mu_prod;
     close_step(p, sc);
   }
 }
@@ -689,6 +604,21 @@ __global__ void __launch_bounds__(kThreads)
   if (retire(p, 1, c) && threadIdx.x == 0) close_step(p, sc);
 }
 
+// Every tensor's norms and trust ratio from the complete chunk slots (a
+// sharded step, after the slots were exchanged): one warp per tensor, the
+// same fixed-order combine as the finaliser of pass 1, so the results equal
+// an unsharded step's bit for bit.
+__global__ void __launch_bounds__(kThreads)
+    finalize_all_kernel(const StepParams p, double coef) {
+  const int warps = (int)(gridDim.x * blockDim.x) >> 5;
+  for (int k = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+       k < p.n_tensors; k += warps) {
+    const TensorDesc td = p.tensors[k];
+    if (td.n_chunks > 0)
+      finalize_tensor<false>(p, k, td.first_chunk, td.n_chunks, coef);
+  }
+}
+
 template <typename K>
 int occupancy_of(K kernel, int* blocks) {
   return (int)cudaOccupancyMaxActiveBlocksPerMultiprocessor(blocks, kernel,
@@ -785,6 +715,14 @@ int launch_lars_pass2(const StepParams& p, int grad_bf16, int copy_bf16,
     case 2: return lars_p2<false, __nv_bfloat16>(p, grid, s);
     default: return lars_p2<true, __nv_bfloat16>(p, grid, s);
   }
+}
+
+int launch_finalize_all(const StepParams& p, double coef, void* stream) {
+  const int warps_per_block = kThreads / 32;
+  const int grid = (p.n_tensors + warps_per_block - 1) / warps_per_block;
+  finalize_all_kernel<<<grid < 1 ? 1 : grid, kThreads, 0,
+                        static_cast<cudaStream_t>(stream)>>>(p, coef);
+  return (int)cudaGetLastError();
 }
 
 int occupancy_lamb_pass1(int grad_bf16, int* blocks) {

@@ -107,8 +107,10 @@ cudaError_t na_setup(int dev, NaDevice** out) {
 // ---- set-up kernel: builds the tables inside the scratch array -------------
 // One CTA of 1024 threads.  Reads the per-tensor sizes, mask and pointer
 // arrays the host copied into the scratch, and writes the tensor table,
-// pointer table (with the 128-bit alignment flag), chunk table, tickets,
-// default results (ratio 1, norms 0), status and work counters.
+// pointer table (with the 128-bit alignment flag), tickets, default results
+// (ratio 1, norms 0), status and work counters; then every thread writes
+// every 1024th chunk of the chunk table, finding its tensor by a binary
+// search over the tensors' first chunks.
 constexpr int kSetupThreads = 1024;
 constexpr int kPerThread = kNaMaxTensors / kSetupThreads;   // 4
 
@@ -172,15 +174,6 @@ __global__ void __launch_bounds__(kSetupThreads)
                     (!tp.copy || (uintptr_t)tp.copy % 8 == 0);
     tp.vec_ok = ok ? 1u : 0u;
     ptrs[k] = tp;
-    for (int64_t j = 0; j < local[i]; ++j) {
-      const int64_t off = j * kNaChunk;
-      const int64_t rem = d - off;
-      ChunkDesc c;
-      c.offset = off;
-      c.tensor = k;
-      c.len = (int32_t)(rem < kNaChunk ? rem : kNaChunk);
-      chunks[first + j] = c;
-    }
     first += local[i];
     tickets[k] = 0u;
     ratio[k] = 1.0;
@@ -190,6 +183,25 @@ __global__ void __launch_bounds__(kSetupThreads)
   if (t == 0) {
     *status = 0u;
     counters[0] = counters[1] = counters[2] = counters[3] = 0u;
+  }
+  __syncthreads();   // the tensor table is complete
+  const int64_t n_chunks = part[kSetupThreads - 1];
+  for (int64_t c = t; c < n_chunks; c += kSetupThreads) {
+    // the last tensor whose first chunk is <= c (a 0-chunk tensor shares its
+    // first chunk with the next one, which comes later and wins)
+    int lo = 0, hi = n - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) / 2;
+      if (tens[mid].first_chunk <= c) lo = mid;
+      else hi = mid - 1;
+    }
+    const int64_t off = (c - tens[lo].first_chunk) * kNaChunk;
+    const int64_t rem = tens[lo].numel - off;
+    ChunkDesc cd;
+    cd.offset = off;
+    cd.tensor = lo;
+    cd.len = (int32_t)(rem < kNaChunk ? rem : kNaChunk);
+    chunks[c] = cd;
   }
 }
 
@@ -239,6 +251,11 @@ extern "C" LAMB_API lamb_status_t lamb_step_noalloc(
     if (d < 0)
       return na_fail(LAMB_ERR_INVALID_ARG,
                      "lamb_step_noalloc: sizes[%d] is negative", k);
+    if (d > (int64_t)kNaMaxChunks * kNaChunk)   // before any rounding sum
+      return na_fail(LAMB_ERR_INVALID_ARG,
+                     "lamb_step_noalloc: sizes[%d] = %lld exceeds the %lld "
+                     "parameters the scratch holds", k, (long long)d,
+                     (long long)kNaMaxChunks * kNaChunk);
     n_chunks += (d + kNaChunk - 1) / kNaChunk;
     if (n_chunks > kNaMaxChunks)
       return na_fail(LAMB_ERR_INVALID_ARG,
@@ -295,8 +312,12 @@ extern "C" LAMB_API lamb_status_t lamb_step_noalloc(
                    cudaGetErrorString(e));
 
   // ---- the two LAMB passes on tables inside the scratch --------------------
+  // The flags check above admits BIAS_CORRECTION and INCREMENT_STEP only:
+  // the fields of the schedule, the gradient check and the N-LAMB product
+  // stay zero / NULL here, which is what those two flags need.
   StepParams sp;
   std::memset(&sp, 0, sizeof(sp));
+  fill_hyper(h, &sp);
   sp.chunks = reinterpret_cast<const ChunkDesc*>(s + kOffChunks);
   sp.tensors = reinterpret_cast<const TensorDesc*>(s + kOffTensors);
   sp.ptrs = reinterpret_cast<const TensorPtrs*>(s + kOffPtrs);
@@ -310,21 +331,6 @@ extern "C" LAMB_API lamb_status_t lamb_step_noalloc(
   sp.status = reinterpret_cast<uint32_t*>(s + kOffStatus);
   sp.d_step = d_step;
   sp.d_lr = d_lr;
-  sp.b1 = (float)h.beta1;
-  sp.omb1 = (float)(1.0 - h.beta1);
-  sp.b2 = (float)h.beta2;
-  sp.omb2 = (float)(1.0 - h.beta2);
-  sp.eps = (float)h.eps;
-  sp.wd = (float)h.weight_decay;
-  sp.beta1 = h.beta1;
-  sp.beta2 = h.beta2;
-  sp.log2_beta1 = std::log2(h.beta1);
-  sp.log2_beta2 = std::log2(h.beta2);
-  sp.gamma_l = h.gamma_l;
-  sp.gamma_u = h.gamma_u;
-  sp.trust = h.trust_coef;
-  sp.phi = h.phi;
-  sp.flags = h.flags;
   sp.n_chunks = (int32_t)n_chunks;
   const int gbf = grad_dtype == LAMB_BF16 ? 1 : 0;
   auto grid_of = [&](int occ) {

@@ -1,0 +1,770 @@
+// sm_103a kernel of the on-chip single-touch LAMB / LARS step.
+//
+// Algorithm 2 needs ||w_k|| and ||u_k|| (u = r + lambda_k w) of a WHOLE tensor
+// before any of its elements may change.  The two-pass kernels therefore read
+// m, v, w twice from HBM (40 B per parameter with bf16 g and a bf16 copy).
+// This kernel reads and writes every operand once (28 B per parameter) by
+// keeping, between the two halves of the step, each element's w and u in the
+// shared memory of the SM that formed them.
+//
+// One cooperative launch per step: one CTA per SM (all resident at once),
+// 512 threads, ~223 KB of shared memory holding up to 223 rows of 128
+// elements (w and u in fp32, 1 KB per row).  The host planner (planner.cpp,
+// plan_onchip) cuts the tensors into ROUNDS of consecutive whole tensors
+// whose rows fit the grid (~4.3M parameters on 152 SMs).  Each CTA owns a
+// fixed slice of a round's rows, in pieces (a piece = the rows of one tensor
+// in one CTA, at most 16 per CTA); warp w takes rows w, w + 16, ...  Per
+// round:
+//
+//   pass 1   each warp keeps 2 x kPairs rows in flight: w and m of a row are
+//            copied (cp.async) straight into the row's shared-memory slot, g
+//            and v into registers.  For each arrived row: the new m, v (Alg. 2
+//            moment lines; Alg. 1 momentum for LARS) go back to HBM, u
+//            replaces m in the slot, and the warp's fixed-tree fp32 sums of
+//            w^2 and u^2 are kept per row; per piece, the row sums are added
+//            in row order (compensated two-float sums) into the piece's slot.
+//   barrier  grid-wide
+//   ratio    every CTA adds the slots of each of its tensors in slot order
+//            (two-float) and forms rho_k = phi(||w||)/||u|| in fp32 (1 on a
+//            zero norm; LARS: kappa phi(||w||)/||m||); the CTA holding the
+//            tensor's first piece exports rho_k and the norms.
+//   pass 2   w <- w - eta rho_k u from shared memory (+ the bf16 copy): no HBM
+//            reads at all.
+//
+// The reductions avoid fp64: GB300 issues fp64 at a small fraction of its
+// fp32 rate, and the compensated two-float sums keep ~44 bits.
+//
+// A tensor with more rows than the grid holds (BERT's 30522 x 1024 word
+// embedding) is not the kernel's: the two-pass kernels update it, over a chunk
+// table of such tensors only, before this launch.
+//
+// The partial sums have a fixed shape given by the plan, so the result does
+// not depend on timing: every run is bitwise identical.  The element
+// arithmetic is the two-pass kernels' (lamb_device.cuh), so m, v and u are
+// bit-identical to theirs; only the summation of the norms differs.
+//
+// The barrier is a generation barrier whose words reset themselves, so the
+// step can be replayed from a CUDA graph.  Its wait is bounded: a CTA that
+// waits longer than the plan's limit (1 s by default) sets
+// LAMB_STATUS_WAIT_TIMEOUT and an abort word; every other waiter then gives
+// up too and the launch returns.  A launch that finds the abort word set does
+// nothing; the plan must be destroyed.
+#include "lamb_device.cuh"
+
+namespace lamb {
+namespace {
+
+constexpr int kOptLars = 3;
+
+// ---------------------------------------------------------------------------
+// PTX helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];"
+               : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], %2;"
+               : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
+__device__ __forceinline__ void red_add_release(uint32_t* p, uint32_t v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;"
+               :: "l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ void st_relaxed(uint32_t* p, uint32_t v) {
+  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;"
+               :: "l"(p), "r"(v) : "memory");
+}
+
+// 16-byte asynchronous copy global -> shared (L2 only), in this thread's
+// current group
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  const uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;"
+               :: "r"(s), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Two-float sums (a value is hi + lo): TwoSum of the high parts, the error
+// and the low parts folded in, then renormalised.  All inputs here are
+// non-negative sums of squares, for which this keeps ~44 significant bits.
+// ---------------------------------------------------------------------------
+struct F2 {
+  float hi, lo;
+};
+
+__device__ __forceinline__ F2 ff_add(F2 a, F2 b) {
+  const float s = __fadd_rn(a.hi, b.hi);
+  const float bb = __fsub_rn(s, a.hi);
+  const float e = __fadd_rn(__fsub_rn(a.hi, __fsub_rn(s, bb)),
+                            __fsub_rn(b.hi, bb));
+  const float t = __fadd_rn(e, __fadd_rn(a.lo, b.lo));
+  const float hi = __fadd_rn(s, t);
+  return F2{hi, __fsub_rn(t, __fsub_rn(hi, s))};
+}
+
+__device__ __forceinline__ F2 warp_sum_ff(F2 x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    F2 y;
+    y.hi = __shfl_down_sync(0xffffffffu, x.hi, o);
+    y.lo = __shfl_down_sync(0xffffffffu, x.lo, o);
+    x = ff_add(x, y);
+  }
+  return x;
+}
+
+// The tables of one round (double-buffered: one round's pass 2 runs inside
+// the next round's pass 1).
+struct OcTables {
+  OcPiece piece[kOcMaxPieces];
+  float s[kOcMaxPieces];           // eta rho_k of each piece's tensor
+  float dd[kOcMaxPieces];          // eta lambda_k (decoupled decay) or 0
+  uint8_t row_piece[kOcMaxRows];
+  int np, nr;                      // pieces and rows of this CTA's slice
+};
+
+struct OcShared {
+  OcTables tab[2];
+  float4 red[kOcMaxPieces][kOcWarps];  // per piece and warp: two-float
+                                       // sums of w^2 (x, y) and u^2 (z, w)
+  LambConsts k;
+  int64_t t;
+  float lr;
+  int skip;
+  int ok;
+  uint32_t unused_draw;
+};
+
+// Grid-wide barrier (cooperative launch: every CTA is resident).  Arrivals
+// count up (acq_rel: each CTA's writes, ordered before thread 0 by the CTA
+// barrier, are released with its arrival); the last arrival resets the count
+// and advances the generation with a release that the waiters acquire.
+// Returns false if the launch gives up (see the file header).
+__device__ __noinline__ bool grid_sync(const OcParams& q, uint32_t* status,
+                                       int* s_ok) {
+  __syncthreads();
+  if (gridDim.x == 1 && q.extra_arrivals == 0) return true;
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    uint32_t* count = q.bar + kBarCount;
+    uint32_t* gen = q.bar + kBarGen;
+    const uint32_t g0 = ld_acquire_u32(gen);
+    const uint32_t need = gridDim.x + (uint32_t)q.extra_arrivals;
+    if (atom_add_acq_rel(count, 1u) + 1u == need) {
+      st_relaxed(count, 0u);
+      red_add_release(gen, 1u);
+    } else {
+      const uint64_t t0 = global_ns();
+      uint32_t polls = 0;
+      while (ld_acquire_u32(gen) == g0) {
+        if ((++polls & 63u) == 0u) {
+          if (ld_acquire_u32(q.bar + kBarAbort)) {
+            ok = 0;
+            break;
+          }
+          if (global_ns() - t0 > (uint64_t)q.wait_limit_ns) {
+            atomicOr(status, kStatusWaitTimeout);
+            atomicExch(q.bar + kBarAbort, 1u);
+            ok = 0;
+            break;
+          }
+        }
+      }
+    }
+    *s_ok = ok;
+  }
+  __syncthreads();
+  return *s_ok != 0;
+}
+
+// ---------------------------------------------------------------------------
+// Gradient registers: kept as loaded (bf16 pairs stay packed) until the row
+// is computed, so nothing waits on the load before then.
+// ---------------------------------------------------------------------------
+template <typename GT> struct GradRaw;
+
+template <> struct GradRaw<float> {
+  using T = float4;
+  __device__ static T load4(const float* p) {
+    return __ldcs(reinterpret_cast<const float4*>(p));
+  }
+  __device__ static T load_n(const float* p, int c) {
+    float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (c > 0) x.x = __ldcs(p);
+    if (c > 1) x.y = __ldcs(p + 1);
+    if (c > 2) x.z = __ldcs(p + 2);
+    if (c > 3) x.w = __ldcs(p + 3);
+    return x;
+  }
+  __device__ static float4 widen(const T& x) { return x; }
+};
+
+template <> struct GradRaw<__nv_bfloat16> {
+  using T = uint2;
+  __device__ static T load4(const __nv_bfloat16* p) {
+    return __ldcs(reinterpret_cast<const uint2*>(p));
+  }
+  __device__ static T load_n(const __nv_bfloat16* p, int c) {
+    const unsigned short* h = reinterpret_cast<const unsigned short*>(p);
+    uint32_t b[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (j < c) b[j] = __ldcs(h + j);
+    return make_uint2(b[0] | (b[1] << 16), b[2] | (b[3] << 16));
+  }
+  // bf16 -> f32 is exact: the pattern is the top half of the f32
+  __device__ static float4 widen(const T& u) {
+    return make_float4(__uint_as_float(u.x << 16),
+                       __uint_as_float(u.x & 0xffff0000u),
+                       __uint_as_float(u.y << 16),
+                       __uint_as_float(u.y & 0xffff0000u));
+  }
+};
+
+// Stores elements i..i+c-1 of x into `dst` (evict-first).
+__device__ __forceinline__ void store4(float* dst, int64_t i, int c, bool vec,
+                                       const float4& x) {
+  if (c == 4 && vec) {
+    st4_last(dst + i, x);
+    return;
+  }
+  const float y[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    if (j < c) dst[i + j] = y[j];
+}
+
+__device__ __forceinline__ void store_copy4(void* dst, int64_t i, int c,
+                                            bool vec, const float4& x) {
+  if (c == 4 && vec) {
+    st_copy4(dst, i, x);
+    return;
+  }
+  const float y[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    if (j < c) st_copy1(dst, i + j, y[j]);
+}
+
+// Pass 1 of one element: the new moments (Alg. 2) or momentum (Alg. 1), and
+// the direction u whose norm the trust ratio needs.
+template <int kOpt>
+__device__ __forceinline__ float elem1(float g, float& m, float& v, float w,
+                                       float lam, const LambConsts& k) {
+  if (kOpt == kOptLars) {
+    m = lars_momentum(g, m, w, lam, k.b1, k.omb1);
+    return m;
+  }
+  lamb_moments(g, m, v, k);
+  return kOpt ? nlamb_direction<kOpt>(m, v, g, w, lam, k)
+              : lamb_direction(m, v, w, lam, k);
+}
+
+// Four elements of pass 1: moments in m, v; u in u; valid elements (j < c)
+// add w^2 and u^2 to sw, su; invalid ones give u = 0.
+template <int kOpt>
+__device__ __forceinline__ void row1(const float4& g, float4& m, float4& v,
+                                     const float4& w, float4& u, int c,
+                                     float lam, const LambConsts& k, float& sw,
+                                     float& su) {
+  float gg[4] = {g.x, g.y, g.z, g.w}, mm[4] = {m.x, m.y, m.z, m.w},
+        vv[4] = {v.x, v.y, v.z, v.w}, ww[4] = {w.x, w.y, w.z, w.w}, uu[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (j < c) {
+      uu[j] = elem1<kOpt>(gg[j], mm[j], vv[j], ww[j], lam, k);
+      sw = __fmaf_rn(ww[j], ww[j], sw);
+      su = __fmaf_rn(uu[j], uu[j], su);
+    } else {
+      uu[j] = 0.f;
+    }
+  }
+  m = make_float4(mm[0], mm[1], mm[2], mm[3]);
+  v = make_float4(vv[0], vv[1], vv[2], vv[3]);
+  u = make_float4(uu[0], uu[1], uu[2], uu[3]);
+}
+
+__device__ __forceinline__ float4 update4(const float4& w, const float4& u,
+                                          float s, float dd) {
+  float4 o;
+  o.x = __fmaf_rn(-s, u.x, w.x);
+  o.y = __fmaf_rn(-s, u.y, w.y);
+  o.z = __fmaf_rn(-s, u.z, w.z);
+  o.w = __fmaf_rn(-s, u.w, w.w);
+  if (dd != 0.f) {   // decoupled decay; skipped, not added as 0 (signed 0)
+    o.x = __fmaf_rn(-dd, w.x, o.x);
+    o.y = __fmaf_rn(-dd, w.y, o.y);
+    o.z = __fmaf_rn(-dd, w.z, o.z);
+    o.w = __fmaf_rn(-dd, w.w, o.w);
+  }
+  return o;
+}
+
+// ---------------------------------------------------------------------------
+// Pass 1.  Row slot layout: float4 index row * 64 + lane holds lane's w,
+// row * 64 + 32 + lane its m until the row is computed, then its u.  Warp w
+// owns rows w, w + kOcWarps, ... of every round; i counts a warp's rows.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int warp_rows(int n_rows) {
+  const int warp = threadIdx.x >> 5;
+  return n_rows > warp ? (n_rows - warp + kOcWarps - 1) / kOcWarps : 0;
+}
+
+template <int kOpt, typename GT>
+__device__ __forceinline__ void ring_issue(const OcTables& T, float4* rows,
+                                           int i, int nw,
+                                           typename GradRaw<GT>::T& g,
+                                           float4& v, int& cnt) {
+  constexpr bool kV = kOpt != kOptLars;
+  cnt = 0;
+  if (i < nw) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int row = warp + i * kOcWarps;
+    const OcPiece& P = T.piece[T.row_piece[row]];
+    const int e = (row - P.first_row) * kOcRow + lane * 4;
+    cnt = min(max(P.len - e, 0), 4);
+    const int64_t x = P.offset + e;
+    const GT* gp = static_cast<const GT*>(P.g) + x;
+    float4* slot_w = rows + row * 64 + lane;
+    float4* slot_m = slot_w + 32;
+    if (cnt == 4 && (P.flags & kOcVec)) {
+      cp_async16(slot_w, P.w + x);
+      cp_async16(slot_m, P.m + x);
+      g = GradRaw<GT>::load4(gp);
+      if (kV) v = ld4_last(P.v + x);
+    } else {   // ragged tail or unaligned tensor: element-wise, zeros past cnt
+      float4 w4 = make_float4(0.f, 0.f, 0.f, 0.f), m4 = w4, v4 = w4;
+      float* wa = &w4.x;
+      float* ma = &m4.x;
+      float* va = &v4.x;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (j < cnt) {
+          wa[j] = P.w[x + j];
+          ma[j] = P.m[x + j];
+          if (kV) va[j] = P.v[x + j];
+        }
+      }
+      *slot_w = w4;
+      *slot_m = m4;
+      g = GradRaw<GT>::load_n(gp, cnt);
+      v = v4;
+    }
+  }
+}
+
+// One arrived row: the new m, v to HBM, u over m in the slot; the lane's sums
+// of its (up to) four w^2 and u^2 in sw, su.
+template <int kOpt, typename GT>
+__device__ __forceinline__ void ring_consume(const OcTables& T, float4* rows,
+                                             int i,
+                                             const typename GradRaw<GT>::T& g,
+                                             const float4& v, int cnt,
+                                             const LambConsts& k, float wd,
+                                             bool decoupled, float& sw,
+                                             float& su) {
+  constexpr bool kV = kOpt != kOptLars;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = warp + i * kOcWarps;
+  const OcPiece& P = T.piece[T.row_piece[row]];
+  const float lam = decoupled ? 0.f : P.decay * wd;
+  float4* slot_w = rows + row * 64 + lane;
+  float4* slot_m = slot_w + 32;
+  const float4 w4 = *slot_w;
+  float4 m4 = *slot_m, v4 = v, u4;
+  sw = 0.f;
+  su = 0.f;
+  row1<kOpt>(GradRaw<GT>::widen(g), m4, v4, w4, u4, cnt, lam, k, sw, su);
+  if (cnt > 0) {
+    const int64_t x = P.offset + (row - P.first_row) * kOcRow + lane * 4;
+    const bool vec = (P.flags & kOcVec) != 0;
+    store4(P.m, x, cnt, vec, m4);
+    if (kV) store4(P.v, x, cnt, vec, v4);
+  }
+  *slot_m = u4;
+}
+
+// Per-lane two-float sums of w^2 and u^2 over a warp's rows of one piece;
+// flushed (warp tree, then red[piece][warp]) when the next row belongs to
+// another piece.  Every (piece, warp) entry starts at zero each round.
+struct PieceAcc {
+  F2 w, u;
+  __device__ void add(float sw, float su) {
+    w = ff_add(w, F2{sw, 0.f});
+    u = ff_add(u, F2{su, 0.f});
+  }
+  __device__ void flush(OcShared& sh, int piece) {
+    const F2 a = warp_sum_ff(w), b = warp_sum_ff(u);
+    if ((threadIdx.x & 31) == 0)
+      sh.red[piece][threadIdx.x >> 5] = make_float4(a.hi, a.lo, b.hi, b.lo);
+    w = u = F2{0.f, 0.f};
+  }
+};
+
+// Adds row i's sums; flushes if row i is the warp's last row of its piece.
+__device__ __forceinline__ void acc_row(OcShared& sh, const OcTables& T,
+                                        PieceAcc& acc, int i, int nw, float sw,
+                                        float su) {
+  const int warp = threadIdx.x >> 5;
+  const int piece = T.row_piece[warp + i * kOcWarps];
+  acc.add(sw, su);
+  if (i + 1 >= nw || T.row_piece[warp + (i + 1) * kOcWarps] != piece)
+    acc.flush(sh, piece);
+}
+
+// Pass 2 of row i of a round whose ratios are known: w <- w - eta rho_k u
+// (+ decoupled decay, + the bf16 copy), from the row's slot.
+template <bool kCopy>
+__device__ __forceinline__ void pass2_row(const OcTables& T,
+                                          const float4* rows, int i) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = warp + i * kOcWarps;
+  const int j = T.row_piece[row];
+  const OcPiece& P = T.piece[j];
+  const int e = (row - P.first_row) * kOcRow + lane * 4;
+  const int c = min(max(P.len - e, 0), 4);
+  if (c > 0) {
+    const float4 o = update4(rows[row * 64 + lane],
+                             rows[row * 64 + 32 + lane], T.s[j], T.dd[j]);
+    const bool vec = (P.flags & kOcVec) != 0;
+    store4(P.w, P.offset + e, c, vec, o);
+    if (kCopy) store_copy4(P.copy, P.offset + e, c, vec, o);
+  }
+}
+
+// Pass 1 of the round with tables `cur` (if any), with pass 2 of the previous
+// round (tables `prev`, if any) folded in: a slot's previous row is written
+// back just before the next round's copy into it is issued, so the stores of
+// one round overlap the loads of the next.  Each warp keeps one pair of rows
+// in flight.
+template <int kOpt, typename GT, bool kCopy>
+__device__ __forceinline__ void fused_pass(OcShared& sh, float4* rows,
+                                           const OcTables* prev,
+                                           const OcTables* cur,
+                                           const LambConsts& k, float wd,
+                                           bool decoupled) {
+  const int nwp = prev ? warp_rows(prev->nr) : 0;
+  const int nwc = cur ? warp_rows(cur->nr) : 0;
+  int done2 = 0;   // rows of the previous round written back
+  typename GradRaw<GT>::T g0, g1;
+  float4 v0, v1;
+  int c0 = 0, c1 = 0;
+  PieceAcc acc{F2{0.f, 0.f}, F2{0.f, 0.f}};
+  for (; done2 < min(2, nwp); ++done2) pass2_row<kCopy>(*prev, rows, done2);
+  if (nwc > 0) {
+    ring_issue<kOpt, GT>(*cur, rows, 0, nwc, g0, v0, c0);
+    ring_issue<kOpt, GT>(*cur, rows, 1, nwc, g1, v1, c1);
+  }
+  cp_async_commit();
+  for (int i = 0; i < nwc; i += 2) {
+    cp_async_wait<0>();   // rows i, i + 1 have landed
+    float sw0, su0, sw1 = 0.f, su1 = 0.f;
+    ring_consume<kOpt, GT>(*cur, rows, i, g0, v0, c0, k, wd, decoupled, sw0,
+                           su0);
+    if (i + 1 < nwc)
+      ring_consume<kOpt, GT>(*cur, rows, i + 1, g1, v1, c1, k, wd, decoupled,
+                             sw1, su1);
+    acc_row(sh, *cur, acc, i, nwc, sw0, su0);
+    if (i + 1 < nwc) acc_row(sh, *cur, acc, i + 1, nwc, sw1, su1);
+    for (; done2 < min(i + 4, nwp); ++done2)
+      pass2_row<kCopy>(*prev, rows, done2);
+    ring_issue<kOpt, GT>(*cur, rows, i + 2, nwc, g0, v0, c0);
+    ring_issue<kOpt, GT>(*cur, rows, i + 3, nwc, g1, v1, c1);
+    cp_async_commit();
+  }
+  cp_async_wait<0>();
+  for (; done2 < nwp; ++done2) pass2_row<kCopy>(*prev, rows, done2);
+}
+
+// ---------------------------------------------------------------------------
+// Tables, norms and trust ratio
+// ---------------------------------------------------------------------------
+// Loads round r's slice of this CTA into T (two CTA barriers inside).
+__device__ __forceinline__ void load_tables(OcTables& T, const OcParams& q,
+                                            int r) {
+  const OcSlice sl = q.slices[r * (int)gridDim.x + (int)blockIdx.x];
+  if ((int)threadIdx.x < sl.n_pieces)
+    T.piece[threadIdx.x] = q.pieces[sl.piece_begin + (int)threadIdx.x];
+  if (threadIdx.x == 0) {
+    T.np = sl.n_pieces;
+    T.nr = sl.n_rows;
+  }
+  __syncthreads();
+  if ((int)threadIdx.x < sl.n_rows) {
+    int j = 0;
+    for (int i = 1; i < sl.n_pieces; ++i)
+      if (T.piece[i].first_row <= (int)threadIdx.x) j = i;
+    T.row_piece[threadIdx.x] = (uint8_t)j;
+  }
+  __syncthreads();
+}
+
+__device__ __forceinline__ void zero_red(OcShared& sh) {
+  if ((int)threadIdx.x < kOcMaxPieces * kOcWarps)
+    (&sh.red[0][0])[threadIdx.x] = make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
+// Per piece (one warp each): the warps' sums in warp order -> its slot.
+__device__ __forceinline__ void piece_sums(const OcShared& sh,
+                                           const OcTables& T,
+                                           const OcParams& q) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int j = warp; j < T.np; j += kOcWarps) {
+    const float4 x = lane < kOcWarps ? sh.red[j][lane]
+                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+    const F2 a = warp_sum_ff(F2{x.x, x.y}), b = warp_sum_ff(F2{x.z, x.w});
+    if (lane == 0)
+      q.slots[T.piece[j].slot] = make_float4(a.hi, a.lo, b.hi, b.lo);
+  }
+}
+
+__device__ __forceinline__ float phi_f(float z, const StepParams& p) {
+  if (p.phi == 1) {  // clip; comparisons keep NaN as NaN
+    const float gl = (float)p.gamma_l, gu = (float)p.gamma_u;
+    if (z < gl) return gl;
+    if (z > gu) return gu;
+  }
+  return z;
+}
+
+// Warp-wide, per piece: the tensor's slots in slot order (lane-strided, four
+// loads in flight, then a fixed tree) -> ||w||, ||u||, rho_k (Alg. 2 last
+// line with the zero-norm rule; LARS: times kappa), eta rho_k and eta
+// lambda_k for pass 2; exports where this CTA holds the tensor's first piece.
+__device__ __forceinline__ void piece_ratio(const StepParams& p,
+                                            const OcParams& q,
+                                            const OcPiece& P, float coef,
+                                            float lr, bool decoupled,
+                                            float* s_out, float* dd_out) {
+  const int lane = threadIdx.x & 31;
+  F2 a{0.f, 0.f}, b{0.f, 0.f};
+  for (int i = lane; i < P.t_nslots; i += 4 * 32) {
+    float4 x[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int k = i + 32 * j;
+      x[j] = k < P.t_nslots ? __ldcg(&q.slots[P.t_slot + k])
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      a = ff_add(a, F2{x[j].x, x[j].y});
+      b = ff_add(b, F2{x[j].z, x[j].w});
+    }
+  }
+  a = warp_sum_ff(a);
+  b = warp_sum_ff(b);
+  if (lane == 0) {
+    const float aw = __fadd_rn(a.hi, a.lo), au = __fadd_rn(b.hi, b.lo);
+    const float wn = __fsqrt_rn(aw), un = __fsqrt_rn(au);
+    float rho = 1.f;                                   // zero-norm rule
+    if (!(wn == 0.f || un == 0.f))
+      rho = __fdiv_rn(__fmul_rn(coef, phi_f(wn, p)), un);
+    *s_out = __fmul_rn(lr, rho);
+    *dd_out = decoupled ? __fmul_rn(lr, __fmul_rn(P.decay, p.wd)) : 0.f;
+    if (P.flags & kOcExport) {
+      p.ratio[P.tensor] = (double)rho;
+      p.wnorm[P.tensor] = (double)wn;
+      p.unorm[P.tensor] = (double)un;
+      if (!isfinite(a.hi) || !isfinite(b.hi))
+        atomicOr(p.status, kStatusNonfinite);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// The kernel
+// ---------------------------------------------------------------------------
+template <int kOpt, typename GT, bool kCopy>
+__global__ void __launch_bounds__(kOcThreads, 1)
+    onchip_step_kernel(const StepParams p, const OcParams q) {
+  extern __shared__ float4 s_rows[];   // rows x (w[128] | m, then u[128])
+  __shared__ OcShared sh;
+  constexpr bool kLars = kOpt == kOptLars;
+  constexpr int kNest = kLars ? 0 : kOpt;
+  const int warp = threadIdx.x >> 5;
+
+  // a launch after one that gave up does nothing
+  if (ld_acquire_u32(q.bar + kBarAbort)) return;
+
+  // ---- per-launch constants ------------------------------------------------
+  if (!kLars) {
+    step_constants<kNest, false>(p, &sh.unused_draw, &sh.skip, &sh.k, &sh.t);
+  } else if (threadIdx.x == 0) {
+    const int64_t t = p.d_step ? *p.d_step : int64_t(0);
+    sh.t = t;
+    sh.skip = 0;
+    sh.k = LambConsts{p.b1, p.omb1, p.b2, p.omb2, 1.f, 1.f, p.eps,
+                      0.f, 0.f, 0.f, 0.f};
+    if (blockIdx.x == 0) {
+      StepScalars sc{};
+      sc.t = t;
+      sc.c1 = 1.f;
+      sc.c2 = 1.f;
+      sc.lr = step_lr(p, t);
+      *p.scal = sc;
+    }
+  }
+  zero_red(sh);
+  __syncthreads();
+  if (sh.skip) return;   // a step count < 1 (status set by CTA 0)
+  if (threadIdx.x == 0) sh.lr = step_lr(p, sh.t);
+  __syncthreads();
+  const LambConsts k = sh.k;
+  const float lr = sh.lr;
+  const bool decoupled = !kLars && (p.flags & kFlagDecoupledDecay) != 0;
+  const float wd = p.wd;
+  const float coef = kLars ? (float)p.trust : 1.f;
+
+  if (q.n_rounds > 0) {
+    load_tables(sh.tab[0], q, 0);
+    fused_pass<kOpt, GT, kCopy>(sh, s_rows, nullptr, &sh.tab[0], k, wd,
+                                decoupled);
+    __syncthreads();
+  }
+  for (int r = 0; r < q.n_rounds; ++r) {
+    OcTables& T = sh.tab[r & 1];
+    OcTables* next = r + 1 < q.n_rounds ? &sh.tab[(r + 1) & 1] : nullptr;
+    piece_sums(sh, T, q);
+    if (next) load_tables(*next, q, r + 1);
+    if (!grid_sync(q, p.status, &sh.ok)) return;
+    zero_red(sh);
+    for (int j = warp; j < T.np; j += kOcWarps)
+      piece_ratio(p, q, T.piece[j], coef, lr, decoupled, &T.s[j], &T.dd[j]);
+    __syncthreads();
+    fused_pass<kOpt, GT, kCopy>(sh, s_rows, &T, next, k, wd, decoupled);
+    __syncthreads();   // T's buffer is reloaded for round r + 2
+  }
+  // every CTA read t (and the N-LAMB product) before the first barrier
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    const StepScalars sc = *p.scal;
+    if (kNest && p.d_mu_product) *p.d_mu_product = sc.mu_prod;
+    close_step(p, sc);
+  }
+}
+
+template <int kOpt, typename GT, bool kCopy>
+int launch_one(const StepParams& p, const OcParams& q, int grid, int rows,
+               cudaStream_t s) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kOcThreads);
+  cfg.dynamicSmemBytes = (size_t)rows * kOcRowBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeCooperative;
+  at[0].val.cooperative = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return (int)cudaLaunchKernelEx(&cfg, onchip_step_kernel<kOpt, GT, kCopy>, p,
+                                 q);
+}
+
+template <int kOpt, typename GT>
+int launch_copy(const StepParams& p, const OcParams& q, int copy, int grid,
+                int rows, cudaStream_t s) {
+  return copy ? launch_one<kOpt, GT, true>(p, q, grid, rows, s)
+              : launch_one<kOpt, GT, false>(p, q, grid, rows, s);
+}
+
+template <int kOpt>
+int launch_opt(const StepParams& p, const OcParams& q, int g_bf16, int copy,
+               int grid, int rows, cudaStream_t s) {
+  return g_bf16 ? launch_copy<kOpt, __nv_bfloat16>(p, q, copy, grid, rows, s)
+                : launch_copy<kOpt, float>(p, q, copy, grid, rows, s);
+}
+
+// Static shared memory of the largest instantiation, and the dynamic limit
+// raised on every instantiation.
+template <int kOpt, typename GT, bool kCopy>
+int prepare_one(int dyn_bytes, int* static_bytes) {
+  auto* f = onchip_step_kernel<kOpt, GT, kCopy>;
+  if (dyn_bytes < 0) {
+    cudaFuncAttributes a;
+    const cudaError_t e = cudaFuncGetAttributes(&a, f);
+    if (e != cudaSuccess) return (int)e;
+    if ((int)a.sharedSizeBytes > *static_bytes)
+      *static_bytes = (int)a.sharedSizeBytes;
+    return 0;
+  }
+  return (int)cudaFuncSetAttribute(
+      f, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn_bytes);
+}
+
+template <int kOpt>
+int prepare_opt(int dyn_bytes, int* static_bytes) {
+  int rc = prepare_one<kOpt, float, false>(dyn_bytes, static_bytes);
+  if (!rc) rc = prepare_one<kOpt, float, true>(dyn_bytes, static_bytes);
+  if (!rc) rc = prepare_one<kOpt, __nv_bfloat16, false>(dyn_bytes, static_bytes);
+  if (!rc) rc = prepare_one<kOpt, __nv_bfloat16, true>(dyn_bytes, static_bytes);
+  return rc;
+}
+
+int prepare_all(int dyn_bytes, int* static_bytes) {
+  int rc = prepare_opt<0>(dyn_bytes, static_bytes);
+  if (!rc) rc = prepare_opt<1>(dyn_bytes, static_bytes);
+  if (!rc) rc = prepare_opt<2>(dyn_bytes, static_bytes);
+  if (!rc) rc = prepare_opt<3>(dyn_bytes, static_bytes);
+  return rc;
+}
+
+}  // namespace
+
+int onchip_prepare(int device, int* rows_per_cta) {
+  int optin = 0;
+  cudaError_t e = cudaDeviceGetAttribute(
+      &optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, device);
+  if (e != cudaSuccess) return (int)e;
+  int static_bytes = 0;
+  int rc = prepare_all(-1, &static_bytes);
+  if (rc) return rc;
+  int rows = (optin - static_bytes) / kOcRowBytes;
+  if (rows > kOcMaxRows) rows = kOcMaxRows;
+  if (rows < 1) return (int)cudaErrorInvalidConfiguration;
+  rc = prepare_all(rows * kOcRowBytes, &static_bytes);
+  if (rc) return rc;
+  // the launch needs one resident CTA per SM
+  int blocks = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+      &blocks, onchip_step_kernel<0, __nv_bfloat16, true>, kOcThreads,
+      (size_t)rows * kOcRowBytes);
+  if (e != cudaSuccess) return (int)e;
+  if (blocks < 1) return (int)cudaErrorInvalidConfiguration;
+  *rows_per_cta = rows;
+  return 0;
+}
+
+int launch_onchip(const StepParams& p, const OcParams& q, int opt,
+                  int grad_bf16, int copy_bf16, int grid, int rows_per_cta,
+                  void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch (opt) {
+    case 0: return launch_opt<0>(p, q, grad_bf16, copy_bf16, grid, rows_per_cta, s);
+    case 1: return launch_opt<1>(p, q, grad_bf16, copy_bf16, grid, rows_per_cta, s);
+    case 2: return launch_opt<2>(p, q, grad_bf16, copy_bf16, grid, rows_per_cta, s);
+    default: return launch_opt<3>(p, q, grad_bf16, copy_bf16, grid, rows_per_cta, s);
+  }
+}
+
+}  // namespace lamb

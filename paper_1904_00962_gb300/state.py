@@ -87,13 +87,17 @@ class LambPlan:
 
     def __init__(self, state: DeviceState, decay_mask=None, *, device=None,
                  chunk_elems=0, blocks_per_sm=0, algorithm=0, l2_budget_mb=0,
-                 lag_items=0):
+                 lag_items=0, wait_limit_ms=0, test_unmet_wait=False,
+                 onchip_max_ctas=0, onchip_rows=0, tail_elems=0,
+                 shard_world=0, shard_rank=0):
         self.state = state
         dev = state.device.index if device is None else device
         self.handle = B.lamb_plan_create(
             state.sizes, decay_mask, _dtype_code(state.grad_dtype),
             _dtype_code(state.copy_dtype), dev or 0, chunk_elems,
-            blocks_per_sm, algorithm, l2_budget_mb, lag_items)
+            blocks_per_sm, algorithm, l2_budget_mb, lag_items, wait_limit_ms,
+            test_unmet_wait, onchip_max_ctas, onchip_rows, tail_elems,
+            shard_world, shard_rank)
         self.n = len(state.sizes)
         self.bind()
 
@@ -140,6 +144,38 @@ class LambPlan:
         B.lamb_plan_copy_grad_norms(self.handle, *(t.data_ptr() for t in out),
                                     stream=_stream(stream))
         return out
+
+    # -- sharded step (data-parallel) -------------------------------------
+    def shard_pass1(self, hyper, optimizer, d_step, d_lr, d_mu_product=None,
+                    momentum_decay=0.0, stream=None):
+        B.lamb_shard_pass1(self.handle, hyper, optimizer, momentum_decay,
+                           d_step.data_ptr() if d_step is not None else 0,
+                           d_lr.data_ptr() if d_lr is not None else 0,
+                           d_mu_product.data_ptr()
+                           if d_mu_product is not None else 0, _stream(stream))
+
+    def shard_pass2(self, hyper, optimizer, d_step, d_lr, d_mu_product=None,
+                    momentum_decay=0.0, stream=None):
+        B.lamb_shard_pass2(self.handle, hyper, optimizer, momentum_decay,
+                           d_step.data_ptr() if d_step is not None else 0,
+                           d_lr.data_ptr() if d_lr is not None else 0,
+                           d_mu_product.data_ptr()
+                           if d_mu_product is not None else 0, _stream(stream))
+
+    def partials(self, stream=None) -> torch.Tensor:
+        """A device copy of the per-chunk sums (for an all-reduce)."""
+        _, n = B.lamb_plan_partials(self.handle)
+        out = torch.empty(n, dtype=torch.float32, device=self.state.device)
+        B.lamb_plan_copy_partials(self.handle, out.data_ptr(), False,
+                                  _stream(stream))
+        return out
+
+    def set_partials(self, t: torch.Tensor, stream=None) -> None:
+        """Put the (all-reduced) per-chunk sums back into the plan."""
+        _, n = B.lamb_plan_partials(self.handle)
+        assert t.dtype == torch.float32 and t.numel() == n and t.is_contiguous()
+        B.lamb_plan_copy_partials(self.handle, t.data_ptr(), True,
+                                  _stream(stream))
 
     def query(self, clear=False, stream=None) -> int:
         return B.lamb_plan_query(self.handle, clear, _stream(stream))

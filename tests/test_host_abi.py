@@ -66,7 +66,7 @@ def test_binding_constants_match_header_defines():
 
 
 def test_abi_version(lib):
-    assert B.lamb_abi_version() == 1
+    assert B.lamb_abi_version() == 2
 
 
 def test_header_compiles_as_c():
@@ -173,8 +173,39 @@ def test_planner_capacity_too_small(lib):
     t = (ctypes.c_int32 * 2)()
     o = (ctypes.c_int64 * 2)()
     ln = (ctypes.c_int32 * 2)()
-    st = lib.lamb_layout_chunks(sz, 1, 1024, t, o, ln, 2, ctypes.byref(n))
+    st = lib.lamb_layout_chunks(sz, 1, 1024, 0, t, o, ln, 2, ctypes.byref(n))
     assert st == B.LAMB_ERR_INVALID_ARG and n.value == 10
+
+
+@pytest.mark.parametrize("tail", [1, 2048, 5000, 100000, 10 ** 9])
+def test_chunk_table_tail_chunks(lib, tail):
+    """Within `tail` elements of either end of the layout (tensors laid end
+    to end) the chunks are short; elsewhere they are full; every element is
+    covered once, in tensor order, and no chunk spans two tensors."""
+    rng = np.random.default_rng(tail)
+    sizes = [0, 3, 70000, 1, 16384 * 5 + 7, *rng.integers(1, 90000, 20).tolist(),
+             33000, 0]
+    chunk, small = 16384, B.LAMB_TAIL_CHUNK_ELEMS
+    t, o, ln = B.lamb_layout_chunks(sizes, chunk, tail)
+    total = sum(sizes)
+    starts = np.concatenate([[0], np.cumsum(sizes)[:-1]])
+    pos = starts[t] + o                          # position in the layout
+    assert np.all(np.diff(t) >= 0) and np.all(o % 1024 == 0)
+    for k, s in enumerate(sizes):
+        sel = t == k
+        if s == 0:
+            assert not sel.any()
+            continue
+        offs, lens = o[sel], ln[sel]
+        assert offs[0] == 0 and offs[-1] + lens[-1] == s
+        np.testing.assert_array_equal(offs[1:], offs[:-1] + lens[:-1])
+    in_tail = (pos < tail) | (pos + chunk > total - tail)
+    assert np.all(ln[in_tail] <= small)
+    # away from the ends a chunk is short only where its tensor ends
+    ends = pos + ln == starts[t] + np.asarray(sizes)[t]
+    assert np.all((ln[~in_tail] == chunk) | ends[~in_tail])
+    if tail >= total:
+        assert np.all(ln <= small)
 
 
 # ---------------------------------------------------------------------------
@@ -294,7 +325,11 @@ def test_noalloc_validates_before_touching_the_device(lib):
         (dict(sizes=()), B.LAMB_ERR_INVALID_ARG, "n_tensors"),
         (dict(sizes=(1,) * 4097), B.LAMB_ERR_INVALID_ARG, "4096"),
         (dict(sizes=(8, -1)), B.LAMB_ERR_INVALID_ARG, "negative"),
-        (dict(sizes=((1 << 31) + 1,)), B.LAMB_ERR_INVALID_ARG, "chunks"),
+        (dict(sizes=((1 << 31) + 1,)), B.LAMB_ERR_INVALID_ARG, "exceeds"),
+        # sizes near INT64_MAX must not wrap around the chunk count
+        (dict(sizes=((1 << 63) - 1,)), B.LAMB_ERR_INVALID_ARG, "exceeds"),
+        (dict(sizes=((1 << 63) - 16384,)), B.LAMB_ERR_INVALID_ARG, "exceeds"),
+        (dict(sizes=(1 << 30, 1 << 30, 1)), B.LAMB_ERR_INVALID_ARG, "chunks"),
         (dict(grad=7), B.LAMB_ERR_UNSUPPORTED_DTYPE, "grad_dtype"),
         (dict(copy=B.LAMB_F32), B.LAMB_ERR_UNSUPPORTED_DTYPE, "copy_dtype"),
         (dict(copy=B.LAMB_BF16), B.LAMB_ERR_INVALID_ARG, "w_copy"),

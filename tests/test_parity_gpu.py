@@ -297,7 +297,10 @@ def test_ragged_full_size(algo):
             assert math.isclose(d, lr * un[k], rel_tol=2e-3, abs_tol=1e-30), k
         else:
             phi = min(max(wn[k], h.gamma_l), h.gamma_u)
-            assert math.isclose(ratio[k] * un[k], phi, rel_tol=1e-12), k
+            # fp64 ratio (two-pass, single-touch): exact to fp64 rounding;
+            # the on-chip kernel forms rho = RN32(phi / ||u||) in fp32
+            assert math.isclose(ratio[k] * un[k], phi,
+                                rel_tol=2.5e-7 if algo == 3 else 1e-12), k
             assert math.isclose(d, lr * phi, rel_tol=2e-3), (k, d, lr * phi)
     for k in L.zero_w:
         assert ratio[k] == 1.0 and wn[k] == 0.0

@@ -90,8 +90,9 @@ def _prepared(L, step=2, **kw):
 
 @pytest.mark.parametrize("grad_dtype,copy_dtype", [("f32", None),
                                                     ("bf16", "bf16")])
-@pytest.mark.parametrize("algo", [1, 2], ids=["two_pass_plan",
-                                              "single_touch_plan"])
+@pytest.mark.parametrize("algo", [1, 2, 3], ids=["two_pass_plan",
+                                                 "single_touch_plan",
+                                                 "on_chip_plan"])
 @pytest.mark.parametrize("lars", [False, True], ids=["lamb", "lars"])
 def test_grad_norms_match_oracle_and_leave_the_step_unchanged(
         grad_dtype, copy_dtype, algo, lars):
@@ -329,10 +330,11 @@ def test_skip_decision_is_taken_on_the_device_inside_a_graph():
 @pytest.mark.parametrize("grad_dtype,copy_dtype", [("f32", None),
                                                     ("bf16", "bf16")])
 @pytest.mark.parametrize("kind", ["lamb", "nlamb", "nnlamb"])
-def test_decoupled_decay_matches_oracle(grad_dtype, copy_dtype, kind):
+@pytest.mark.parametrize("algo", [1, 3], ids=["two_pass", "on_chip"])
+def test_decoupled_decay_matches_oracle(grad_dtype, copy_dtype, kind, algo):
     L = _layout(grad_dtype, copy_dtype)
     h = W.Hyper(lr=2e-3, weight_decay=0.05, phi="clip", gamma_u=10.0)
-    G = _prepared(L)
+    G = _prepared(L, algorithm=algo)
     G.d_prod = torch.full((1,), 0.5, dtype=torch.float64, device="cuda:0")
     lr = f32(h.lr)
     _with_flags(G, kind, h, lr, 2, decoupled_decay=True)
