@@ -31,3 +31,18 @@ def gpu():
         pytest.fail("test marked gpu but no CUDA device is visible")
     import torch
     return torch.device("cuda:0")
+
+
+def pytest_sessionfinish(session, exitstatus):
+    """With LAMB_FLOOR_STATS set, write how often the parity tolerance floors
+    decided a comparison (gpu_util.FLOOR_STATS) to that file as JSON."""
+    path = os.environ.get("LAMB_FLOOR_STATS")
+    if not path:
+        return
+    try:
+        import gpu_util
+    except Exception:  # pragma: no cover - CPU-only runs
+        return
+    import json
+    with open(path, "w") as f:
+        json.dump(gpu_util.FLOOR_STATS, f, indent=1, sort_keys=True)

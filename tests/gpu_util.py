@@ -69,6 +69,31 @@ def _nan_aware_ok(err, bound, got, ref):
     return np.all((err <= bound) | both_nan)
 
 
+# How often the tolerance floors decide a comparison: per test, the elements
+# compared, those whose error exceeds tol * |ref| but not tol * floor (they
+# pass only because of a floor), and the worst plain relative error
+# |gpu - ref| / |ref|.  Written out by conftest when LAMB_FLOOR_STATS names a
+# file.
+FLOOR_STATS = {}
+
+
+def _floor_stat(array, err, ref, scale, tol):
+    import os
+    test = os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0]
+    ref = np.abs(ref)
+    fin = np.isfinite(err) & np.isfinite(ref)
+    floored = fin & (err > tol * ref) & (err <= tol * scale)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        rel = np.where(fin & (ref > 0), err / np.where(ref > 0, ref, 1.0), 0.0)
+    st = FLOOR_STATS.setdefault(test, {})
+    a = st.setdefault(array, {"n": 0, "floored": 0, "worst_plain_rel": 0.0,
+                              "tol": tol})
+    a["n"] += int(err.size)
+    a["floored"] += int(floored.sum())
+    if rel.size:
+        a["worst_plain_rel"] = max(a["worst_plain_rel"], float(np.max(rel)))
+
+
 def rel_max(err, scale):
     with np.errstate(divide="ignore", invalid="ignore"):
         r = np.where(scale > 0, err / scale, np.where(err > 0, np.inf, 0.0))
@@ -99,6 +124,8 @@ def compare_lamb(got_w, got_m, got_v, ref, w_old, m_old, g64, beta1, tol,
     ew, em = np.abs(got_w - ref.w), np.abs(got_m - ref.m)
     assert _nan_aware_ok(ew, tol * sw, got_w, ref.w), f"w err {rel_max(ew, sw)}"
     assert _nan_aware_ok(em, tol * sm, got_m, ref.m), f"m err {rel_max(em, sm)}"
+    _floor_stat("w", ew, ref.w, sw, tol)
+    _floor_stat("m", em, ref.m, sm, tol)
     out = {"w": rel_max(ew, sw), "m": rel_max(em, sm), "_sw": sw}
     if got_v is not None:
         got_v = got_v.astype(np.float64)
@@ -126,6 +153,8 @@ def compare_lars(got_w, got_m, ref, w_old, m_old, g64, beta1, lam, tol,
     ew, em = np.abs(got_w - ref.w), np.abs(got_m - ref.m)
     assert _nan_aware_ok(ew, tol * sw, got_w, ref.w), f"w err {rel_max(ew, sw)}"
     assert _nan_aware_ok(em, tol * sm, got_m, ref.m), f"m err {rel_max(em, sm)}"
+    _floor_stat("w", ew, ref.w, sw, tol)
+    _floor_stat("m", em, ref.m, sm, tol)
     return {"w": rel_max(ew, sw), "m": rel_max(em, sm), "_sw": sw}
 
 
@@ -163,6 +192,8 @@ def compare_nlamb(got_w, got_m, got_v, ref, w_old, m_old, g64, h, t, lr, lam,
     assert _nan_aware_ok(em, tol * sm, got_m, ref.m), f"m err {rel_max(em, sm)}"
     assert _nan_aware_ok(ev, tol * np.abs(ref.v), got_v, ref.v), \
         f"v err {rel_max(ev, np.abs(ref.v))}"
+    _floor_stat("w", ew, ref.w, sw, tol)
+    _floor_stat("m", em, ref.m, sm, tol)
     return {"w": rel_max(ew, sw), "m": rel_max(em, sm), "_sw": sw}
 
 

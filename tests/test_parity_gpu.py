@@ -259,7 +259,7 @@ def test_ragged_full_size(algo):
         st.view("g", k).zero_()
     rng = np.random.default_rng(7)
     sizes = np.array(L.sizes)
-    ks = set(rng.choice(L.n_tensors, 120, replace=False).tolist())
+    ks = set(rng.choice(L.n_tensors, 1000, replace=False).tolist())
     ks |= set(np.argsort(sizes)[-3:].tolist()) | set(np.argsort(sizes)[:5].tolist())
     ks |= set(list(L.zero_w)[:10]) | set(list(L.zero_g)[:10])
     ks = sorted(int(k) for k in ks)
