@@ -57,18 +57,26 @@ BYTES_PASS1 = 2 + 4 + 4 + 4 + 4 + 4      # read g,m,v,w ; write m,v = 22
 BYTES_PASS2 = 4 + 4 + 4 + 4 + 2          # read m,v,w ; write w, copy = 18
 BYTES_STEP = BYTES_PASS1 + BYTES_PASS2   # 40
 BYTES_SINGLE_TOUCH = 2 + 12 + 12 + 2     # 28
-# per algorithm: kernels of one step, their algorithmic bytes per parameter,
-# and the committed ncu summary holding their measured DRAM traffic
-ALGO_CODES = {"auto": 0, "two_pass": 1, "single_touch": 2, "on_chip": 3}
-KERNELS = {
-    1: (["lamb_pass1_kernel<bf16>", "lamb_pass2_kernel<copy>"],
-        [BYTES_PASS1, BYTES_PASS2],
-        os.path.join(ROOT, "profiles", "lamb_kernels_bert_large.md")),
-    # the single-touch kernel is held to the 28 B/param single-touch model
-    # (the embedding, too large for L2, really moves 40 B/param)
-    2: (["fused_step_kernel<lamb,bf16,copy>"], [BYTES_SINGLE_TOUCH],
-        os.path.join(ROOT, "profiles", "lamb_fused_bert_large.md")),
+ALGO_CODES = {"auto": 0, "two_pass": 1, "on_chip": 3}
+# the committed ncu summaries holding measured DRAM traffic per launch, per
+# (algorithm, layout, optimizer), and the kernel sources they were taken on
+TWO_PASS_SOURCES = ("lamb_kernels.cu", "lamb_device.cuh", "lamb_internal.h")
+ONCHIP_SOURCES = ("lamb_onchip.cu", "lamb_device.cuh", "lamb_internal.h")
+PROFILES = {
+    (1, "bert_large", "lamb"): (
+        os.path.join(ROOT, "profiles", "lamb_kernels_bert_large.md"),
+        None, TWO_PASS_SOURCES),
+    (3, "resnet50", "lamb"): (
+        os.path.join(ROOT, "profiles", "onchip_step_small_layouts.md"),
+        "resnet50/lamb", ONCHIP_SOURCES),
+    (3, "resnet50", "lars"): (
+        os.path.join(ROOT, "profiles", "onchip_step_small_layouts.md"),
+        "resnet50/lars", ONCHIP_SOURCES),
 }
+# kept for the tests of the committed two-pass summary
+KERNELS = {1: (["lamb_pass1_kernel<bf16>", "lamb_pass2_kernel<copy>"],
+               [BYTES_PASS1, BYTES_PASS2], PROFILES[(1, "bert_large",
+                                                     "lamb")][0])}
 
 
 def two_pass_bytes(opt, gb, cb):
@@ -103,9 +111,6 @@ def kernel_model(opt, algo, gb, cb, variant="plain", streamed_frac=0.0):
         names, per = kernel_model(opt, 1, gb, cb, variant)
         return ([n + "(streamed)" for n in names] + on[0],
                 [b * f for b in per] + on[1])
-    if algo == 2 and opt in ("lamb", "lars") and variant == "plain":
-        return ([f"fused_step_kernel<{opt},g{8 * gb},copy{8 * cb}>"],
-                [single_touch_bytes(opt, gb, cb)])
     defer = variant == "skip_nonfinite"
     if opt == "lars":
         if defer:
@@ -138,10 +143,6 @@ def parse_args():
                     help="step algorithm of the plan (auto = library default)")
     ap.add_argument("--chunk-elems", type=int, default=0,
                     help="two-pass chunk size (0 = library default)")
-    ap.add_argument("--lag-items", type=int, default=0,
-                    help="single-touch schedule lag (0 = library default)")
-    ap.add_argument("--l2-budget-mb", type=int, default=0,
-                    help="single-touch L2 budget (0 = library default)")
     ap.add_argument("--layout", default="bert_large",
                     choices=["bert_large", "bert_base", "resnet50", "ragged",
                              "mlp"],
@@ -173,12 +174,12 @@ def load_peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_hash():
-    """sha256 (16 hex digits) of the two-pass kernels' code with comments and
+def kernel_source_hash(sources=TWO_PASS_SOURCES):
+    """sha256 (16 hex digits) of the kernels' code with comments and
     whitespace removed, so that editing a comment does not invalidate the
     committed ncu traffic figures while any change of code does."""
     h = hashlib.sha256()
-    for name in ("lamb_kernels.cu", "lamb_device.cuh", "lamb_internal.h"):
+    for name in sources:
         with open(os.path.join(ROOT, "paper_1904_00962_gb300", "csrc",
                                name)) as f:
             src = f.read()
@@ -188,18 +189,21 @@ def kernel_source_hash():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(profile_file, kernel_idx):
+def profiled_traffic(profile_file, kernel_idx, key=None,
+                     sources=TWO_PASS_SOURCES):
     """Per-launch DRAM bytes from the committed ncu summary, if it was taken
-    on the current kernel source; else None."""
+    on the current kernel source; else None.  A summary covering several
+    workloads labels its lines traffic_bytes_per_launch[<key>][<i>]."""
     try:
         text = open(profile_file).read()
     except OSError:
         return None
     m = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", text)
-    if not m or m.group(1) != kernel_source_hash():
+    if not m or m.group(1) != kernel_source_hash(sources):
         return None
-    m = re.search(rf"traffic_bytes_per_launch\[{kernel_idx}\]:\s*([0-9.e+]+)",
-                  text)
+    label = "" if key is None else rf"\[{re.escape(key)}\]"
+    m = re.search(rf"traffic_bytes_per_launch{label}\[{kernel_idx}\]:\s*"
+                  r"([0-9.e+]+)", text)
     return float(m.group(1)) if m else None
 
 
@@ -521,8 +525,7 @@ def run_ours(args):
         st.upload("w", k, L.weights(k))
         st.upload("g", k, L.grad(k, 1))
     plan = LambPlan(st, L.decay, algorithm=ALGO_CODES[args.algo],
-                    chunk_elems=args.chunk_elems,
-                    lag_items=args.lag_items, l2_budget_mb=args.l2_budget_mb)
+                    chunk_elems=args.chunk_elems)
     info = plan.info()
     algo = info["algorithm"]
     streamed = 0
@@ -532,9 +535,8 @@ def run_ours(args):
     kernel_names, kernel_bytes = kernel_model(
         opt, algo, 2 if L.grad_dtype == "bf16" else 4,
         2 if L.copy_dtype == "bf16" else 0, args.variant, streamed / P)
-    profile_file = KERNELS[algo][2] if algo in KERNELS and (
-        args.layout == "bert_large" and opt == "lamb" and
-        args.variant == "plain") else None
+    profile = PROFILES.get((algo, args.layout, opt)) if (
+        args.variant == "plain" and args.layers == 24) else None
     d_step = torch.ones(1, dtype=torch.int64, device=dev)
     d_lr = torch.full((1,), float(np.float32(h.lr)), dtype=torch.float32,
                       device=dev)
@@ -627,8 +629,7 @@ def run_ours(args):
     d2h = L.n_tensors * 8
     g_dev = [st.g, torch.empty_like(st.g)]
     plan2 = LambPlan(st, L.decay, algorithm=ALGO_CODES[args.algo],
-                     chunk_elems=args.chunk_elems, lag_items=args.lag_items,
-                     l2_budget_mb=args.l2_budget_mb)
+                     chunk_elems=args.chunk_elems)
     es = st.g.element_size()
     B.lamb_plan_bind(plan2.handle, st.ptrs("w"),
                      [g_dev[1].data_ptr() + es * o for o in st.offsets],
@@ -693,11 +694,10 @@ def run_ours(args):
     dom = int(np.argmax(per_launch_ms))
     alg_bytes = kernel_bytes[dom] * P
     achieved = alg_bytes / (per_launch_ms[dom] * 1e-3) / 1e9
-    traffic = profiled_traffic(profile_file, dom) if profile_file else None
+    traffic = profiled_traffic(profile[0], dom, profile[1], profile[2]) \
+        if profile else None
     ms_step = ms_total / args.steps
-    step_bytes = sum(kernel_bytes) if algo != 2 \
-        else two_pass_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
-                            2 if L.copy_dtype == "bf16" else 0)
+    step_bytes = sum(kernel_bytes)
     single_bytes = single_touch_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
                                       2 if L.copy_dtype == "bf16" else 0)
     two_bytes = two_pass_bytes(opt, 2 if L.grad_dtype == "bf16" else 4,
@@ -761,7 +761,7 @@ def run_ours(args):
         "single_touch_bytes_per_param": single_bytes,
         "frac_of_peak_single_touch_model": single_bytes * P /
         (ms_step * 1e-3) / 1e9 / peak,
-        "algorithm": {1: "two_pass", 2: "single_touch", 3: "on_chip"}[algo],
+        "algorithm": {1: "two_pass", 3: "on_chip"}[algo],
         "kernels": {kernel_names[i]: {"ms_per_launch": per_launch_ms[i],
                                       "alg_bytes_per_param": kernel_bytes[i]}
                     for i in range(len(kernel_names))},

@@ -52,7 +52,7 @@
 extern "C" {
 #endif
 
-#define LAMB_ABI_VERSION 2
+#define LAMB_ABI_VERSION 3
 
 /* Only the entry points below are exported from liblamb.so. */
 #if defined(__GNUC__)
@@ -123,12 +123,9 @@ typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
 #define LAMB_STATUS_BAD_STEP  0x2u      /* *d_step < 1 with bias correction:
                                            the step was skipped, nothing was
                                            written                          */
-#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* single-touch or on-chip: a wait
-                                           inside the kernel (single-touch: a
-                                           pass-2 item for its tensor's
-                                           norms, or a stage of the operand
-                                           pipeline, ~0.5 s; on-chip: a grid
-                                           barrier, wait_limit_ms) gave up
+#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* on-chip: a grid-barrier wait
+                                           inside the kernel (wait_limit_ms)
+                                           gave up
                                            and the rest of the launch gave up
                                            with it, so the step is
                                            incomplete and the plan must be
@@ -167,14 +164,7 @@ typedef struct {
                                      (lamb_plan_get_info reports the choice) */
 #define LAMB_ALGO_TWO_PASS 1      /* two streaming kernels per step: 40 B of
                                      HBM traffic per parameter (bf16 g/copy) */
-#define LAMB_ALGO_SINGLE_TOUCH 2  /* one kernel per step; pass 2 of a tensor
-                                     follows its pass 1 closely enough to read
-                                     m, v, w back from L2: ~28 B/parameter
-                                     for tensors whose state fits the L2
-                                     budget.  Work items are fused chunks of
-                                     LAMB_FUSED_CHUNK_ELEMS elements.  LAMB
-                                     and LARS only; N-LAMB and the flagged
-                                     variants run two-pass on such a plan  */
+/* 2 is not assigned (plan creation rejects it)                           */
 #define LAMB_ALGO_ON_CHIP 3       /* one cooperative kernel per step (one CTA
                                      per SM).  Consecutive tensors are taken in
                                      rounds that fit the grid's shared memory
@@ -191,7 +181,6 @@ typedef struct {
                                      decoupled decay and the schedule; the
                                      gradient check and the skip mode run
                                      two-pass on such a plan               */
-#define LAMB_FUSED_CHUNK_ELEMS 4096
 #define LAMB_ONCHIP_ROW_ELEMS 128
 #define LAMB_TAIL_CHUNK_ELEMS 2048
 
@@ -202,12 +191,6 @@ typedef struct {
   int32_t blocks_per_sm; /* resident CTAs per SM for the persistent grid;
                             0 = as many as the occupancy calculator allows */
   int32_t algorithm;     /* LAMB_ALGO_*                                     */
-  int32_t l2_budget_mb;  /* single-touch: tensors whose w, m, v take at most
-                            this many MiB keep them in L2 between the
-                            passes; 0 = half the device's L2               */
-  int32_t lag_items;     /* single-touch: work items between a tensor's last
-                            pass-1 item and its pass-2 block; 0 = 12 per
-                            CTA of the grid, about what it holds in flight */
   int32_t wait_limit_ms; /* on-chip: a grid-barrier wait gives up after this
                             long (LAMB_STATUS_WAIT_TIMEOUT); 0 = 1000      */
   int32_t test_unmet_wait; /* on-chip, for tests of the give-up path only:
@@ -252,11 +235,7 @@ typedef struct {
   int32_t bound;             /* 1 after a successful lamb_plan_bind         */
   int32_t n_vector_tensors;  /* tensors on the vectorised path (after bind) */
   int64_t device_bytes;      /* device memory owned by the plan             */
-  int32_t algorithm;         /* LAMB_ALGO_TWO_PASS or LAMB_ALGO_SINGLE_TOUCH */
-  int32_t n_resident_tensors;/* single-touch: tensors kept in L2            */
-  int64_t n_items;           /* single-touch: work items per step           */
-  int64_t lag_items;         /* single-touch: schedule lag                  */
-  int64_t l2_budget_bytes;   /* single-touch: residency budget              */
+  int32_t algorithm;         /* LAMB_ALGO_TWO_PASS or LAMB_ALGO_ON_CHIP     */
   int32_t n_rounds;          /* on-chip: rounds per step                    */
   int32_t n_streamed_tensors;/* on-chip: tensors too large for a round,
                                 updated by the two-pass kernels            */
@@ -329,7 +308,7 @@ LAMB_API lamb_status_t lars_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
 /* One N-LAMB step (appendix Algorithm 3: Nesterov momentum in the first
  * moment) or, with nesterov_second_moment = 1, one NN-LAMB step (Algorithm
  * 4: also in the second moment), over every tensor.  Uses w, g, m, v and
- * the two-pass kernels (also on a single-touch plan).
+ * the two-pass kernels, or the on-chip kernel on an on-chip plan.
  *   hyper          beta1, beta2, eps, weight_decay, phi as for lamb_step;
  *                  the bias-correction flag is ignored (the Nesterov forms
  *                  carry their own corrections); INCREMENT_STEP honoured
@@ -403,8 +382,9 @@ LAMB_API lamb_status_t lamb_plan_get_info(lamb_plan_t plan, lamb_plan_info_t* in
  * stream around every kernel it launches (up to 4096 steps are kept).
  * lamb_plan_read_timing waits for those events, returns the number of steps
  * recorded and the summed device time of each kernel in milliseconds
- * (ms_per_kernel[0..n_kernels-1]; a two-pass step launches 2 kernels, a
- * single-touch step 1; entries past the step's kernels are 0), and clears
+ * (ms_per_kernel[0..n_kernels-1]; a two-pass step launches 2 kernels, an
+ * on-chip step 1, or 3 when it streams tensors through the two-pass kernels
+ * first; entries past the step's kernels are 0), and clears
  * the record. */
 LAMB_API lamb_status_t lamb_plan_set_timing(lamb_plan_t plan, int32_t enable);
 LAMB_API lamb_status_t lamb_plan_read_timing(lamb_plan_t plan, int32_t* n_steps,
@@ -478,21 +458,6 @@ LAMB_API lamb_status_t lamb_step_noalloc(
     const void* const* g, void* const* m, void* const* v,
     void* const* w_copy, const lamb_hyper_t* hyper, int64_t* d_step,
     const float* d_lr, double* d_ratio, cudaStream_t stream);
-
-/* Host-only planner, no device needed: the work-item order a single-touch
- * plan would use.  Each item is (fused chunk index << 1) | is_pass2; fused
- * chunks hold LAMB_FUSED_CHUNK_ELEMS elements, numbered in tensor order.  l2_budget_bytes and
- * lag_items as in lamb_plan_options_t (both required, > 0).  Writes up to
- * `capacity` items, the total into *n_items and, if `resident` is not NULL,
- * one residency flag per tensor.  INVALID_ARG on bad input or capacity too
- * small (n_items is still written). */
-LAMB_API lamb_status_t lamb_layout_schedule(const int64_t* sizes,
-                                            int32_t n_tensors,
-                                            int64_t l2_budget_bytes,
-                                            int64_t lag_items,
-                                            uint32_t* items, int64_t capacity,
-                                            int64_t* n_items,
-                                            uint8_t* resident);
 
 /* Host-only planner, no device needed: the rounds of an on-chip plan
  * (LAMB_ALGO_ON_CHIP) with `grid` CTAs of rows_per_cta rows (1..224) each.

@@ -51,7 +51,7 @@ EXPORTED = ["lamb_plan_create", "lamb_plan_bind", "lamb_step", "lars_step",
             "lamb_plan_query", "lamb_plan_get_info",
             "lamb_plan_set_timing", "lamb_plan_read_timing",
             "lamb_plan_destroy", "lamb_layout_chunks", "lamb_last_error",
-            "lamb_abi_version", "lamb_step_noalloc", "lamb_layout_schedule",
+            "lamb_abi_version", "lamb_step_noalloc",
             "nlamb_step", "lamb_plan_grad_norms", "lamb_plan_copy_grad_norms",
             "lamb_layout_rounds", "lamb_shard_pass1", "lamb_shard_pass2",
             "lamb_plan_partials", "lamb_layout_shard",
@@ -79,9 +79,7 @@ class lamb_hyper_t(Structure):
 
 LAMB_ALGO_AUTO = 0
 LAMB_ALGO_TWO_PASS = 1
-LAMB_ALGO_SINGLE_TOUCH = 2
 LAMB_ALGO_ON_CHIP = 3
-LAMB_FUSED_CHUNK_ELEMS = 4096     # work item of a single-touch step
 LAMB_ONCHIP_ROW_ELEMS = 128       # row of an on-chip step
 LAMB_TAIL_CHUNK_ELEMS = 2048      # chunks near the ends of a two-pass layout
 LAMB_OPT_LAMB = 0
@@ -93,8 +91,7 @@ LAMB_STATUS_WAIT_TIMEOUT = 0x4
 
 class lamb_plan_options_t(Structure):
     _fields_ = [("chunk_elems", c_int32), ("blocks_per_sm", c_int32),
-                ("algorithm", c_int32), ("l2_budget_mb", c_int32),
-                ("lag_items", c_int32), ("wait_limit_ms", c_int32),
+                ("algorithm", c_int32), ("wait_limit_ms", c_int32),
                 ("test_unmet_wait", c_int32), ("onchip_max_ctas", c_int32),
                 ("onchip_rows", c_int32), ("tail_elems", c_int64),
                 ("shard_world", c_int32), ("shard_rank", c_int32)]
@@ -108,8 +105,6 @@ class lamb_plan_info_t(Structure):
                 ("grad_dtype", c_int32), ("copy_dtype", c_int32),
                 ("bound", c_int32), ("n_vector_tensors", c_int32),
                 ("device_bytes", c_int64), ("algorithm", c_int32),
-                ("n_resident_tensors", c_int32), ("n_items", c_int64),
-                ("lag_items", c_int64), ("l2_budget_bytes", c_int64),
                 ("n_rounds", c_int32), ("n_streamed_tensors", c_int32),
                 ("rows_per_cta", c_int32), ("row_elems", c_int32),
                 ("tail_elems", c_int64), ("shard_world", c_int32),
@@ -159,9 +154,6 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                        POINTER(c_int32), POINTER(c_int64),
                                        POINTER(c_int32), c_int32,
                                        POINTER(c_int32)]
-    lib.lamb_layout_schedule.argtypes = [POINTER(c_int64), c_int32, c_int64,
-                                         c_int64, POINTER(c_uint32), c_int64,
-                                         POINTER(c_int64), POINTER(c_uint8)]
     lib.lamb_step_noalloc.argtypes = [POINTER(c_int64), c_int32,
                                       POINTER(c_uint8), c_int32, c_int32,
                                       POINTER(vp), POINTER(vp), POINTER(vp),
@@ -233,7 +225,7 @@ def make_hyper(*, beta1=0.9, beta2=0.999, eps=1e-6, weight_decay=0.01,
 def lamb_plan_create(sizes, decay_mask=None, grad_dtype=LAMB_F32,
                      copy_dtype=LAMB_DTYPE_NONE, device=0, chunk_elems=0,
                      blocks_per_sm=0, algorithm=LAMB_ALGO_AUTO,
-                     l2_budget_mb=0, lag_items=0, wait_limit_ms=0,
+                     wait_limit_ms=0,
                      test_unmet_wait=False, onchip_max_ctas=0,
                      onchip_rows=0, tail_elems=0, shard_world=0,
                      shard_rank=0) -> int:
@@ -244,8 +236,7 @@ def lamb_plan_create(sizes, decay_mask=None, grad_dtype=LAMB_F32,
     if decay_mask is not None:
         mask = (c_uint8 * max(n, 1))(*[1 if d else 0 for d in decay_mask])
     opts = lamb_plan_options_t(int(chunk_elems), int(blocks_per_sm),
-                               int(algorithm), int(l2_budget_mb),
-                               int(lag_items), int(wait_limit_ms),
+                               int(algorithm), int(wait_limit_ms),
                                int(bool(test_unmet_wait)),
                                int(onchip_max_ctas), int(onchip_rows),
                                int(tail_elems), int(shard_world),
@@ -361,25 +352,6 @@ def lamb_step_noalloc(sizes, decay_mask, grad_dtype, copy_dtype, w, g, m, v,
         _ptr_array(g), _ptr_array(m), _ptr_array(v), _ptr_array(w_copy),
         byref(hyper), c_void_p(d_step or None), c_void_p(d_lr or None),
         c_void_p(d_ratio or None), c_void_p(stream or None)))
-
-
-def lamb_layout_schedule(sizes, l2_budget_bytes, lag_items):
-    """Host-only: (items uint32 array, resident uint8 array) of the
-    single-touch schedule."""
-    lib = load()
-    n = len(sizes)
-    sz = (c_int64 * max(n, 1))(*[int(s) for s in sizes])
-    count = c_int64()
-    res = np.zeros(max(n, 1), dtype=np.uint8)
-    _check(lib.lamb_layout_schedule(sz, n, int(l2_budget_bytes),
-                                    int(lag_items), None, 0, byref(count),
-                                    res.ctypes.data_as(POINTER(c_uint8))))
-    items = np.zeros(max(count.value, 1), dtype=np.uint32)
-    _check(lib.lamb_layout_schedule(sz, n, int(l2_budget_bytes),
-                                    int(lag_items),
-                                    items.ctypes.data_as(POINTER(c_uint32)),
-                                    count.value, byref(count), None))
-    return items[:count.value], res[:n]
 
 
 def lamb_layout_chunks(sizes, chunk_elems=0, tail_elems=0):

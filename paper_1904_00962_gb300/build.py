@@ -21,7 +21,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "liblamb.so")
 
-SOURCES = ["planner.cpp", "lamb_kernels.cu", "lamb_fused.cu", "lamb_onchip.cu",
+SOURCES = ["planner.cpp", "lamb_kernels.cu", "lamb_onchip.cu",
            "lamb_capi.cu", "lamb_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -42,8 +42,6 @@ void lamb::set_last_error(const char* msg) {
 
 namespace {
 
-static_assert(lamb::kFusedChunk == LAMB_FUSED_CHUNK_ELEMS,
-              "the ABI documents the fused chunk size");
 constexpr int kMaxTimedSteps = 4096;
 constexpr int kKernelsPerStep = 3;
 
@@ -80,10 +78,7 @@ struct lamb_plan {
   int num_sms = 0;
   int blocks_per_sm_opt = 0;
   int grid[4] = {0, 0, 0, 0};  // lamb p1, lamb p2, lars p1, lars p2
-  int grid_fused[2] = {0, 0};  // single-touch lamb, lars
   int algorithm = LAMB_ALGO_TWO_PASS;
-  int64_t n_items = 0, lag = 0, l2_budget = 0;
-  int n_resident = 0;
   bool bound = false;
   bool has_v = false;
   int n_vec = 0;
@@ -108,12 +103,6 @@ struct lamb_plan {
   double* grad_norm = nullptr;
   GradCheck* grad_check = nullptr;
   int n_live = 0;               // tensors with at least one chunk
-  // single-touch tables
-  uint2* items = nullptr;
-  FusedTensor* ftensors = nullptr;
-  float2* fslots = nullptr;
-  uint32_t* ftickets = nullptr;
-  uint32_t* ready = nullptr;
   // on-chip single-touch tables
   int oc_grid = 0;
   int oc_rows = 0;              // rows of shared memory per CTA
@@ -228,45 +217,6 @@ lamb_status_t lamb_layout_shard(const int64_t* sizes, int32_t n_tensors,
   return LAMB_OK;
 }
 
-lamb_status_t lamb_layout_schedule(const int64_t* sizes, int32_t n_tensors,
-                                   int64_t l2_budget_bytes, int64_t lag_items,
-                                   uint32_t* items, int64_t capacity,
-                                   int64_t* n_items, uint8_t* resident) {
-  if (!n_items) return fail(LAMB_ERR_INVALID_ARG, "n_items is NULL");
-  if (n_tensors < 1 || !sizes)
-    return fail(LAMB_ERR_INVALID_ARG, "need n_tensors >= 1 and sizes");
-  if (l2_budget_bytes < 1 || lag_items < 1 || capacity < 0 ||
-      (capacity > 0 && !items))
-    return fail(LAMB_ERR_INVALID_ARG, "bad budget, lag or output buffer");
-  char err[256] = "";
-  int64_t total = 0;
-  for (int32_t k = 0; k < n_tensors; ++k) {
-    if (sizes[k] < 0)
-      return fail(LAMB_ERR_INVALID_ARG, "sizes[%d] is negative", k);
-    if (sizes[k] > (int64_t(1) << 62) - total)
-      return fail(LAMB_ERR_INVALID_ARG, "total element count exceeds 2^62");
-    total += sizes[k];
-  }
-  std::vector<FusedChunk> fc;
-  std::vector<FusedTensor> ft;
-  std::vector<uint32_t> it;
-  try {
-    if (plan_fused(sizes, n_tensors, nullptr, 12, l2_budget_bytes, lag_items,
-                   &fc, &ft, &it, err, sizeof(err)))
-      return fail(LAMB_ERR_INVALID_ARG, "%s", err);
-  } catch (const std::bad_alloc&) {
-    return fail(LAMB_ERR_OOM, "host allocation failed");
-  }
-  *n_items = (int64_t)it.size();
-  if (resident)
-    for (int32_t k = 0; k < n_tensors; ++k) resident[k] = (uint8_t)ft[k].resident;
-  if ((int64_t)it.size() > capacity)
-    return capacity == 0 ? LAMB_OK
-                         : fail(LAMB_ERR_INVALID_ARG, "capacity too small");
-  if (!it.empty()) std::memcpy(items, it.data(), it.size() * sizeof(uint32_t));
-  return LAMB_OK;
-}
-
 lamb_status_t lamb_layout_rounds(const int64_t* sizes, int32_t n_tensors,
                                  int32_t grid, int32_t rows_per_cta,
                                  int32_t* piece_round, int32_t* piece_cta,
@@ -354,7 +304,7 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
     return fail(LAMB_ERR_UNSUPPORTED_DTYPE,
                 "copy_dtype %d unsupported (NONE or BF16)", copy_dtype);
   int chunk = kDefaultChunk, bps = 0, algo = LAMB_ALGO_AUTO;
-  int64_t budget_mb = 0, lag_opt = 0, wait_ms = 1000;
+  int64_t wait_ms = 1000;
   int unmet_wait = 0, oc_max_ctas = 0, oc_rows_opt = 0;
   int64_t tail_opt = 0;
   int sh_world = 1, sh_rank = 0;
@@ -364,12 +314,9 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
       return fail(LAMB_ERR_INVALID_ARG, "blocks_per_sm < 0");
     bps = opts->blocks_per_sm;
     algo = opts->algorithm;
-    if (algo < LAMB_ALGO_AUTO || algo > LAMB_ALGO_ON_CHIP)
+    if (algo != LAMB_ALGO_AUTO && algo != LAMB_ALGO_TWO_PASS &&
+        algo != LAMB_ALGO_ON_CHIP)
       return fail(LAMB_ERR_INVALID_ARG, "unknown algorithm %d", algo);
-    if (opts->l2_budget_mb < 0 || opts->lag_items < 0)
-      return fail(LAMB_ERR_INVALID_ARG, "l2_budget_mb and lag_items >= 0");
-    budget_mb = opts->l2_budget_mb;
-    lag_opt = opts->lag_items;
     if (opts->wait_limit_ms < 0)
       return fail(LAMB_ERR_INVALID_ARG, "wait_limit_ms >= 0");
     if (opts->wait_limit_ms) wait_ms = opts->wait_limit_ms;
@@ -482,42 +429,6 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
     if (g < 1) g = 1;
     p->grid[i] = (int)g;
   }
-  // single-touch schedule
-  std::vector<FusedChunk> h_fchunks;
-  std::vector<FusedTensor> h_ftensors;
-  std::vector<uint32_t> h_items;
-  {
-    int focc[2] = {0, 0};
-    rc = occupancy_fused(0, p->grad_bf16, p->copy_bf16, &focc[0]);
-    if (!rc) rc = occupancy_fused(1, p->grad_bf16, p->copy_bf16, &focc[1]);
-    if (rc) {
-      return cuda_fail((cudaError_t)rc, "occupancy query");
-    }
-    for (int i = 0; i < 2; ++i) {
-      int b = focc[i] < 1 ? 1 : focc[i];
-      if (bps > 0 && bps < b) b = bps;
-      p->grid_fused[i] = p->num_sms * b;
-    }
-    int l2 = 0;
-    e = cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, device);
-    if (e != cudaSuccess) {
-      return cuda_fail(e, "cudaDeviceGetAttribute(L2)");
-    }
-    p->l2_budget = budget_mb ? budget_mb << 20 : (int64_t)l2 / 2;
-    p->lag = lag_opt ? lag_opt
-                     : (int64_t)kFusedLagPerCta *
-                           (p->grid_fused[0] > p->grid_fused[1]
-                                ? p->grid_fused[0]
-                                : p->grid_fused[1]);
-    if (plan_fused(sizes, n_tensors, decay_mask, 12, p->l2_budget, p->lag,
-                   &h_fchunks, &h_ftensors, &h_items, err,
-                   sizeof(err))) {
-      return fail(LAMB_ERR_INVALID_ARG, "%s", err);
-    }
-    p->n_items = (int64_t)h_items.size();
-    for (const FusedTensor& t : h_ftensors) p->n_resident += t.resident ? 1 : 0;
-  }
-
   // on-chip rounds
   std::vector<OcSlice> h_slices;
   std::vector<ChunkDesc> h_sub_chunks;
@@ -611,15 +522,6 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   const size_t o_grad_sq = carve(n * sizeof(double));
   const size_t o_grad_norm = carve(n * sizeof(double));
   const size_t o_grad_check = carve(sizeof(GradCheck));
-  const size_t nf = h_fchunks.size();
-  // padded so that a batch of kDrawBatch item records is always readable
-  const size_t n_items_pad =
-      (h_items.size() + kDrawBatch - 1) / kDrawBatch * kDrawBatch;
-  const size_t o_items = carve(n_items_pad * sizeof(uint2));
-  const size_t o_ftensors = carve(n * sizeof(FusedTensor));
-  const size_t o_fslots = carve(nf * sizeof(float2));
-  const size_t o_ftickets = carve(n * sizeof(uint32_t));
-  const size_t o_ready = carve(n * sizeof(uint32_t));
   const size_t o_oc_chunks = carve(h_sub_chunks.size() * sizeof(ChunkDesc));
   const size_t o_oc_tensors = carve(h_sub_tensors.size() * sizeof(TensorDesc));
   const size_t o_oc_slices = carve(h_slices.size() * sizeof(OcSlice));
@@ -647,11 +549,6 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   p->grad_sq = reinterpret_cast<double*>(base + o_grad_sq);
   p->grad_norm = reinterpret_cast<double*>(base + o_grad_norm);
   p->grad_check = reinterpret_cast<GradCheck*>(base + o_grad_check);
-  p->items = reinterpret_cast<uint2*>(base + o_items);
-  p->ftensors = reinterpret_cast<FusedTensor*>(base + o_ftensors);
-  p->fslots = reinterpret_cast<float2*>(base + o_fslots);
-  p->ftickets = reinterpret_cast<uint32_t*>(base + o_ftickets);
-  p->ready = reinterpret_cast<uint32_t*>(base + o_ready);
   p->oc_chunks = reinterpret_cast<ChunkDesc*>(base + o_oc_chunks);
   p->oc_tensors = reinterpret_cast<TensorDesc*>(base + o_oc_tensors);
   p->oc_slices = reinterpret_cast<OcSlice*>(base + o_oc_slices);
@@ -667,20 +564,6 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   if (e == cudaSuccess)
     e = cudaMemcpy(p->tensors, p->h_tensors.data(), n * sizeof(TensorDesc),
                    cudaMemcpyHostToDevice);
-  if (e == cudaSuccess && !h_items.empty()) {
-    // device items carry the tensor and the chunk index directly
-    std::vector<uint2> dev_items(n_items_pad, make_uint2(0u, 0u));
-    for (size_t i = 0; i < h_items.size(); ++i) {
-      const FusedChunk& fc = h_fchunks[h_items[i] >> 1];
-      dev_items[i] = make_uint2(((uint32_t)fc.tensor << 1) | (h_items[i] & 1u),
-                                (uint32_t)fc.index);
-    }
-    e = cudaMemcpy(p->items, dev_items.data(), dev_items.size() * sizeof(uint2),
-                   cudaMemcpyHostToDevice);
-  }
-  if (e == cudaSuccess)
-    e = cudaMemcpy(p->ftensors, h_ftensors.data(), n * sizeof(FusedTensor),
-                   cudaMemcpyHostToDevice);
   if (e == cudaSuccess && !h_sub_chunks.empty())
     e = cudaMemcpy(p->oc_chunks, h_sub_chunks.data(),
                    h_sub_chunks.size() * sizeof(ChunkDesc),
@@ -692,10 +575,6 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   if (e == cudaSuccess && !h_slices.empty())
     e = cudaMemcpy(p->oc_slices, h_slices.data(),
                    h_slices.size() * sizeof(OcSlice), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess) {  // fused launch epoch starts at 1 (ready[] = 0)
-    const uint32_t one = 1u;
-    e = cudaMemcpy(p->counters + 3, &one, sizeof(one), cudaMemcpyHostToDevice);
-  }
   if (e == cudaSuccess) {
     // trust ratio 1 for every tensor until a step computes it; a 0-element
     // tensor keeps it (its norms are 0, and a zero norm gives ratio 1)
@@ -957,27 +836,8 @@ static lamb_status_t run_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
     if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = (uint8_t)n;
     return LAMB_OK;
   }
-  // the single-touch kernel implements the plain step; the gradient check,
-  // the skip mode and decoupled decay run on the two-pass kernels
-  const uint32_t two_pass_only = LAMB_FLAG_GRAD_NORM | LAMB_FLAG_SKIP_NONFINITE |
-                                 LAMB_FLAG_DECOUPLED_DECAY;
-  if (plan->algorithm == LAMB_ALGO_SINGLE_TOUCH &&
-      !(hyper->flags & two_pass_only)) {
-    FusedParams fp;
-    fp.items = plan->items;
-    fp.ftensors = plan->ftensors;
-    fp.fslots = plan->fslots;
-    fp.tickets = plan->ftickets;
-    fp.ready = plan->ready;
-    fp.n_items = (int32_t)plan->n_items;
-    if (!rc)
-      rc = launch_fused(sp, fp, lamb ? 0 : 1, plan->grad_bf16, plan->copy_bf16,
-                        plan->grid_fused[lamb ? 0 : 1], stream);
-    if (!rc && timed) rc = (int)cudaEventRecord(ev[1], stream);
-    if (rc) return cuda_fail((cudaError_t)rc, lamb ? "lamb_step" : "lars_step");
-    if (timed) plan->timed_kernels[(size_t)plan->timed_steps++] = 1;
-    return LAMB_OK;
-  }
+  // two-pass plans, and on-chip plans with the gradient check or the skip
+  // mode
   if (!rc)
     rc = lamb ? launch_lamb_pass1(sp, 0, plan->grad_bf16, plan->grid[0], stream)
               : launch_lars_pass1(sp, plan->grad_bf16, plan->grid[2], stream);
@@ -1277,12 +1137,6 @@ lamb_status_t lamb_plan_get_info(lamb_plan_t plan, lamb_plan_info_t* info) {
   info->n_vector_tensors = plan->n_vec;
   info->device_bytes = (int64_t)plan->arena_bytes;
   info->algorithm = plan->algorithm;
-  info->n_resident_tensors = plan->n_resident;
-  info->n_items = plan->n_items;
-  info->lag_items = plan->lag;
-  info->l2_budget_bytes = plan->l2_budget;
-  if (plan->algorithm == LAMB_ALGO_SINGLE_TOUCH)
-    info->grid_blocks = plan->grid_fused[0];
   if (plan->algorithm == LAMB_ALGO_ON_CHIP) {
     info->grid_blocks = plan->oc_grid;
     info->threads_per_block = kOcThreads;

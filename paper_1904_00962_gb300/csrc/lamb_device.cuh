@@ -1,4 +1,4 @@
-// Device helpers shared by the two-pass and the single-touch kernels: the
+// Device helpers shared by the two-pass and the on-chip kernels: the
 // element arithmetic of Algs. 1-4 (explicit round-to-nearest intrinsics,
 // so every kernel forms bit-identical values), vector loads and stores,
 // warp reductions, and the helpers that close a step.

@@ -94,10 +94,7 @@ struct StepParams {
   const TensorPtrs* ptrs;
   float2* slots;
   uint32_t* tickets;
-  uint32_t* counters;     // [0] pass-1, [1] pass-2, [2] fused work counter,
-                          // [3] launch epoch of the fused kernel (>= 1),
-                          // [4] epoch of a fused launch whose wait gave up,
-                          // [5] fused producers done drawing this launch
+  uint32_t* counters;     // [0] pass-1, [1] pass-2 work counter
   double* ratio;
   double* wnorm;
   double* unorm;
@@ -133,47 +130,6 @@ struct StepParams {
   GradCheck* gcheck;
   int32_t n_tensors;
   int32_t n_live;         // tensors with at least one chunk
-};
-
-// ---------------------------------------------------------------------------
-// Single-touch (fused) step: one persistent kernel (one CTA per SM) that
-// takes work items -- the pass-1 or pass-2 work on one "fused chunk" of
-// kFusedChunk elements -- from a host-built schedule in which the pass-2
-// items of a tensor follow its pass-1 items by a lag of about the items the
-// grid holds in flight, so the m, v, w the pass 1 just touched are still in
-// L2 when the pass 2 reads them.
-// ---------------------------------------------------------------------------
-constexpr int kFusedChunk = 4096;     // elements per fused chunk (a CTA item)
-// items a CTA draws at once (one atomic); the device item list is padded to
-// a multiple of it
-constexpr int kDrawBatch = 4;
-// default schedule lag per CTA of the fused grid: a CTA holds up to ~20
-// items (8 stages, 3 batches drawn ahead, 1 in the consumers)
-constexpr int kFusedLagPerCta = 12;
-
-struct __align__(8) FusedChunk {
-  int32_t tensor;   // tensor index k
-  int32_t index;    // chunk index inside the tensor (offset = index*kFusedChunk)
-};
-
-struct __align__(16) FusedTensor {
-  int64_t numel;
-  int32_t first_chunk;   // in the fused chunk table (slot base)
-  int32_t n_chunks;
-  float decay;           // 1.0f: weight decay applies
-  uint32_t resident;     // 1: keep pass-1 data in L2 (evict_last) for pass 2
-  uint32_t pad[2];
-};
-
-struct FusedParams {
-  const uint2* items;          // x = (tensor << 1) | is_pass2, y = index of
-                               // the fused chunk inside the tensor
-  const FusedTensor* ftensors;
-  float2* fslots;              // per fused chunk (sum w^2, sum u^2), fp32
-  uint32_t* tickets;           // per tensor: chunks whose sums are stored
-  uint32_t* ready;             // per tensor: epoch of the launch that
-                               // finished its norms
-  int32_t n_items;
 };
 
 // ---------------------------------------------------------------------------
@@ -280,9 +236,6 @@ int launch_finalize_all(const StepParams& p, double coef, void* stream);
 // (planner.cpp).
 void shard_range(const ChunkDesc* chunks, int64_t n_chunks, int32_t world,
                  int32_t rank, int64_t* begin, int64_t* end);
-int launch_fused(const StepParams& p, const FusedParams& f, int lars,
-                 int grad_bf16, int copy_bf16, int grid, void* stream);
-int occupancy_fused(int lars, int grad_bf16, int copy_bf16, int* blocks);
 // Resident CTAs per SM of each kernel instantiation (occupancy calculator).
 int occupancy_lamb_pass1(int grad_bf16, int* blocks);
 int occupancy_lamb_pass2(int copy_bf16, int* blocks);
@@ -295,14 +248,6 @@ void fill_hyper(const lamb_hyper_t& h, StepParams* sp);
 
 // Sets the thread-local message returned by lamb_last_error() (lamb_capi.cu).
 void set_last_error(const char* msg);
-
-// Schedule of the single-touch step (planner.cpp): fused chunk table, tensor
-// table (with the L2-residency flag) and the ordered work items.
-int plan_fused(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
-               int64_t bytes_per_param, int64_t l2_budget, int64_t lag,
-               std::vector<FusedChunk>* fchunks,
-               std::vector<FusedTensor>* ftensors,
-               std::vector<uint32_t>* items, char* err, int errlen);
 
 // Host planner (planner.cpp).  Returns 0 on success, else writes a message.
 // Within tail_elems of either end of the layout the chunks hold tail_chunk

@@ -103,82 +103,6 @@ int plan_chunks(const int64_t* sizes, int32_t n, int32_t chunk_elems,
 }  // namespace lamb
 
 // ---------------------------------------------------------------------------
-// Schedule of the single-touch step.
-//
-// Every tensor k of d_k elements becomes ceil(d_k / kFusedChunk) fused
-// chunks.  Work items are emitted in this order:
-// the pass-1 items of tensor 0, 1, 2, ... in turn; the pass-2 items of a
-// tensor whose state fits the L2 budget ("resident") are emitted as one block
-// once `lag` further pass-1 items have been emitted after its last pass-1
-// item (about one wave of workers, so its norms are usually final when the
-// block is reached, while its m, v, w are still in L2); the pass-2 blocks of
-// tensors too large for L2 come last.  Every pass-2 item therefore follows
-// all pass-1 items of its tensor, which is what makes the kernel
-// deadlock-free.
-// ---------------------------------------------------------------------------
-namespace lamb {
-
-int plan_fused(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
-               int64_t bytes_per_param, int64_t l2_budget, int64_t lag,
-               std::vector<FusedChunk>* fchunks,
-               std::vector<FusedTensor>* ftensors,
-               std::vector<uint32_t>* items, char* err, int errlen) {
-  ftensors->assign((size_t)n, FusedTensor{});
-  int64_t nf = 0;
-  for (int32_t k = 0; k < n; ++k) {
-    const int64_t d = sizes[k];
-    const int64_t nk = (d + kFusedChunk - 1) / kFusedChunk;
-    FusedTensor& t = (*ftensors)[(size_t)k];
-    t.numel = d;
-    t.first_chunk = (int32_t)nf;
-    t.n_chunks = (int32_t)nk;
-    t.decay = (decay_mask == nullptr || decay_mask[k]) ? 1.0f : 0.0f;
-    t.resident = (d <= l2_budget / bytes_per_param) ? 1u : 0u;
-    nf += nk;
-    if (nf > (int64_t(1) << 30)) {
-      snprintf(err, errlen, "more than 2^30 fused chunks");
-      return 1;
-    }
-  }
-  fchunks->resize((size_t)nf);
-  for (int32_t k = 0; k < n; ++k) {
-    const FusedTensor& t = (*ftensors)[(size_t)k];
-    for (int32_t j = 0; j < t.n_chunks; ++j)
-      (*fchunks)[(size_t)t.first_chunk + j] = FusedChunk{k, j};
-  }
-  items->clear();
-  items->reserve((size_t)(2 * nf));
-  auto emit_pass2 = [&](int32_t k) {
-    const FusedTensor& t = (*ftensors)[(size_t)k];
-    for (int32_t j = 0; j < t.n_chunks; ++j)
-      items->push_back(((uint32_t)(t.first_chunk + j) << 1) | 1u);
-  };
-  std::vector<std::pair<int64_t, int32_t>> pending;  // (release point, k)
-  size_t head = 0;
-  std::vector<int32_t> tail;
-  int64_t p1 = 0;
-  for (int32_t k = 0; k < n; ++k) {
-    const FusedTensor& t = (*ftensors)[(size_t)k];
-    for (int32_t j = 0; j < t.n_chunks; ++j) {
-      items->push_back((uint32_t)(t.first_chunk + j) << 1);
-      ++p1;
-      while (head < pending.size() && pending[head].first <= p1)
-        emit_pass2(pending[head++].second);
-    }
-    if (t.n_chunks == 0) continue;
-    if (t.resident)
-      pending.emplace_back(p1 + lag, k);
-    else
-      tail.push_back(k);
-  }
-  while (head < pending.size()) emit_pass2(pending[head++].second);
-  for (int32_t k : tail) emit_pass2(k);
-  return 0;
-}
-
-}  // namespace lamb
-
-// ---------------------------------------------------------------------------
 // Rounds of the on-chip single-touch step.
 //
 // A tensor of d elements takes ceil(d / kOcRow) rows.  Tensors are taken in

@@ -86,8 +86,8 @@ class LambPlan:
     """A C-library plan bound to a DeviceState."""
 
     def __init__(self, state: DeviceState, decay_mask=None, *, device=None,
-                 chunk_elems=0, blocks_per_sm=0, algorithm=0, l2_budget_mb=0,
-                 lag_items=0, wait_limit_ms=0, test_unmet_wait=False,
+                 chunk_elems=0, blocks_per_sm=0, algorithm=0, wait_limit_ms=0,
+                 test_unmet_wait=False,
                  onchip_max_ctas=0, onchip_rows=0, tail_elems=0,
                  shard_world=0, shard_rank=0):
         self.state = state
@@ -95,7 +95,7 @@ class LambPlan:
         self.handle = B.lamb_plan_create(
             state.sizes, decay_mask, _dtype_code(state.grad_dtype),
             _dtype_code(state.copy_dtype), dev or 0, chunk_elems,
-            blocks_per_sm, algorithm, l2_budget_mb, lag_items, wait_limit_ms,
+            blocks_per_sm, algorithm, wait_limit_ms,
             test_unmet_wait, onchip_max_ctas, onchip_rows, tail_elems,
             shard_world, shard_rank)
         self.n = len(state.sizes)

@@ -32,8 +32,8 @@ from paper_1904_00962_gb300 import binding as B
 from paper_1904_00962_gb300.state import DeviceState, LambPlan
 
 # the step algorithms of the library
-ALGOS = [1, 2, 3]
-ALGO_IDS = {1: "two_pass", 2: "single_touch", 3: "on_chip"}
+ALGOS = [1, 3]
+ALGO_IDS = {1: "two_pass", 3: "on_chip"}
 
 TOL_STEP = 1e-5
 TOL_CHAIN = 1e-4
@@ -231,15 +231,13 @@ class GpuLayout:
     """A layout's state on the GPU plus a bound plan."""
 
     def __init__(self, layout, *, with_v=True, chunk_elems=0, blocks_per_sm=0,
-                 misalign=None, device="cuda:0", algorithm=1, l2_budget_mb=0,
-                 lag_items=0, **plan_opts):
+                 misalign=None, device="cuda:0", algorithm=1, **plan_opts):
         self.L = layout
         self.st = DeviceState(layout.sizes, grad_dtype=layout.grad_dtype,
                               copy_dtype=layout.copy_dtype, device=device,
                               with_v=with_v, misalign=misalign)
         self.plan = LambPlan(self.st, layout.decay, chunk_elems=chunk_elems,
                              blocks_per_sm=blocks_per_sm, algorithm=algorithm,
-                             l2_budget_mb=l2_budget_mb, lag_items=lag_items,
                              **plan_opts)
         self.d_step = torch.ones(1, dtype=torch.int64, device=device)
         self.d_lr = torch.zeros(1, dtype=torch.float32, device=device)

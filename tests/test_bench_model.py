@@ -45,12 +45,29 @@ def test_kernel_byte_model(opt, gb, cb, variant, per_kernel, two_pass,
         assert sum(got) == two_pass + gb
 
 
-def test_single_touch_model_is_one_kernel():
-    names, got = bench.kernel_model("lamb", 2, 2, 2)
+def test_onchip_model_counts_streamed_tensors_at_two_pass_bytes():
+    names, got = bench.kernel_model("lamb", 3, 2, 2)
     assert len(names) == 1 and got == [28]
+    # a quarter of the parameters streamed through the two-pass kernels
+    names, got = bench.kernel_model("lamb", 3, 2, 2, "plain", 0.25)
+    assert len(names) == 3 and got == [22 * 0.25, 18 * 0.25, 28 * 0.75]
     # the flagged variants run on the two-pass kernels of such a plan
-    names, got = bench.kernel_model("lamb", 2, 2, 2, "grad_norm")
+    names, got = bench.kernel_model("lamb", 3, 2, 2, "grad_norm")
     assert len(names) == 2 and got == [22, 18]
+
+
+def test_profiled_traffic_by_workload_label(tmp_path):
+    f = tmp_path / "multi.md"
+    h = bench.kernel_source_hash(bench.ONCHIP_SOURCES)
+    f.write_text(f"kernel_source_sha256: {h}\n"
+                 "traffic_bytes_per_launch[resnet50/lamb][0]: 6.613e8\n"
+                 "traffic_bytes_per_launch[resnet50/lars][0]: 4.562e8\n")
+    assert bench.profiled_traffic(str(f), 0, "resnet50/lars",
+                                  bench.ONCHIP_SOURCES) == 4.562e8
+    assert bench.profiled_traffic(str(f), 0, "mlp/lamb",
+                                  bench.ONCHIP_SOURCES) is None
+    # the two-pass sources give another hash
+    assert bench.profiled_traffic(str(f), 0, "resnet50/lars") is None
 
 
 def _tree_copy(tmp_path):

@@ -60,13 +60,13 @@ def test_binding_constants_match_header_defines():
             checked += 1
     assert checked >= 12
     for flag in ("LAMB_FLAG_GRAD_NORM", "LAMB_FLAG_SKIP_NONFINITE",
-                 "LAMB_FLAG_DECOUPLED_DECAY", "LAMB_FUSED_CHUNK_ELEMS",
+                 "LAMB_FLAG_DECOUPLED_DECAY", "LAMB_ONCHIP_ROW_ELEMS",
                  "LAMB_STATUS_SKIPPED"):
         assert flag in defs and hasattr(B, flag), flag
 
 
 def test_abi_version(lib):
-    assert B.lamb_abi_version() == 2
+    assert B.lamb_abi_version() == 3
 
 
 def test_header_compiles_as_c():
@@ -206,79 +206,6 @@ def test_chunk_table_tail_chunks(lib, tail):
     assert np.all((ln[~in_tail] == chunk) | ends[~in_tail])
     if tail >= total:
         assert np.all(ln <= small)
-
-
-# ---------------------------------------------------------------------------
-# Single-touch schedule: the precondition of its deadlock freedom
-# ---------------------------------------------------------------------------
-
-def _check_schedule(sizes, budget, lag):
-    items, res = B.lamb_layout_schedule(sizes, budget, lag)
-    c = B.LAMB_FUSED_CHUNK_ELEMS
-    nk = [(s + c - 1) // c for s in sizes]
-    first = np.concatenate([[0], np.cumsum(nk)[:-1]]).astype(np.int64)
-    owner = np.repeat(np.arange(len(sizes)), nk)
-    chunk = (items >> 1).astype(np.int64)
-    p2 = (items & 1).astype(bool)
-    n_f = int(sum(nk))
-    # every fused chunk exactly once per pass
-    assert len(items) == 2 * n_f
-    np.testing.assert_array_equal(np.sort(chunk[~p2]), np.arange(n_f))
-    np.testing.assert_array_equal(np.sort(chunk[p2]), np.arange(n_f))
-    pos = np.arange(len(items))
-    last_p1 = np.full(len(sizes), -1)
-    first_p2 = np.full(len(sizes), len(items))
-    np.maximum.at(last_p1, owner[chunk[~p2]], pos[~p2])
-    np.minimum.at(first_p2, owner[chunk[p2]], pos[p2])
-    for k in range(len(sizes)):
-        if nk[k] == 0:
-            continue
-        # every pass-2 item of k after every pass-1 item of k
-        assert first_p2[k] > last_p1[k], k
-        assert bool(res[k]) == (sizes[k] * 12 <= budget), k
-    # pass 1 runs in tensor order
-    assert np.all(np.diff(owner[chunk[~p2]]) >= 0)
-    # resident tensors wait `lag` pass-1 items (or the end of pass 1);
-    # non-resident tensors' pass-2 items come after all resident ones
-    p1_before = np.cumsum(~p2)
-    n_p1 = int((~p2).sum())
-    for k in range(len(sizes)):
-        if nk[k] == 0 or not res[k]:
-            continue
-        after = p1_before[first_p2[k]] - p1_before[last_p1[k]]
-        assert after >= lag or p1_before[first_p2[k]] == n_p1, k
-    nonres = [k for k in range(len(sizes)) if nk[k] and not res[k]]
-    if nonres:
-        start_tail = min(first_p2[k] for k in nonres)
-        assert np.all(p2[start_tail:])
-        assert all(first_p2[k] > last_p1[j] for k in nonres
-                   for j in range(len(sizes)) if nk[j])
-    return items, res
-
-
-def test_schedule_bert_large(lib):
-    from paper_1904_00962_gb300.workloads import bert_large_layout
-    L = bert_large_layout()
-    items, res = _check_schedule(L.sizes, 63 << 20, 2432)
-    # the word embedding (31M) is the only tensor too large for 63 MiB
-    assert not res[0] and res[1:].all()
-
-
-@pytest.mark.parametrize("seed", range(4))
-def test_schedule_random_layouts(lib, seed):
-    rng = np.random.default_rng(seed)
-    n = int(rng.integers(1, 300))
-    sizes = np.floor(np.exp(rng.uniform(0, np.log(3e6), n))).astype(int)
-    sizes[rng.random(n) < 0.05] = 0
-    _check_schedule(sizes.tolist(), int(rng.integers(1, 64)) << 20,
-                    int(rng.integers(1, 5000)))
-
-
-def test_schedule_rejects_bad_input(lib):
-    for args in (([], 1 << 20, 10), ([10], 0, 10), ([10], 1 << 20, 0),
-                 ([-1], 1 << 20, 10)):
-        with pytest.raises(B.LambError):
-            B.lamb_layout_schedule(*args)
 
 
 # ---------------------------------------------------------------------------

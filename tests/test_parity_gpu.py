@@ -297,7 +297,7 @@ def test_ragged_full_size(algo):
             assert math.isclose(d, lr * un[k], rel_tol=2e-3, abs_tol=1e-30), k
         else:
             phi = min(max(wn[k], h.gamma_l), h.gamma_u)
-            # fp64 ratio (two-pass, single-touch): exact to fp64 rounding;
+            # fp64 ratio (two-pass): exact to fp64 rounding;
             # the on-chip kernel forms rho = RN32(phi / ||u||) in fp32
             assert math.isclose(ratio[k] * un[k], phi,
                                 rel_tol=2.5e-7 if algo == 3 else 1e-12), k
@@ -753,95 +753,6 @@ def test_timing_hook_records_both_kernels(algo):
     assert G.plan.info()["algorithm"] == algo
     B.lamb_plan_set_timing(G.plan.handle, False)
     G.close()
-
-
-# ---------------------------------------------------------------------------
-# Single-touch specifics: edge layouts, schedule knobs, determinism
-# ---------------------------------------------------------------------------
-
-@pytest.mark.parametrize("grad_dtype,copy_dtype", [("f32", None),
-                                                    ("bf16", "bf16")])
-@pytest.mark.parametrize("misalign", [False, True])
-@pytest.mark.parametrize("budget_mb,lag", [(0, 0), (1, 1), (1024, 100000)])
-def test_single_touch_edge_layout(grad_dtype, copy_dtype, misalign, budget_mb,
-                                  lag):
-    L = _edge_layout(grad_dtype, copy_dtype)
-    h = L.hyper
-    G = GpuLayout(L, algorithm=2, l2_budget_mb=budget_mb, lag_items=lag,
-                  misalign={5, 9, 12, 16} if misalign else None)
-    info = G.plan.info()
-    assert info["algorithm"] == 2
-    if budget_mb == 1:        # 1 MiB: only tensors of <= 87381 elements
-        assert info["n_resident_tensors"] == sum(
-            1 for s in L.sizes if s * 12 <= (1 << 20))
-    G.load_weights()
-    G.load_warm_state()
-    G.load_grads(2)
-    lr = f32(h.lr)
-    G.step(2, lr, c_hyper(h))
-    assert G.plan.query(clear=True) == 0
-    ratio, wn, un = G.results()
-    for k in range(L.n_tensors):
-        w, g = L.weights(k), L.grad(k, 2)
-        m, v = L.state_warm(k)
-        ref = _oracle_lamb(L, k, w, g, m, v, 2, lr, h)
-        e = compare_lamb(G.download("w", k), G.download("m", k),
-                         G.download("v", k), ref, w, m,
-                         O.to_f64(g, grad_dtype), h.beta1, TOL_STEP,
-                         upd=(h, 2, lr, h.weight_decay * L.decay[k]))
-        if copy_dtype:
-            check_copy(G.download("copy", k), G.download("w", k), ref.w,
-                       sw=e["_sw"])
-        assert ratio_ok(ratio[k], ref.ratio), (k, ratio[k], ref.ratio)
-    G.close()
-
-
-@pytest.mark.parametrize("lars", [False, True])
-def test_single_touch_bitwise_deterministic_across_schedules(lars):
-    """Chunking is fixed (fused chunks of LAMB_FUSED_CHUNK_ELEMS), so neither the grid,
-    the lag nor the L2 budget may change a single bit of the results."""
-    L = W.resnet50_layout()
-    h = L.lars_hyper if lars else L.hyper
-    snaps = []
-    for bps, lag, budget in ((0, 0, 0), (1, 1, 1), (0, 50000, 4096),
-                             (0, 0, 0)):
-        G = GpuLayout(L, with_v=not lars, blocks_per_sm=bps, lag_items=lag,
-                      l2_budget_mb=budget, algorithm=2)
-        G.load_weights()
-        G.load_warm_state()
-        G.load_grads(4)
-        for t in (4, 5, 6):
-            G.step(t, f32(h.lr), c_hyper(h, lars=lars), lars=lars)
-        assert G.plan.query() == 0
-        snaps.append(_snapshot(G))
-        G.close()
-    for other in snaps[1:]:
-        for a, b in zip(snaps[0], other):
-            assert torch.equal(a, b)
-
-
-def test_single_touch_matches_two_pass_within_tolerance():
-    L = W.bert_base_layout()
-    h = L.hyper
-    outs = []
-    w_before = None
-    for algo in (1, 2):
-        G = GpuLayout(L, algorithm=algo)
-        G.load_weights()
-        G.load_warm_state()
-        G.load_grads(4)
-        w_before = G.st.w.clone()
-        G.step(4, f32(h.lr), c_hyper(h))
-        r, _, _ = G.results()
-        outs.append((G.st.w.clone(), G.st.m.clone(), G.st.v.clone(), r))
-        G.close()
-    (w1, m1, v1, r1), (w2, m2, v2, r2) = outs
-    # the moments do not depend on any reduction: bitwise equal
-    assert torch.equal(m1, m2) and torch.equal(v1, v2)
-    np.testing.assert_allclose(r2, r1, rtol=2 * TOL_RATIO, atol=0)
-    d = (w1.double() - w2.double()).abs()
-    scale = torch.maximum(w1.double().abs(), w_before.double().abs())
-    assert bool(torch.all(d <= TOL_STEP * scale))
 
 
 # ---------------------------------------------------------------------------
