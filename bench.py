@@ -61,7 +61,8 @@ ALGO_CODES = {"auto": 0, "two_pass": 1, "on_chip": 3}
 # the committed ncu summaries holding measured DRAM traffic per launch, per
 # (algorithm, layout, optimizer), and the kernel sources they were taken on
 TWO_PASS_SOURCES = ("lamb_kernels.cu", "lamb_device.cuh", "lamb_internal.h")
-ONCHIP_SOURCES = ("lamb_onchip.cu", "lamb_device.cuh", "lamb_internal.h")
+ONCHIP_SOURCES = ("lamb_onchip.cu", "lamb_onchip.h", "lamb_device.cuh",
+                  "lamb_internal.h")
 PROFILES = {
     (1, "bert_large", "lamb"): (
         os.path.join(ROOT, "profiles", "lamb_kernels_bert_large.md"),
@@ -124,6 +125,52 @@ def kernel_model(opt, algo, gb, cb, variant="plain", streamed_frac=0.0):
     if defer:
         return names, [gb + 12, gb + 12 + 8 + 4 + cb]
     return names, [gb + 12 + 8, 12 + (gb if nest else 0) + 4 + cb]
+
+
+def noalloc_overhead(st, L, hyper, d_step, d_lr, stream, one_step, n=20):
+    """Device time and host enqueue time per call of lamb_step_noalloc
+    against the plan's lamb_step, on the same state, n calls each after
+    three of each untimed.  The no-alloc call rebuilds its tables on the
+    device every call; the difference is its per-call overhead."""
+    from ctypes import byref, c_int64, c_uint8, c_void_p
+    from paper_1904_00962_gb300.state import _dtype_code
+    lib = B.load()
+    k = L.n_tensors
+    sizes = (c_int64 * k)(*[int(x) for x in L.sizes])
+    mask = (c_uint8 * k)(*[1 if d else 0 for d in L.decay])
+    arrs = [B._ptr_array(st.ptrs(x)) for x in ("w", "g", "m", "v", "copy")]
+    gcode, ccode = _dtype_code(st.grad_dtype), _dtype_code(st.copy_dtype)
+    hp = byref(hyper)
+    ds, dl = c_void_p(d_step.data_ptr()), c_void_p(d_lr.data_ptr())
+    sp = c_void_p(stream.cuda_stream)
+
+    def na():
+        rc = lib.lamb_step_noalloc(sizes, k, mask, gcode, ccode, *arrs, hp,
+                                   ds, dl, None, sp)
+        if rc:
+            raise B.LambError(rc, B.lamb_last_error())
+
+    for _ in range(3):
+        na()
+        one_step()
+    res = {}
+    for name, fn in (("plan", one_step), ("noalloc", na)):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        t0 = time.perf_counter()
+        for _ in range(n):
+            fn()
+        t1 = time.perf_counter()
+        e1.record(stream)
+        e1.synchronize()
+        res[name] = (e0.elapsed_time(e1) / n, (t1 - t0) / n * 1e6)
+    return {"calls": n, "ms_per_call": res["noalloc"][0],
+            "plan_ms_per_call": res["plan"][0],
+            "overhead_ms": res["noalloc"][0] - res["plan"][0],
+            "host_us_per_call": res["noalloc"][1],
+            "plan_host_us_per_call": res["plan"][1]}
 
 
 def parse_args():
@@ -680,6 +727,13 @@ def run_ours(args):
     plan2.destroy()
     del g_dev[1]
     clk = clocks.stop() if clocks else None
+    noalloc = None
+    if rank == 0 and opt == "lamb" and args.variant == "plain":
+        try:
+            noalloc = noalloc_overhead(st, L, hyper, d_step, d_lr, stream,
+                                       one_step)
+        except B.LambError as e:   # beyond the entry point's limits
+            noalloc = {"unavailable": str(e)}
 
     if rank != 0:
         plan.destroy()
@@ -783,6 +837,7 @@ def run_ours(args):
                 "steps": k_e2e, "upload_streams": n_up,
                 "overlap": "upload of step s+1 overlaps step s "
                            "(two gradient buffers)"},
+        "noalloc": noalloc,
         "gpu_launches": len(kernel_names) * args.steps,
         "device_status": status,
         "clocks": clk,

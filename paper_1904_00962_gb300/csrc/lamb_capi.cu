@@ -12,6 +12,7 @@
 
 #include "lamb.h"
 #include "lamb_internal.h"
+#include "lamb_onchip.h"
 
 using namespace lamb;
 

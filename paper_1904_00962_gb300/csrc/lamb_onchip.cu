@@ -8,28 +8,32 @@
 // shared memory of the SM that formed them.
 //
 // One cooperative launch per step: one CTA per SM (all resident at once),
-// 512 threads, ~223 KB of shared memory holding up to 223 rows of 128
-// elements (w and u in fp32, 1 KB per row).  The host planner (planner.cpp,
-// plan_onchip) cuts the tensors into ROUNDS of consecutive whole tensors
-// whose rows fit the grid (~4.3M parameters on 152 SMs).  Each CTA owns a
-// fixed slice of a round's rows, in pieces (a piece = the rows of one tensor
-// in one CTA, at most 16 per CTA); warp w takes rows w, w + 16, ...  Per
-// round:
+// 768 threads (24 warps), ~223 KB of shared memory holding up to 224 rows of
+// 128 elements (w and u in fp32, 1 KB per row).  The host planner
+// (planner.cpp, plan_onchip) cuts the tensors into ROUNDS of consecutive
+// whole tensors whose rows fit the grid (~4.3M parameters on 152 SMs).  Each
+// CTA owns a fixed slice of a round's rows, in pieces (a piece = the rows of
+// one tensor in one CTA, at most 16 per CTA); warp w takes rows w, w + 24, ...
+// Per round r:
 //
-//   pass 1   each warp keeps 2 x kPairs rows in flight: w and m of a row are
-//            copied (cp.async) straight into the row's shared-memory slot, g
-//            and v into registers.  For each arrived row: the new m, v (Alg. 2
+//   pass 1   each warp keeps two rows in flight: w and m of a row are copied
+//            (cp.async) straight into the row's shared-memory slot, g and v
+//            into registers.  For each arrived row: the new m, v (Alg. 2
 //            moment lines; Alg. 1 momentum for LARS) go back to HBM, u
-//            replaces m in the slot, and the warp's fixed-tree fp32 sums of
-//            w^2 and u^2 are kept per row; per piece, the row sums are added
-//            in row order (compensated two-float sums) into the piece's slot.
-//   barrier  grid-wide
+//            replaces m in the slot, and each lane adds its elements' w^2 and
+//            u^2 to per-piece two-float sums (a fixed warp tree when the
+//            warp leaves the piece); per piece, the warps' sums are added in
+//            warp order into the piece's slot.
+//   barrier  grid-wide; the CTA loads round r + 1's tables while it waits
 //   ratio    every CTA adds the slots of each of its tensors in slot order
 //            (two-float) and forms rho_k = phi(||w||)/||u|| in fp32 (1 on a
 //            zero norm; LARS: kappa phi(||w||)/||m||); the CTA holding the
 //            tensor's first piece exports rho_k and the norms.
 //   pass 2   w <- w - eta rho_k u from shared memory (+ the bf16 copy): no HBM
-//            reads at all.
+//            reads at all.  It runs inside pass 1 of round r + 1: a row's
+//            slot is written back just before round r + 1's copy into it is
+//            issued, so the stores of one round overlap the loads of the
+//            next.
 //
 // The reductions avoid fp64: GB300 issues fp64 at a small fraction of its
 // fp32 rate, and the compensated two-float sums keep ~44 bits.
@@ -43,13 +47,14 @@
 // arithmetic is the two-pass kernels' (lamb_device.cuh), so m, v and u are
 // bit-identical to theirs; only the summation of the norms differs.
 //
-// The barrier is a generation barrier whose words reset themselves, so the
+// The barrier counts arrivals in a 64-bit word that is never reset, so the
 // step can be replayed from a CUDA graph.  Its wait is bounded: a CTA that
 // waits longer than the plan's limit (1 s by default) sets
 // LAMB_STATUS_WAIT_TIMEOUT and an abort word; every other waiter then gives
 // up too and the launch returns.  A launch that finds the abort word set does
 // nothing; the plan must be destroyed.
 #include "lamb_device.cuh"
+#include "lamb_onchip.h"
 
 namespace lamb {
 namespace {
@@ -72,21 +77,19 @@ __device__ __forceinline__ uint64_t global_ns() {
   return t;
 }
 
-__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
-  uint32_t old;
-  asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], %2;"
-               : "=r"(old) : "l"(p), "r"(v) : "memory");
+__device__ __forceinline__ uint64_t ld_acquire_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];"
+               : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ uint64_t atom_add_acq_rel_u64(uint64_t* p,
+                                                         uint64_t v) {
+  uint64_t old;
+  asm volatile("atom.add.acq_rel.gpu.global.u64 %0, [%1], %2;"
+               : "=l"(old) : "l"(p), "l"(v) : "memory");
   return old;
-}
-
-__device__ __forceinline__ void red_add_release(uint32_t* p, uint32_t v) {
-  asm volatile("red.release.gpu.global.add.u32 [%0], %1;"
-               :: "l"(p), "r"(v) : "memory");
-}
-
-__device__ __forceinline__ void st_relaxed(uint32_t* p, uint32_t v) {
-  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;"
-               :: "l"(p), "r"(v) : "memory");
 }
 
 // 16-byte asynchronous copy global -> shared (L2 only), in this thread's
@@ -154,30 +157,43 @@ struct OcShared {
   int skip;
   int ok;
   uint32_t unused_draw;
+  uint64_t target;       // count the current grid barrier waits for
 };
 
-// Grid-wide barrier (cooperative launch: every CTA is resident).  Arrivals
-// count up (acq_rel: each CTA's writes, ordered before thread 0 by the CTA
-// barrier, are released with its arrival); the last arrival resets the count
-// and advances the generation with a release that the waiters acquire.
-// Returns false if the launch gives up (see the file header).
-__device__ __noinline__ bool grid_sync(const OcParams& q, uint32_t* status,
-                                       int* s_ok) {
+// Grid-wide barrier (cooperative launch: every CTA is resident), split in an
+// arrival and a wait so that a CTA can do independent work in between.  The
+// plan's 64-bit count of arrivals only grows: every launch adds n_rounds x
+// grid, so a launch starts at a multiple of the grid, and an arrival that
+// finds the count at `old` completes when it reaches the next multiple of
+// the barrier's size above `old`.  The arrival (acq_rel, after the CTA
+// barrier) releases the CTA's writes; the wait acquires everyone's.  Nothing
+// is reset, so the step can be replayed from a CUDA graph.
+__device__ __forceinline__ void grid_arrive(const OcParams& q,
+                                            uint64_t* s_target) {
   __syncthreads();
-  if (gridDim.x == 1 && q.extra_arrivals == 0) return true;
+  if (threadIdx.x == 0) {
+    const uint64_t need = gridDim.x + (uint64_t)q.extra_arrivals;
+    if (gridDim.x == 1 && q.extra_arrivals == 0) {
+      *s_target = 0;   // nobody to wait for
+      return;
+    }
+    uint64_t* count = reinterpret_cast<uint64_t*>(q.bar + kBarCount);
+    const uint64_t old = atom_add_acq_rel_u64(count, 1u);
+    *s_target = (old / need + 1u) * need;
+  }
+}
+
+// Returns false if the launch gives up (see the file header).
+__device__ __noinline__ bool grid_wait(const OcParams& q, uint32_t* status,
+                                       const uint64_t* s_target, int* s_ok) {
   if (threadIdx.x == 0) {
     int ok = 1;
-    uint32_t* count = q.bar + kBarCount;
-    uint32_t* gen = q.bar + kBarGen;
-    const uint32_t g0 = ld_acquire_u32(gen);
-    const uint32_t need = gridDim.x + (uint32_t)q.extra_arrivals;
-    if (atom_add_acq_rel(count, 1u) + 1u == need) {
-      st_relaxed(count, 0u);
-      red_add_release(gen, 1u);
-    } else {
+    const uint64_t target = *s_target;
+    const uint64_t* count = reinterpret_cast<const uint64_t*>(q.bar + kBarCount);
+    if (target != 0 && ld_acquire_u64(count) < target) {
       const uint64_t t0 = global_ns();
       uint32_t polls = 0;
-      while (ld_acquire_u32(gen) == g0) {
+      while (ld_acquire_u64(count) < target) {
         if ((++polls & 63u) == 0u) {
           if (ld_acquire_u32(q.bar + kBarAbort)) {
             ok = 0;
@@ -647,8 +663,9 @@ __global__ void __launch_bounds__(kOcThreads, 1)
     OcTables& T = sh.tab[r & 1];
     OcTables* next = r + 1 < q.n_rounds ? &sh.tab[(r + 1) & 1] : nullptr;
     piece_sums(sh, T, q);
-    if (next) load_tables(*next, q, r + 1);
-    if (!grid_sync(q, p.status, &sh.ok)) return;
+    grid_arrive(q, &sh.target);
+    if (next) load_tables(*next, q, r + 1);   // while the others arrive
+    if (!grid_wait(q, p.status, &sh.target, &sh.ok)) return;
     zero_red(sh);
     for (int j = warp; j < T.np; j += kOcWarps)
       piece_ratio(p, q, T.piece[j], coef, lr, decoupled, &T.s[j], &T.dd[j]);

@@ -15,6 +15,7 @@
 #include <vector>
 
 #include "lamb_internal.h"
+#include "lamb_onchip.h"
 
 namespace lamb {
 
