@@ -275,6 +275,34 @@ def nlamb_step(plan, hyper: lamb_hyper_t, momentum_decay, nesterov_second_moment
                              c_void_p(stream or None)))
 
 
+def step_call(kind, plan, hyper: lamb_hyper_t, d_step, d_lr, stream=0,
+              momentum_decay=0.0, d_mu_product=0):
+    """A zero-argument callable that runs one lamb_step ("lamb"), lars_step
+    ("lars") or nlamb_step ("nlamb", "nnlamb") with its arguments marshalled
+    once, for loops that repeat the same step.  The callable keeps `hyper`
+    alive and reads it at each call."""
+    lib = load()
+    p, hp = c_void_p(plan), byref(hyper)
+    ds, dl = c_void_p(d_step or None), c_void_p(d_lr or None)
+    s = c_void_p(stream or None)
+    if kind == "lamb":
+        fn, args = lib.lamb_step, (p, hp, ds, dl, s)
+    elif kind == "lars":
+        fn, args = lib.lars_step, (p, hp, ds, dl, s)
+    elif kind in ("nlamb", "nnlamb"):
+        fn, args = lib.nlamb_step, (p, hp, c_double(momentum_decay),
+                                    c_int32(kind == "nnlamb"), ds, dl,
+                                    c_void_p(d_mu_product or None), s)
+    else:
+        raise ValueError(f"unknown step kind {kind!r}")
+
+    def call():
+        st = fn(*args)
+        if st:
+            _check(st)
+    return call
+
+
 def lamb_plan_trust_ratios(plan):
     r, w, u = c_void_p(), c_void_p(), c_void_p()
     _check(load().lamb_plan_trust_ratios(c_void_p(plan), byref(r), byref(w),

@@ -84,12 +84,9 @@ __device__ __forceinline__ uint64_t ld_acquire_u64(const uint64_t* p) {
   return v;
 }
 
-__device__ __forceinline__ uint64_t atom_add_acq_rel_u64(uint64_t* p,
-                                                         uint64_t v) {
-  uint64_t old;
-  asm volatile("atom.add.acq_rel.gpu.global.u64 %0, [%1], %2;"
-               : "=l"(old) : "l"(p), "l"(v) : "memory");
-  return old;
+__device__ __forceinline__ void red_add_release_u64(uint64_t* p, uint64_t v) {
+  asm volatile("red.release.gpu.global.add.u64 [%0], %1;"
+               :: "l"(p), "l"(v) : "memory");
 }
 
 // 16-byte asynchronous copy global -> shared (L2 only), in this thread's
@@ -157,38 +154,44 @@ struct OcShared {
   int skip;
   int ok;
   uint32_t unused_draw;
-  uint64_t target;       // count the current grid barrier waits for
+  uint64_t base;         // the barrier count when this launch started
 };
 
 // Grid-wide barrier (cooperative launch: every CTA is resident), split in an
 // arrival and a wait so that a CTA can do independent work in between.  The
-// plan's 64-bit count of arrivals only grows: every launch adds n_rounds x
-// grid, so a launch starts at a multiple of the grid, and an arrival that
-// finds the count at `old` completes when it reaches the next multiple of
-// the barrier's size above `old`.  The arrival (acq_rel, after the CTA
-// barrier) releases the CTA's writes; the wait acquires everyone's.  Nothing
-// is reset, so the step can be replayed from a CUDA graph.
-__device__ __forceinline__ void grid_arrive(const OcParams& q,
-                                            uint64_t* s_target) {
+// plan's 64-bit count of arrivals only grows: a launch adds n_rounds x grid,
+// so every launch starts at a multiple of the grid.  Thread 0 reads the
+// count before its CTA first arrives, when fewer than `grid` arrivals of this
+// launch can have happened, so rounding the value down to a multiple of the
+// grid gives the launch's base; barrier r then completes at base + (r + 1)
+// grid.  The arrival is a release reduction (no reply to wait for); the wait
+// acquires.  Nothing is reset, so the step can be replayed from a CUDA
+// graph.
+__device__ __forceinline__ uint64_t grid_base(const OcParams& q) {
+  const uint64_t c =
+      ld_acquire_u64(reinterpret_cast<const uint64_t*>(q.bar + kBarCount));
+  return c - c % gridDim.x;
+}
+
+__device__ __forceinline__ void grid_arrive(const OcParams& q) {
   __syncthreads();
-  if (threadIdx.x == 0) {
-    const uint64_t need = gridDim.x + (uint64_t)q.extra_arrivals;
-    if (gridDim.x == 1 && q.extra_arrivals == 0) {
-      *s_target = 0;   // nobody to wait for
-      return;
-    }
-    uint64_t* count = reinterpret_cast<uint64_t*>(q.bar + kBarCount);
-    const uint64_t old = atom_add_acq_rel_u64(count, 1u);
-    *s_target = (old / need + 1u) * need;
-  }
+  if (threadIdx.x == 0 && !(gridDim.x == 1 && q.extra_arrivals == 0))
+    red_add_release_u64(reinterpret_cast<uint64_t*>(q.bar + kBarCount), 1u);
+}
+
+// Target of barrier r (0 = nobody to wait for).  Test plans add arrivals
+// that never come, so the first wait runs out.
+__device__ __forceinline__ uint64_t grid_target(const OcParams& q,
+                                                uint64_t base, int r) {
+  if (gridDim.x == 1 && q.extra_arrivals == 0) return 0;
+  return base + (uint64_t)(r + 1) * gridDim.x + (uint64_t)q.extra_arrivals;
 }
 
 // Returns false if the launch gives up (see the file header).
 __device__ __noinline__ bool grid_wait(const OcParams& q, uint32_t* status,
-                                       const uint64_t* s_target, int* s_ok) {
+                                       uint64_t target, int* s_ok) {
   if (threadIdx.x == 0) {
     int ok = 1;
-    const uint64_t target = *s_target;
     const uint64_t* count = reinterpret_cast<const uint64_t*>(q.bar + kBarCount);
     if (target != 0 && ld_acquire_u64(count) < target) {
       const uint64_t t0 = global_ns();
@@ -564,8 +567,12 @@ __device__ __forceinline__ float phi_f(float z, const StepParams& p) {
   return z;
 }
 
-// Warp-wide, per piece: the tensor's slots in slot order (lane-strided, four
-// loads in flight, then a fixed tree) -> ||w||, ||u||, rho_k (Alg. 2 last
+// Slot loads a lane keeps in flight when forming a ratio: a tensor has at
+// most one slot per CTA, so 8 x 32 covers a 152-SM grid in one round trip.
+constexpr int kRatioLoads = 8;
+
+// Warp-wide, per piece: the tensor's slots in slot order (lane-strided,
+// kRatioLoads loads in flight, then a fixed tree) -> ||w||, ||u||, rho_k (Alg. 2 last
 // line with the zero-norm rule; LARS: times kappa), eta rho_k and eta
 // lambda_k for pass 2; exports where this CTA holds the tensor's first piece.
 __device__ __forceinline__ void piece_ratio(const StepParams& p,
@@ -575,16 +582,16 @@ __device__ __forceinline__ void piece_ratio(const StepParams& p,
                                             float* s_out, float* dd_out) {
   const int lane = threadIdx.x & 31;
   F2 a{0.f, 0.f}, b{0.f, 0.f};
-  for (int i = lane; i < P.t_nslots; i += 4 * 32) {
-    float4 x[4];
+  for (int i = lane; i < P.t_nslots; i += kRatioLoads * 32) {
+    float4 x[kRatioLoads];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < kRatioLoads; ++j) {
       const int k = i + 32 * j;
       x[j] = k < P.t_nslots ? __ldcg(&q.slots[P.t_slot + k])
                             : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < kRatioLoads; ++j) {
       a = ff_add(a, F2{x[j].x, x[j].y});
       b = ff_add(b, F2{x[j].z, x[j].w});
     }
@@ -623,6 +630,7 @@ __global__ void __launch_bounds__(kOcThreads, 1)
 
   // a launch after one that gave up does nothing
   if (ld_acquire_u32(q.bar + kBarAbort)) return;
+  if (threadIdx.x == 0) sh.base = grid_base(q);   // before the first arrival
 
   // ---- per-launch constants ------------------------------------------------
   if (!kLars) {
@@ -663,9 +671,9 @@ __global__ void __launch_bounds__(kOcThreads, 1)
     OcTables& T = sh.tab[r & 1];
     OcTables* next = r + 1 < q.n_rounds ? &sh.tab[(r + 1) & 1] : nullptr;
     piece_sums(sh, T, q);
-    grid_arrive(q, &sh.target);
+    grid_arrive(q);
     if (next) load_tables(*next, q, r + 1);   // while the others arrive
-    if (!grid_wait(q, p.status, &sh.target, &sh.ok)) return;
+    if (!grid_wait(q, p.status, grid_target(q, sh.base, r), &sh.ok)) return;
     zero_red(sh);
     for (int j = warp; j < T.np; j += kOcWarps)
       piece_ratio(p, q, T.piece[j], coef, lr, decoupled, &T.s[j], &T.dd[j]);

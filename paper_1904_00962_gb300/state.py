@@ -125,6 +125,17 @@ class LambPlan:
                      d_lr.data_ptr(), d_mu_product.data_ptr(),
                      _stream(stream))
 
+    def step_call(self, kind, hyper, d_step: torch.Tensor, d_lr: torch.Tensor,
+                  d_mu_product: torch.Tensor = None, momentum_decay=0.004,
+                  stream=None):
+        """binding.step_call on this plan: a zero-argument callable for one
+        step, with the device pointers and the stream taken now."""
+        return B.step_call(kind, self.handle, hyper,
+                           d_step.data_ptr() if d_step is not None else 0,
+                           d_lr.data_ptr(), _stream(stream), momentum_decay,
+                           d_mu_product.data_ptr()
+                           if d_mu_product is not None else 0)
+
     def results(self, stream=None):
         """(ratio, wnorm, unorm) as new float64 device tensors."""
         dev = self.state.device

@@ -486,6 +486,39 @@ def test_graph_replay_equals_eager(algo):
     G.close()
 
 
+@algos
+@pytest.mark.parametrize("lars", [False, True], ids=["lamb", "lars"])
+def test_step_call_equals_the_plain_binding(algo, lars):
+    """binding.step_call marshals the arguments once; the steps it runs must
+    be the ones lamb_step / lars_step run, bit for bit."""
+    L = W.bert_layout(1, 64, 256, vocab=500, positions=32, name="stepcall")
+    h = L.hyper
+    hyp = c_hyper(h, increment=True, lars=lars)
+    snaps = []
+    for use_call in (False, True):
+        G = GpuLayout(L, with_v=not lars, algorithm=algo)
+        G.load_weights()
+        G.load_warm_state()
+        G.d_step.fill_(2)
+        G.d_lr.fill_(f32(h.lr))
+        call = G.plan.step_call("lars" if lars else "lamb", hyp, G.d_step,
+                                G.d_lr)
+        for t in (2, 3, 4):
+            G.load_grads(t)
+            if use_call:
+                call()
+            elif lars:
+                G.plan.lars_step(hyp, G.d_step, G.d_lr)
+            else:
+                G.plan.lamb_step(hyp, G.d_step, G.d_lr)
+        assert G.plan.query(clear=True) == 0
+        assert int(G.d_step.item()) == 5
+        snaps.append(_snapshot(G))
+        G.close()
+    for a, b in zip(*snaps):
+        assert torch.equal(a, b)
+
+
 # ---------------------------------------------------------------------------
 # Checkpoint / resume: state is caller-owned, the plan is stateless
 # ---------------------------------------------------------------------------
