@@ -115,7 +115,7 @@ struct lamb_plan {
   std::vector<OcPiece> h_oc_pieces;   // without pointers (filled by bind)
   OcSlice* oc_slices = nullptr;
   OcPiece* oc_pieces = nullptr;
-  float4* oc_slots = nullptr;
+  uint64_t* oc_slots = nullptr;
   uint32_t* oc_bar = nullptr;
   // the streamed tensors' chunk table for the two-pass kernels
   int64_t oc_n_chunks = 0;
@@ -527,7 +527,7 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   const size_t o_oc_tensors = carve(h_sub_tensors.size() * sizeof(TensorDesc));
   const size_t o_oc_slices = carve(h_slices.size() * sizeof(OcSlice));
   const size_t o_oc_pieces = carve(p->h_oc_pieces.size() * sizeof(OcPiece));
-  const size_t o_oc_slots = carve((size_t)p->oc_n_slots * sizeof(float4));
+  const size_t o_oc_slots = carve((size_t)p->oc_n_slots * 2 * sizeof(uint64_t));
   const size_t o_oc_bar = carve(kBarWords * sizeof(uint32_t));
   p->arena_bytes = off;
   e = cudaMalloc(&p->arena, p->arena_bytes);
@@ -554,7 +554,7 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
   p->oc_tensors = reinterpret_cast<TensorDesc*>(base + o_oc_tensors);
   p->oc_slices = reinterpret_cast<OcSlice*>(base + o_oc_slices);
   p->oc_pieces = reinterpret_cast<OcPiece*>(base + o_oc_pieces);
-  p->oc_slots = reinterpret_cast<float4*>(base + o_oc_slots);
+  p->oc_slots = reinterpret_cast<uint64_t*>(base + o_oc_slots);
   p->oc_bar = reinterpret_cast<uint32_t*>(base + o_oc_bar);
 
   // zero everything (tickets, counters, status, results, pointer table)

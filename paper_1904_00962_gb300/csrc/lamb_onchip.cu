@@ -23,12 +23,16 @@
 //            replaces m in the slot, and each lane adds its elements' w^2 and
 //            u^2 to per-piece two-float sums (a fixed warp tree when the
 //            warp leaves the piece); per piece, the warps' sums are added in
-//            warp order into the piece's slot.
-//   barrier  grid-wide; the CTA loads round r + 1's tables while it waits
-//   ratio    every CTA adds the slots of each of its tensors in slot order
-//            (two-float) and forms rho_k = phi(||w||)/||u|| in fp32 (1 on a
-//            zero norm; LARS: kappa phi(||w||)/||m||); the CTA holding the
-//            tensor's first piece exports rho_k and the norms.
+//            warp order into the piece's slot, tagged with the launch.
+//   exchange the CTA loads round r + 1's tables; then, for each of its
+//            tensors, it reloads the tensor's slots (written by every CTA
+//            that holds a piece of it) until all carry this launch's tag.
+//            No grid-wide barrier is needed: nothing else passes between
+//            CTAs.
+//   ratio    the slots in slot order (two-float) give rho_k =
+//            phi(||w||)/||u|| in fp32 (1 on a zero norm; LARS: kappa
+//            phi(||w||)/||m||); the CTA holding the tensor's first piece
+//            exports rho_k and the norms.
 //   pass 2   w <- w - eta rho_k u from shared memory (+ the bf16 copy): no HBM
 //            reads at all.  It runs inside pass 1 of round r + 1: a row's
 //            slot is written back just before round r + 1's copy into it is
@@ -47,12 +51,13 @@
 // arithmetic is the two-pass kernels' (lamb_device.cuh), so m, v and u are
 // bit-identical to theirs; only the summation of the norms differs.
 //
-// The barrier counts arrivals in a 64-bit word that is never reset, so the
-// step can be replayed from a CUDA graph.  Its wait is bounded: a CTA that
-// waits longer than the plan's limit (1 s by default) sets
-// LAMB_STATUS_WAIT_TIMEOUT and an abort word; every other waiter then gives
-// up too and the launch returns.  A launch that finds the abort word set does
-// nothing; the plan must be destroyed.
+// The tags come from a launch epoch that the last CTA of a launch advances,
+// so the step can be replayed from a CUDA graph.  The wait for a tensor's
+// slots is bounded: a CTA that waits longer than the plan's limit (1 s by
+// default) sets LAMB_STATUS_WAIT_TIMEOUT and an abort word; every other
+// waiter then gives up too and the launch returns.  A launch that finds the
+// abort word set does nothing; the plan must be destroyed.  The last CTA to
+// finish also closes the step (t + 1, the scheduled eta, the N-LAMB product).
 #include "lamb_device.cuh"
 #include "lamb_onchip.h"
 
@@ -77,16 +82,28 @@ __device__ __forceinline__ uint64_t global_ns() {
   return t;
 }
 
-__device__ __forceinline__ uint64_t ld_acquire_u64(const uint64_t* p) {
+__device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t* p) {
   uint64_t v;
-  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];"
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];"
                : "=l"(v) : "l"(p) : "memory");
   return v;
 }
 
-__device__ __forceinline__ void red_add_release_u64(uint64_t* p, uint64_t v) {
-  asm volatile("red.release.gpu.global.add.u64 [%0], %1;"
+__device__ __forceinline__ void st_relaxed_u64(uint64_t* p, uint64_t v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;"
                :: "l"(p), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t* p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], %2;"
+               : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+
+__device__ __forceinline__ void st_relaxed_u32(uint32_t* p, uint32_t v) {
+  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;"
+               :: "l"(p), "r"(v) : "memory");
 }
 
 // 16-byte asynchronous copy global -> shared (L2 only), in this thread's
@@ -154,67 +171,42 @@ struct OcShared {
   int skip;
   int ok;
   uint32_t unused_draw;
-  uint64_t base;         // the barrier count when this launch started
+  uint32_t epoch;        // the plan's launch epoch when this launch started
 };
 
-// Grid-wide barrier (cooperative launch: every CTA is resident), split in an
-// arrival and a wait so that a CTA can do independent work in between.  The
-// plan's 64-bit count of arrivals only grows: a launch adds n_rounds x grid,
-// so every launch starts at a multiple of the grid.  Thread 0 reads the
-// count before its CTA first arrives, when fewer than `grid` arrivals of this
-// launch can have happened, so rounding the value down to a multiple of the
-// grid gives the launch's base; barrier r then completes at base + (r + 1)
-// grid.  The arrival is a release reduction (no reply to wait for); the wait
-// acquires.  Nothing is reset, so the step can be replayed from a CUDA
-// graph.
-__device__ __forceinline__ uint64_t grid_base(const OcParams& q) {
-  const uint64_t c =
-      ld_acquire_u64(reinterpret_cast<const uint64_t*>(q.bar + kBarCount));
-  return c - c % gridDim.x;
+// Exchange of the piece sums between CTAs, without a grid barrier.  A
+// piece's slot is two 64-bit words, (sum w^2) and (sum u^2), each holding a
+// two-float value: hi in the low half, lo in the high half with its four
+// lowest bits replaced by a tag (lo is at most half an ulp of hi, so the
+// truncation changes the sum by less than 2^-44 of it).  Every launch writes
+// every slot once, with the tag (epoch + 1) mod 16 of its own launch; a CTA
+// that needs a tensor's sums reloads its slots until every word carries that
+// tag.  The words are written and read with single-copy-atomic relaxed 64-bit
+// accesses, so a word with the right tag holds the right value, and no other
+// data passes between CTAs: no fence is needed.  Slots keep the previous
+// launch's tag until overwritten, and the plan zeroes them (tag 0) while the
+// first launch uses tag 1.  The epoch advances when the last CTA of a launch
+// finishes (a ticket), so the next launch, which starts after this one ends,
+// reads the new value.  Nothing is reset by the host: the step can be
+// replayed from a CUDA graph.
+__device__ __forceinline__ uint64_t slot_word(F2 x, uint32_t tag) {
+  return (uint64_t)__float_as_uint(x.hi) |
+         ((uint64_t)((__float_as_uint(x.lo) & ~0xFu) | tag) << 32);
 }
-
-__device__ __forceinline__ void grid_arrive(const OcParams& q) {
-  __syncthreads();
-  if (threadIdx.x == 0 && !(gridDim.x == 1 && q.extra_arrivals == 0))
-    red_add_release_u64(reinterpret_cast<uint64_t*>(q.bar + kBarCount), 1u);
+__device__ __forceinline__ F2 slot_value(uint64_t x) {
+  return F2{__uint_as_float((uint32_t)x),
+            __uint_as_float((uint32_t)(x >> 32) & ~0xFu)};
 }
-
-// Target of barrier r (0 = nobody to wait for).  Test plans add arrivals
-// that never come, so the first wait runs out.
-__device__ __forceinline__ uint64_t grid_target(const OcParams& q,
-                                                uint64_t base, int r) {
-  if (gridDim.x == 1 && q.extra_arrivals == 0) return 0;
-  return base + (uint64_t)(r + 1) * gridDim.x + (uint64_t)q.extra_arrivals;
+__device__ __forceinline__ bool slot_tagged(uint64_t x, uint32_t tag) {
+  return ((uint32_t)(x >> 32) & 0xFu) == tag;
 }
-
-// Returns false if the launch gives up (see the file header).
-__device__ __noinline__ bool grid_wait(const OcParams& q, uint32_t* status,
-                                       uint64_t target, int* s_ok) {
-  if (threadIdx.x == 0) {
-    int ok = 1;
-    const uint64_t* count = reinterpret_cast<const uint64_t*>(q.bar + kBarCount);
-    if (target != 0 && ld_acquire_u64(count) < target) {
-      const uint64_t t0 = global_ns();
-      uint32_t polls = 0;
-      while (ld_acquire_u64(count) < target) {
-        if ((++polls & 63u) == 0u) {
-          if (ld_acquire_u32(q.bar + kBarAbort)) {
-            ok = 0;
-            break;
-          }
-          if (global_ns() - t0 > (uint64_t)q.wait_limit_ns) {
-            atomicOr(status, kStatusWaitTimeout);
-            atomicExch(q.bar + kBarAbort, 1u);
-            ok = 0;
-            break;
-          }
-        }
-      }
-    }
-    *s_ok = ok;
-  }
-  __syncthreads();
-  return *s_ok != 0;
+// Tag of this launch's slots; test plans wait for a tag nobody writes.
+__device__ __forceinline__ uint32_t write_tag(uint32_t epoch) {
+  return (epoch + 1u) & 0xFu;
+}
+__device__ __forceinline__ uint32_t wait_tag(const OcParams& q,
+                                             uint32_t epoch) {
+  return (epoch + 1u + (uint32_t)q.extra_arrivals) & 0xFu;
 }
 
 // ---------------------------------------------------------------------------
@@ -544,17 +536,21 @@ __device__ __forceinline__ void zero_red(OcShared& sh) {
     (&sh.red[0][0])[threadIdx.x] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
-// Per piece (one warp each): the warps' sums in warp order -> its slot.
+// Per piece (one warp each): the warps' sums in warp order -> its slot,
+// tagged with this launch's tag.
 __device__ __forceinline__ void piece_sums(const OcShared& sh,
                                            const OcTables& T,
-                                           const OcParams& q) {
+                                           const OcParams& q, uint32_t tag) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int j = warp; j < T.np; j += kOcWarps) {
     const float4 x = lane < kOcWarps ? sh.red[j][lane]
                                      : make_float4(0.f, 0.f, 0.f, 0.f);
     const F2 a = warp_sum_ff(F2{x.x, x.y}), b = warp_sum_ff(F2{x.z, x.w});
-    if (lane == 0)
-      q.slots[T.piece[j].slot] = make_float4(a.hi, a.lo, b.hi, b.lo);
+    if (lane == 0) {
+      uint64_t* w = q.slots + 2 * (size_t)T.piece[j].slot;
+      st_relaxed_u64(w, slot_word(a, tag));
+      st_relaxed_u64(w + 1, slot_word(b, tag));
+    }
   }
 }
 
@@ -567,33 +563,68 @@ __device__ __forceinline__ float phi_f(float z, const StepParams& p) {
   return z;
 }
 
-// Slot loads a lane keeps in flight when forming a ratio: a tensor has at
-// most one slot per CTA, so 8 x 32 covers a 152-SM grid in one round trip.
+// Slots a lane keeps in flight when forming a ratio: a tensor has at most
+// one slot per CTA, so 8 x 32 covers a 152-SM grid in one round trip.
 constexpr int kRatioLoads = 8;
 
 // Warp-wide, per piece: the tensor's slots in slot order (lane-strided,
-// kRatioLoads loads in flight, then a fixed tree) -> ||w||, ||u||, rho_k (Alg. 2 last
-// line with the zero-norm rule; LARS: times kappa), eta rho_k and eta
-// lambda_k for pass 2; exports where this CTA holds the tensor's first piece.
-__device__ __forceinline__ void piece_ratio(const StepParams& p,
-                                            const OcParams& q,
-                                            const OcPiece& P, float coef,
-                                            float lr, bool decoupled,
-                                            float* s_out, float* dd_out) {
+// kRatioLoads slots in flight, reloaded until every word carries this
+// launch's tag, then a fixed tree) -> ||w||, ||u||, rho_k (Alg. 2 last line
+// with the zero-norm rule; LARS: times kappa), eta rho_k and eta lambda_k
+// for pass 2; exports where this CTA holds the tensor's first piece.  Returns
+// false if the wait gave up (see the file header).
+__device__ __forceinline__ bool piece_ratio(const StepParams& p,
+                                         const OcParams& q, const OcPiece& P,
+                                         float coef, float lr, bool decoupled,
+                                         uint32_t tag, float* s_out,
+                                         float* dd_out) {
   const int lane = threadIdx.x & 31;
+  const uint64_t* slots = q.slots + 2 * (size_t)P.t_slot;
+  const uint64_t zero = slot_word(F2{0.f, 0.f}, tag);
   F2 a{0.f, 0.f}, b{0.f, 0.f};
-  for (int i = lane; i < P.t_nslots; i += kRatioLoads * 32) {
-    float4 x[kRatioLoads];
+  for (int base = 0; base < P.t_nslots; base += kRatioLoads * 32) {
+    uint64_t x[kRatioLoads][2];
 #pragma unroll
     for (int j = 0; j < kRatioLoads; ++j) {
-      const int k = i + 32 * j;
-      x[j] = k < P.t_nslots ? __ldcg(&q.slots[P.t_slot + k])
-                            : make_float4(0.f, 0.f, 0.f, 0.f);
+      const int k = base + lane + 32 * j;
+      x[j][0] = k < P.t_nslots ? ld_relaxed_u64(slots + 2 * k) : zero;
+      x[j][1] = k < P.t_nslots ? ld_relaxed_u64(slots + 2 * k + 1) : zero;
+    }
+    uint64_t t0 = 0;
+    for (uint32_t polls = 0;; ++polls) {
+      bool ready = true;
+#pragma unroll
+      for (int j = 0; j < kRatioLoads; ++j)
+        ready = ready && slot_tagged(x[j][0], tag) && slot_tagged(x[j][1], tag);
+      if (__all_sync(0xffffffffu, ready)) break;
+      if (polls == 0) t0 = global_ns();
+      if ((polls & 15u) == 15u) {   // warp-uniform: every lane counts alike
+        int stop = 0;
+        if (lane == 0) {
+          if (ld_acquire_u32(q.bar + kBarAbort)) {
+            stop = 1;
+          } else if (global_ns() - t0 > (uint64_t)q.wait_limit_ns) {
+            atomicOr(p.status, kStatusWaitTimeout);
+            atomicExch(q.bar + kBarAbort, 1u);
+            stop = 1;
+          }
+        }
+        if (__shfl_sync(0xffffffffu, stop, 0)) return false;
+      }
+#pragma unroll
+      for (int j = 0; j < kRatioLoads; ++j) {
+        const int k = base + lane + 32 * j;
+        if (k < P.t_nslots) {
+          if (!slot_tagged(x[j][0], tag)) x[j][0] = ld_relaxed_u64(slots + 2 * k);
+          if (!slot_tagged(x[j][1], tag))
+            x[j][1] = ld_relaxed_u64(slots + 2 * k + 1);
+        }
+      }
     }
 #pragma unroll
     for (int j = 0; j < kRatioLoads; ++j) {
-      a = ff_add(a, F2{x[j].x, x[j].y});
-      b = ff_add(b, F2{x[j].z, x[j].w});
+      a = ff_add(a, slot_value(x[j][0]));
+      b = ff_add(b, slot_value(x[j][1]));
     }
   }
   a = warp_sum_ff(a);
@@ -614,6 +645,7 @@ __device__ __forceinline__ void piece_ratio(const StepParams& p,
         atomicOr(p.status, kStatusNonfinite);
     }
   }
+  return true;
 }
 
 // ---------------------------------------------------------------------------
@@ -630,7 +662,7 @@ __global__ void __launch_bounds__(kOcThreads, 1)
 
   // a launch after one that gave up does nothing
   if (ld_acquire_u32(q.bar + kBarAbort)) return;
-  if (threadIdx.x == 0) sh.base = grid_base(q);   // before the first arrival
+  if (threadIdx.x == 0) sh.epoch = ld_acquire_u32(q.bar + kBarEpoch);
 
   // ---- per-launch constants ------------------------------------------------
   if (!kLars) {
@@ -670,19 +702,30 @@ __global__ void __launch_bounds__(kOcThreads, 1)
   for (int r = 0; r < q.n_rounds; ++r) {
     OcTables& T = sh.tab[r & 1];
     OcTables* next = r + 1 < q.n_rounds ? &sh.tab[(r + 1) & 1] : nullptr;
-    piece_sums(sh, T, q);
-    grid_arrive(q);
-    if (next) load_tables(*next, q, r + 1);   // while the others arrive
-    if (!grid_wait(q, p.status, grid_target(q, sh.base, r), &sh.ok)) return;
+    piece_sums(sh, T, q, write_tag(sh.epoch));
+    if (threadIdx.x == 0) sh.ok = 1;
+    if (next)
+      load_tables(*next, q, r + 1);   // while the other CTAs finish
+    else
+      __syncthreads();
     zero_red(sh);
     for (int j = warp; j < T.np; j += kOcWarps)
-      piece_ratio(p, q, T.piece[j], coef, lr, decoupled, &T.s[j], &T.dd[j]);
+      if (!piece_ratio(p, q, T.piece[j], coef, lr, decoupled,
+                       wait_tag(q, sh.epoch), &T.s[j], &T.dd[j]))
+        sh.ok = 0;
     __syncthreads();
+    if (!sh.ok) return;   // the launch gave up
     fused_pass<kOpt, GT, kCopy>(sh, s_rows, &T, next, k, wd, decoupled);
     __syncthreads();   // T's buffer is reloaded for round r + 2
   }
-  // every CTA read t (and the N-LAMB product) before the first barrier
-  if (blockIdx.x == 0 && threadIdx.x == 0) {
+  // The last CTA to finish advances the epoch and closes the step: every
+  // CTA read t (and the N-LAMB product) before its ticket, which releases
+  // it; CTA 0 stored the step scalars before its own.
+  __syncthreads();
+  if (threadIdx.x == 0 &&
+      atom_add_acq_rel(q.bar + kBarTicket, 1u) == gridDim.x - 1u) {
+    st_relaxed_u32(q.bar + kBarTicket, 0u);
+    st_relaxed_u32(q.bar + kBarEpoch, sh.epoch + 1u);
     const StepScalars sc = *p.scal;
     if (kNest && p.d_mu_product) *p.d_mu_product = sc.mu_prod;
     close_step(p, sc);

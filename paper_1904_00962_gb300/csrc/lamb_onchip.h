@@ -8,9 +8,10 @@
 //   TensorDesc oc_tensors[]   their tensor table
 //   OcSlice    slices[n_rounds][grid]   8 B  one CTA's part of a round
 //   OcPiece    pieces[]                80 B  rows of one tensor in one CTA
-//   float4     slots[n_pieces]         16 B  per piece: two-float sums of
-//                                             w^2 and u^2
-//   uint32     bar[kBarWords]                the grid barrier's words
+//   uint64     slots[n_pieces][2]      16 B  per piece: two-float sums of
+//                                             w^2 and u^2, tagged by launch
+//   uint32     bar[kBarWords]                launch epoch, finish ticket,
+//                                             abort word
 #pragma once
 #include <stdint.h>
 
@@ -66,18 +67,18 @@ struct __align__(8) OcSlice {   // one CTA's part of a resident round
   int16_t n_rows;
 };
 
-// Words of the plan's barrier block (uint32 indices; each group on its own
-// 128-byte line)
-constexpr int kBarCount = 0;     // words 0-1: 64-bit count of all arrivals
-                                 // at the plan's grid barriers (never reset)
-constexpr int kBarAbort = 32;    // a wait gave up: the plan is unusable
-constexpr int kBarWords = 64;
+// Words of the plan's launch block (uint32 indices; each on its own 128-byte
+// line)
+constexpr int kBarEpoch = 0;     // launches of the plan that finished
+constexpr int kBarTicket = 32;   // CTAs of the current launch that finished
+constexpr int kBarAbort = 64;    // a wait gave up: the plan is unusable
+constexpr int kBarWords = 96;
 
 struct OcParams {
   const OcSlice* slices;  // [n_rounds][grid]
   const OcPiece* pieces;
-  float4* slots;          // per piece: sum w^2 and sum u^2, each as a
-                          // two-float value (hi, lo)
+  uint64_t* slots;        // per piece, 2 words: sum w^2 and sum u^2, each
+                          // a two-float value with the launch's tag
   uint32_t* bar;          // kBarWords words, see kBar*
   int32_t n_rounds;
   int32_t extra_arrivals; // > 0 only in tests of the give-up path
