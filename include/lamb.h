@@ -123,9 +123,9 @@ typedef enum { LAMB_PHI_IDENTITY = 0, LAMB_PHI_CLIP = 1 } lamb_phi_t;
 #define LAMB_STATUS_BAD_STEP  0x2u      /* *d_step < 1 with bias correction:
                                            the step was skipped, nothing was
                                            written                          */
-#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* on-chip: a grid-barrier wait
-                                           inside the kernel (wait_limit_ms)
-                                           gave up
+#define LAMB_STATUS_WAIT_TIMEOUT 0x4u   /* on-chip: a wait for the other
+                                           CTAs' partial sums inside the
+                                           kernel (wait_limit_ms) gave up
                                            and the rest of the launch gave up
                                            with it, so the step is
                                            incomplete and the plan must be
@@ -159,8 +159,9 @@ typedef struct {
 /* lamb_plan_options_t.algorithm */
 #define LAMB_ALGO_AUTO 0          /* the library's default: on-chip when the
                                      whole layout fits one on-chip round (one
-                                     launch, one grid barrier; ~4.2M
-                                     parameters on a GB300), else two-pass
+                                     launch, one exchange of partial sums;
+                                     ~4.3M parameters on a GB300), else
+                                     two-pass
                                      (lamb_plan_get_info reports the choice) */
 #define LAMB_ALGO_TWO_PASS 1      /* two streaming kernels per step: 40 B of
                                      HBM traffic per parameter (bf16 g/copy) */
@@ -169,11 +170,12 @@ typedef struct {
                                      per SM).  Consecutive tensors are taken in
                                      rounds that fit the grid's shared memory
                                      (rows of LAMB_ONCHIP_ROW_ELEMS elements,
-                                     ~223 rows per SM: ~4.3M parameters on
+                                     ~217 rows per SM: ~4.3M parameters on
                                      152 SMs): pass 1 reads g, m, v, w once and
-                                     keeps w and the direction on chip across
-                                     a grid barrier, pass 2 writes w from
-                                     there -- 28 B/parameter (bf16 g/copy).  A
+                                     keeps w and the direction on chip while
+                                     the CTAs exchange their partial sums,
+                                     pass 2 writes w from there -- 28
+                                     B/parameter (bf16 g/copy).  A
                                      tensor larger than a round ("streamed")
                                      goes through the two-pass kernels first
                                      (40 B/parameter; 3 launches per step
@@ -191,14 +193,15 @@ typedef struct {
   int32_t blocks_per_sm; /* resident CTAs per SM for the persistent grid;
                             0 = as many as the occupancy calculator allows */
   int32_t algorithm;     /* LAMB_ALGO_*                                     */
-  int32_t wait_limit_ms; /* on-chip: a grid-barrier wait gives up after this
-                            long (LAMB_STATUS_WAIT_TIMEOUT); 0 = 1000      */
+  int32_t wait_limit_ms; /* on-chip: a CTA's wait for the other CTAs'
+                            partial sums gives up after this long
+                            (LAMB_STATUS_WAIT_TIMEOUT); 0 = 1000           */
   int32_t test_unmet_wait; /* on-chip, for tests of the give-up path only:
-                            nonzero makes every grid barrier wait for one
-                            arrival more than the grid makes, so the first
-                            wait runs out after wait_limit_ms and the launch
-                            returns with LAMB_STATUS_WAIT_TIMEOUT.  0 for
-                            every real use                                 */
+                            nonzero makes every CTA wait for partial sums
+                            tagged for a launch that never comes, so the
+                            first wait runs out after wait_limit_ms and the
+                            launch returns with LAMB_STATUS_WAIT_TIMEOUT.  0
+                            for every real use                             */
   int32_t onchip_max_ctas; /* on-chip: at most this many CTAs (one per SM);
                             0 = the SM count                               */
   int32_t onchip_rows;   /* on-chip: rows of shared memory per CTA, at most
