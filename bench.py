@@ -68,10 +68,10 @@ PROFILES = {
         os.path.join(ROOT, "profiles", "lamb_kernels_bert_large.md"),
         None, TWO_PASS_SOURCES),
     (3, "resnet50", "lamb"): (
-        os.path.join(ROOT, "profiles", "onchip_step_small_layouts.md"),
+        os.path.join(ROOT, "profiles", "onchip_step_kernel.md"),
         "resnet50/lamb", ONCHIP_SOURCES),
     (3, "resnet50", "lars"): (
-        os.path.join(ROOT, "profiles", "onchip_step_small_layouts.md"),
+        os.path.join(ROOT, "profiles", "onchip_step_kernel.md"),
         "resnet50/lars", ONCHIP_SOURCES),
 }
 # kept for the tests of the committed two-pass summary
