@@ -312,3 +312,71 @@ def test_last_error_is_thread_local(lib):
 def test_product_path_fails_loudly_without_library(tmp_path):
     with pytest.raises(B.LambLibraryMissing):
         B.load(str(tmp_path / "missing.so"))
+
+
+# ---------------------------------------------------------------------------
+# On-chip round planner (host only)
+# ---------------------------------------------------------------------------
+
+def _check_rounds(sizes, grid, rpc):
+    p, n_rounds = B.lamb_layout_rounds(sizes, grid, rpc)
+    row = B.LAMB_ONCHIP_ROW_ELEMS
+    cap = grid * rpc
+    rows_of = [(s + row - 1) // row for s in sizes]
+    streamed = p["round"] < 0
+    # tensors too large for a round are streamed whole, and only those
+    np.testing.assert_array_equal(
+        np.sort(p["tensor"][streamed]),
+        [k for k, r in enumerate(rows_of) if r > cap])
+    assert np.all(p["len"][streamed] == np.asarray(sizes)[p["tensor"][streamed]])
+    on = ~streamed
+    # every element of every other non-empty tensor is in exactly one piece,
+    # in order, whole rows except at the tensor's end, all in one round
+    for k, s in enumerate(sizes):
+        if rows_of[k] == 0 or rows_of[k] > cap:
+            assert not np.any(p["tensor"][on] == k), k
+            continue
+        sel = np.flatnonzero(on & (p["tensor"] == k))
+        off, ln = p["offset"][sel], p["len"][sel]
+        assert off[0] == 0 and off[-1] + ln[-1] == s, k
+        np.testing.assert_array_equal(off[1:], off[:-1] + ln[:-1])
+        assert np.all(off % row == 0)
+        assert np.all(p["rows"][sel] == (ln + row - 1) // row)
+        assert len(set(p["round"][sel].tolist())) == 1, k
+    # per (round, CTA): at most 16 pieces, rows packed from 0, within rpc
+    assert 0 <= p["round"][on].min(initial=0) and \
+        p["round"][on].max(initial=-1) < n_rounds
+    assert np.all((p["cta"][on] >= 0) & (p["cta"][on] < grid))
+    for r in range(n_rounds):
+        for c in np.unique(p["cta"][on & (p["round"] == r)]):
+            sel = np.flatnonzero(on & (p["round"] == r) & (p["cta"] == c))
+            assert len(sel) <= 16
+            fr, nr = p["first_row"][sel], p["rows"][sel]
+            assert fr[0] == 0
+            np.testing.assert_array_equal(fr[1:], fr[:-1] + nr[:-1])
+            assert fr[-1] + nr[-1] <= rpc
+    return p, n_rounds
+
+
+@pytest.mark.parametrize("grid,rpc", [(152, 217), (4, 8), (7, 3), (1, 224)])
+def test_rounds_cover_every_tensor_once(lib, grid, rpc):
+    rng = np.random.default_rng(grid * 1000 + rpc)
+    sizes = [0, 1, 127, 128, 129, 4096, 100003] + \
+        rng.integers(0, 3 * 128 * rpc, 60).tolist()
+    _check_rounds(sizes, grid, rpc)
+
+
+def test_rounds_of_the_paper_layouts(lib):
+    from paper_1904_00962_gb300.workloads import (bert_large_layout,
+                                                   resnet50_layout)
+    p, n = _check_rounds(resnet50_layout().sizes, 152, 217)
+    assert n == 7 and not np.any(p["round"] < 0)
+    p, n = _check_rounds(bert_large_layout().sizes, 152, 217)
+    # only the word embedding (30522 x 1024) is streamed
+    assert n == 74 and p["tensor"][p["round"] < 0].tolist() == [0]
+
+
+def test_rounds_reject_bad_input(lib):
+    for args in (([10], 0, 8), ([10], 4, 0), ([10], 4, 225), ([-1], 4, 8)):
+        with pytest.raises(B.LambError):
+            B.lamb_layout_rounds(*args)
