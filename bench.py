@@ -579,6 +579,9 @@ def run_ours(args):
                     chunk_elems=args.chunk_elems)
     info = plan.info()
     algo = info["algorithm"]
+    if args.algo == "auto" and opt == "lars" and algo == 3 and \
+            info["n_rounds"] > 1:
+        algo = 1   # AUTO runs LARS over several rounds on the two-pass kernels
     streamed = 0
     if algo == 3:
         cap = info["grid_blocks"] * info["rows_per_cta"] * info["row_elems"]

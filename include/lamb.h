@@ -157,11 +157,12 @@ typedef struct {
 } lamb_hyper_t;
 
 /* lamb_plan_options_t.algorithm */
-#define LAMB_ALGO_AUTO 0          /* the library's default: on-chip when the
-                                     whole layout fits one on-chip round (one
-                                     launch, one exchange of partial sums;
-                                     ~4.3M parameters on a GB300), else
-                                     two-pass
+#define LAMB_ALGO_AUTO 0          /* the library's default: on-chip when no
+                                     tensor is larger than an on-chip round
+                                     (~4.3M parameters on a GB300), else
+                                     two-pass; on such an on-chip plan,
+                                     lars_step over more than one round runs
+                                     the two-pass kernels
                                      (lamb_plan_get_info reports the choice) */
 #define LAMB_ALGO_TWO_PASS 1      /* two streaming kernels per step: 40 B of
                                      HBM traffic per parameter (bf16 g/copy) */

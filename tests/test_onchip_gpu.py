@@ -281,16 +281,31 @@ def test_onchip_barrier_wait_gives_up_and_a_new_plan_works():
     G.close()
 
 
-def test_auto_picks_on_chip_for_one_round_layouts_only():
-    """LAMB_ALGO_AUTO: the on-chip step when the whole layout is one round
-    (the tiny MLP), the two-pass step otherwise (ResNet-50: several rounds;
-    BERT-base: its word embedding exceeds a round)."""
-    for name, want in (("mlp", ON_CHIP), ("resnet50", B.LAMB_ALGO_TWO_PASS),
+def test_auto_picks_on_chip_unless_a_tensor_is_streamed():
+    """LAMB_ALGO_AUTO: the on-chip step when no tensor is larger than a round
+    (the tiny MLP, one round; ResNet-50, seven rounds), the two-pass step
+    otherwise (BERT-base: its word embedding exceeds a round).  On ResNet-50,
+    lamb_step runs the on-chip kernel (one launch) and lars_step the two
+    two-pass kernels."""
+    for name, want in (("mlp", ON_CHIP), ("resnet50", ON_CHIP),
                        ("bert_base", B.LAMB_ALGO_TWO_PASS)):
         L = W.get_layout(name)
         G = GpuLayout(L, algorithm=B.LAMB_ALGO_AUTO)
         info = G.plan.info()
         assert info["algorithm"] == want, name
         if want == ON_CHIP:
-            assert info["n_rounds"] == 1 and info["n_streamed_tensors"] == 0
+            assert info["n_streamed_tensors"] == 0
+            assert info["n_rounds"] == (1 if name == "mlp" else 7)
+        if name == "resnet50":
+            G.load_weights()
+            G.load_warm_state()
+            G.load_grads(2)
+            h = L.hyper
+            for lars, launches in ((False, 1), (True, 2)):
+                B.lamb_plan_set_timing(G.plan.handle, True)
+                G.step(2, f32(h.lr), c_hyper(h, lars=lars), lars=lars)
+                n, ms = B.lamb_plan_read_timing(G.plan.handle, 3)
+                B.lamb_plan_set_timing(G.plan.handle, False)
+                assert n == 1 and sum(x > 0 for x in ms) == launches, (lars, ms)
+            assert G.plan.query(clear=True) == 0
         G.close()
