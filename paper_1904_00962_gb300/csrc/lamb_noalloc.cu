@@ -110,7 +110,8 @@ cudaError_t na_setup(int dev, NaDevice** out) {
 // pointer table (with the 128-bit alignment flag), tickets, default results
 // (ratio 1, norms 0), status and work counters; then every thread writes
 // every 1024th chunk of the chunk table, finding its tensor by a binary
-// search over the tensors' first chunks.
+// search over the tensors' first chunks, kept in shared memory with the
+// length of each tensor's last chunk.
 constexpr int kSetupThreads = 1024;
 constexpr int kPerThread = kNaMaxTensors / kSetupThreads;   // 4
 
@@ -132,6 +133,8 @@ __global__ void __launch_bounds__(kSetupThreads)
   uint32_t* counters = reinterpret_cast<uint32_t*>(s + kOffCounters);
 
   __shared__ int64_t part[kSetupThreads];
+  __shared__ int32_t s_first[kNaMaxTensors];     // first chunk of tensor k
+  __shared__ int32_t s_lastlen[kNaMaxTensors];   // length of its last chunk
   const int t = threadIdx.x;
   // chunk counts of this thread's tensors, then an exclusive scan
   int64_t local[kPerThread];
@@ -161,6 +164,8 @@ __global__ void __launch_bounds__(kSetupThreads)
     td.n_chunks = (int32_t)local[i];
     td.decay = (!has_mask || mask[k]) ? 1.0f : 0.0f;
     tens[k] = td;
+    s_first[k] = (int32_t)first;
+    s_lastlen[k] = (int32_t)(d - (local[i] - 1) * kNaChunk);
     TensorPtrs tp{};
     tp.w = static_cast<float*>(raw[0 * kNaMaxTensors + k]);
     tp.g = raw[1 * kNaMaxTensors + k];
@@ -185,22 +190,22 @@ __global__ void __launch_bounds__(kSetupThreads)
     counters[0] = counters[1] = counters[2] = counters[3] = 0u;
   }
   __syncthreads();   // the tensor table is complete
-  const int64_t n_chunks = part[kSetupThreads - 1];
-  for (int64_t c = t; c < n_chunks; c += kSetupThreads) {
+  const int32_t n_chunks = (int32_t)part[kSetupThreads - 1];
+  for (int32_t c = t; c < n_chunks; c += kSetupThreads) {
     // the last tensor whose first chunk is <= c (a 0-chunk tensor shares its
     // first chunk with the next one, which comes later and wins)
     int lo = 0, hi = n - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) / 2;
-      if (tens[mid].first_chunk <= c) lo = mid;
+      if (s_first[mid] <= c) lo = mid;
       else hi = mid - 1;
     }
-    const int64_t off = (c - tens[lo].first_chunk) * kNaChunk;
-    const int64_t rem = tens[lo].numel - off;
+    // tensor lo holds chunk c; its chunks end where the next tensor's begin
+    const int32_t end = lo + 1 < n ? s_first[lo + 1] : n_chunks;
     ChunkDesc cd;
-    cd.offset = off;
+    cd.offset = (int64_t)(c - s_first[lo]) * kNaChunk;
     cd.tensor = lo;
-    cd.len = (int32_t)(rem < kNaChunk ? rem : kNaChunk);
+    cd.len = c + 1 == end ? s_lastlen[lo] : kNaChunk;
     chunks[c] = cd;
   }
 }

@@ -172,6 +172,7 @@ struct OcShared {
   int ok;
   uint32_t unused_draw;
   uint32_t epoch;        // the plan's launch epoch when this launch started
+  uint32_t abort;        // the plan's abort word when this launch started
 };
 
 // Exchange of the piece sums between CTAs, without a grid barrier.  A
@@ -512,22 +513,33 @@ __device__ __forceinline__ void fused_pass(OcShared& sh, float4* rows,
 // Tables, norms and trust ratio
 // ---------------------------------------------------------------------------
 // Loads round r's slice of this CTA into T (two CTA barriers inside).
-__device__ __forceinline__ void load_tables(OcTables& T, const OcParams& q,
-                                            int r) {
+// Round r's pieces of this CTA into T, by the calling threads with index
+// i = 0..kOcMaxPieces - 1 (the row map follows after a CTA barrier).
+__device__ __forceinline__ void load_pieces(OcTables& T, const OcParams& q,
+                                            int r, int i) {
   const OcSlice sl = q.slices[r * (int)gridDim.x + (int)blockIdx.x];
-  if ((int)threadIdx.x < sl.n_pieces)
-    T.piece[threadIdx.x] = q.pieces[sl.piece_begin + (int)threadIdx.x];
-  if (threadIdx.x == 0) {
+  if (i < sl.n_pieces) T.piece[i] = q.pieces[sl.piece_begin + i];
+  if (i == 0) {
     T.np = sl.n_pieces;
     T.nr = sl.n_rows;
   }
-  __syncthreads();
-  if ((int)threadIdx.x < sl.n_rows) {
+}
+
+// The piece of each row of T's slice.
+__device__ __forceinline__ void piece_rows(OcTables& T) {
+  if ((int)threadIdx.x < T.nr) {
     int j = 0;
-    for (int i = 1; i < sl.n_pieces; ++i)
+    for (int i = 1; i < T.np; ++i)
       if (T.piece[i].first_row <= (int)threadIdx.x) j = i;
     T.row_piece[threadIdx.x] = (uint8_t)j;
   }
+}
+
+__device__ __forceinline__ void load_tables(OcTables& T, const OcParams& q,
+                                            int r) {
+  load_pieces(T, q, r, (int)threadIdx.x);
+  __syncthreads();
+  piece_rows(T);
   __syncthreads();
 }
 
@@ -658,13 +670,19 @@ __global__ void __launch_bounds__(kOcThreads, 1)
   __shared__ OcShared sh;
   constexpr bool kLars = kOpt == kOptLars;
   constexpr int kNest = kLars ? 0 : kOpt;
-  const int warp = threadIdx.x >> 5;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  // a launch after one that gave up does nothing
-  if (ld_acquire_u32(q.bar + kBarAbort)) return;
-  if (threadIdx.x == 0) sh.epoch = ld_acquire_u32(q.bar + kBarEpoch);
-
-  // ---- per-launch constants ------------------------------------------------
+  // ---- prologue: the launch's independent loads run in separate warps and
+  // meet at the first CTA barrier -- the abort and epoch words (the last
+  // warp), eta (the warp before it), round 0's pieces (warp 8), and the step
+  // count with the constants formed from it (warps 0-5)
+  if (warp == kOcWarps - 1 && lane == 0) {
+    sh.abort = ld_acquire_u32(q.bar + kBarAbort);
+    sh.epoch = ld_acquire_u32(q.bar + kBarEpoch);
+  }
+  if (warp == kOcWarps - 2 && lane == 0)
+    sh.lr = (p.flags & kFlagLrSchedule) ? 0.f : *p.d_lr;
+  if (warp == 8 && q.n_rounds > 0) load_pieces(sh.tab[0], q, 0, lane);
   if (!kLars) {
     step_constants<kNest, false>(p, &sh.unused_draw, &sh.skip, &sh.k, &sh.t);
   } else if (threadIdx.x == 0) {
@@ -684,8 +702,12 @@ __global__ void __launch_bounds__(kOcThreads, 1)
   }
   zero_red(sh);
   __syncthreads();
-  if (sh.skip) return;   // a step count < 1 (status set by CTA 0)
-  if (threadIdx.x == 0) sh.lr = step_lr(p, sh.t);
+  // a launch after one that gave up does nothing more; a step count < 1 is
+  // skipped (status set by CTA 0)
+  if (sh.abort || sh.skip) return;
+  if (threadIdx.x == 0 && (p.flags & kFlagLrSchedule))
+    sh.lr = step_lr(p, sh.t);
+  if (q.n_rounds > 0) piece_rows(sh.tab[0]);
   __syncthreads();
   const LambConsts k = sh.k;
   const float lr = sh.lr;
@@ -694,7 +716,6 @@ __global__ void __launch_bounds__(kOcThreads, 1)
   const float coef = kLars ? (float)p.trust : 1.f;
 
   if (q.n_rounds > 0) {
-    load_tables(sh.tab[0], q, 0);
     fused_pass<kOpt, GT, kCopy>(sh, s_rows, nullptr, &sh.tab[0], k, wd,
                                 decoupled);
     __syncthreads();
