@@ -295,7 +295,13 @@ LAMB_API lamb_status_t lamb_plan_bind(lamb_plan_t plan, void* const* w,
  * Updates w, m, v in place (and the bf16 copy); g is read only.  Writes the
  * per-tensor norms and trust ratios (lamb_plan_trust_ratios).  No host
  * synchronisation, allocation or pageable copy: capturable in a CUDA graph,
- * and replays of the graph read the current *d_step and *d_lr. */
+ * and replays of the graph read the current *d_step and *d_lr.
+ * On an on-chip plan the step is one cooperative launch that holds every SM
+ * and whose CTAs wait for each other's partial sums: do not run on-chip
+ * steps of two plans at the same time on different streams (a wait that
+ * cannot be met gives up after wait_limit_ms with LAMB_STATUS_WAIT_TIMEOUT
+ * and leaves the plan unusable).  Steps of one plan, like all steps, must
+ * not overlap either. */
 LAMB_API lamb_status_t lamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
                         int64_t* d_step, const float* d_lr,
                         cudaStream_t stream);
