@@ -26,8 +26,8 @@ namespace lamb {
 // one CTA per SM.  The tensors are cut into rounds: runs of whole tensors whose
 // elements fit the grid's shared memory.  Every CTA owns a fixed slice of a
 // round's rows (kOcRow elements each), keeps w and the update direction of its
-// rows in shared memory across a grid barrier, and writes the new w from
-// there.  A tensor too large for one round is "streamed": the two-pass kernels
+// rows in shared memory while the CTAs exchange their partial sums, and writes
+// the new w from there.  A tensor too large for one round is "streamed": the two-pass kernels
 // take it, over a chunk table of such tensors only, before the on-chip launch.
 // ---------------------------------------------------------------------------
 constexpr int kOcThreads = 768;
@@ -81,8 +81,9 @@ struct OcParams {
                           // a two-float value with the launch's tag
   uint32_t* bar;          // kBarWords words, see kBar*
   int32_t n_rounds;
-  int32_t extra_arrivals; // > 0 only in tests of the give-up path
-  int64_t wait_limit_ns;  // a barrier wait gives up after this long
+  int32_t extra_arrivals; // > 0 only in tests of the give-up path: the
+                          // CTAs wait for a launch tag nobody writes
+  int64_t wait_limit_ns;  // a wait for partial sums gives up after this long
 };
 
 // Host planner of the on-chip step (planner.cpp).  grid CTAs, rows_per_cta

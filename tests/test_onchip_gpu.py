@@ -2,8 +2,9 @@
 fp64 oracle, on grids and shared-memory sizes small enough that the edge
 layout needs several resident rounds, pieces split across CTAs and streamed
 tensors; plus its agreement with the two-pass kernels, its determinism, and
-the bounded grid-barrier wait giving up (a wait made to run out on purpose:
-nothing faults, the launch returns with LAMB_STATUS_WAIT_TIMEOUT)."""
+the bounded wait for the other CTAs' partial sums giving up (a wait made to
+run out on purpose: nothing faults, the launch returns with
+LAMB_STATUS_WAIT_TIMEOUT)."""
 import math
 
 import numpy as np
@@ -235,9 +236,9 @@ def test_onchip_bitwise_repeatable(lars):
         assert torch.equal(a, b)
 
 
-def test_onchip_barrier_wait_gives_up_and_a_new_plan_works():
-    """A plan whose grid barriers wait for one arrival more than the grid
-    makes (a test-only option): the first wait runs out after 20 ms, every
+def test_onchip_wait_gives_up_and_a_new_plan_works():
+    """A plan whose CTAs wait for partial sums tagged for a launch that never
+    comes (a test-only option): the first wait runs out after 20 ms, every
     CTA returns, the status word says LAMB_STATUS_WAIT_TIMEOUT, the context
     stays usable, later steps of that plan do nothing, and a new plan on the
     same state computes the step correctly."""
@@ -255,8 +256,8 @@ def test_onchip_barrier_wait_gives_up_and_a_new_plan_works():
     torch.cuda.synchronize()                 # the launch returned
     st = G.plan.query(clear=True)
     assert st & B.LAMB_STATUS_WAIT_TIMEOUT
-    # the launch gave up at its first barrier: only round 0's pass 1 ran, so
-    # no weight changed
+    # the launch gave up at its first exchange: only round 0's pass 1 ran,
+    # so no weight changed
     assert torch.equal(G.st.w, w0)
     G.load_warm_state()
     G.step(2, lr, c_hyper(h))                # an aborted plan does nothing
