@@ -151,13 +151,28 @@ __device__ __forceinline__ F2 warp_sum_ff(F2 x) {
   return x;
 }
 
+// A row of a round's slice, formed once when the round's tables are loaded so
+// that the per-row work does not walk the piece table; packed in 32 bits to
+// leave the shared memory to the rows themselves: bits 0-15 the row's index
+// inside its tensor (a resident tensor has fewer than 2^16 rows), 16-23 its
+// element count (1..kOcRow), 24-27 its piece, 28 whether the piece's arrays
+// take 16-byte accesses.
+struct OcRow {
+  uint32_t bits;
+  __device__ int64_t x() const { return (int64_t)(bits & 0xFFFFu) * kOcRow; }
+  __device__ int cnt() const { return (int)((bits >> 16) & 0xFFu); }
+  __device__ int piece() const { return (int)((bits >> 24) & 0xFu); }
+  __device__ bool vec() const { return (bits >> 28) & 1u; }
+};
+static_assert(kOcRow <= 255 && kOcMaxPieces <= 16, "OcRow fields");
+
 // The tables of one round (double-buffered: one round's pass 2 runs inside
 // the next round's pass 1).
 struct OcTables {
   OcPiece piece[kOcMaxPieces];
   float s[kOcMaxPieces];           // eta rho_k of each piece's tensor
   float dd[kOcMaxPieces];          // eta lambda_k (decoupled decay) or 0
-  uint8_t row_piece[kOcMaxRows];
+  OcRow row[kOcMaxRows];           // per row of the slice
   int np, nr;                      // pieces and rows of this CTA's slice
 };
 
@@ -353,14 +368,14 @@ __device__ __forceinline__ void ring_issue(const OcTables& T, float4* rows,
   if (i < nw) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int row = warp + i * kOcWarps;
-    const OcPiece& P = T.piece[T.row_piece[row]];
-    const int e = (row - P.first_row) * kOcRow + lane * 4;
-    cnt = min(max(P.len - e, 0), 4);
-    const int64_t x = P.offset + e;
+    const OcRow R = T.row[row];
+    const OcPiece& P = T.piece[R.piece()];
+    cnt = min(max(R.cnt() - lane * 4, 0), 4);
+    const int64_t x = R.x() + lane * 4;
     const GT* gp = static_cast<const GT*>(P.g) + x;
     float4* slot_w = rows + row * 64 + lane;
     float4* slot_m = slot_w + 32;
-    if (cnt == 4 && (P.flags & kOcVec)) {
+    if (cnt == 4 && R.vec()) {
       cp_async16(slot_w, P.w + x);
       cp_async16(slot_m, P.m + x);
       g = GradRaw<GT>::load4(gp);
@@ -399,7 +414,8 @@ __device__ __forceinline__ void ring_consume(const OcTables& T, float4* rows,
   constexpr bool kV = kOpt != kOptLars;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = warp + i * kOcWarps;
-  const OcPiece& P = T.piece[T.row_piece[row]];
+  const OcRow R = T.row[row];
+  const OcPiece& P = T.piece[R.piece()];
   const float lam = decoupled ? 0.f : P.decay * wd;
   float4* slot_w = rows + row * 64 + lane;
   float4* slot_m = slot_w + 32;
@@ -409,10 +425,9 @@ __device__ __forceinline__ void ring_consume(const OcTables& T, float4* rows,
   su = 0.f;
   row1<kOpt>(GradRaw<GT>::widen(g), m4, v4, w4, u4, cnt, lam, k, sw, su);
   if (cnt > 0) {
-    const int64_t x = P.offset + (row - P.first_row) * kOcRow + lane * 4;
-    const bool vec = (P.flags & kOcVec) != 0;
-    store4(P.m, x, cnt, vec, m4);
-    if (kV) store4(P.v, x, cnt, vec, v4);
+    const int64_t x = R.x() + lane * 4;
+    store4(P.m, x, cnt, R.vec(), m4);
+    if (kV) store4(P.v, x, cnt, R.vec(), v4);
   }
   *slot_m = u4;
 }
@@ -439,9 +454,9 @@ __device__ __forceinline__ void acc_row(OcShared& sh, const OcTables& T,
                                         PieceAcc& acc, int i, int nw, float sw,
                                         float su) {
   const int warp = threadIdx.x >> 5;
-  const int piece = T.row_piece[warp + i * kOcWarps];
+  const int piece = T.row[warp + i * kOcWarps].piece();
   acc.add(sw, su);
-  if (i + 1 >= nw || T.row_piece[warp + (i + 1) * kOcWarps] != piece)
+  if (i + 1 >= nw || T.row[warp + (i + 1) * kOcWarps].piece() != piece)
     acc.flush(sh, piece);
 }
 
@@ -452,16 +467,15 @@ __device__ __forceinline__ void pass2_row(const OcTables& T,
                                           const float4* rows, int i) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = warp + i * kOcWarps;
-  const int j = T.row_piece[row];
-  const OcPiece& P = T.piece[j];
-  const int e = (row - P.first_row) * kOcRow + lane * 4;
-  const int c = min(max(P.len - e, 0), 4);
+  const OcRow R = T.row[row];
+  const int j = R.piece();
+  const int c = min(max(R.cnt() - lane * 4, 0), 4);
   if (c > 0) {
     const float4 o = update4(rows[row * 64 + lane],
                              rows[row * 64 + 32 + lane], T.s[j], T.dd[j]);
-    const bool vec = (P.flags & kOcVec) != 0;
-    store4(P.w, P.offset + e, c, vec, o);
-    if (kCopy) store_copy4(P.copy, P.offset + e, c, vec, o);
+    const int64_t x = R.x() + lane * 4;
+    store4(T.piece[j].w, x, c, R.vec(), o);
+    if (kCopy) store_copy4(T.piece[j].copy, x, c, R.vec(), o);
   }
 }
 
@@ -525,13 +539,19 @@ __device__ __forceinline__ void load_pieces(OcTables& T, const OcParams& q,
   }
 }
 
-// The piece of each row of T's slice.
+// The row records of T's slice: each row's piece, first element and count.
 __device__ __forceinline__ void piece_rows(OcTables& T) {
-  if ((int)threadIdx.x < T.nr) {
+  const int row = (int)threadIdx.x;
+  if (row < T.nr) {
     int j = 0;
     for (int i = 1; i < T.np; ++i)
-      if (T.piece[i].first_row <= (int)threadIdx.x) j = i;
-    T.row_piece[threadIdx.x] = (uint8_t)j;
+      if (T.piece[i].first_row <= row) j = i;
+    const OcPiece& P = T.piece[j];
+    const int r_in = row - P.first_row;   // row inside the piece
+    const uint32_t t_row = (uint32_t)(P.offset / kOcRow) + (uint32_t)r_in;
+    const uint32_t cnt = (uint32_t)min(P.len - r_in * kOcRow, kOcRow);
+    T.row[row].bits = (t_row & 0xFFFFu) | (cnt << 16) | ((uint32_t)j << 24) |
+                      ((P.flags & kOcVec) ? (1u << 28) : 0u);
   }
 }
 

@@ -35,6 +35,8 @@ constexpr int kOcWarps = kOcThreads / 32;
 constexpr int kOcRow = 128;          // elements per row: one float4 per lane
 constexpr int kOcMaxPieces = 16;     // pieces per CTA and round
 constexpr int kOcMaxRows = 224;      // rows per CTA (the plan may use fewer)
+constexpr int kOcMaxTensorRows = 65535;   // rows of a resident tensor (the
+                                          // kernel's row records hold 16 bits)
 constexpr int kOcRowBytes = 2 * kOcRow * 4;   // w and u of a row, fp32
 
 enum : uint32_t { kOcVec = 1u,       // arrays aligned for 4-element access

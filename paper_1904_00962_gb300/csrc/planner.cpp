@@ -264,7 +264,8 @@ int plan_onchip(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
   for (int32_t k = 0; k < n; ++k) {
     const int64_t r = rows_of(k);
     if (r == 0) continue;         // 0-element tensor: ratio 1, no work
-    if (r > cap) {                // streamed: the two-pass kernels take it
+    if (r > cap || r > kOcMaxTensorRows) {   // streamed: the two-pass
+                                             // kernels take it
       streamed->push_back(k);
       continue;
     }

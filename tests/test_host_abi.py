@@ -321,7 +321,8 @@ def test_product_path_fails_loudly_without_library(tmp_path):
 def _check_rounds(sizes, grid, rpc):
     p, n_rounds = B.lamb_layout_rounds(sizes, grid, rpc)
     row = B.LAMB_ONCHIP_ROW_ELEMS
-    cap = grid * rpc
+    # a resident tensor has at most 65,535 rows (the kernel's row records)
+    cap = min(grid * rpc, 65535)
     rows_of = [(s + row - 1) // row for s in sizes]
     streamed = p["round"] < 0
     # tensors too large for a round are streamed whole, and only those
@@ -364,6 +365,13 @@ def test_rounds_cover_every_tensor_once(lib, grid, rpc):
     sizes = [0, 1, 127, 128, 129, 4096, 100003] + \
         rng.integers(0, 3 * 128 * rpc, 60).tolist()
     _check_rounds(sizes, grid, rpc)
+
+
+def test_rounds_stream_tensors_beyond_65535_rows(lib):
+    row = B.LAMB_ONCHIP_ROW_ELEMS
+    sizes = [65535 * row, 65536 * row - 5, 10, 70000 * row]
+    p, n = _check_rounds(sizes, 400, 224)      # 89,600 rows per round
+    assert sorted(p["tensor"][p["round"] < 0].tolist()) == [1, 3]
 
 
 def test_rounds_of_the_paper_layouts(lib):
