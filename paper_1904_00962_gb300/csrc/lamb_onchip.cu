@@ -156,13 +156,14 @@ __device__ __forceinline__ F2 warp_sum_ff(F2 x) {
 // leave the shared memory to the rows themselves: bits 0-15 the row's index
 // inside its tensor (a resident tensor has fewer than 2^16 rows), 16-23 its
 // element count (1..kOcRow), 24-27 its piece, 28 whether the piece's arrays
-// take 16-byte accesses.
+// take 16-byte accesses, 29 whether it is its warp's last row of its piece.
 struct OcRow {
   uint32_t bits;
   __device__ int64_t x() const { return (int64_t)(bits & 0xFFFFu) * kOcRow; }
   __device__ int cnt() const { return (int)((bits >> 16) & 0xFFu); }
   __device__ int piece() const { return (int)((bits >> 24) & 0xFu); }
   __device__ bool vec() const { return (bits >> 28) & 1u; }
+  __device__ bool last() const { return (bits >> 29) & 1u; }
 };
 static_assert(kOcRow <= 255 && kOcMaxPieces <= 16, "OcRow fields");
 
@@ -317,14 +318,23 @@ __device__ __forceinline__ void row1(const float4& g, float4& m, float4& v,
                                      float& su) {
   float gg[4] = {g.x, g.y, g.z, g.w}, mm[4] = {m.x, m.y, m.z, m.w},
         vv[4] = {v.x, v.y, v.z, v.w}, ww[4] = {w.x, w.y, w.z, w.w}, uu[4];
+  if (c == 4) {   // a full row: the same operations, without the guards
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    if (j < c) {
+    for (int j = 0; j < 4; ++j) {
       uu[j] = elem1<kOpt>(gg[j], mm[j], vv[j], ww[j], lam, k);
       sw = __fmaf_rn(ww[j], ww[j], sw);
       su = __fmaf_rn(uu[j], uu[j], su);
-    } else {
-      uu[j] = 0.f;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (j < c) {
+        uu[j] = elem1<kOpt>(gg[j], mm[j], vv[j], ww[j], lam, k);
+        sw = __fmaf_rn(ww[j], ww[j], sw);
+        su = __fmaf_rn(uu[j], uu[j], su);
+      } else {
+        uu[j] = 0.f;
+      }
     }
   }
   m = make_float4(mm[0], mm[1], mm[2], mm[3]);
@@ -454,10 +464,9 @@ __device__ __forceinline__ void acc_row(OcShared& sh, const OcTables& T,
                                         PieceAcc& acc, int i, int nw, float sw,
                                         float su) {
   const int warp = threadIdx.x >> 5;
-  const int piece = T.row[warp + i * kOcWarps].piece();
+  const OcRow R = T.row[warp + i * kOcWarps];
   acc.add(sw, su);
-  if (i + 1 >= nw || T.row[warp + (i + 1) * kOcWarps].piece() != piece)
-    acc.flush(sh, piece);
+  if (R.last()) acc.flush(sh, R.piece());
 }
 
 // Pass 2 of row i of a round whose ratios are known: w <- w - eta rho_k u
@@ -540,18 +549,27 @@ __device__ __forceinline__ void load_pieces(OcTables& T, const OcParams& q,
 }
 
 // The row records of T's slice: each row's piece, first element and count.
+__device__ __forceinline__ int piece_of_row(const OcTables& T, int row) {
+  int j = 0;
+  for (int i = 1; i < T.np; ++i)
+    if (T.piece[i].first_row <= row) j = i;
+  return j;
+}
+
 __device__ __forceinline__ void piece_rows(OcTables& T) {
   const int row = (int)threadIdx.x;
   if (row < T.nr) {
-    int j = 0;
-    for (int i = 1; i < T.np; ++i)
-      if (T.piece[i].first_row <= row) j = i;
+    const int j = piece_of_row(T, row);
+    // the warp that takes this row next takes row + kOcWarps
+    const bool last = row + kOcWarps >= T.nr ||
+                      piece_of_row(T, row + kOcWarps) != j;
     const OcPiece& P = T.piece[j];
     const int r_in = row - P.first_row;   // row inside the piece
     const uint32_t t_row = (uint32_t)(P.offset / kOcRow) + (uint32_t)r_in;
     const uint32_t cnt = (uint32_t)min(P.len - r_in * kOcRow, kOcRow);
     T.row[row].bits = (t_row & 0xFFFFu) | (cnt << 16) | ((uint32_t)j << 24) |
-                      ((P.flags & kOcVec) ? (1u << 28) : 0u);
+                      ((P.flags & kOcVec) ? (1u << 28) : 0u) |
+                      (last ? (1u << 29) : 0u);
   }
 }
 
