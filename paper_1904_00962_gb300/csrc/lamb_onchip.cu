@@ -372,15 +372,15 @@ template <int kOpt, typename GT>
 __device__ __forceinline__ void ring_issue(const OcTables& T, float4* rows,
                                            int i, int nw,
                                            typename GradRaw<GT>::T& g,
-                                           float4& v, int& cnt) {
+                                           float4& v, OcRow& R) {
   constexpr bool kV = kOpt != kOptLars;
-  cnt = 0;
+  R.bits = 0u;   // no row: no elements
   if (i < nw) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int row = warp + i * kOcWarps;
-    const OcRow R = T.row[row];
+    R = T.row[row];
     const OcPiece& P = T.piece[R.piece()];
-    cnt = min(max(R.cnt() - lane * 4, 0), 4);
+    const int cnt = min(max(R.cnt() - lane * 4, 0), 4);
     const int64_t x = R.x() + lane * 4;
     const GT* gp = static_cast<const GT*>(P.g) + x;
     float4* slot_w = rows + row * 64 + lane;
@@ -411,20 +411,21 @@ __device__ __forceinline__ void ring_issue(const OcTables& T, float4* rows,
   }
 }
 
-// One arrived row: the new m, v to HBM, u over m in the slot; the lane's sums
-// of its (up to) four w^2 and u^2 in sw, su.
+// One arrived row (its record R as ring_issue read it): the new m, v to HBM,
+// u over m in the slot; the lane's sums of its (up to) four w^2 and u^2 in
+// sw, su.
 template <int kOpt, typename GT>
 __device__ __forceinline__ void ring_consume(const OcTables& T, float4* rows,
                                              int i,
                                              const typename GradRaw<GT>::T& g,
-                                             const float4& v, int cnt,
+                                             const float4& v, OcRow R,
                                              const LambConsts& k, float wd,
                                              bool decoupled, float& sw,
                                              float& su) {
   constexpr bool kV = kOpt != kOptLars;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = warp + i * kOcWarps;
-  const OcRow R = T.row[row];
+  const int cnt = min(max(R.cnt() - lane * 4, 0), 4);
   const OcPiece& P = T.piece[R.piece()];
   const float lam = decoupled ? 0.f : P.decay * wd;
   float4* slot_w = rows + row * 64 + lane;
@@ -459,12 +460,10 @@ struct PieceAcc {
   }
 };
 
-// Adds row i's sums; flushes if row i is the warp's last row of its piece.
-__device__ __forceinline__ void acc_row(OcShared& sh, const OcTables& T,
-                                        PieceAcc& acc, int i, int nw, float sw,
-                                        float su) {
-  const int warp = threadIdx.x >> 5;
-  const OcRow R = T.row[warp + i * kOcWarps];
+// Adds a row's sums; flushes if the row (record R) is its warp's last row of
+// its piece.
+__device__ __forceinline__ void acc_row(OcShared& sh, PieceAcc& acc, OcRow R,
+                                        float sw, float su) {
   acc.add(sw, su);
   if (R.last()) acc.flush(sh, R.piece());
 }
@@ -504,28 +503,28 @@ __device__ __forceinline__ void fused_pass(OcShared& sh, float4* rows,
   int done2 = 0;   // rows of the previous round written back
   typename GradRaw<GT>::T g0, g1;
   float4 v0, v1;
-  int c0 = 0, c1 = 0;
+  OcRow r0{0u}, r1{0u};
   PieceAcc acc{F2{0.f, 0.f}, F2{0.f, 0.f}};
   for (; done2 < min(2, nwp); ++done2) pass2_row<kCopy>(*prev, rows, done2);
   if (nwc > 0) {
-    ring_issue<kOpt, GT>(*cur, rows, 0, nwc, g0, v0, c0);
-    ring_issue<kOpt, GT>(*cur, rows, 1, nwc, g1, v1, c1);
+    ring_issue<kOpt, GT>(*cur, rows, 0, nwc, g0, v0, r0);
+    ring_issue<kOpt, GT>(*cur, rows, 1, nwc, g1, v1, r1);
   }
   cp_async_commit();
   for (int i = 0; i < nwc; i += 2) {
     cp_async_wait<0>();   // rows i, i + 1 have landed
     float sw0, su0, sw1 = 0.f, su1 = 0.f;
-    ring_consume<kOpt, GT>(*cur, rows, i, g0, v0, c0, k, wd, decoupled, sw0,
+    ring_consume<kOpt, GT>(*cur, rows, i, g0, v0, r0, k, wd, decoupled, sw0,
                            su0);
     if (i + 1 < nwc)
-      ring_consume<kOpt, GT>(*cur, rows, i + 1, g1, v1, c1, k, wd, decoupled,
+      ring_consume<kOpt, GT>(*cur, rows, i + 1, g1, v1, r1, k, wd, decoupled,
                              sw1, su1);
-    acc_row(sh, *cur, acc, i, nwc, sw0, su0);
-    if (i + 1 < nwc) acc_row(sh, *cur, acc, i + 1, nwc, sw1, su1);
+    acc_row(sh, acc, r0, sw0, su0);
+    if (i + 1 < nwc) acc_row(sh, acc, r1, sw1, su1);
     for (; done2 < min(i + 4, nwp); ++done2)
       pass2_row<kCopy>(*prev, rows, done2);
-    ring_issue<kOpt, GT>(*cur, rows, i + 2, nwc, g0, v0, c0);
-    ring_issue<kOpt, GT>(*cur, rows, i + 3, nwc, g1, v1, c1);
+    ring_issue<kOpt, GT>(*cur, rows, i + 2, nwc, g0, v0, r0);
+    ring_issue<kOpt, GT>(*cur, rows, i + 3, nwc, g1, v1, r1);
     cp_async_commit();
   }
   cp_async_wait<0>();
