@@ -159,7 +159,8 @@ typedef struct {
 /* lamb_plan_options_t.algorithm */
 #define LAMB_ALGO_AUTO 0          /* the library's default: on-chip when no
                                      tensor is larger than an on-chip round
-                                     (~4.3M parameters on a GB300), else
+                                     (~4.3M parameters on a GB300) and the
+                                     layout takes at most 32 rounds, else
                                      two-pass; on such an on-chip plan,
                                      lars_step over more than one round runs
                                      the two-pass kernels

@@ -314,3 +314,19 @@ def test_auto_picks_on_chip_unless_a_tensor_is_streamed():
                 assert n == 1 and sum(x > 0 for x in ms) == launches, (lars, ms)
             assert G.plan.query(clear=True) == 0
         G.close()
+
+
+@pytest.mark.parametrize("n,want", [(20, ON_CHIP), (40, B.LAMB_ALGO_TWO_PASS)])
+def test_auto_takes_two_pass_beyond_32_rounds(n, want):
+    """AUTO's round limit: with 4 CTAs of 8 rows (4,096 elements a round),
+    n tensors of 4,000 elements take n rounds; 20 stay on-chip, 40 do not."""
+    L = W.Layout(name="rounds", names=[f"t{i}" for i in range(n)],
+                 shapes=[(4000,)] * n, decay=[1] * n,
+                 init=[("normal", 0.02)] * n, grad_sigma=[1e-3] * n)
+    G = GpuLayout(L, algorithm=B.LAMB_ALGO_AUTO, onchip_max_ctas=4,
+                  onchip_rows=8)
+    info = G.plan.info()
+    assert info["algorithm"] == want
+    if want == ON_CHIP:
+        assert info["n_rounds"] == n
+    G.close()
