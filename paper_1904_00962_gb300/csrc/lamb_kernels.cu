@@ -105,31 +105,14 @@ __device__ __noinline__ void finalize_tensor(const StepParams& p, int k,
   const int lane = threadIdx.x & 31;
   double aw = 0.0, au = 0.0, ag = 0.0;
   float az = 0.f;
-  // each lane adds slots lane, lane + 32, ... in that order; the loads of
-  // kBatch of them are issued before the adds, so a tensor of thousands of
-  // chunks (BERT's word embedding: 1,908) costs a few L2 round trips, not
-  // one per slot
-  constexpr int kBatch = 8;
-  for (int base = 0; base < n; base += 32 * kBatch) {
-    float2 s[kBatch], q[kBatch];
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      const int i = base + lane + 32 * j;
-      if (i < n) {
-        s[j] = __ldcg(&p.slots[first + i]);
-        if (kGn) q[j] = __ldcg(&p.grad_slots[first + i]);
-      }
-    }
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      if (base + lane + 32 * j < n) {
-        aw += (double)s[j].x;
-        au += (double)s[j].y;
-        if (kGn) {
-          ag += (double)q[j].x;
-          az += q[j].y;
-        }
-      }
+  for (int i = lane; i < n; i += 32) {
+    const float2 s = __ldcg(&p.slots[first + i]);
+    aw += (double)s.x;
+    au += (double)s.y;
+    if (kGn) {
+      const float2 q = __ldcg(&p.grad_slots[first + i]);
+      ag += (double)q.x;
+      az += q.y;
     }
   }
 #pragma unroll
