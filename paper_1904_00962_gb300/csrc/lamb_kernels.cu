@@ -94,18 +94,23 @@ __device__ __forceinline__ void finalize_grad(const StepParams& p) {
   }
 }
 
-// Warp 0 of the CTA that finished tensor k's last chunk: fixed-order fp64
-// combine of the chunk slots -> norms and trust ratio.  Resets the ticket.
-// With the gradient check (kGn) it also forms the tensor's sum g^2 and
-// whether any of its elements was Inf/NaN, and counts the tensor done.
+// All threads of the CTA that finished tensor k's last chunk: fixed-order
+// fp64 combine of the chunk slots -> norms and trust ratio.  Thread t adds
+// slots t, t + kThreads, ... in that order; each warp adds its lanes, then
+// warp 0 the warps, in fixed trees.  Spreading the slots over the whole CTA
+// keeps a tensor of thousands of chunks (BERT's word embedding: 1,908) to a
+// few dependent L2 loads per thread.  Resets the ticket.  With the gradient
+// check (kGn) it also forms the tensor's sum g^2 and whether any of its
+// elements was Inf/NaN, and counts the tensor done.
 template <bool kGn>
 __device__ __noinline__ void finalize_tensor(const StepParams& p, int k,
                                              int first, int n, double coef) {
+  __shared__ double s_fin[4][kWarps];
   __threadfence();
-  const int lane = threadIdx.x & 31;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   double aw = 0.0, au = 0.0, ag = 0.0;
   float az = 0.f;
-  for (int i = lane; i < n; i += 32) {
+  for (int i = (int)threadIdx.x; i < n; i += kThreads) {
     const float2 s = __ldcg(&p.slots[first + i]);
     aw += (double)s.x;
     au += (double)s.y;
@@ -117,6 +122,27 @@ __device__ __noinline__ void finalize_tensor(const StepParams& p, int k,
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
+    aw += __shfl_down_sync(0xffffffffu, aw, o);
+    au += __shfl_down_sync(0xffffffffu, au, o);
+    if (kGn) {
+      ag += __shfl_down_sync(0xffffffffu, ag, o);
+      az += __shfl_down_sync(0xffffffffu, az, o);
+    }
+  }
+  if (lane == 0) {
+    s_fin[0][warp] = aw;
+    s_fin[1][warp] = au;
+    s_fin[2][warp] = ag;
+    s_fin[3][warp] = (double)az;
+  }
+  __syncthreads();
+  if (warp != 0) return;
+  aw = lane < kWarps ? s_fin[0][lane] : 0.0;
+  au = lane < kWarps ? s_fin[1][lane] : 0.0;
+  ag = lane < kWarps ? s_fin[2][lane] : 0.0;
+  az = lane < kWarps ? (float)s_fin[3][lane] : 0.f;
+#pragma unroll
+  for (int o = kWarps / 2; o > 0; o >>= 1) {
     aw += __shfl_down_sync(0xffffffffu, aw, o);
     au += __shfl_down_sync(0xffffffffu, au, o);
     if (kGn) {
@@ -168,7 +194,7 @@ __device__ __forceinline__ void publish_chunk(const StepParams& p, int c,
     }
   }
   __syncthreads();
-  if (*s_last && threadIdx.x < 32)
+  if (*s_last)   // the whole CTA
     finalize_tensor<kGn>(p, ch.tensor, td.first_chunk, td.n_chunks, coef);
 }
 
@@ -610,12 +636,12 @@ __global__ void __launch_bounds__(kThreads)
 // an unsharded step's bit for bit.
 __global__ void __launch_bounds__(kThreads)
     finalize_all_kernel(const StepParams p, double coef) {
-  const int warps = (int)(gridDim.x * blockDim.x) >> 5;
-  for (int k = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
-       k < p.n_tensors; k += warps) {
+  // one CTA per tensor, as when pass 1 finalises it: the same sums
+  for (int k = (int)blockIdx.x; k < p.n_tensors; k += (int)gridDim.x) {
     const TensorDesc td = p.tensors[k];
     if (td.n_chunks > 0)
       finalize_tensor<false>(p, k, td.first_chunk, td.n_chunks, coef);
+    __syncthreads();   // the finaliser's shared sums are reused
   }
 }
 
@@ -718,8 +744,7 @@ int launch_lars_pass2(const StepParams& p, int grad_bf16, int copy_bf16,
 }
 
 int launch_finalize_all(const StepParams& p, double coef, void* stream) {
-  const int warps_per_block = kThreads / 32;
-  const int grid = (p.n_tensors + warps_per_block - 1) / warps_per_block;
+  const int grid = p.n_tensors < 4096 ? p.n_tensors : 4096;
   finalize_all_kernel<<<grid < 1 ? 1 : grid, kThreads, 0,
                         static_cast<cudaStream_t>(stream)>>>(p, coef);
   return (int)cudaGetLastError();
