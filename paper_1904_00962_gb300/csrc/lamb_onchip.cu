@@ -8,13 +8,15 @@
 // shared memory of the SM that formed them.
 //
 // One cooperative launch per step: one CTA per SM (all resident at once),
-// 768 threads (24 warps), ~223 KB of shared memory holding up to 224 rows of
-// 128 elements (w and u in fp32, 1 KB per row).  The host planner
-// (planner.cpp, plan_onchip) cuts the tensors into ROUNDS of consecutive
-// whole tensors whose rows fit the grid (~4.3M parameters on 152 SMs).  Each
-// CTA owns a fixed slice of a round's rows, in pieces (a piece = the rows of
-// one tensor in one CTA, at most 16 per CTA); warp w takes rows w, w + 24, ...
-// Per round r:
+// 768 threads (24 warps), ~221 KB of dynamic shared memory holding up to 224
+// rows of 128 elements (w and u in fp32, 1 KB per row; 216 on a GB300).  The
+// host planner (planner.cpp, plan_onchip) cuts the tensors into ROUNDS of
+// consecutive whole tensors whose rows fit the grid (~4.2M parameters on 152
+// SMs).  Each CTA owns a fixed slice of a round's rows, in pieces (a piece =
+// the rows of one tensor in one CTA, at most 16 per CTA); warp w takes rows
+// w, w + 24, ...  When a round's tables are loaded, every row gets a 32-bit
+// record (its row inside the tensor, its count, its piece, its flags), which
+// is all the per-row work reads.  Per round r:
 //
 //   pass 1   each warp keeps two rows in flight: w and m of a row are copied
 //            (cp.async) straight into the row's shared-memory slot, g and v
@@ -50,6 +52,9 @@
 // not depend on timing: every run is bitwise identical.  The element
 // arithmetic is the two-pass kernels' (lamb_device.cuh), so m, v and u are
 // bit-identical to theirs; only the summation of the norms differs.
+//
+// The prologue's independent loads (the abort and epoch words, eta, round 0's
+// pieces, the step count) run in separate warps and meet at one CTA barrier.
 //
 // The tags come from a launch epoch that the last CTA of a launch advances,
 // so the step can be replayed from a CUDA graph.  The wait for a tensor's

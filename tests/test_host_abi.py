@@ -388,3 +388,9 @@ def test_rounds_reject_bad_input(lib):
     for args in (([10], 0, 8), ([10], 4, 0), ([10], 4, 225), ([-1], 4, 8)):
         with pytest.raises(B.LambError):
             B.lamb_layout_rounds(*args)
+
+
+def test_step_call_rejects_an_unknown_step(lib):
+    hyper = B.make_hyper()
+    with pytest.raises(ValueError):
+        B.step_call("adamw", 0, hyper, 0, 0)
