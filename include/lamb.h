@@ -172,7 +172,7 @@ typedef struct {
                                      per SM).  Consecutive tensors are taken in
                                      rounds that fit the grid's shared memory
                                      (rows of LAMB_ONCHIP_ROW_ELEMS elements,
-                                     ~217 rows per SM: ~4.3M parameters on
+                                     216 rows per SM: ~4.2M parameters on
                                      152 SMs): pass 1 reads g, m, v, w once and
                                      keeps w and the direction on chip while
                                      the CTAs exchange their partial sums,
