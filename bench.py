@@ -18,7 +18,9 @@ One JSON line is printed by rank 0:
             CUDA events on the launching stream over K steps
   e2e       the same metric through the same C-ABI call, but every step also
             copies that step's bf16 gradients host->device from pinned memory
-            and reads the step's result (the per-tensor trust ratios) back
+            and reads the step's result (the per-tensor trust ratios) back;
+            upload_gbs is the rate the loop moved gradients at, h2d_copy_gbs
+            that of a plain pinned copy of the same bytes, timed alone
   roofline  the dominant kernel's algorithmic bytes / its event-timed
             duration, against the measured HBM copy bandwidth
   cpu_baseline  the fp64 oracle on a bounded sample, on this host's cores
@@ -742,6 +744,19 @@ def run_ours(args):
     ms_e2e = e2.elapsed_time(e3)
     ms_e2e = max_over_ranks(ms_e2e, dev)
     assert math.isfinite(float(ratio_host[(k_e2e - 1) % 2][0]))
+    # The host link's own rate, outside the timed region: plain uploads of
+    # the same gradient bytes with nothing else running.
+    c0 = torch.cuda.Event(enable_timing=True)
+    c1 = torch.cuda.Event(enable_timing=True)
+    us = up_streams[0]
+    us.wait_stream(stream)
+    c0.record(us)
+    with torch.cuda.stream(us):
+        for _ in range(4):
+            g_dev[1].copy_(g_host, non_blocking=True)
+    c1.record(us)
+    c1.synchronize()
+    h2d_copy_gbs = 4 * h2d / (c0.elapsed_time(c1) * 1e6)
     calls.pop(plan2.handle, None)
     plan2.destroy()
     del g_dev[1]
@@ -855,6 +870,8 @@ def run_ours(args):
         "e2e": {"value": P * world * k_e2e / (ms_e2e * 1e-3), "unit": UNIT,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": k_e2e, "upload_streams": n_up,
+                "upload_gbs": h2d * k_e2e / (ms_e2e * 1e6),
+                "h2d_copy_gbs": h2d_copy_gbs,
                 "overlap": "upload of step s+1 overlaps step s "
                            "(two gradient buffers)"},
         "noalloc": noalloc,
