@@ -206,6 +206,9 @@ def parse_args():
                              "decoupled"],
                     help="optional step flags: the fused gradient check, "
                          "skip-on-non-finite, or decoupled weight decay")
+    ap.add_argument("--shard-world", type=int, default=0,
+                    help="time the sharded step of this many ranks, run in "
+                         "turn on one GPU, instead of the plain step")
     ap.add_argument("--layers", type=int, default=24,
                     help="encoder layers of the layout (24 = BERT-large; "
                          "fewer only for small profiling captures)")
@@ -533,6 +536,27 @@ def run_reference(args):
 # our arm
 # ---------------------------------------------------------------------------
 
+def layout_hyper(L, opt, variant="plain"):
+    """The layout's hyper-parameters for optimizer `opt` (LARS takes the
+    layout's own LARS settings, else lr 1, kappa 1e-3, no bias correction)
+    and the C-ABI struct for one step with them (t incremented per step)."""
+    from paper_1904_00962_gb300 import binding as B
+    lars = opt == "lars"
+    h = L.lars_hyper if (lars and L.lars_hyper) else L.hyper
+    if lars and not L.lars_hyper:
+        h = type(h)(lr=1.0, beta1=0.9, weight_decay=1e-4, trust_coef=1e-3,
+                    bias_correction=False)
+    hyper = B.make_hyper(beta1=h.beta1, beta2=h.beta2, eps=h.eps,
+                         weight_decay=h.weight_decay, phi=h.phi,
+                         gamma_l=h.gamma_l, gamma_u=h.gamma_u,
+                         trust_coef=h.trust_coef,
+                         bias_correction=not lars, increment_step=True,
+                         grad_norm=variant == "grad_norm",
+                         skip_nonfinite=variant == "skip_nonfinite",
+                         decoupled_decay=variant == "decoupled")
+    return h, hyper
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -567,10 +591,7 @@ def run_ours(args):
     if args.variant != "plain":
         workload += f"_{args.variant}"
     lars = opt == "lars"
-    h = L.lars_hyper if (lars and L.lars_hyper) else L.hyper
-    if lars and not L.lars_hyper:
-        h = type(h)(lr=1.0, beta1=0.9, weight_decay=1e-4, trust_coef=1e-3,
-                    bias_correction=False)
+    h, hyper = layout_hyper(L, opt, args.variant)
     P = L.n_params
     st = DeviceState(L.sizes, grad_dtype=L.grad_dtype,
                      copy_dtype=L.copy_dtype, device=dev, with_v=not lars)
@@ -597,14 +618,6 @@ def run_ours(args):
     d_lr = torch.full((1,), float(np.float32(h.lr)), dtype=torch.float32,
                       device=dev)
     d_prod = torch.ones(1, dtype=torch.float64, device=dev)
-    hyper = B.make_hyper(beta1=h.beta1, beta2=h.beta2, eps=h.eps,
-                         weight_decay=h.weight_decay, phi=h.phi,
-                         gamma_l=h.gamma_l, gamma_u=h.gamma_u,
-                         trust_coef=h.trust_coef,
-                         bias_correction=not lars, increment_step=True,
-                         grad_norm=args.variant == "grad_norm",
-                         skip_nonfinite=args.variant == "skip_nonfinite",
-                         decoupled_decay=args.variant == "decoupled")
 
     stream = torch.cuda.current_stream(dev)
     # one step per call, arguments marshalled once per plan
@@ -887,10 +900,186 @@ def run_ours(args):
     return 0
 
 
+def run_shard(args):
+    """The data-parallel (sharded) step of a W-way split, timed per rank on
+    one GPU: each step runs every rank's lamb_shard_pass1, then adds the
+    ranks' per-chunk sums arrays and puts the total back into every plan (what
+    an all-reduce over NCCL leaves on each rank; here device copies and adds,
+    outside the ranks' timings), then every rank's lamb_shard_pass2.  A rank's
+    time is its two launches, timed with events on the launching stream.  The
+    line gives the slowest rank's time per step beside the unsharded two-pass
+    step's time divided by W, which a perfectly split step would reach.
+    --chunk-elems sets the sharded plans' chunk size (the unsharded plan
+    keeps the library default)."""
+    import numpy as np
+    import torch
+
+    from paper_1904_00962_gb300 import binding as B
+    from paper_1904_00962_gb300 import build as build_mod
+    from paper_1904_00962_gb300.state import DeviceState, LambPlan
+    from paper_1904_00962_gb300.workloads import get_layout
+
+    rank, world, _ = dist_env()
+    if world > 1:   # the emulation is a one-process, one-GPU measurement
+        if rank == 0:
+            print(json.dumps({"impl": "ours", "unavailable":
+                              "--shard-world runs as one process on one GPU"}))
+        return 0
+    n_ranks = args.shard_world
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    if not os.path.exists(B.LIB_PATH):
+        build_mod.build()
+    B.load()
+    L = get_layout(args.layout)
+    opt = args.optimizer
+    h, hyper = layout_hyper(L, opt)
+    code = {"lamb": B.LAMB_OPT_LAMB, "lars": B.LAMB_OPT_LARS,
+            "nlamb": B.LAMB_OPT_NLAMB, "nnlamb": B.LAMB_OPT_NNLAMB}[opt]
+    psi = 0.004
+    st = DeviceState(L.sizes, grad_dtype=L.grad_dtype,
+                     copy_dtype=L.copy_dtype, device=dev,
+                     with_v=opt != "lars")
+    for k in range(L.n_tensors):
+        st.upload("w", k, L.weights(k))
+        st.upload("g", k, L.grad(k, 1))
+    stream = torch.cuda.current_stream(dev)
+    full = LambPlan(st, L.decay, algorithm=B.LAMB_ALGO_TWO_PASS)
+    plans = [LambPlan(st, L.decay, algorithm=B.LAMB_ALGO_TWO_PASS,
+                      chunk_elems=args.chunk_elems, shard_world=n_ranks,
+                      shard_rank=r)
+             for r in range(n_ranks)]
+    infos = [p.info() for p in plans]
+    lr32 = float(np.float32(h.lr))
+
+    def scalars():
+        return (torch.ones(1, dtype=torch.int64, device=dev),
+                torch.full((1,), lr32, dtype=torch.float32, device=dev),
+                torch.ones(1, dtype=torch.float64, device=dev))
+
+    sc = [scalars() for _ in range(n_ranks + 1)]   # the last: unsharded
+    nested = opt in ("nlamb", "nnlamb")
+    full_step = full.step_call(opt, hyper, sc[-1][0], sc[-1][1],
+                               sc[-1][2] if nested else None, psi, stream)
+    _, n_sums = B.lamb_plan_partials(plans[0].handle)
+    bufs = [torch.empty(n_sums, dtype=torch.float32, device=dev)
+            for _ in range(n_ranks)]
+    total = torch.empty(n_sums, dtype=torch.float32, device=dev)
+    sid = stream.cuda_stream
+
+    def pass_(r, second):
+        d_step, d_lr, d_prod = sc[r]
+        fn = plans[r].shard_pass2 if second else plans[r].shard_pass1
+        fn(hyper, code, d_step, d_lr, d_prod if nested else None,
+           momentum_decay=psi, stream=stream)
+
+    def exchange():
+        for r, p in enumerate(plans):
+            B.lamb_plan_copy_partials(p.handle, bufs[r].data_ptr(), False,
+                                      sid)
+        torch.sum(torch.stack(bufs), 0, out=total)
+        for p in plans:
+            B.lamb_plan_copy_partials(p.handle, total.data_ptr(), True, sid)
+
+    def sharded_step(ev=None):
+        for r in range(n_ranks):
+            if ev:
+                ev[r][0].record(stream)
+            pass_(r, False)
+            if ev:
+                ev[r][1].record(stream)
+        exchange()
+        for r in range(n_ranks):
+            if ev:
+                ev[r][2].record(stream)
+            pass_(r, True)
+            if ev:
+                ev[r][3].record(stream)
+
+    for _ in range(args.warmup):
+        full_step()
+        sharded_step()
+    for d_step, _, _ in sc:
+        d_step.fill_(1000)
+    torch.cuda.synchronize(dev)
+
+    gpu_id = None
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        gpu_id = None
+    clocks = ClockSampler(gpu_id)
+    time.sleep(0.3)
+    wall0 = _dt.datetime.now()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        full_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    ms_full = e0.elapsed_time(e1) / args.steps
+    # The host enqueues a sharded step (2W launches, 4W events and the
+    # emulated exchange) more slowly than small layouts run it, so a short
+    # spin kernel holds the GPU while every timed step is enqueued: the
+    # events then time the launches alone, never a wait for the host.  The
+    # timed steps are capped so that all of them fit the stream's queue.
+    ops = 9 * n_ranks + 3   # stream operations per sharded step
+    k_shard = max(1, min(args.steps, 800 // ops))
+    t0 = time.perf_counter()
+    sharded_step()
+    torch.cuda.synchronize(dev)
+    host_s = time.perf_counter() - t0
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(4)]
+            for _ in range(n_ranks)] for _ in range(k_shard)]
+    torch.cuda._sleep(int(min(1.0, 3 * k_shard * host_s) * 2.1e9))  # cycles
+    for k in range(k_shard):
+        sharded_step(evs[k])
+    torch.cuda.synchronize(dev)
+    wall1 = _dt.datetime.now()
+    clocks.mark(wall0, wall1)
+    p1 = [sum(evs[k][r][0].elapsed_time(evs[k][r][1])
+              for k in range(k_shard)) / k_shard for r in range(n_ranks)]
+    p2 = [sum(evs[k][r][2].elapsed_time(evs[k][r][3])
+              for k in range(k_shard)) / k_shard for r in range(n_ranks)]
+    per_rank = [a + b for a, b in zip(p1, p2)]
+    status = [p.query(clear=True) for p in plans + [full]]
+    clk = clocks.stop()
+    worst = max(per_rank)
+    line = {
+        "metric": "sharded step: slowest rank's time per step "
+                  "(every rank's launches run in turn on one GPU)",
+        "value": worst, "unit": "ms", "higher_is_better": False,
+        "world": n_ranks, "steps": k_shard, "unsharded_steps": args.steps,
+        "warmup": args.warmup, "per_rank_ms": per_rank, "pass1_ms": p1, "pass2_ms": p2,
+        "rank_chunks": [i["shard_chunk_end"] - i["shard_chunk_begin"]
+                        for i in infos],
+        "chunk_elems": infos[0]["chunk_elems"],
+        "unsharded_ms": ms_full, "ideal_ms": ms_full / n_ranks,
+        "ideal_over_slowest": ms_full / n_ranks / worst,
+        "sums_exchanged_bytes": 4 * n_sums,
+        "exchange": "per-chunk sums added on the device outside the ranks' "
+                    "timings (an all-reduce over NCCL on several GPUs)",
+        "dtype": "f32", "data": "synthetic",
+        "config": {"workload": f"{args.layout}_layout"
+                   + ("" if opt == "lamb" else f"_{opt}"),
+                   "n_params": L.n_params, "n_tensors": L.n_tensors,
+                   "grad_dtype": L.grad_dtype, "optimizer": opt,
+                   "step_t": 1000, "l2": "inputs larger than L2"},
+        "device_status": status, "clocks": clk,
+    }
+    print(json.dumps(line))
+    for p in plans + [full]:
+        p.destroy()
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.shard_world > 1:
+        return run_shard(args)
     return run_ours(args)
 
 

@@ -111,3 +111,33 @@ def test_committed_kernel_profile_has_the_parsed_fields():
     assert "kernel_source_sha256:" in text
     for i in range(2):
         assert f"traffic_bytes_per_launch[{i}]:" in text
+
+
+def test_layout_hyper_takes_the_layouts_lars_settings_or_the_default():
+    from paper_1904_00962_gb300 import binding as B
+    from paper_1904_00962_gb300.workloads import get_layout
+    rn = get_layout("resnet50")
+    h, c = bench.layout_hyper(rn, "lars")
+    assert h is rn.lars_hyper and c.trust_coef == pytest.approx(h.trust_coef)
+    assert not (c.flags & B.LAMB_FLAG_BIAS_CORRECTION)
+    mlp = get_layout("mlp")
+    h, c = bench.layout_hyper(mlp, "lars")
+    assert (h.lr, h.trust_coef, h.bias_correction) == (1.0, 1e-3, False)
+    h, c = bench.layout_hyper(get_layout("bert_large"), "lamb", "decoupled")
+    assert c.flags & B.LAMB_FLAG_BIAS_CORRECTION
+    assert c.flags & B.LAMB_FLAG_DECOUPLED_DECAY
+    assert c.flags & B.LAMB_FLAG_INCREMENT_STEP
+
+
+def test_shard_timing_declines_under_several_ranks():
+    """--shard-world is a one-process measurement: under torchrun every rank
+    exits 0 and rank 0 prints an `unavailable` line, before any device use."""
+    import json
+    import subprocess
+    env = dict(os.environ, RANK="0", LOCAL_RANK="0", WORLD_SIZE="2")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"),
+                        "--shard-world", "2"], capture_output=True, text=True,
+                       env=env, cwd=ROOT, timeout=300)
+    assert r.returncode == 0, r.stderr
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    assert "unavailable" in line
