@@ -631,7 +631,7 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // Every tensor's norms and trust ratio from the complete chunk slots (a
-// sharded step, after the slots were exchanged): one warp per tensor, the
+// sharded step, after the slots were exchanged): one CTA per tensor, the
 // same fixed-order combine as the finaliser of pass 1, so the results equal
 // an unsharded step's bit for bit.
 __global__ void __launch_bounds__(kThreads)
