@@ -215,7 +215,8 @@ typedef struct {
                             chunks a pass draws are short; 0 = none (the
                             default: measured slower on every layout here,
                             the short chunks' per-chunk cost outweighs the
-                            shorter tail)                                  */
+                            shorter tail).  A tail needs chunk_elems >=
+                            LAMB_TAIL_CHUNK_ELEMS                          */
   int32_t shard_world;   /* data-parallel shards of the step (0 or 1: the
                             plan covers every chunk).  With shard_world = W
                             the plan owns chunk range shard_rank of W
@@ -411,7 +412,8 @@ LAMB_API lamb_status_t lamb_plan_destroy(lamb_plan_t plan);
  * uses the tail reported by lamb_plan_get_info.  Writes up to `capacity`
  * rows into the three host arrays (any may be NULL when capacity is 0) and
  * the total row count into *n_chunks.  INVALID_ARG on bad sizes, chunk_elems
- * or tail_elems (< 0), or capacity too small (n_chunks is still written). */
+ * or tail_elems (< 0, or > 0 with chunk_elems < LAMB_TAIL_CHUNK_ELEMS), or
+ * capacity too small (n_chunks is still written). */
 LAMB_API lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
                                  int32_t chunk_elems, int64_t tail_elems,
                                  int32_t* chunk_tensor, int64_t* chunk_offset,
@@ -560,8 +562,10 @@ LAMB_API lamb_status_t lamb_plan_copy_partials(lamb_plan_t plan, float* buf,
 /* Host-only: the chunk range [*chunk_begin, *chunk_end) of shard `rank` of
  * `world` for the chunk table lamb_layout_chunks(sizes, chunk_elems,
  * tail_elems) gives: the chunks whose first element, counted over the layout
- * (tensors laid end to end), lies in [total rank / world, total (rank + 1) /
- * world).  A range may be empty.  INVALID_ARG on bad input. */
+ * (tensors laid end to end), lies in [floor(total rank / world),
+ * floor(total (rank + 1) / world)), total being the layout's element count.
+ * The ranges of ranks 0..world-1 are contiguous and cover every chunk once;
+ * a range may be empty.  INVALID_ARG on bad input. */
 LAMB_API lamb_status_t lamb_layout_shard(const int64_t* sizes,
                                          int32_t n_tensors,
                                          int32_t chunk_elems,
