@@ -411,9 +411,10 @@ LAMB_API lamb_status_t lamb_plan_destroy(lamb_plan_t plan);
  * they hold LAMB_TAIL_CHUNK_ELEMS; a chunk never spans two tensors.  A plan
  * uses the tail reported by lamb_plan_get_info.  Writes up to `capacity`
  * rows into the three host arrays (any may be NULL when capacity is 0) and
- * the total row count into *n_chunks.  INVALID_ARG on bad sizes, chunk_elems
- * or tail_elems (< 0, or > 0 with chunk_elems < LAMB_TAIL_CHUNK_ELEMS), or
- * capacity too small (n_chunks is still written). */
+ * the total row count into *n_chunks.  capacity 0 only counts: LAMB_OK with
+ * *n_chunks written.  INVALID_ARG on bad sizes, chunk_elems or tail_elems
+ * (< 0, or > 0 with chunk_elems < LAMB_TAIL_CHUNK_ELEMS), or a capacity
+ * above 0 that is too small (n_chunks is still written). */
 LAMB_API lamb_status_t lamb_layout_chunks(const int64_t* sizes, int32_t n_tensors,
                                  int32_t chunk_elems, int64_t tail_elems,
                                  int32_t* chunk_tensor, int64_t* chunk_offset,
@@ -481,8 +482,9 @@ LAMB_API lamb_status_t lamb_step_noalloc(
  * whole tensor as its elements and 0 rows.
  * Writes up to `capacity` pieces (the output arrays may be NULL when
  * capacity is 0), the total into *n_pieces and the round count into
- * *n_rounds.  INVALID_ARG on bad input or capacity too small (the counts are
- * still written).  lamb_plan_create uses the same planner with the device's
+ * *n_rounds.  capacity 0 only counts: LAMB_OK with the counts written.
+ * INVALID_ARG on bad input or a capacity above 0 that is too small (the
+ * counts are still written).  lamb_plan_create uses the same planner with the device's
  * SM count (at most; at least 32 rows per CTA) and shared-memory rows
  * (lamb_plan_get_info reports both). */
 LAMB_API lamb_status_t lamb_layout_rounds(

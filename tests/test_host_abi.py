@@ -82,6 +82,66 @@ def test_header_compiles_as_c():
     assert res.returncode == 0, res.stderr
 
 
+def test_c_program_links_and_plans(lib, tmp_path):
+    """A plain C99 program, linked against the shared library with nothing
+    but include/lamb.h, uses the host-only entry points: the ABI version,
+    the chunk table, a shard range and the on-chip rounds of a small layout,
+    and a rejected plan creation with its error message."""
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    src = tmp_path / "user.c"
+    src.write_text(r"""
+#include <stdio.h>
+#include <string.h>
+#include "lamb.h"
+int main(void) {
+  const int64_t sizes[4] = {1000000, 1024, 0, 70000};
+  int32_t t[128], len[128], n = 0;
+  int64_t off[128], total = 0, b = 0, e = 0;
+  if (lamb_abi_version() != LAMB_ABI_VERSION) return 10;
+  if (lamb_layout_chunks(sizes, 4, 16384, 0, t, off, len, 128, &n) != LAMB_OK)
+    return 11;
+  for (int i = 0; i < n; ++i) total += len[i];
+  if (total != 1071024) return 12;
+  if (lamb_layout_shard(sizes, 4, 16384, 0, 2, 1, &b, &e) != LAMB_OK)
+    return 13;
+  int64_t pieces = 0;
+  int32_t rounds = 0;
+  if (lamb_layout_rounds(sizes, 4, 152, 216, NULL, NULL, NULL, NULL, NULL,
+                         NULL, NULL, 0, &pieces, &rounds) != LAMB_OK)
+    return 14;                     /* capacity 0: the counts only */
+  lamb_plan_t plan = NULL;
+  if (lamb_plan_create(NULL, 4, NULL, LAMB_F32, LAMB_DTYPE_NONE, 0, NULL,
+                       &plan) !=
+      LAMB_ERR_INVALID_ARG || plan != NULL || strlen(lamb_last_error()) == 0)
+    return 15;
+  printf("%d %lld %lld %lld %d\n", n, (long long)b, (long long)e,
+         (long long)pieces, rounds);
+  return 0;
+}
+""")
+    build_dir = os.path.dirname(B.LIB_PATH)
+    exe = tmp_path / "user"
+    res = subprocess.run([gcc, "-std=c99", "-Wall", "-Werror",
+                          "-I", os.path.join(ROOT, "include"),
+                          "-I", "/usr/local/cuda/include", str(src),
+                          "-o", str(exe), "-L", build_dir, "-llamb",
+                          "-Wl,-rpath," + build_dir],
+                         capture_output=True, text=True)
+    assert res.returncode == 0, res.stderr
+    run = subprocess.run([str(exe)], capture_output=True, text=True,
+                         timeout=60)
+    assert run.returncode == 0, (run.returncode, run.stderr)
+    n, b, e, pieces, rounds = map(int, run.stdout.split())
+    t, o, ln = B.lamb_layout_chunks([1000000, 1024, 0, 70000], 16384)
+    assert n == len(t)
+    assert (b, e) == B.lamb_layout_shard([1000000, 1024, 0, 70000], 2, 1,
+                                         16384, 0)
+    p, n_rounds = B.lamb_layout_rounds([1000000, 1024, 0, 70000], 152, 216)
+    assert (pieces, rounds) == (len(p["round"]), n_rounds)
+
+
 def test_struct_layouts_match_ctypes(tmp_path):
     """sizeof and field offsets of the ABI structs, as a C compiler lays
     them out from include/lamb.h, equal the ctypes mirrors in binding.py."""
