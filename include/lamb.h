@@ -159,7 +159,7 @@ typedef struct {
 /* lamb_plan_options_t.algorithm */
 #define LAMB_ALGO_AUTO 0          /* the library's default: on-chip when no
                                      tensor is larger than an on-chip round
-                                     (~4.3M parameters on a GB300) and the
+                                     (~4.2M parameters on a GB300) and the
                                      layout takes at most 32 rounds, else
                                      two-pass; on such an on-chip plan,
                                      lars_step over more than one round runs
@@ -290,8 +290,9 @@ LAMB_API lamb_status_t lamb_plan_bind(lamb_plan_t plan, void* const* w,
 
 /* One LAMB step (Algorithm 2) over every tensor, enqueued on `stream`.
  *   d_step  DEVICE int64: t (>= 1 when bias correction is on).  Needed when
- *           LAMB_FLAG_BIAS_CORRECTION or LAMB_FLAG_INCREMENT_STEP is set,
- *           else may be NULL.
+ *           LAMB_FLAG_BIAS_CORRECTION, LAMB_FLAG_INCREMENT_STEP or
+ *           LAMB_FLAG_LR_SCHEDULE is set, else may be NULL (INVALID_ARG
+ *           when it is NULL but needed).
  *   d_lr    DEVICE float: eta_t for this step (with LAMB_FLAG_LR_SCHEDULE:
  *           NULL, or where the step writes the eta_t it computed).
  * Updates w, m, v in place (and the bf16 copy); g is read only.  Writes the
@@ -311,8 +312,8 @@ LAMB_API lamb_status_t lamb_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
 /* One LARS step (Algorithm 1 with trust coefficient kappa) over every
  * tensor.  Uses w, g, m (v is not touched).  beta1 is the momentum; the
  * momentum is damped by (1-beta1) as in Algorithm 1.  d_step is read only for
- * LAMB_FLAG_INCREMENT_STEP (may be NULL otherwise).  Same capture and
- * ownership rules as lamb_step. */
+ * LAMB_FLAG_INCREMENT_STEP and LAMB_FLAG_LR_SCHEDULE (may be NULL otherwise).
+ * Same capture and ownership rules as lamb_step. */
 LAMB_API lamb_status_t lars_step(lamb_plan_t plan, const lamb_hyper_t* hyper,
                         int64_t* d_step, const float* d_lr,
                         cudaStream_t stream);
@@ -484,9 +485,9 @@ LAMB_API lamb_status_t lamb_step_noalloc(
  * capacity is 0), the total into *n_pieces and the round count into
  * *n_rounds.  capacity 0 only counts: LAMB_OK with the counts written.
  * INVALID_ARG on bad input or a capacity above 0 that is too small (the
- * counts are still written).  lamb_plan_create uses the same planner with the device's
- * SM count (at most; at least 32 rows per CTA) and shared-memory rows
- * (lamb_plan_get_info reports both). */
+ * counts are still written).  lamb_plan_create uses the same planner with
+ * the device's SM count (at most; at least 32 rows per CTA) and
+ * shared-memory rows (lamb_plan_get_info reports both). */
 LAMB_API lamb_status_t lamb_layout_rounds(
     const int64_t* sizes, int32_t n_tensors, int32_t grid,
     int32_t rows_per_cta, int32_t* piece_round, int32_t* piece_cta,
