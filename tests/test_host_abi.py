@@ -63,6 +63,11 @@ def test_binding_constants_match_header_defines():
                  "LAMB_FLAG_DECOUPLED_DECAY", "LAMB_ONCHIP_ROW_ELEMS",
                  "LAMB_STATUS_SKIPPED"):
         assert flag in defs and hasattr(B, flag), flag
+    # and every enumerator (status codes, dtypes, phi) by name and value
+    enums = dict(re.findall(r"\b(LAMB_[A-Z0-9_]+)\s*=\s*(-?\d+)", hdr))
+    assert len(enums) == 11
+    for name, val in enums.items():
+        assert getattr(B, name) == int(val), name
 
 
 def test_abi_version(lib):
