@@ -70,6 +70,30 @@ def test_binding_constants_match_header_defines():
         assert getattr(B, name) == int(val), name
 
 
+def test_binding_signatures_match_the_header(lib):
+    """Every declared entry point's ctypes argtypes have the declaration's
+    arity, the same integer width or double for each scalar, and a pointer
+    for each pointer (plans and streams are pointers too)."""
+    text = open(HEADER).read()
+    decls = re.findall(r"LAMB_API\s+[\w\s\*]+?\b(\w+)\s*\(([^)]*)\)\s*;",
+                       text, re.S)
+    assert len(decls) == len(_declared())
+    scalar = {"int32_t": ctypes.c_int32, "int64_t": ctypes.c_int64,
+              "double": ctypes.c_double}
+    for name, params in decls:
+        ps = [p.strip() for p in params.split(",")]
+        ps = [] if ps == ["void"] else ps
+        at = getattr(lib, name).argtypes or []
+        assert len(at) == len(ps), name
+        for p, t in zip(ps, at):
+            base = p.replace("const", "").split()[0]
+            if "*" in p or base in ("lamb_plan_t", "cudaStream_t"):
+                assert t in (ctypes.c_void_p, ctypes.c_char_p) or \
+                    issubclass(t, ctypes._Pointer), (name, p)
+            else:
+                assert t is scalar[base], (name, p)
+
+
 def test_abi_version(lib):
     assert B.lamb_abi_version() == 3
 
