@@ -289,7 +289,8 @@ int plan_onchip(const int64_t* sizes, int32_t n, const uint8_t* decay_mask,
 // ---------------------------------------------------------------------------
 // Shards of a chunk table (the data-parallel split of the step): rank r of W
 // takes the chunks whose first element, counted over the layout, lies in
-// [total r / W, total (r + 1) / W).  Every rank computes the same split.
+// [floor(total r / W), floor(total (r + 1) / W)).  Every rank computes the
+// same split.
 // ---------------------------------------------------------------------------
 namespace lamb {
 
