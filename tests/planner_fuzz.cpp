@@ -190,6 +190,10 @@ bool check_rounds(const std::vector<int64_t>& sizes,
         CHECK(p.first_row == row && p.n_rows >= 1);
         row += p.n_rows;
         CHECK(p.offset % kOcRow == 0 && p.offset == covered[p.tensor]);
+        // the kernel's row record holds a row's index inside its tensor in
+        // 16 bits, its element count in 8 and its piece in 4
+        CHECK(p.offset / kOcRow + p.n_rows <= 65536);
+        CHECK(j < 16 && kOcRow < 256);
         CHECK(p.len >= 1 && p.len <= (int64_t)p.n_rows * kOcRow &&
               p.len > (int64_t)(p.n_rows - 1) * kOcRow);
         covered[p.tensor] += p.len;
