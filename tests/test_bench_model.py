@@ -141,3 +141,35 @@ def test_shard_timing_declines_under_several_ranks():
     assert r.returncode == 0, r.stderr
     line = json.loads(r.stdout.strip().splitlines()[-1])
     assert "unavailable" in line
+
+
+def test_clock_record_keeps_the_timed_window_and_its_reasons(tmp_path,
+                                                             monkeypatch):
+    """bench.py's clock sampler, fed by a stand-in nvidia-smi: only samples
+    inside the marked window count, the median SM clock and the maximum are
+    taken from them, and a throttle reason is reported when any of those
+    samples shows it active."""
+    import datetime as dt
+    import stat
+    rows = [  # time, sm, max, power, active, hw, hw_thermal, sw_thermal, cap
+        ("10:00:00.000", 1000, 2070, "Not Active", "Not Active"),   # before
+        ("10:00:00.200", 2070, 2070, "Not Active", "Not Active"),
+        ("10:00:00.300", 2050, 2070, "Not Active", "Active"),
+        ("10:00:00.400", 2070, 2070, "Not Active", "Not Active"),
+        ("10:00:00.900", 900, 2070, "Active", "Not Active"),       # after
+    ]
+    lines = [f"2026/12/02 {t}, {sm}, {mx}, 950.00, 0x0, {hw}, Not Active, "
+             f"Not Active, {cap}" for t, sm, mx, hw, cap in rows]
+    fake = tmp_path / "nvidia-smi"
+    fake.write_text("#!/bin/sh\ncat <<'EOF_'\n" + "\n".join(lines) +
+                    "\nEOF_\nexec sleep 30\n")
+    fake.chmod(fake.stat().st_mode | stat.S_IEXEC)
+    monkeypatch.setenv("PATH", f"{tmp_path}:{os.environ['PATH']}")
+    cs = bench.ClockSampler()
+    import time
+    time.sleep(0.5)   # let the stand-in print
+    cs.mark(dt.datetime(2026, 12, 2, 10, 0, 0, 100000),
+            dt.datetime(2026, 12, 2, 10, 0, 0, 500000))
+    rec = cs.stop()
+    assert rec == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "samples": 3,
+                   "reasons": ["sw_power_cap"]}
