@@ -382,9 +382,11 @@ static lamb_status_t plan_create(const int64_t* sizes, int32_t n_tensors,
                                           : "sizes is NULL");
   }
   p->h_tensors.resize((size_t)n_tensors);
-  // validates the sizes before the device is touched
+  // validates the sizes, the chunk size and the tail before the device is
+  // touched
   if (plan_chunks(sizes, n_tensors, chunk, nullptr, 0, &nch,
-                  p->h_tensors.data(), decay_mask, err, sizeof(err))) {
+                  p->h_tensors.data(), decay_mask, err, sizeof(err),
+                  tail_opt, kTailChunk)) {
     return fail(LAMB_ERR_INVALID_ARG, "%s", err);
   }
   for (int k = 0; k < n_tensors; ++k) p->n_params += sizes[k];

@@ -320,6 +320,16 @@ def test_create_validates_before_touching_the_device(lib):
     with pytest.raises(B.LambError) as ei:
         B.lamb_plan_create([10], device=-1)
     assert ei.value.status == B.LAMB_ERR_INVALID_ARG
+    with pytest.raises(B.LambError) as ei:   # a tail needs 2048+ chunks
+        B.lamb_plan_create([10], chunk_elems=1024, tail_elems=5000)
+    assert ei.value.status == B.LAMB_ERR_INVALID_ARG
+    for bad in (dict(tail_elems=-1), dict(wait_limit_ms=-1),
+                dict(algorithm=2), dict(blocks_per_sm=-1),
+                dict(onchip_rows=-1), dict(shard_world=2, shard_rank=2),
+                dict(shard_world=0, shard_rank=1)):
+        with pytest.raises(B.LambError) as ei:
+            B.lamb_plan_create([10], **bad)
+        assert ei.value.status == B.LAMB_ERR_INVALID_ARG, bad
 
 
 
